@@ -1,0 +1,118 @@
+"""Pins of the oracle's binary64 decode attention (paper Sec. 4: attention over the
+reconstructed cache) by closed forms, invariants and special cases."""
+import math
+import os
+
+import numpy as np
+import pytest
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _bits(x):
+    x = np.asarray(x, np.float32)
+    u = x.view(np.uint32)
+    return ((u.astype(np.uint64) + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+def _f32(bits):
+    return (bits.astype(np.uint32) << 16).view(np.float32)
+
+
+def test_zero_query_gives_mean_of_values(oracle):
+    rng = np.random.default_rng(0)
+    V = rng.standard_normal((1, 2, 9, 128))
+    K = rng.standard_normal((1, 2, 9, 128))
+    q = np.zeros((1, 4, 128), np.uint16)
+    out = oracle.attention_layer(q, K, V, 0.0883883476)
+    for qh in range(4):
+        assert np.allclose(out[0, qh], V[0, qh // 2].mean(0), atol=1e-14)
+
+
+def test_identical_keys_give_mean(oracle):
+    rng = np.random.default_rng(1)
+    V = rng.standard_normal((1, 1, 6, 128))
+    K = np.repeat(rng.standard_normal((1, 1, 1, 128)), 6, axis=2)
+    q = _bits(rng.standard_normal((1, 3, 128)))
+    out = oracle.attention_layer(q, K, V, 0.1)
+    for qh in range(3):
+        assert np.allclose(out[0, qh], V[0, 0].mean(0), atol=1e-13)
+
+
+def test_two_token_closed_form(oracle):
+    # q = e_0, keys differ only in channel 0: scores sigma*a, sigma*b; the output
+    # is the logistic mix sigmoid(sigma (a - b)) v1 + (1 - .) v2.
+    q = np.zeros((1, 1, 128), np.float32)
+    q[0, 0, 0] = 1.0
+    K = np.zeros((1, 1, 2, 128))
+    K[0, 0, 0, 0], K[0, 0, 1, 0] = 2.5, -1.0
+    V = np.zeros((1, 1, 2, 128))
+    V[0, 0, 0, :], V[0, 0, 1, :] = 1.0, 3.0
+    sigma = 0.75
+    out = oracle.attention_layer(_bits(q), K, V, sigma)
+    w = 1.0 / (1.0 + math.exp(-sigma * (2.5 - -1.0)))
+    assert np.allclose(out[0, 0], w * 1.0 + (1 - w) * 3.0, atol=1e-15)
+
+
+def test_dominant_key_selects_its_value(oracle):
+    rng = np.random.default_rng(2)
+    K = rng.standard_normal((1, 1, 5, 128)) * 0.01
+    K[0, 0, 3, :] = 50.0
+    V = rng.standard_normal((1, 1, 5, 128))
+    q = _bits(np.ones((1, 1, 128)))
+    out = oracle.attention_layer(q, K, V, 1.0)
+    assert np.allclose(out[0, 0], V[0, 0, 3], atol=1e-12)
+
+
+def test_token_permutation_invariance(oracle):
+    rng = np.random.default_rng(3)
+    K = rng.standard_normal((2, 2, 17, 128))
+    V = rng.standard_normal((2, 2, 17, 128))
+    q = _bits(rng.standard_normal((2, 6, 128)))
+    perm = rng.permutation(17)
+    a = oracle.attention_layer(q, K, V, 0.09)
+    b = oracle.attention_layer(q, K[:, :, perm], V[:, :, perm], 0.09)
+    assert np.allclose(a, b, atol=1e-13)
+
+
+def test_grouped_query_mapping(oracle):
+    # KV head 0 values are all 1, KV head 1 values all 2: query heads 0,1 read
+    # head 0 and 2,3 read head 1 (contiguous groups), whatever the scores.
+    rng = np.random.default_rng(4)
+    K = rng.standard_normal((1, 2, 8, 128))
+    V = np.stack([np.full((8, 128), 1.0), np.full((8, 128), 2.0)])[None]
+    q = _bits(rng.standard_normal((1, 4, 128)))
+    out = oracle.attention_layer(q, K, V, 0.09)
+    assert np.allclose(out[0, :, 0], [1, 1, 2, 2], atol=1e-14)
+
+
+def test_softmax_weights_sum_to_one(oracle):
+    # with V = 1 everywhere the output is exactly the sum of the weights
+    rng = np.random.default_rng(5)
+    K = rng.standard_normal((1, 1, 300, 128)) * 4
+    V = np.ones((1, 1, 300, 128))
+    q = _bits(rng.standard_normal((1, 2, 128)) * 3)
+    out = oracle.attention_layer(q, K, V, 0.0883883476)
+    assert np.allclose(out, 1.0, atol=1e-13)
+
+
+def _storage_rows():
+    rows = []
+    with open(os.path.join(GOLDEN, "storage_model.txt")) as f:
+        for line in f:
+            if line.strip() and not line.startswith("#"):
+                name, frac, ko, printed = [p.strip() for p in line.split("|")]
+                rows.append((name, float(frac), int(ko), float(printed)))
+    return rows
+
+
+@pytest.mark.parametrize("name,frac,keys_only,printed", _storage_rows())
+def test_storage_model_matches_paper(oracle, name, frac, keys_only, printed):
+    got = oracle.image_bits_per_elem(2, 32, frac, keys_only)
+    assert round(got, 2) == printed
+
+
+def test_storage_k_only_saving_about_22_percent(oracle):
+    kv = oracle.image_bits_per_elem(2, 32, 0.125, 0)
+    ko = oracle.image_bits_per_elem(2, 32, 0.125, 1)
+    assert round(100 * (kv - ko) / kv) == 22
