@@ -1,0 +1,218 @@
+/*
+ * headguard.h -- C ABI of the HeadGuard mixed-precision KV-cache library
+ * (GB300 / sm_103a).
+ *
+ * The library implements the data-parallel path of "HeadGuard: Selective Head
+ * Protection for Low-Bit VLM KV-Cache Quantization":
+ *   - quantize and bit-pack each layer's image-token keys / values with one of
+ *     three base quantizers (Sec. 1 per-token min-max RTN; Sec. 4 KIVI-style
+ *     per-channel keys / per-token values; Sec. 4 AKVQ-style Hadamard-128
+ *     rotation + per-token RTN), keeping the protected KV heads' image keys
+ *     (and values, unless keys-only) and every text token in BF16 (Sec. 3,
+ *     "Applying protection");
+ *   - reconstruct the cache as floating point (Sec. 4, simulated quantization:
+ *     values rounded to the quantizer's levels and reconstructed as floats);
+ *   - grouped-query decode attention that reads packed 2/4-bit codes and BF16
+ *     entries in one pass.
+ *
+ * Conventions shared by every entry point
+ *   Memory     The caller owns every byte.  The library never allocates device
+ *              memory; the cache lives in a caller-provided device "arena",
+ *              and decode attention uses a caller-provided workspace.  The
+ *              only host allocation is the hg_cache descriptor itself.
+ *   Tensors    Device tensors are dense row-major BF16 (uint16 bit patterns)
+ *              unless stated otherwise, head_dim = 128, and must be 16-byte
+ *              aligned.
+ *   Streams    Every device operation is enqueued on the given stream
+ *              (hg_stream_t is cudaStream_t; NULL means the legacy default
+ *              stream) and returns before the GPU work completes.
+ *   Errors     Arguments are validated on the host before anything is
+ *              launched; a call that returns an error has enqueued nothing and
+ *              changed no state.  HG_ERR_CUDA reports a launch error returned
+ *              by the CUDA runtime (cudaGetLastError after the launch).
+ *              Device code performs no waits of any kind.
+ *   Threads    A hg_cache may be used from one host thread at a time.
+ */
+#ifndef HEADGUARD_H
+#define HEADGUARD_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Same type as cudaStream_t, declared without the CUDA headers. */
+typedef struct CUstream_st *hg_stream_t;
+
+typedef enum hg_status {
+    HG_OK = 0,
+    HG_ERR_INVALID_ARG = 1,        /* null pointer, out-of-range index or size     */
+    HG_ERR_ALIGNMENT = 2,          /* a device pointer is not 16-byte aligned       */
+    HG_ERR_UNSUPPORTED = 3,        /* valid but not implemented (head_dim != 128 ..) */
+    HG_ERR_WORKSPACE_TOO_SMALL = 4,/* decode workspace smaller than required         */
+    HG_ERR_CAPACITY = 5,           /* append beyond max_new_tokens                   */
+    HG_ERR_CUDA = 6,               /* the CUDA runtime reported an error             */
+    HG_ERR_ARENA_TOO_SMALL = 7     /* cache arena smaller than hg_cache_layout says  */
+} hg_status;
+
+/* Base quantizers (Sec. 1 and Sec. 4). */
+typedef enum hg_base {
+    HG_BASE_MINMAX_TOKEN = 0,   /* per-token min-max, round to nearest level         */
+    HG_BASE_KIVI = 1,           /* keys per channel over 32-token groups, values per
+                                   token over 32-channel groups, BF16 residual window */
+    HG_BASE_AKVQ_HADAMARD = 2   /* keys rotated by the orthonormal Hadamard-128, then
+                                   per-token; values per-token, unrotated             */
+} hg_base;
+
+/* Cache geometry.  K/V of one layer are [batch][num_kv_heads][seq_len][head_dim].
+ * The image tokens are the contiguous span [img_start, img_start + img_len), the
+ * same for every batch row; every other prefill token is text (Sec. 3: text K/V
+ * stay BF16).  max_new_tokens is the decode-time capacity for appended tokens. */
+typedef struct hg_shape {
+    int32_t batch;
+    int32_t num_layers;
+    int32_t num_kv_heads;     /* 1..64 */
+    int32_t num_q_heads;      /* multiple of num_kv_heads, G = num_q_heads / num_kv_heads <= 16 */
+    int32_t head_dim;         /* must be 128 (the paper's heads, Sec. 5.4) */
+    int32_t seq_len;          /* prefill length T >= 1 */
+    int32_t img_start;
+    int32_t img_len;          /* img_start + img_len <= seq_len */
+    int32_t max_new_tokens;
+} hg_shape;
+
+/* Quantizer configuration.  bits in {2, 4}.  keys_only selects K-only protection
+ * (Sec. 3: protected heads keep image keys BF16, their image values follow the
+ * base).  The KIVI-style group sizes must be 32; kivi_residual >= 0 is the number
+ * of trailing prefill tokens kept BF16.  Unused fields are ignored for other bases. */
+typedef struct hg_quant_config {
+    int32_t base;
+    int32_t bits;
+    int32_t keys_only;
+    int32_t kivi_group_tokens;
+    int32_t kivi_group_channels;
+    int32_t kivi_residual;
+} hg_quant_config;
+
+/* Opaque host-side descriptor of a cache arena (offsets, mask, appended counts). */
+typedef struct hg_cache hg_cache;
+
+/* Class of a (layer, KV head), from the protection mask (Sec. 3). */
+typedef enum hg_head_class {
+    HG_HEAD_QUANTIZED = 0,  /* image K and V follow the base quantizer          */
+    HG_HEAD_KEYS_ONLY = 1,  /* protected, keys-only: image K BF16, image V coded */
+    HG_HEAD_PROTECTED = 2   /* protected K+V: image K and V BF16                 */
+} hg_head_class;
+
+/* Where one (layer, KV head) lives in the arena.  Offsets are bytes from the
+ * arena base of element [b = 0][t = 0]; each *_bstride is the byte stride
+ * between batch rows; an absent region has offset UINT64_MAX.
+ *   kb / vb   BF16 [batch][bf16_capacity][128]: the head's BF16 tokens in
+ *             prefill order (text, image tokens not quantized), then appended
+ *             tokens.  bf16_prefill of them come from the prefill.
+ *   kq / kqm  key codes / metadata (quantized class only).  Per-token bases:
+ *             codes uint32 [batch][nq][4*bits] (128 codes, channel order, packed
+ *             LSB-first, 32/bits per word), metadata float2 {scale, zero}
+ *             [batch][nq].  KIVI-style: codes [batch][nq/32][128][bits] (one
+ *             32-token group of one channel, token order), metadata
+ *             [batch][nq/32][128].
+ *   vq / vqm  value codes [batch][nq][4*bits] (channel order), metadata
+ *             [batch][nq][groups], groups = 1 (per token) or 4 (KIVI-style,
+ *             channels 32j..32j+31).
+ *   kimg      BF16 [batch][nq][128] image keys of a keys-only protected head.
+ * Quantized image tokens are [img_start, img_start + nq); nq equals img_len
+ * except for KIVI-style, where only whole 32-token groups inside
+ * [img_start, min(img_start + img_len, seq_len - kivi_residual)) are coded. */
+typedef struct hg_head_regions {
+    int32_t head_class;
+    int32_t nq;
+    int32_t bf16_prefill;
+    int32_t bf16_capacity;
+    uint64_t kb, vb, kq, kqm, vq, vqm, kimg;
+    uint64_t kb_bstride, kq_bstride, kqm_bstride, vq_bstride, vqm_bstride, kimg_bstride;
+} hg_head_regions;
+
+/* Bytes of device arena a cache of this shape / config / mask needs.
+ * head_mask: host uint8 [num_layers][num_kv_heads], non-zero = protected
+ * (Sec. 3, Eq. 2's selected set P).  Host only; no CUDA call. */
+hg_status hg_cache_layout(const hg_shape *shape, const hg_quant_config *config,
+                          const uint8_t *head_mask, size_t *arena_bytes);
+
+/* Create the descriptor of a cache stored in `arena` (device, 256-byte aligned,
+ * at least hg_cache_layout bytes; its contents need no initialisation).  The
+ * descriptor copies shape, config and mask.  Host only; no CUDA call.
+ * The arena must outlive the descriptor's use; hg_cache_destroy frees only the
+ * descriptor. */
+hg_status hg_cache_create(const hg_shape *shape, const hg_quant_config *config,
+                          const uint8_t *head_mask, void *arena, size_t arena_bytes,
+                          hg_cache **out);
+void hg_cache_destroy(hg_cache *cache);
+
+/* Region map of one (layer, head).  Host only. */
+hg_status hg_cache_head_regions(const hg_cache *cache, int32_t layer, int32_t head,
+                                hg_head_regions *out);
+
+/* Number of decode tokens appended so far to `layer` (host state). */
+int32_t hg_cache_appended(const hg_cache *cache, int32_t layer);
+
+/* Forget appended tokens (all layers); device memory is not touched. */
+hg_status hg_cache_reset_appended(hg_cache *cache);
+
+/* Quantize-pack layers [layer_begin, layer_begin + layer_count) from their BF16
+ * prefill K/V (Sec. 3 protection over a Sec. 1 / Sec. 4 base).  k and v are HOST
+ * arrays of layer_count DEVICE pointers, each [batch][num_kv_heads][seq_len][128]
+ * BF16; they are only read and may be freed once the stream work completes.
+ * Writes every region of those layers.  Packed codes and fp32 (scale, zero)
+ * follow the group quantizer: scale = (max - min) / (2^bits - 1), code =
+ * round-half-even((x - min) / scale), zero = min, codes 0 when scale == 0. */
+hg_status hg_quantize_kv(hg_cache *cache, int32_t layer_begin, int32_t layer_count,
+                         const void *const *k, const void *const *v, hg_stream_t stream);
+
+/* Reconstruct one layer as floating point (Sec. 4: code * scale + zero, the
+ * AKVQ-style keys rotated back).  k_out / v_out: device
+ * [batch][num_kv_heads][seq_len + appended][128], fp32 when out_fp32 != 0, else
+ * BF16 (round to nearest even), tokens in original order followed by the
+ * appended ones.  BF16 entries are copied exactly. */
+hg_status hg_dequantize_kv(const hg_cache *cache, int32_t layer, void *k_out, void *v_out,
+                           int32_t out_fp32, hg_stream_t stream);
+
+/* Append one decode token's K/V to layers [layer_begin, +layer_count) (text
+ * tokens stay BF16, Sec. 3).  k_new / v_new: device BF16
+ * [layer_count][batch][num_kv_heads][128].  Returns HG_ERR_CAPACITY if a layer
+ * already holds max_new_tokens appended tokens.  Advances the host-side count. */
+hg_status hg_append_kv(hg_cache *cache, int32_t layer_begin, int32_t layer_count,
+                       const void *k_new, const void *v_new, hg_stream_t stream);
+
+/* Workspace bytes hg_decode_attention needs for a launch over layer_count
+ * layers (any appended count up to max_new_tokens). */
+hg_status hg_decode_workspace_size(const hg_cache *cache, int32_t layer_count, size_t *bytes);
+
+/* Zero a workspace (cudaMemsetAsync).  Required once before its first use;
+ * decode attention leaves it zeroed again on completion. */
+hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
+
+/* Grouped-query decode attention of one step over layers
+ * [layer_begin, +layer_count), reading packed codes and BF16 entries in one
+ * pass.  q: device BF16 [layer_count][batch][num_q_heads][128]; out: device
+ * BF16, same shape.  Query head qh attends with KV head qh / G over every
+ * token of that head (prefill text, image, appended), with
+ * score = softmax_scale * <q, k>; softmax_scale <= 0 selects 1/sqrt(128).
+ * workspace: device, >= hg_decode_workspace_size(layer_count) bytes, zeroed
+ * once by hg_workspace_clear; one launch at a time may use it. */
+hg_status hg_decode_attention(const hg_cache *cache, int32_t layer_begin, int32_t layer_count,
+                              const void *q, void *out, float softmax_scale,
+                              void *workspace, size_t workspace_bytes, hg_stream_t stream);
+
+/* Sec. 5.4 storage accounting of the arena's image-token regions: bits per
+ * image K/V element actually stored (codes + 64-bit metadata + BF16 entries). */
+hg_status hg_cache_image_bits_per_elem(const hg_cache *cache, double *bits);
+
+/* Static description of a status code. */
+const char *hg_status_string(hg_status status);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* HEADGUARD_H */

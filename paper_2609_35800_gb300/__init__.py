@@ -1,0 +1,247 @@
+"""HeadGuard mixed-precision KV cache for GB300 -- Python binding of the C ABI.
+
+Thin ctypes marshalling over ``libheadguard.so`` (declared in
+``include/headguard.h``): every function here has the C entry point's name,
+converts its arguments (torch tensors -> device pointers, streams -> handles)
+and raises :class:`HGError` on a non-zero status.  All computation happens in
+the library's CUDA kernels; there is no Python or CPU fallback, and importing
+the compute functions without the built library raises.
+"""
+import ctypes
+import os
+
+from . import build as _build
+
+__all__ = [
+    "HGError", "Shape", "QuantConfig", "HeadRegions", "Cache",
+    "HG_BASE_MINMAX_TOKEN", "HG_BASE_KIVI", "HG_BASE_AKVQ_HADAMARD",
+    "HG_HEAD_QUANTIZED", "HG_HEAD_KEYS_ONLY", "HG_HEAD_PROTECTED",
+    "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
+    "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
+    "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_decode_attention",
+    "hg_cache_image_bits_per_elem", "hg_status_string", "library", "library_path",
+]
+
+HG_BASE_MINMAX_TOKEN = 0
+HG_BASE_KIVI = 1
+HG_BASE_AKVQ_HADAMARD = 2
+HG_HEAD_QUANTIZED = 0
+HG_HEAD_KEYS_ONLY = 1
+HG_HEAD_PROTECTED = 2
+NONE_OFFSET = (1 << 64) - 1
+
+STATUS = {
+    0: "HG_OK", 1: "HG_ERR_INVALID_ARG", 2: "HG_ERR_ALIGNMENT", 3: "HG_ERR_UNSUPPORTED",
+    4: "HG_ERR_WORKSPACE_TOO_SMALL", 5: "HG_ERR_CAPACITY", 6: "HG_ERR_CUDA",
+    7: "HG_ERR_ARENA_TOO_SMALL",
+}
+
+
+class HGError(RuntimeError):
+    def __init__(self, status, where):
+        self.status = status
+        super().__init__("%s: %s (%s)" % (where, STATUS.get(status, status),
+                                          hg_status_string(status)))
+
+
+class Shape(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "batch", "num_layers", "num_kv_heads", "num_q_heads", "head_dim", "seq_len",
+        "img_start", "img_len", "max_new_tokens")]
+
+
+class QuantConfig(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_int32) for n in (
+        "base", "bits", "keys_only", "kivi_group_tokens", "kivi_group_channels",
+        "kivi_residual")]
+
+
+class HeadRegions(ctypes.Structure):
+    _fields_ = ([(n, ctypes.c_int32) for n in ("head_class", "nq", "bf16_prefill",
+                                                "bf16_capacity")] +
+                [(n, ctypes.c_uint64) for n in ("kb", "vb", "kq", "kqm", "vq", "vqm", "kimg",
+                                                 "kb_bstride", "kq_bstride", "kqm_bstride",
+                                                 "vq_bstride", "vqm_bstride", "kimg_bstride")])
+
+
+_lib = None
+
+
+def library_path():
+    return _build.LIB
+
+
+def library():
+    """Load libheadguard.so (it must have been built by build.build())."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB
+    if not os.path.exists(path):
+        raise RuntimeError("libheadguard.so is not built (%s); run "
+                           "paper_2609_35800_gb300.build.build() first" % path)
+    L = ctypes.CDLL(path)
+    P, i32, sz = ctypes.c_void_p, ctypes.c_int32, ctypes.c_size_t
+    st = ctypes.c_int
+    sigs = {
+        "hg_cache_layout": ([P, P, P, ctypes.POINTER(sz)], st),
+        "hg_cache_create": ([P, P, P, P, sz, ctypes.POINTER(P)], st),
+        "hg_cache_destroy": ([P], None),
+        "hg_cache_head_regions": ([P, i32, i32, ctypes.POINTER(HeadRegions)], st),
+        "hg_cache_appended": ([P, i32], i32),
+        "hg_cache_reset_appended": ([P], st),
+        "hg_quantize_kv": ([P, i32, i32, P, P, P], st),
+        "hg_dequantize_kv": ([P, i32, P, P, i32, P], st),
+        "hg_append_kv": ([P, i32, i32, P, P, P], st),
+        "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
+        "hg_workspace_clear": ([P, sz, P], st),
+        "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
+        "hg_cache_image_bits_per_elem": ([P, ctypes.POINTER(ctypes.c_double)], st),
+        "hg_status_string": ([st], ctypes.c_char_p),
+    }
+    for name, (args, res) in sigs.items():
+        f = getattr(L, name)
+        f.argtypes = args
+        f.restype = res
+    _lib = L
+    return L
+
+
+def _check(status, where):
+    if status != 0:
+        raise HGError(status, where)
+
+
+def _ptr(x):
+    """Device/host address of a tensor (data_ptr), an int, or None."""
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    return x.data_ptr()
+
+
+def _stream(stream):
+    """cudaStream_t handle: a torch.cuda.Stream, an int, or None (current torch stream)."""
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+def _mask_bytes(mask):
+    import numpy as np
+    m = np.ascontiguousarray(np.asarray(mask, dtype=np.uint8))
+    return m, m.ctypes.data_as(ctypes.c_void_p)
+
+
+class Cache:
+    """Owning handle of an hg_cache descriptor (the arena stays caller-owned)."""
+
+    def __init__(self, handle, arena, shape, config, mask):
+        self.handle = handle
+        self.arena = arena
+        self.shape = shape
+        self.config = config
+        self.mask = mask
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.hg_cache_destroy(self.handle)
+            self.handle = None
+
+
+def hg_status_string(status):
+    return library().hg_status_string(int(status)).decode()
+
+
+def hg_cache_layout(shape, config, head_mask):
+    m, mp = _mask_bytes(head_mask)
+    out = ctypes.c_size_t(0)
+    _check(library().hg_cache_layout(ctypes.byref(shape), ctypes.byref(config), mp,
+                                     ctypes.byref(out)), "hg_cache_layout")
+    return out.value
+
+
+def hg_cache_create(shape, config, head_mask, arena, arena_bytes=None):
+    """Create the descriptor of a cache stored in `arena` (a device tensor or address)."""
+    m, mp = _mask_bytes(head_mask)
+    if arena_bytes is None:
+        arena_bytes = arena.numel() * arena.element_size()
+    h = ctypes.c_void_p()
+    _check(library().hg_cache_create(ctypes.byref(shape), ctypes.byref(config), mp, _ptr(arena),
+                                     arena_bytes, ctypes.byref(h)), "hg_cache_create")
+    return Cache(h, arena, shape, config, m.copy())
+
+
+def hg_cache_destroy(cache):
+    if cache.handle:
+        library().hg_cache_destroy(cache.handle)
+        cache.handle = None
+
+
+def hg_cache_head_regions(cache, layer, head):
+    out = HeadRegions()
+    _check(library().hg_cache_head_regions(cache.handle, layer, head, ctypes.byref(out)),
+           "hg_cache_head_regions")
+    return out
+
+
+def hg_cache_appended(cache, layer):
+    return library().hg_cache_appended(cache.handle, layer)
+
+
+def hg_cache_reset_appended(cache):
+    _check(library().hg_cache_reset_appended(cache.handle), "hg_cache_reset_appended")
+
+
+def hg_quantize_kv(cache, layer_begin, k_list, v_list, stream=None):
+    n = len(k_list)
+    assert len(v_list) == n
+    karr = (ctypes.c_void_p * n)(*[_ptr(k) for k in k_list])
+    varr = (ctypes.c_void_p * n)(*[_ptr(v) for v in v_list])
+    _check(library().hg_quantize_kv(cache.handle, layer_begin, n, karr, varr, _stream(stream)),
+           "hg_quantize_kv")
+
+
+def hg_dequantize_kv(cache, layer, k_out, v_out, out_fp32, stream=None):
+    _check(library().hg_dequantize_kv(cache.handle, layer, _ptr(k_out), _ptr(v_out),
+                                      1 if out_fp32 else 0, _stream(stream)), "hg_dequantize_kv")
+
+
+def hg_append_kv(cache, layer_begin, layer_count, k_new, v_new, stream=None):
+    _check(library().hg_append_kv(cache.handle, layer_begin, layer_count, _ptr(k_new),
+                                  _ptr(v_new), _stream(stream)), "hg_append_kv")
+
+
+def hg_decode_workspace_size(cache, layer_count):
+    out = ctypes.c_size_t(0)
+    _check(library().hg_decode_workspace_size(cache.handle, layer_count, ctypes.byref(out)),
+           "hg_decode_workspace_size")
+    return out.value
+
+
+def hg_workspace_clear(workspace, nbytes=None, stream=None):
+    if nbytes is None:
+        nbytes = workspace.numel() * workspace.element_size()
+    _check(library().hg_workspace_clear(_ptr(workspace), nbytes, _stream(stream)),
+           "hg_workspace_clear")
+
+
+def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, workspace,
+                        workspace_bytes=None, stream=None):
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(library().hg_decode_attention(cache.handle, layer_begin, layer_count, _ptr(q),
+                                         _ptr(out), float(softmax_scale), _ptr(workspace),
+                                         workspace_bytes, _stream(stream)),
+           "hg_decode_attention")
+
+
+def hg_cache_image_bits_per_elem(cache):
+    out = ctypes.c_double(0)
+    _check(library().hg_cache_image_bits_per_elem(cache.handle, ctypes.byref(out)),
+           "hg_cache_image_bits_per_elem")
+    return out.value

@@ -1,0 +1,384 @@
+// Host runtime of the HeadGuard C ABI (include/headguard.h): argument
+// validation, arena layout, decode work decomposition and kernel launches.
+// Every check runs before anything is enqueued; no device memory is
+// allocated here.
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "../../include/headguard.h"
+#include "hg_internal.h"
+#include "hg_layout.cuh"
+
+using namespace hg;
+
+struct hg_cache {
+  hg_shape shape;
+  hg_quant_config cfg;
+  Dims d;
+  std::vector<uint64_t> layer_mask;
+  std::vector<uint64_t> layer_base;
+  std::vector<int> appended;
+  char* arena;
+  size_t arena_bytes;
+  size_t needed_bytes;
+};
+
+namespace {
+
+constexpr int kTargetItems = 1024;  // decode work items per launch (~6.7 per SM on 152 SMs)
+
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* mask, Dims* d) {
+  if (!sh || !c || !mask) return HG_ERR_INVALID_ARG;
+  if (sh->batch < 1 || sh->num_layers < 1 || sh->num_kv_heads < 1 || sh->num_q_heads < 1 ||
+      sh->seq_len < 1 || sh->img_start < 0 || sh->img_len < 0 || sh->max_new_tokens < 0)
+    return HG_ERR_INVALID_ARG;
+  if ((int64_t)sh->img_start + sh->img_len > sh->seq_len) return HG_ERR_INVALID_ARG;
+  if (sh->num_q_heads % sh->num_kv_heads != 0) return HG_ERR_INVALID_ARG;
+  if (sh->head_dim != kD) return HG_ERR_UNSUPPORTED;
+  if (sh->num_kv_heads > kMaxHeads) return HG_ERR_UNSUPPORTED;
+  if (sh->num_q_heads / sh->num_kv_heads > kMaxG) return HG_ERR_UNSUPPORTED;
+  if (c->base != HG_BASE_MINMAX_TOKEN && c->base != HG_BASE_KIVI && c->base != HG_BASE_AKVQ_HADAMARD)
+    return HG_ERR_INVALID_ARG;
+  if (c->bits != 2 && c->bits != 4) return HG_ERR_UNSUPPORTED;
+  if (c->keys_only != 0 && c->keys_only != 1) return HG_ERR_INVALID_ARG;
+  if (c->base == HG_BASE_KIVI) {
+    if (c->kivi_group_tokens != kKiviGroup || c->kivi_group_channels != kKiviGroup)
+      return HG_ERR_UNSUPPORTED;
+    if (c->kivi_residual < 0) return HG_ERR_INVALID_ARG;
+  }
+  // every offset of a layer must stay far inside 64-bit and every token index in int
+  const int64_t tok = (int64_t)sh->seq_len + sh->max_new_tokens;
+  if (tok > (1 << 28)) return HG_ERR_UNSUPPORTED;
+  if ((int64_t)sh->batch * sh->num_kv_heads > 65535) return HG_ERR_UNSUPPORTED;  // grid.y
+
+  d->B = sh->batch;
+  d->L = sh->num_layers;
+  d->H = sh->num_kv_heads;
+  d->Hq = sh->num_q_heads;
+  d->G = sh->num_q_heads / sh->num_kv_heads;
+  d->T = sh->seq_len;
+  d->s = sh->img_start;
+  d->n = sh->img_len;
+  d->S_new = sh->max_new_tokens;
+  d->base = c->base;
+  d->bits = c->bits;
+  d->keys_only = c->keys_only;
+  d->residual = c->base == HG_BASE_KIVI ? c->kivi_residual : 0;
+  d->nq = quantized_count(d->T, d->s, d->n, d->base, d->residual);
+  return HG_OK;
+}
+
+uint64_t layer_mask_bits(const uint8_t* mask, int layer, int H) {
+  uint64_t m = 0;
+  for (int h = 0; h < H; ++h)
+    if (mask[(size_t)layer * H + h]) m |= (1ull << h);
+  return m;
+}
+
+// Arena layout: layer blocks back to back, each 256-byte aligned.
+size_t compute_layout(const Dims& d, const uint8_t* mask, std::vector<uint64_t>* bases,
+                      std::vector<uint64_t>* masks) {
+  uint64_t off = 0;
+  for (int l = 0; l < d.L; ++l) {
+    const uint64_t m = layer_mask_bits(mask, l, d.H);
+    const LayerGeom g = layer_geom(d, m);
+    if (bases) bases->push_back(off);
+    if (masks) masks->push_back(m);
+    off += g.size;
+  }
+  return (size_t)off;
+}
+
+bool range_ok(const hg_cache* c, int32_t begin, int32_t count) {
+  return c && count >= 1 && begin >= 0 && (int64_t)begin + count <= c->d.L;
+}
+
+// Chunk scale k: BF16 chunks of 128k tokens, coded chunks of 512k tokens.
+// The largest k that still gives kTargetItems items (appended = 0) wins.
+int chunk_scale(const hg_cache* c, int begin, int count) {
+  const Dims& d = c->d;
+  for (int k = 32; k > 1; k >>= 1) {
+    int64_t items = 0;
+    for (int l = begin; l < begin + count; ++l)
+      items += (int64_t)d.B * layer_items_per_row(d, c->layer_mask[l], 0, 128 * k, 512 * k);
+    if (items >= kTargetItems) return k;
+  }
+  return 1;
+}
+
+size_t ws_size_for(const hg_cache* c, int count, int k) {
+  return (size_t)ws_bytes(c->d, count, 128 * k, 512 * k);
+}
+
+hg_status cuda_status(cudaError_t e) { return e == cudaSuccess ? HG_OK : HG_ERR_CUDA; }
+
+void fill_table(const hg_cache* c, int begin, int count, LayerTable* t) {
+  for (int i = 0; i < count; ++i) {
+    t->base[i] = c->layer_base[begin + i];
+    t->mask[i] = c->layer_mask[begin + i];
+  }
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* hg_status_string(hg_status s) {
+  switch (s) {
+    case HG_OK: return "ok";
+    case HG_ERR_INVALID_ARG: return "invalid argument";
+    case HG_ERR_ALIGNMENT: return "device pointer not 16-byte aligned";
+    case HG_ERR_UNSUPPORTED: return "unsupported configuration";
+    case HG_ERR_WORKSPACE_TOO_SMALL: return "decode workspace too small";
+    case HG_ERR_CAPACITY: return "appended tokens exceed max_new_tokens";
+    case HG_ERR_CUDA: return "CUDA runtime error";
+    case HG_ERR_ARENA_TOO_SMALL: return "cache arena too small";
+  }
+  return "unknown status";
+}
+
+hg_status hg_cache_layout(const hg_shape* shape, const hg_quant_config* config,
+                          const uint8_t* head_mask, size_t* arena_bytes) {
+  Dims d;
+  const hg_status st = validate(shape, config, head_mask, &d);
+  if (st != HG_OK) return st;
+  if (!arena_bytes) return HG_ERR_INVALID_ARG;
+  *arena_bytes = compute_layout(d, head_mask, nullptr, nullptr);
+  return HG_OK;
+}
+
+hg_status hg_cache_create(const hg_shape* shape, const hg_quant_config* config,
+                          const uint8_t* head_mask, void* arena, size_t arena_bytes,
+                          hg_cache** out) {
+  Dims d;
+  const hg_status st = validate(shape, config, head_mask, &d);
+  if (st != HG_OK) return st;
+  if (!out || !arena) return HG_ERR_INVALID_ARG;
+  if ((reinterpret_cast<uintptr_t>(arena) & (kAlign - 1)) != 0) return HG_ERR_ALIGNMENT;
+  hg_cache* c = new (std::nothrow) hg_cache();
+  if (!c) return HG_ERR_INVALID_ARG;
+  c->shape = *shape;
+  c->cfg = *config;
+  c->d = d;
+  c->needed_bytes = compute_layout(d, head_mask, &c->layer_base, &c->layer_mask);
+  if (arena_bytes < c->needed_bytes) {
+    delete c;
+    return HG_ERR_ARENA_TOO_SMALL;
+  }
+  c->appended.assign(d.L, 0);
+  c->arena = static_cast<char*>(arena);
+  c->arena_bytes = arena_bytes;
+  *out = c;
+  return HG_OK;
+}
+
+void hg_cache_destroy(hg_cache* cache) { delete cache; }
+
+hg_status hg_cache_head_regions(const hg_cache* c, int32_t layer, int32_t head, hg_head_regions* out) {
+  if (!c || !out || layer < 0 || layer >= c->d.L || head < 0 || head >= c->d.H) return HG_ERR_INVALID_ARG;
+  const LayerGeom g = layer_geom(c->d, c->layer_mask[layer]);
+  const HeadGeom hd = head_geom(c->d, g, head);
+  const uint64_t base = c->layer_base[layer];
+  auto abs = [&](uint64_t off) { return off == kNone ? kNone : base + off; };
+  out->head_class = hd.cls;
+  out->nq = c->d.nq;
+  out->bf16_prefill = hd.bf16_prefill;
+  out->bf16_capacity = hd.cap;
+  out->kb = abs(hd.kb);
+  out->vb = abs(hd.vb);
+  out->kq = abs(hd.kq);
+  out->kqm = abs(hd.kqm);
+  out->vq = abs(hd.vq);
+  out->vqm = abs(hd.vqm);
+  out->kimg = abs(hd.kimg);
+  out->kb_bstride = hd.kb_bs;
+  out->kq_bstride = hd.kq_bs;
+  out->kqm_bstride = hd.kqm_bs;
+  out->vq_bstride = hd.vq_bs;
+  out->vqm_bstride = hd.vqm_bs;
+  out->kimg_bstride = hd.kimg_bs;
+  return HG_OK;
+}
+
+int32_t hg_cache_appended(const hg_cache* c, int32_t layer) {
+  if (!c || layer < 0 || layer >= c->d.L) return -1;
+  return c->appended[layer];
+}
+
+hg_status hg_cache_reset_appended(hg_cache* c) {
+  if (!c) return HG_ERR_INVALID_ARG;
+  for (auto& a : c->appended) a = 0;
+  return HG_OK;
+}
+
+hg_status hg_quantize_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count,
+                         const void* const* k, const void* const* v, hg_stream_t stream) {
+  if (!range_ok(c, layer_begin, layer_count) || !k || !v) return HG_ERR_INVALID_ARG;
+  for (int i = 0; i < layer_count; ++i) {
+    if (!k[i] || !v[i]) return HG_ERR_INVALID_ARG;
+    if (!aligned16(k[i]) || !aligned16(v[i])) return HG_ERR_ALIGNMENT;
+  }
+  const Dims& d = c->d;
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    QuantizeParams p;
+    std::memset(&p, 0, sizeof p);
+    p.d = d;
+    p.arena = c->arena;
+    p.n_layers = n;
+    p.tile_origin = d.s % 32;
+    p.n_tiles = (d.T - p.tile_origin + 32 + 31) / 32;
+    fill_table(c, layer_begin + done, n, &p.lt);
+    for (int i = 0; i < n; ++i) {
+      p.k[i] = static_cast<const uint16_t*>(k[done + i]);
+      p.v[i] = static_cast<const uint16_t*>(v[done + i]);
+    }
+    const hg_status st = cuda_status(launch_quantize(p, reinterpret_cast<cudaStream_t>(stream)));
+    if (st != HG_OK) return st;
+  }
+  for (int i = 0; i < layer_count; ++i) c->appended[layer_begin + i] = 0;
+  return HG_OK;
+}
+
+hg_status hg_dequantize_kv(const hg_cache* c, int32_t layer, void* k_out, void* v_out,
+                           int32_t out_fp32, hg_stream_t stream) {
+  if (!range_ok(c, layer, 1) || !k_out || !v_out) return HG_ERR_INVALID_ARG;
+  if (!aligned16(k_out) || !aligned16(v_out)) return HG_ERR_ALIGNMENT;
+  DequantParams p;
+  std::memset(&p, 0, sizeof p);
+  p.d = c->d;
+  p.arena = c->arena;
+  p.layer_base = c->layer_base[layer];
+  p.mask = c->layer_mask[layer];
+  p.appended = c->appended[layer];
+  p.out_fp32 = out_fp32 ? 1 : 0;
+  p.k_out = k_out;
+  p.v_out = v_out;
+  return cuda_status(launch_dequantize(p, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+hg_status hg_append_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count, const void* k_new,
+                       const void* v_new, hg_stream_t stream) {
+  if (!range_ok(c, layer_begin, layer_count) || !k_new || !v_new) return HG_ERR_INVALID_ARG;
+  if (!aligned16(k_new) || !aligned16(v_new)) return HG_ERR_ALIGNMENT;
+  for (int i = 0; i < layer_count; ++i)
+    if (c->appended[layer_begin + i] >= c->d.S_new) return HG_ERR_CAPACITY;
+  const Dims& d = c->d;
+  const size_t layer_elems = (size_t)d.B * d.H * kD;
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    AppendParams p;
+    std::memset(&p, 0, sizeof p);
+    p.d = d;
+    p.arena = c->arena;
+    p.n_layers = n;
+    fill_table(c, layer_begin + done, n, &p.lt);
+    for (int i = 0; i < n; ++i) p.appended[i] = c->appended[layer_begin + done + i];
+    p.k_new = static_cast<const uint16_t*>(k_new) + (size_t)done * layer_elems;
+    p.v_new = static_cast<const uint16_t*>(v_new) + (size_t)done * layer_elems;
+    const hg_status st = cuda_status(launch_append(p, reinterpret_cast<cudaStream_t>(stream)));
+    if (st != HG_OK) return st;
+  }
+  for (int i = 0; i < layer_count; ++i) c->appended[layer_begin + i] += 1;
+  return HG_OK;
+}
+
+hg_status hg_decode_workspace_size(const hg_cache* c, int32_t layer_count, size_t* bytes) {
+  if (!c || !bytes || layer_count < 1 || layer_count > c->d.L) return HG_ERR_INVALID_ARG;
+  // a launch over more than kMaxLayersPerLaunch layers reuses the workspace per group
+  const int per = std::min<int>(layer_count, kMaxLayersPerLaunch);
+  int kmin = 32;
+  for (int b = 0; b + per <= c->d.L; ++b) kmin = std::min(kmin, chunk_scale(c, b, per));
+  *bytes = ws_size_for(c, per, kmin);
+  return HG_OK;
+}
+
+hg_status hg_workspace_clear(void* ws, size_t bytes, hg_stream_t stream) {
+  if (!ws) return HG_ERR_INVALID_ARG;
+  return cuda_status(cudaMemsetAsync(ws, 0, bytes, reinterpret_cast<cudaStream_t>(stream)));
+}
+
+hg_status hg_decode_attention(const hg_cache* c, int32_t layer_begin, int32_t layer_count,
+                              const void* q, void* out, float softmax_scale, void* ws,
+                              size_t ws_bytes_given, hg_stream_t stream) {
+  if (!range_ok(c, layer_begin, layer_count) || !q || !out || !ws) return HG_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || !aligned16(ws)) return HG_ERR_ALIGNMENT;
+  if (!(softmax_scale == softmax_scale)) return HG_ERR_INVALID_ARG;  // NaN
+  const Dims& d = c->d;
+  const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)kD);
+  const size_t layer_elems = (size_t)d.B * d.Hq * kD;
+  // validate every group before launching any
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    const int k = chunk_scale(c, layer_begin + done, n);
+    if (ws_bytes_given < ws_size_for(c, n, k)) return HG_ERR_WORKSPACE_TOO_SMALL;
+  }
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    const int k = chunk_scale(c, layer_begin + done, n);
+    DecodeParams p;
+    std::memset(&p, 0, sizeof p);
+    p.d = d;
+    p.arena = c->arena;
+    p.n_layers = n;
+    p.cb = 128 * k;
+    p.cq = 512 * k;
+    p.max_items = max_head_items(d, p.cb, p.cq);
+    p.scale_log2 = scale * 1.4426950408889634f;
+    p.q = static_cast<const uint16_t*>(q) + (size_t)done * layer_elems;
+    p.out = static_cast<uint16_t*>(out) + (size_t)done * layer_elems;
+    p.counters = static_cast<uint32_t*>(ws);
+    p.partials = reinterpret_cast<float*>(static_cast<char*>(ws) + ws_counter_bytes(d, n));
+    fill_table(c, layer_begin + done, n, &p.lt);
+    int grid_x = 0;
+    for (int i = 0; i < n; ++i) {
+      const int l = layer_begin + done + i;
+      p.appended[i] = c->appended[l];
+      p.items_per_row[i] = layer_items_per_row(d, c->layer_mask[l], c->appended[l], p.cb, p.cq);
+      grid_x = std::max(grid_x, p.items_per_row[i] * d.B);
+    }
+    const hg_status st = cuda_status(launch_decode(p, grid_x, reinterpret_cast<cudaStream_t>(stream)));
+    if (st != HG_OK) return st;
+  }
+  return HG_OK;
+}
+
+hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {
+  if (!c || !bits) return HG_ERR_INVALID_ARG;
+  const Dims& d = c->d;
+  if (d.n == 0) return HG_ERR_INVALID_ARG;
+  // stored bits over all image K/V elements of the cache
+  double stored = 0.0;
+  const double code_bits = (double)d.bits * kD;                 // per coded token vector
+  const double kmeta_tok = d.base == kKivi ? 64.0 * kD / kKiviGroup : 64.0;
+  const double vmeta_tok = 64.0 * vgroups(d);
+  for (int l = 0; l < d.L; ++l) {
+    for (int h = 0; h < d.H; ++h) {
+      const int cls = head_class(d, c->layer_mask[l], h);
+      const double coded = d.nq, bf16 = d.n - d.nq;
+      double kb = 0, vb = 0;
+      if (cls == kQuantized) {
+        kb = coded * (code_bits + kmeta_tok) + bf16 * 16.0 * kD;
+        vb = coded * (code_bits + vmeta_tok) + bf16 * 16.0 * kD;
+      } else if (cls == kKeysOnly) {
+        kb = (double)d.n * 16.0 * kD;
+        vb = coded * (code_bits + vmeta_tok) + bf16 * 16.0 * kD;
+      } else {
+        kb = vb = (double)d.n * 16.0 * kD;
+      }
+      stored += (kb + vb) * d.B;
+    }
+  }
+  *bits = stored / ((double)d.L * d.H * d.B * d.n * kD * 2.0);
+  return HG_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,110 @@
+// Device helpers shared by the HeadGuard kernels: BF16 conversion, warp
+// reductions, the warp-distributed Hadamard-128 butterflies and the group
+// quantizer.  Every float operation that decides a stored bit (codes, scale,
+// zero, reconstructed values) uses an explicit round-to-nearest intrinsic so
+// that the compiler can neither fuse nor reorder it.
+#pragma once
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "hg_layout.cuh"
+
+namespace hg {
+
+__device__ __forceinline__ float bf16_to_f32(uint32_t h16) { return __uint_as_float(h16 << 16); }
+
+// Two BF16 packed in a 32-bit word -> two floats (low half first).
+__device__ __forceinline__ void bf16x2_to_f32(uint32_t w, float& lo, float& hi) {
+  lo = __uint_as_float(w << 16);
+  hi = __uint_as_float(w & 0xffff0000u);
+}
+
+// fp32 -> BF16 bits, round to nearest even (finite inputs and infinities).
+__device__ __forceinline__ uint32_t f32_to_bf16_rn(float f) {
+  uint32_t u = __float_as_uint(f);
+  if ((u & 0x7fffffffu) > 0x7f800000u) return 0x7fc0u;  // NaN
+  u += 0x7fffu + ((u >> 16) & 1u);
+  return u >> 16;
+}
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+  return v;
+}
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// fl32(1/sqrt(128)) -- bit pattern 0x3DB504F3.
+__device__ __forceinline__ float hadamard_c() { return __uint_as_float(0x3DB504F3u); }
+
+// Normalised Walsh-Hadamard transform of a 128-vector spread over a warp, lane
+// l holding channels 4l..4l+3 (Sylvester order).  Stages h = 1, 2 are inside a
+// lane, h = 4..64 pair lane l with lane l ^ (h/4).  Each butterfly maps
+// (a, b) = (x[j], x[j+h]) to (a + b, a - b); the 1/sqrt(128) factor is one
+// multiply after the last stage.  Self-inverse.
+__device__ __forceinline__ void fwht128_warp(float (&x)[4], int lane) {
+  const float a0 = __fadd_rn(x[0], x[1]), a1 = __fsub_rn(x[0], x[1]);
+  const float a2 = __fadd_rn(x[2], x[3]), a3 = __fsub_rn(x[2], x[3]);
+  x[0] = __fadd_rn(a0, a2);
+  x[2] = __fsub_rn(a0, a2);
+  x[1] = __fadd_rn(a1, a3);
+  x[3] = __fsub_rn(a1, a3);
+#pragma unroll
+  for (int m = 1; m < 32; m <<= 1) {
+    const bool upper = (lane & m) != 0;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const float p = __shfl_xor_sync(0xffffffffu, x[i], m);
+      x[i] = upper ? __fsub_rn(p, x[i]) : __fadd_rn(x[i], p);
+    }
+  }
+  const float c = hadamard_c();
+#pragma unroll
+  for (int i = 0; i < 4; ++i) x[i] = __fmul_rn(x[i], c);
+}
+
+// Group quantizer over a group spread across GL consecutive lanes (aligned),
+// 4 values per lane.  min / max by butterflies (exact), signed zeros folded to
+// +0, scale = (max - min) / (2^bits - 1), code = round-half-even((x - min) /
+// scale) clamped to the levels, codes 0 when scale == 0, zero = min.
+template <int GL>
+__device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, uint32_t (&code)[4],
+                                                float& scale, float& zero) {
+  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
+  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
+#pragma unroll
+  for (int o = 1; o < GL; o <<= 1) {
+    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+  }
+  mn = __fadd_rn(mn, 0.0f);
+  mx = __fadd_rn(mx, 0.0f);
+  const float levels = (float)((1 << bits) - 1);
+  scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  zero = mn;
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    if (scale == 0.0f) {
+      code[i] = 0u;
+    } else {
+      const float q = __fdiv_rn(__fsub_rn(x[i], mn), scale);
+      float r = rintf(q);
+      r = fminf(fmaxf(r, 0.0f), levels);
+      code[i] = (uint32_t)r;
+    }
+  }
+}
+
+// Reconstruction fl32(fl32(code * scale) + zero).
+__device__ __forceinline__ float dequant1(uint32_t code, float scale, float zero) {
+  return __fadd_rn(__fmul_rn((float)code, scale), zero);
+}
+
+__device__ __forceinline__ uint4 ldg16(const void* p) { return __ldg(reinterpret_cast<const uint4*>(p)); }
+__device__ __forceinline__ uint2 ldg8(const void* p) { return __ldg(reinterpret_cast<const uint2*>(p)); }
+
+}  // namespace hg

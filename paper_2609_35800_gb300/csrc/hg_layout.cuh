@@ -1,0 +1,196 @@
+// Arena geometry of the mixed-precision KV cache, shared by the host runtime
+// and the kernels.  Everything here is arithmetic on the cache dimensions and
+// one layer's 64-bit protection mask (Sec. 3, "Applying protection"), so a
+// kernel can locate any (layer, batch row, head) region from two words per
+// layer held in its launch parameters.
+#pragma once
+#include <stdint.h>
+
+#ifdef __CUDACC__
+#define HG_HD __host__ __device__ __forceinline__
+#else
+#define HG_HD inline
+#endif
+
+namespace hg {
+
+constexpr int kD = 128;            // head_dim (the paper's 128-d heads, Sec. 5.4)
+constexpr int kMaxHeads = 64;      // one bit per KV head in a uint64 mask
+constexpr int kMaxG = 16;          // query heads per KV head
+constexpr int kMaxLayersPerLaunch = 64;
+constexpr int kKiviGroup = 32;     // KIVI-style key group (tokens) and value group (channels)
+constexpr uint64_t kAlign = 256;   // region alignment inside the arena
+constexpr uint64_t kNone = ~0ull;
+
+enum Base : int { kMinMax = 0, kKivi = 1, kAkvq = 2 };
+enum HeadClass : int { kQuantized = 0, kKeysOnly = 1, kProtected = 2 };
+
+struct Dims {
+  int B, L, H, Hq, G, T, s, n, nq, S_new;
+  int base, bits, keys_only, residual;
+};
+
+HG_HD uint64_t align_up(uint64_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
+
+HG_HD int popc64(uint64_t x) {
+#ifdef __CUDA_ARCH__
+  return __popcll(x);
+#else
+  return __builtin_popcountll(x);
+#endif
+}
+
+// Image tokens eligible for low precision: [s, s + nq).  Whole span for the
+// per-token bases; whole 32-token key groups before the BF16 residual window
+// for KIVI-style.
+HG_HD int quantized_count(int T, int s, int n, int base, int residual) {
+  if (base != kKivi) return n;
+  int end = s + n;
+  if (T - residual < end) end = T - residual;
+  int span = end - s;
+  if (span <= 0) return 0;
+  return (span / kKiviGroup) * kKiviGroup;
+}
+
+// Bytes per token of one head's packed codes (128 codes).
+HG_HD uint64_t code_bytes_per_token(const Dims& d) { return (uint64_t)kD * d.bits / 8; }
+// Key metadata bytes for nq tokens of one batch row of one head.
+HG_HD uint64_t kmeta_bytes(const Dims& d) {
+  return d.base == kKivi ? (uint64_t)(d.nq / kKiviGroup) * kD * 8 : (uint64_t)d.nq * 8;
+}
+// Value metadata groups per token.
+HG_HD int vgroups(const Dims& d) { return d.base == kKivi ? kD / kKiviGroup : 1; }
+
+struct LayerGeom {
+  uint64_t mask;
+  int n_prot, n_U, n_PK, n_PKV, n_VQ;
+  uint64_t kb, vb, kq, kqm, vq, vqm, kimg, size;  // region offsets relative to the layer base
+  uint64_t bf16_bytes;                             // size of the kb (and vb) region
+};
+
+HG_HD int cap_unprot(const Dims& d) { return d.T - d.nq + d.S_new; }
+
+HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
+  LayerGeom g;
+  g.mask = mask;
+  g.n_prot = popc64(mask);
+  g.n_U = d.H - g.n_prot;
+  g.n_PK = d.keys_only ? g.n_prot : 0;
+  g.n_PKV = d.keys_only ? 0 : g.n_prot;
+  g.n_VQ = g.n_U + g.n_PK;
+  const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
+  const uint64_t tok_bf16 = (uint64_t)d.H * cap_unprot(d) + (uint64_t)g.n_PKV * nq;
+  g.bf16_bytes = align_up(B * tok_bf16 * kD * 2);
+  uint64_t off = 0;
+  g.kb = off; off += g.bf16_bytes;
+  g.vb = off; off += g.bf16_bytes;
+  g.kq = off; off += align_up((uint64_t)g.n_U * B * nq * code_bytes_per_token(d));
+  g.kqm = off; off += align_up((uint64_t)g.n_U * B * kmeta_bytes(d));
+  g.vq = off; off += align_up((uint64_t)g.n_VQ * B * nq * code_bytes_per_token(d));
+  g.vqm = off; off += align_up((uint64_t)g.n_VQ * B * nq * vgroups(d) * 8);
+  g.kimg = off; off += align_up((uint64_t)g.n_PK * B * nq * kD * 2);
+  g.size = off;
+  return g;
+}
+
+HG_HD int head_class(const Dims& d, uint64_t mask, int h) {
+  if (!((mask >> h) & 1ull)) return kQuantized;
+  return d.keys_only ? kKeysOnly : kProtected;
+}
+
+// One (layer, head): offsets of element [b=0][t=0] relative to the layer base,
+// and byte strides between batch rows.
+struct HeadGeom {
+  int cls;
+  int bf16_prefill;  // BF16 tokens that come from the prefill
+  int cap;           // BF16 capacity (prefill + max_new_tokens)
+  uint64_t kb, vb, kq, kqm, vq, vqm, kimg;
+  uint64_t kb_bs, kq_bs, kqm_bs, vq_bs, vqm_bs, kimg_bs;
+};
+
+HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
+  HeadGeom r;
+  const uint64_t below = (h == 0) ? 0ull : (g.mask & ((h >= 64) ? ~0ull : ((1ull << h) - 1ull)));
+  const int prot_below = popc64(below);
+  const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
+  r.cls = head_class(d, g.mask, h);
+  r.bf16_prefill = (r.cls == kProtected) ? d.T : d.T - d.nq;
+  r.cap = r.bf16_prefill + d.S_new;
+  const uint64_t pkv_below = d.keys_only ? 0ull : (uint64_t)prot_below;
+  const uint64_t tok_before = (uint64_t)h * cap_unprot(d) + pkv_below * nq;
+  r.kb_bs = (uint64_t)r.cap * kD * 2;
+  r.kb = g.kb + B * tok_before * kD * 2;
+  r.vb = g.vb + B * tok_before * kD * 2;
+  r.kq_bs = nq * code_bytes_per_token(d);
+  r.kqm_bs = kmeta_bytes(d);
+  r.vq_bs = nq * code_bytes_per_token(d);
+  r.vqm_bs = nq * vgroups(d) * 8;
+  r.kimg_bs = nq * kD * 2;
+  r.kq = r.kqm = r.vq = r.vqm = r.kimg = kNone;
+  if (r.cls == kQuantized) {
+    const uint64_t u = (uint64_t)(h - prot_below);
+    r.kq = g.kq + u * B * r.kq_bs;
+    r.kqm = g.kqm + u * B * r.kqm_bs;
+  }
+  if (r.cls != kProtected) {
+    const uint64_t vr = d.keys_only ? (uint64_t)h : (uint64_t)(h - prot_below);
+    r.vq = g.vq + vr * B * r.vq_bs;
+    r.vqm = g.vqm + vr * B * r.vqm_bs;
+  }
+  if (r.cls == kKeysOnly) {
+    r.kimg = g.kimg + (uint64_t)prot_below * B * r.kimg_bs;
+  }
+  return r;
+}
+
+// Position of prefill token t in a head's BF16 region, or -1 when the token is
+// stored in the quantized (or keys-only image) regions.
+HG_HD int bf16_pos(const Dims& d, int cls, int t) {
+  if (cls == kProtected) return t;
+  if (t < d.s) return t;
+  if (t < d.s + d.nq) return -1;
+  return t - d.nq;
+}
+
+// ---------------------------------------------------------------------------
+// Decode work decomposition.  Each (layer, batch row, KV head) is split into
+// chunks of at most cb BF16 tokens and cq coded tokens; a work item is one
+// chunk.  Items of one layer are numbered batch-row major, then head, then
+// BF16 chunks before coded chunks.
+// ---------------------------------------------------------------------------
+HG_HD int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+HG_HD int head_items(const Dims& d, int cls, int appended, int cb, int cq, int* n_bf16_items) {
+  const int lb = ((cls == kProtected) ? d.T : d.T - d.nq) + appended;
+  const int nb = cdiv(lb, cb);
+  const int nqi = (cls == kProtected) ? 0 : cdiv(d.nq, cq);
+  if (n_bf16_items) *n_bf16_items = nb;
+  return nb + nqi;
+}
+
+HG_HD int layer_items_per_row(const Dims& d, uint64_t mask, int appended, int cb, int cq) {
+  int tot = 0;
+  for (int h = 0; h < d.H; ++h) tot += head_items(d, head_class(d, mask, h), appended, cb, cq, nullptr);
+  return tot;
+}
+
+// Largest number of items any head can have (appended = max_new_tokens).
+HG_HD int max_head_items(const Dims& d, int cb, int cq) {
+  int a = head_items(d, kQuantized, d.S_new, cb, cq, nullptr);
+  int b = head_items(d, d.keys_only ? kKeysOnly : kProtected, d.S_new, cb, cq, nullptr);
+  return a > b ? a : b;
+}
+
+// Decode workspace: a counter per (layer, row, head), then partial results
+// [layer][row][head][split][G][kD + 2] floats (m, l, o[kD]).
+HG_HD uint64_t ws_counter_bytes(const Dims& d, int n_layers) {
+  return align_up((uint64_t)n_layers * d.B * d.H * 4);
+}
+HG_HD uint64_t ws_partial_floats_per_split(const Dims& d) { return (uint64_t)d.G * (kD + 2); }
+HG_HD uint64_t ws_bytes(const Dims& d, int n_layers, int cb, int cq) {
+  return ws_counter_bytes(d, n_layers) +
+         align_up((uint64_t)n_layers * d.B * d.H * max_head_items(d, cb, cq) *
+                  ws_partial_floats_per_split(d) * 4);
+}
+
+}  // namespace hg

@@ -1,0 +1,314 @@
+// Quantize-pack, dequantize and append kernels of the HeadGuard KV cache.
+//
+// Quantize (Sec. 3 "Applying protection" over the Sec. 1 / Sec. 4 bases):
+// one CTA per (32-token tile, batch row, KV head, layer).  The head's class
+// and the image span are resolved once per CTA, so protected heads and text
+// tokens take a uniform BF16 copy path.  A warp owns one token at a time,
+// each lane four consecutive channels; per-token groups reduce their min /
+// max with warp butterflies, KIVI-style value groups (32 channels) with
+// 8-lane butterflies, and KIVI-style key groups (32 tokens of one channel) are
+// quantized by one thread per channel from a shared-memory copy of the tile.
+#include <cuda_runtime.h>
+
+#include "hg_common.cuh"
+#include "hg_internal.h"
+
+namespace hg {
+
+namespace {
+
+constexpr int kThreads = 128;
+constexpr int kTile = 32;
+constexpr unsigned kFull = 0xffffffffu;
+
+// Pack one token's 128 codes (lane l holds channels 4l..4l+3) in channel order,
+// LSB-first, and store its 4*bits words.
+__device__ __forceinline__ void store_token_codes(uint32_t* row, const uint32_t (&c)[4], int bits,
+                                                  int lane) {
+  if (bits == 2) {
+    uint32_t x = (c[0] | (c[1] << 2) | (c[2] << 4) | (c[3] << 6)) << (8 * (lane & 3));
+    x |= __shfl_xor_sync(kFull, x, 1);
+    x |= __shfl_xor_sync(kFull, x, 2);
+    if ((lane & 3) == 0) row[lane >> 2] = x;
+  } else {
+    uint32_t x = (c[0] | (c[1] << 4) | (c[2] << 8) | (c[3] << 12)) << (16 * (lane & 1));
+    x |= __shfl_xor_sync(kFull, x, 1);
+    if ((lane & 1) == 0) row[lane >> 1] = x;
+  }
+}
+
+// Codes of channels 4l..4l+3 of one token from its packed row.
+__device__ __forceinline__ void load_token_codes(const uint32_t* row, int bits, int lane,
+                                                 uint32_t (&c)[4]) {
+  if (bits == 2) {
+    const uint32_t byte = (__ldg(row + (lane >> 2)) >> (8 * (lane & 3))) & 0xffu;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) c[i] = (byte >> (2 * i)) & 3u;
+  } else {
+    const uint32_t half = (__ldg(row + (lane >> 1)) >> (16 * (lane & 1))) & 0xffffu;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) c[i] = (half >> (4 * i)) & 15u;
+  }
+}
+
+__device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
+  bf16x2_to_f32(w.x, x[0], x[1]);
+  bf16x2_to_f32(w.y, x[2], x[3]);
+}
+
+// One 32-value group held by a single thread (KIVI-style key channel group).
+__device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGroup], int bits,
+                                                      uint32_t (&code)[kKiviGroup], float& scale,
+                                                      float& zero) {
+  float mn = x[0], mx = x[0];
+#pragma unroll
+  for (int e = 1; e < kKiviGroup; ++e) {
+    mn = fminf(mn, x[e]);
+    mx = fmaxf(mx, x[e]);
+  }
+  mn = __fadd_rn(mn, 0.0f);
+  mx = __fadd_rn(mx, 0.0f);
+  const float levels = (float)((1 << bits) - 1);
+  scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  zero = mn;
+#pragma unroll
+  for (int e = 0; e < kKiviGroup; ++e) {
+    if (scale == 0.0f) {
+      code[e] = 0u;
+    } else {
+      float r = rintf(__fdiv_rn(__fsub_rn(x[e], mn), scale));
+      r = fminf(fmaxf(r, 0.0f), levels);
+      code[e] = (uint32_t)r;
+    }
+  }
+}
+
+__global__ void __launch_bounds__(kThreads)
+quantize_kernel(const __grid_constant__ QuantizeParams p) {
+  const Dims& d = p.d;
+  const int tile = blockIdx.x, bh = blockIdx.y, li = blockIdx.z;
+  const int b = bh / d.H, h = bh % d.H;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+
+  int t0 = p.tile_origin - kTile + kTile * tile;
+  int t1 = t0 + kTile;
+  if (t0 < 0) t0 = 0;
+  if (t1 > d.T) t1 = d.T;
+  if (t0 >= t1) return;
+
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+  const HeadGeom hd = head_geom(d, g, h);
+  char* Lb = p.arena + p.lt.base[li];
+  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T;
+  const uint16_t* K = p.k[li] + row0 * kD;
+  const uint16_t* V = p.v[li] + row0 * kD;
+  const int qs = d.s, qe = d.s + d.nq;
+  const int W = kD * d.bits / 32;  // code words per token
+  // A whole KIVI-style key group of a quantized head: tokens [t0, t0 + 32).
+  const bool kivi_k_tile = (d.base == kKivi) && (hd.cls == kQuantized) && t0 >= qs && t1 <= qe;
+
+  __shared__ __align__(16) uint16_t ktile[kTile][kD];
+
+  // Issue every load of this warp's tokens first (8 tokens x (K, V) x 8 bytes / lane).
+  uint2 kr[kTile / 4], vr[kTile / 4];
+#pragma unroll
+  for (int i = 0; i < kTile / 4; ++i) {
+    const int t = t0 + warp + 4 * i;
+    if (t < t1) {
+      kr[i] = ldg8(K + (size_t)t * kD + lane * 4);
+      vr[i] = ldg8(V + (size_t)t * kD + lane * 4);
+    }
+  }
+
+#pragma unroll
+  for (int i = 0; i < kTile / 4; ++i) {
+    const int t = t0 + warp + 4 * i;
+    if (t >= t1) break;
+    const bool coded = (t >= qs) && (t < qe);
+    const int ti = t - qs;
+
+    // ---- key ----
+    if (coded && hd.cls == kQuantized) {
+      if (d.base == kKivi) {
+        *reinterpret_cast<uint2*>(&ktile[t - t0][lane * 4]) = kr[i];
+      } else {
+        float x[4];
+        bf16x4_to_f32(kr[i], x);
+        if (d.base == kAkvq) fwht128_warp(x, lane);  // rotate, then per-token RTN
+        uint32_t c[4];
+        float sc, z;
+        quantize_group4<32>(x, d.bits, c, sc, z);
+        uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W;
+        store_token_codes(crow, c, d.bits, lane);
+        if (lane == 0)
+          reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs)[ti] = make_float2(sc, z);
+      }
+    } else if (coded && hd.cls == kKeysOnly) {
+      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) =
+          kr[i];
+    } else {
+      const int pos = bf16_pos(d, hd.cls, t);
+      *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
+          kr[i];
+    }
+
+    // ---- value (never rotated) ----
+    if (coded && hd.cls != kProtected) {
+      float x[4];
+      bf16x4_to_f32(vr[i], x);
+      uint32_t c[4];
+      float sc, z;
+      float2* meta = reinterpret_cast<float2*>(Lb + hd.vqm + b * hd.vqm_bs) + (size_t)ti * vgroups(d);
+      if (d.base == kKivi) {
+        quantize_group4<8>(x, d.bits, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
+        if ((lane & 7) == 0) meta[lane >> 3] = make_float2(sc, z);
+      } else {
+        quantize_group4<32>(x, d.bits, c, sc, z);
+        if (lane == 0) meta[0] = make_float2(sc, z);
+      }
+      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W;
+      store_token_codes(crow, c, d.bits, lane);
+    } else {
+      const int pos = bf16_pos(d, hd.cls, t);
+      *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
+          vr[i];
+    }
+  }
+
+  if (!kivi_k_tile) return;  // uniform over the CTA
+  __syncthreads();
+  // KIVI-style keys: thread c quantizes channel c over the 32-token group.
+  const int c = threadIdx.x;
+  float x[kKiviGroup];
+#pragma unroll
+  for (int e = 0; e < kKiviGroup; ++e) x[e] = bf16_to_f32(ktile[e][c]);
+  uint32_t code[kKiviGroup];
+  float sc, z;
+  quantize_group_serial(x, d.bits, code, sc, z);
+  const int grp = (t0 - qs) / kKiviGroup;
+  uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * d.bits;
+  const int per = 32 / d.bits;
+  for (int w = 0; w < d.bits; ++w) {
+    uint32_t word = 0;
+    for (int e = 0; e < per; ++e) word |= code[w * per + e] << (d.bits * e);
+    dst[w] = word;
+  }
+  reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs)[(size_t)grp * kD + c] = make_float2(sc, z);
+}
+
+// Reconstruct one layer as floats in original token order (then appended).
+__global__ void __launch_bounds__(kThreads)
+dequantize_kernel(const __grid_constant__ DequantParams p) {
+  const Dims& d = p.d;
+  const int bh = blockIdx.y;
+  const int b = bh / d.H, h = bh % d.H;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int Tt = d.T + p.appended;
+  const LayerGeom g = layer_geom(d, p.mask);
+  const HeadGeom hd = head_geom(d, g, h);
+  const char* Lb = p.arena + p.layer_base;
+  const int qs = d.s, qe = d.s + d.nq;
+  const int W = kD * d.bits / 32;
+
+  for (int t = blockIdx.x * kTile + warp; t < min(Tt, (int)(blockIdx.x + 1) * kTile); t += 4) {
+    const bool coded = (t >= qs) && (t < qe);
+    const int ti = t - qs;
+    const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : bf16_pos(d, hd.cls, t);
+    float xk[4], xv[4];
+    if (coded && hd.cls == kQuantized) {
+      uint32_t c[4];
+      if (d.base == kKivi) {
+        const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
+        const int per = 32 / d.bits;
+        const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs);
+        const float2* meta = reinterpret_cast<const float2*>(Lb + hd.kqm + b * hd.kqm_bs);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const size_t row = (size_t)grp * kD + lane * 4 + i;
+          const uint32_t w = __ldg(codes + row * d.bits + e / per);
+          const uint32_t code = (w >> (d.bits * (e % per))) & ((1u << d.bits) - 1u);
+          const float2 m = __ldg(meta + row);
+          xk[i] = dequant1(code, m.x, m.y);
+        }
+      } else {
+        load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
+                         d.bits, lane, c);
+        const float2 m = __ldg(reinterpret_cast<const float2*>(Lb + hd.kqm + b * hd.kqm_bs) + ti);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) xk[i] = dequant1(c[i], m.x, m.y);
+        if (d.base == kAkvq) fwht128_warp(xk, lane);  // inverse rotation (H is self-inverse)
+      }
+    } else if (coded && hd.cls == kKeysOnly) {
+      bf16x4_to_f32(ldg8(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2), xk);
+    } else {
+      bf16x4_to_f32(ldg8(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2), xk);
+    }
+    if (coded && hd.cls != kProtected) {
+      uint32_t c[4];
+      load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+                       d.bits, lane, c);
+      const float2* meta = reinterpret_cast<const float2*>(Lb + hd.vqm + b * hd.vqm_bs) +
+                           (size_t)ti * vgroups(d);
+      const float2 m = __ldg(meta + (d.base == kKivi ? (lane >> 3) : 0));
+#pragma unroll
+      for (int i = 0; i < 4; ++i) xv[i] = dequant1(c[i], m.x, m.y);
+    } else {
+      bf16x4_to_f32(ldg8(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2), xv);
+    }
+    const size_t o = (((size_t)b * d.H + h) * Tt + t) * kD + lane * 4;
+    if (p.out_fp32) {
+      reinterpret_cast<float4*>(p.k_out)[o / 4] = make_float4(xk[0], xk[1], xk[2], xk[3]);
+      reinterpret_cast<float4*>(p.v_out)[o / 4] = make_float4(xv[0], xv[1], xv[2], xv[3]);
+    } else {
+      reinterpret_cast<uint2*>(p.k_out)[o / 4] =
+          make_uint2(f32_to_bf16_rn(xk[0]) | (f32_to_bf16_rn(xk[1]) << 16),
+                     f32_to_bf16_rn(xk[2]) | (f32_to_bf16_rn(xk[3]) << 16));
+      reinterpret_cast<uint2*>(p.v_out)[o / 4] =
+          make_uint2(f32_to_bf16_rn(xv[0]) | (f32_to_bf16_rn(xv[1]) << 16),
+                     f32_to_bf16_rn(xv[2]) | (f32_to_bf16_rn(xv[3]) << 16));
+    }
+  }
+}
+
+// One decode token per (layer, row, head) into the head's BF16 region.
+__global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ AppendParams p) {
+  const Dims& d = p.d;
+  const int li = blockIdx.x, bh = blockIdx.y;
+  const int b = bh / d.H, h = bh % d.H;
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+  const HeadGeom hd = head_geom(d, g, h);
+  char* Lb = p.arena + p.lt.base[li];
+  const int pos = hd.bf16_prefill + p.appended[li];
+  const size_t src = (((size_t)li * d.B + b) * d.H + h) * kD;
+  const int lane = threadIdx.x & 31;
+  if (threadIdx.x < 32) {
+    *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
+        ldg8(p.k_new + src + lane * 4);
+  } else {
+    *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
+        ldg8(p.v_new + src + lane * 4);
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
+  dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
+  quantize_kernel<<<grid, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s) {
+  const int Tt = p.d.T + p.appended;
+  dim3 grid((Tt + kTile - 1) / kTile, p.d.B * p.d.H, 1);
+  dequantize_kernel<<<grid, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
+  dim3 grid(p.n_layers, p.d.B * p.d.H, 1);
+  append_kernel<<<grid, 64, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+}  // namespace hg

@@ -1,0 +1,100 @@
+"""Parity helpers: compare the library's arena, reconstruction and attention with
+the CPU oracle on the same seeded inputs (test infrastructure)."""
+import numpy as np
+import torch
+
+import oracle
+import paper_2609_35800_gb300 as hg
+
+ATOL, RTOL = 2e-3, 1e-2   # attention tolerance (allclose form) on BF16 outputs
+
+
+def bits16(t):
+    """BF16 tensor -> host uint16 numpy bit patterns."""
+    return t.detach().contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def f32_from_bits(b):
+    return (b.astype(np.uint32) << 16).view(np.float32)
+
+
+def bf16_rne(x):
+    """fp32 -> BF16 bits, round to nearest even (numpy, independent of the GPU)."""
+    u = np.ascontiguousarray(x, np.float32).view(np.uint32).astype(np.uint64)
+    return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
+def oracle_layer(runner, layer, k_bits, v_bits):
+    w = runner.w
+    return oracle.quantize_layer(k_bits, v_bits, w.img_start, w.image, w.base, w.bits,
+                                 runner.mask[layer], int(w.keys_only), w.kivi_group_tokens,
+                                 w.kivi_group_channels, w.kivi_residual)
+
+
+def _slice(arena, off, nbytes, dtype):
+    return arena[off: off + nbytes].view(dtype)
+
+
+def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, rows=None):
+    """Bit-exact comparison of every region of one layer (or the given heads / rows)."""
+    w = runner.w
+    if arena is None:
+        arena = runner.arena.cpu().numpy()
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    s, nq = w.img_start, o["nq"]
+    W = 128 * w.bits // 32
+    heads = range(H) if heads is None else heads
+    rows = range(B) if rows is None else rows
+    for h in heads:
+        r = hg.hg_cache_head_regions(runner.cache, layer, h)
+        assert r.nq == nq
+        cls = r.head_class
+        if cls == hg.HG_HEAD_PROTECTED:
+            toks = np.arange(T)
+        else:
+            toks = np.concatenate([np.arange(0, s), np.arange(s + nq, T)])
+        assert r.bf16_prefill == toks.size
+        for b in rows:
+            kb = _slice(arena, r.kb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
+            vb = _slice(arena, r.vb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
+            assert np.array_equal(kb, k_bits[b, h, toks]), (layer, h, b, "kb")
+            assert np.array_equal(vb, v_bits[b, h, toks]), (layer, h, b, "vb")
+            if cls == hg.HG_HEAD_QUANTIZED and nq:
+                kw = _slice(arena, r.kq + b * r.kq_bstride, nq * W * 4, np.uint32)
+                km = _slice(arena, r.kqm + b * r.kqm_bstride, r.kqm_bstride, np.uint32)
+                assert np.array_equal(kw, o["k_words"][b, h]), (layer, h, b, "kq")
+                assert np.array_equal(km, o["k_meta"][b, h].view(np.uint32)), (layer, h, b, "kqm")
+            if cls != hg.HG_HEAD_PROTECTED and nq:
+                vw = _slice(arena, r.vq + b * r.vq_bstride, nq * W * 4, np.uint32)
+                vm = _slice(arena, r.vqm + b * r.vqm_bstride, r.vqm_bstride, np.uint32)
+                assert np.array_equal(vw, o["v_words"][b, h]), (layer, h, b, "vq")
+                assert np.array_equal(vm, o["v_meta"][b, h].view(np.uint32)), (layer, h, b, "vqm")
+            if cls == hg.HG_HEAD_KEYS_ONLY and nq:
+                ki = _slice(arena, r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)
+                assert np.array_equal(ki, k_bits[b, h, s:s + nq]), (layer, h, b, "kimg")
+
+
+def attention_reference(runner, o, q_bits, appended_k, appended_v, sigma):
+    """fp64 oracle attention of one layer over the reconstruction + appended tokens.
+
+    appended_k/v: list of uint16 [B][H][128] (one per appended step)."""
+    K = o["k_att"]
+    V = o["v_deq"].astype(np.float64)
+    if appended_k:
+        ak = np.stack([f32_from_bits(a) for a in appended_k], axis=2).astype(np.float64)
+        av = np.stack([f32_from_bits(a) for a in appended_v], axis=2).astype(np.float64)
+        K = np.concatenate([K, ak], axis=2)
+        V = np.concatenate([V, av], axis=2)
+    return oracle.attention_layer(q_bits, K, V, sigma)
+
+
+def assert_close(got_bf16_bits, ref, where=""):
+    g = f32_from_bits(got_bf16_bits).astype(np.float64)
+    err = np.abs(g - ref)
+    bad = err > ATOL + RTOL * np.abs(ref)
+    if bad.any():
+        i = np.argwhere(bad)[0]
+        raise AssertionError("%s: %d / %d outside tolerance; first at %s got %r ref %r "
+                             "(max abs err %.3g)" % (where, bad.sum(), bad.size, tuple(i),
+                                                     g[tuple(i)], ref[tuple(i)], err.max()))
+    return float(err.max())

@@ -1,0 +1,190 @@
+"""Host-only tests of the C ABI: the library loads, exports every declared entry
+point, validates arguments before touching the GPU, and lays the arena out as
+the storage model says.  No CUDA call is made here."""
+import ctypes
+import os
+import re
+
+import numpy as np
+import pytest
+
+import paper_2609_35800_gb300 as hg
+from paper_2609_35800_gb300 import build, workloads as wl
+from paper_2609_35800_gb300.runner import config_of, shape_of
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return hg.library()
+
+
+def _declared():
+    txt = open(os.path.join(ROOT, "include", "headguard.h")).read()
+    txt = re.sub(r"/\*.*?\*/", "", txt, flags=re.S)
+    return sorted(set(re.findall(r"\b(hg_[a-z0-9_]+)\s*\(", txt)))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = _declared()
+    assert len(names) >= 14
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def _shape(**kw):
+    d = dict(batch=2, num_layers=3, num_kv_heads=4, num_q_heads=28, head_dim=128, seq_len=300,
+             img_start=20, img_len=256, max_new_tokens=8)
+    d.update(kw)
+    return hg.Shape(**d)
+
+
+def _cfg(**kw):
+    d = dict(base=0, bits=2, keys_only=0, kivi_group_tokens=32, kivi_group_channels=32,
+             kivi_residual=32)
+    d.update(kw)
+    return hg.QuantConfig(**d)
+
+
+def _status(f, *a):
+    return f(*a)
+
+
+@pytest.mark.parametrize("shape_kw,cfg_kw,status", [
+    (dict(head_dim=64), {}, 3),
+    (dict(num_q_heads=30), {}, 1),
+    (dict(img_start=100, img_len=256), {}, 1),
+    (dict(num_kv_heads=65, num_q_heads=65), {}, 3),
+    (dict(num_kv_heads=1, num_q_heads=17), {}, 3),
+    (dict(seq_len=0, img_len=0, img_start=0), {}, 1),
+    (dict(batch=0), {}, 1),
+    ({}, dict(bits=3), 3),
+    ({}, dict(base=7), 1),
+    ({}, dict(base=1, kivi_group_tokens=16), 3),
+    ({}, dict(base=1, kivi_residual=-1), 1),
+    ({}, dict(keys_only=2), 1),
+])
+def test_layout_validation(lib, shape_kw, cfg_kw, status):
+    mask = np.zeros((3, max(4, shape_kw.get("num_kv_heads", 4))), np.uint8)
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_cache_layout(_shape(**shape_kw), _cfg(**cfg_kw), mask)
+    assert e.value.status == status
+
+
+def _fake_cache(w, arena_addr=1 << 40):
+    mask = wl.protection_mask(w).numpy()
+    sh, cf = shape_of(w), config_of(w)
+    n = hg.hg_cache_layout(sh, cf, mask)
+    return hg.hg_cache_create(sh, cf, mask, arena_addr, n), n, mask
+
+
+def test_create_checks_arena(lib):
+    w = wl.WORKLOADS["tiny"]
+    mask = wl.protection_mask(w).numpy()
+    sh, cf = shape_of(w), config_of(w)
+    n = hg.hg_cache_layout(sh, cf, mask)
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_cache_create(sh, cf, mask, 1 << 40, n - 1)
+    assert e.value.status == 7
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_cache_create(sh, cf, mask, (1 << 40) + 16, n)
+    assert e.value.status == 2
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+def test_regions_tile_the_arena_without_overlap(lib, name):
+    w = wl.WORKLOADS[name]
+    cache, n, mask = _fake_cache(w)
+    base = 1 << 40
+    spans = []
+    W = 128 * w.bits // 8
+    for l in range(w.layers):
+        for h in range(w.kv_heads):
+            r = hg.hg_cache_head_regions(cache, l, h)
+            B = w.batch
+            assert r.head_class == (0 if not mask[l, h] else (1 if w.keys_only else 2))
+            spans.append((r.kb, B * r.kb_bstride))
+            spans.append((r.vb, B * r.kb_bstride))
+            assert r.kb_bstride == r.bf16_capacity * 256
+            if r.kq != hg.NONE_OFFSET:
+                assert r.kq_bstride == r.nq * W
+                spans.append((r.kq, B * r.kq_bstride))
+                spans.append((r.kqm, B * r.kqm_bstride))
+            if r.vq != hg.NONE_OFFSET:
+                spans.append((r.vq, B * r.vq_bstride))
+                spans.append((r.vqm, B * r.vqm_bstride))
+            if r.kimg != hg.NONE_OFFSET:
+                spans.append((r.kimg, B * r.kimg_bstride))
+            for off in (r.kb, r.vb, r.kq, r.vq, r.kimg):
+                if off != hg.NONE_OFFSET:
+                    assert off % 16 == 0
+    spans = sorted(s for s in spans if s[1] > 0)
+    for (a, la), (b, _) in zip(spans, spans[1:]):
+        assert a + la <= b, (a, la, b)
+    assert spans[-1][0] + spans[-1][1] <= n
+
+
+def test_image_storage_matches_paper_storage_model(lib, oracle):
+    # exactly 1/8 of the heads protected, 2-bit min-max, no text outside the image:
+    # the arena's image bits/elem equals the Sec. 5.4 model with 64-bit metadata.
+    for keys_only in (0, 1):
+        w = wl.custom("st", 2, 1, 8, 8, 0, 64, 0, wl.BASE_MINMAX, 2, keys_only,
+                      protected=[(0, 3), (1, 6)])
+        cache, _, _ = _fake_cache(w)
+        got = hg.hg_cache_image_bits_per_elem(cache)
+        want = oracle.image_bits_per_elem(2, 64, 0.125, keys_only)
+        assert got == pytest.approx(want, rel=1e-12)
+    w = wl.custom("st", 1, 1, 8, 8, 0, 64, 0, wl.BASE_MINMAX, 2, 0, protected=[])
+    cache, _, _ = _fake_cache(w)
+    assert hg.hg_cache_image_bits_per_elem(cache) == pytest.approx(2.5)
+    assert oracle.image_bits_per_elem(2, 64, 0.0, 0) == pytest.approx(2.5)
+
+
+def test_calls_validate_before_any_launch(lib):
+    w = wl.custom("v", 2, 1, 8, 2, 8, 64, 8, wl.BASE_MINMAX, 2, 0, decode_steps=0,
+                  protected=[(0, 0)])
+    cache, n, _ = _fake_cache(w)
+    base = 1 << 40
+    # null / misaligned inputs
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_quantize_kv(cache, 0, [0, 0], [base, base], stream=0)
+    assert e.value.status == 1
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_quantize_kv(cache, 0, [base + 8], [base], stream=0)
+    assert e.value.status == 2
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_quantize_kv(cache, 1, [base, base], [base, base], stream=0)  # layers 1..2 of 2
+    assert e.value.status == 1
+    # capacity 0: appending fails before launching
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_append_kv(cache, 0, 1, base, base, stream=0)
+    assert e.value.status == 5
+    # workspace too small
+    need = hg.hg_decode_workspace_size(cache, 2)
+    assert need > 0
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_decode_attention(cache, 0, 2, base, base, 0.0, base, need - 1, stream=0)
+    assert e.value.status == 4
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_decode_attention(cache, 0, 2, base, base, float("nan"), base, need, stream=0)
+    assert e.value.status == 1
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_dequantize_kv(cache, 2, base, base, 1, stream=0)
+    assert e.value.status == 1
+    assert hg.hg_cache_appended(cache, 0) == 0
+    assert hg.hg_cache_appended(cache, 5) == -1
+
+
+def test_workspace_size_grows_with_layers(lib):
+    w = wl.WORKLOADS["qwen25vl7b"]
+    cache, _, _ = _fake_cache(w)
+    one = hg.hg_decode_workspace_size(cache, 1)
+    allw = hg.hg_decode_workspace_size(cache, w.layers)
+    assert 0 < one < allw
+
+
+def test_status_strings(lib):
+    for s in range(8):
+        assert isinstance(hg.hg_status_string(s), str) and hg.hg_status_string(s)

@@ -1,0 +1,165 @@
+"""GPU parity of the CUDA path against the CPU oracle, through the C ABI.
+
+Packed codes, fp32 metadata and BF16 copies must be bit-identical; the fp32
+reconstruction (hg_dequantize_kv) must be bit-identical; decode attention
+must match the fp64 oracle within |g - r| <= 2e-3 + 1e-2 |r| element-wise.
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2609_35800_gb300 as hg
+from paper_2609_35800_gb300 import workloads as wl
+from paper_2609_35800_gb300.runner import CacheRunner
+
+from parity import (assert_close, attention_reference, bf16_rne, bits16, check_arena_layer,
+                    oracle_layer)
+
+pytestmark = pytest.mark.gpu
+
+SIGMA = float(np.float32(1.0 / np.sqrt(128.0)))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_35800_gb300 import build
+    build.build()
+    hg.library()
+
+
+M, K, A = wl.BASE_MINMAX, wl.BASE_KIVI, wl.BASE_AKVQ
+
+# name, layers, batch, q_heads, kv_heads, prefix, image, suffix, base, bits, keys_only, steps, protected, residual
+CASES = [
+    ("minmax2_gqa7", 2, 1, 28, 4, 32, 256, 32, M, 2, 0, 3, [(0, 1), (1, 3)], 32),
+    ("minmax4_g2_b2", 1, 2, 4, 2, 10, 70, 5, M, 4, 0, 3, [(0, 0)], 32),
+    ("minmax2_konly", 2, 2, 8, 4, 7, 200, 9, M, 2, 1, 2, [(0, 2), (1, 0), (1, 1)], 32),
+    ("kivi2_konly_mha", 1, 2, 4, 4, 3, 100, 40, K, 2, 1, 3, [(0, 1)], 32),
+    ("kivi4_residual_in_image", 1, 1, 8, 2, 5, 80, 10, K, 4, 0, 2, [(0, 1)], 32),
+    ("kivi2_unaligned_start", 2, 1, 4, 4, 13, 130, 45, K, 2, 0, 2, [(1, 2)], 32),
+    ("akvq4_g4_b3", 1, 3, 16, 4, 64, 333, 17, A, 4, 0, 3, [(0, 3)], 32),
+    ("akvq2_konly", 1, 2, 8, 4, 20, 150, 30, A, 2, 1, 2, [(0, 0), (0, 2)], 32),
+    ("no_image", 1, 1, 8, 2, 40, 0, 30, M, 2, 0, 2, [(0, 0)], 32),
+    ("image_at_start_and_end", 1, 2, 8, 4, 0, 300, 0, M, 2, 0, 2, [(0, 2)], 32),
+    ("all_protected", 1, 1, 8, 2, 16, 100, 16, A, 4, 0, 2, [(0, 0), (0, 1)], 32),
+    ("none_protected", 1, 1, 8, 2, 16, 100, 16, K, 2, 0, 2, [], 0),
+    ("g16", 1, 1, 32, 2, 16, 200, 16, M, 4, 0, 2, [(0, 1)], 32),
+    ("long_multisplit", 1, 1, 28, 4, 50, 3000, 50, M, 2, 0, 2, [(0, 0)], 32),
+]
+
+
+def _workload(case):
+    (name, L, B, Hq, H, pre, img, suf, base, bits, ko, steps, prot, R) = case
+    return wl.custom(name, L, B, Hq, H, pre, img, suf, base, bits, ko, decode_steps=steps,
+                     seed=7, protected=prot, residual=R)
+
+
+def _run_and_check(w, layer_batched=True):
+    runner = CacheRunner(w)
+    kept = runner.quantize_all(keep=True)
+    torch.cuda.synchronize()
+    arena = runner.arena.cpu().numpy()
+    outs = []
+    for l, (k, v) in enumerate(kept):
+        kb, vb = bits16(k), bits16(v)
+        o = oracle_layer(runner, l, kb, vb)
+        check_arena_layer(runner, l, kb, vb, o, arena=arena)
+        outs.append(o)
+    # decode steps (append + attention), compared after every step
+    app_k = [[] for _ in range(w.layers)]
+    app_v = [[] for _ in range(w.layers)]
+    for step in range(w.decode_steps):
+        k_new, v_new = wl.step_new_kv(w, step, "cuda")
+        q = wl.step_query(w, step, "cuda")
+        out = torch.empty_like(q)
+        hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
+        if layer_batched:
+            hg.hg_decode_attention(runner.cache, 0, w.layers, q, out, SIGMA, runner.ws,
+                                   runner.ws_bytes)
+        else:
+            for l in range(w.layers):
+                hg.hg_decode_attention(runner.cache, l, 1, q[l], out[l], SIGMA, runner.ws,
+                                       runner.ws_bytes)
+        torch.cuda.synchronize()
+        kn, vn, qb, ob = bits16(k_new), bits16(v_new), bits16(q), bits16(out)
+        for l in range(w.layers):
+            app_k[l].append(kn[l])
+            app_v[l].append(vn[l])
+            ref = attention_reference(runner, outs[l], qb[l], app_k[l], app_v[l], SIGMA)
+            assert_close(ob[l], ref, "%s layer %d step %d" % (w.name, l, step))
+    return runner, kept, outs
+
+
+@pytest.mark.parametrize("case", CASES, ids=[c[0] for c in CASES])
+def test_quantize_and_decode_parity(case):
+    _run_and_check(_workload(case))
+
+
+def test_tiny_workload_parity():
+    _run_and_check(wl.WORKLOADS["tiny"])
+
+
+@pytest.mark.parametrize("case", [CASES[0], CASES[3], CASES[6]], ids=["minmax", "kivi", "akvq"])
+def test_per_layer_launches(case):
+    _run_and_check(_workload(case), layer_batched=False)
+
+
+@pytest.mark.parametrize("case", [CASES[1], CASES[2], CASES[4], CASES[5], CASES[7]],
+                         ids=["minmax4", "minmax2_konly", "kivi4", "kivi2", "akvq2"])
+def test_dequantize_bit_exact(case):
+    w = _workload(case)
+    runner = CacheRunner(w)
+    kept = runner.quantize_all(keep=True)
+    # append one step so the appended tail is reconstructed too
+    k_new, v_new = wl.step_new_kv(w, 0, "cuda")
+    hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
+    Tt = w.seq_len + 1
+    for l, (k, v) in enumerate(kept):
+        o = oracle_layer(runner, l, bits16(k), bits16(v))
+        k32 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
+        v32 = torch.empty_like(k32)
+        hg.hg_dequantize_kv(runner.cache, l, k32, v32, True)
+        k16 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.bfloat16, device="cuda")
+        v16 = torch.empty_like(k16)
+        hg.hg_dequantize_kv(runner.cache, l, k16, v16, False)
+        torch.cuda.synchronize()
+        kd = np.concatenate([o["k_deq"], (bits16(k_new[l]).astype(np.uint32) << 16)
+                             .view(np.float32)[:, :, None]], axis=2)
+        vd = np.concatenate([o["v_deq"], (bits16(v_new[l]).astype(np.uint32) << 16)
+                             .view(np.float32)[:, :, None]], axis=2)
+        assert np.array_equal(k32.cpu().numpy().view(np.uint32), kd.view(np.uint32))
+        assert np.array_equal(v32.cpu().numpy().view(np.uint32), vd.view(np.uint32))
+        assert np.array_equal(bits16(k16), bf16_rne(kd))
+        assert np.array_equal(bits16(v16), bf16_rne(vd))
+
+
+def test_quantize_is_idempotent_and_resets_appended():
+    w = _workload(CASES[0])
+    runner = CacheRunner(w)
+    kept = runner.quantize_all(keep=True)
+    runner.decode_step(0)
+    assert hg.hg_cache_appended(runner.cache, 0) == 1
+    a1 = runner.arena.clone()
+    hg.hg_quantize_kv(runner.cache, 0, [k for k, _ in kept], [v for _, v in kept])
+    torch.cuda.synchronize()
+    assert hg.hg_cache_appended(runner.cache, 0) == 0
+    # every prefill region is rewritten identically
+    l = 0
+    r = hg.hg_cache_head_regions(runner.cache, l, 0)
+    span = slice(r.kq, r.kq + r.kq_bstride)
+    assert torch.equal(a1[span], runner.arena[span])
+
+
+def test_capacity_error_leaves_state():
+    w = _workload(CASES[1])
+    runner = CacheRunner(w)
+    runner.quantize_all()
+    for s in range(w.decode_steps):
+        runner.decode_step(s)
+    k_new, v_new = wl.step_new_kv(w, 0, "cuda")
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
+    assert e.value.status == 5
+    assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
