@@ -1,0 +1,528 @@
+#!/usr/bin/env python
+"""Benchmark of the HeadGuard mixed-precision KV-cache path on one GB300.
+
+One step = the whole path over one synthetic cache: quantize-pack every layer
+from its BF16 prefill (one launch per 64 layers), then `decode_steps` decode
+steps, each appending one token per (layer, row, KV head) and running decode
+attention over all layers (one launch each).  Inputs are resident in HBM when
+timing starts; L2 is flushed (a 512 MiB write) before every timed launch
+group, and every group is timed with CUDA events on the launching stream.
+
+value     = algorithmic bytes of a step / summed device time of the step (GB/s)
+roofline  = decode attention (the dominant kernel): its algorithmic bytes per
+            launch / its mean event-timed duration, against MEASURED_PEAKS.json
+e2e       = the same bytes / time of a step driven from pinned HOST buffers
+            through the C ABI (H2D of prefill, queries and new K/V; D2H of
+            the attention outputs inside the timed region)
+--impl reference times the CPU oracle on a bounded sample of the same step.
+"""
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = ("decode-attn + quantize achieved HBM GB/s (% of 8 TB/s) and decode tokens/s, 1 GB300")
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+L2_FLUSH_BYTES = 512 << 20
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="headguard", choices=["headguard", "reference"])
+    ap.add_argument("--workload", default="qwen25vl7b")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# Algorithmic bytes (inputs read + outputs written, no workspace traffic)
+# ---------------------------------------------------------------------------
+
+def geometry_bytes(runner):
+    """Algorithmic bytes of quantize (per step), decode (per decode step, list),
+    append (per decode step), from the library's region map."""
+    import paper_2609_35800_gb300 as hg
+    w = runner.w
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    code_tok = 128 * w.bits // 8
+    q_rows = w.layers * B * w.q_heads * 256
+    quant = 0
+    dec_static = 0          # cache bytes read per decode step excluding appended tokens
+    bf16_heads = 0          # (layer, head) pairs: appended tokens are read per head
+    for l in range(w.layers):
+        for h in range(H):
+            r = hg.hg_cache_head_regions(runner.cache, l, h)
+            nq = r.nq
+            per_b_write = r.bf16_prefill * 512
+            per_b_read_dec = r.bf16_prefill * 512
+            if r.head_class == hg.HG_HEAD_QUANTIZED:
+                per_b_write += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
+                per_b_read_dec += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
+            elif r.head_class == hg.HG_HEAD_KEYS_ONLY:
+                per_b_write += nq * 256 + nq * code_tok + r.vqm_bstride
+                per_b_read_dec += nq * 256 + nq * code_tok + r.vqm_bstride
+            quant += B * (T * 512 + per_b_write)
+            dec_static += B * per_b_read_dec
+            bf16_heads += 1
+    decode = []
+    for s in range(w.decode_steps):
+        appended = s + 1
+        decode.append(dec_static + bf16_heads * B * appended * 512 + 2 * q_rows)
+    append = 4 * w.layers * B * H * 256
+    return quant, decode, append
+
+
+# ---------------------------------------------------------------------------
+# clocks
+# ---------------------------------------------------------------------------
+
+CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+
+class ClockSampler:
+    def __init__(self, device_index):
+        self.proc = None
+        self.idx = device_index
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + CLOCK_FIELDS, "--format=csv,noheader,nounits",
+                 "-i", str(self.idx), "-lms", "200"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        self.lines = []
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                out, _ = self.proc.communicate()
+            self.lines = [l for l in out.splitlines() if l.strip()]
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in getattr(self, "lines", []):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower() == "active":
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# roofline inputs
+# ---------------------------------------------------------------------------
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            return json.load(f), "measured"
+    except (OSError, ValueError):
+        return {"hbm_gbs": FALLBACK_HBM_GBS}, "fallback"
+
+
+def kernel_source_hash():
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2609_35800_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode() + f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload):
+    """DRAM bytes per decode launch from the committed ncu summary, if it was
+    taken on the current kernel sources (else None)."""
+    path = os.path.join(ROOT, "profiles", "decode_attention_%s.md" % workload)
+    try:
+        txt = open(path).read()
+    except OSError:
+        return None
+    m_src = re.search(r"source_sha256_16:\s*([0-9a-f]+)", txt)
+    m_tr = re.search(r"dram_bytes_per_launch:\s*([0-9.eE+]+)", txt)
+    if not m_src or not m_tr or m_src.group(1) != kernel_source_hash():
+        return None
+    return float(m_tr.group(1))
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_sample(w, n_layers, n_steps):
+    """Time the oracle on the first n_layers layers: quantize, then n_steps decode
+    steps of attention over those layers.  Returns (bytes, seconds, threads)."""
+    import numpy as np
+    import torch
+
+    import oracle
+    from paper_2609_35800_gb300 import workloads as wl
+
+    mask = wl.protection_mask(w).numpy()
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    sigma = float(np.float32(1.0 / np.sqrt(128.0)))
+
+    def bits(t):
+        return t.contiguous().view(torch.int16).numpy().view(np.uint16)
+
+    secs = 0.0
+    nbytes = 0
+    outs = []
+    for l in range(n_layers):
+        k, v = wl.layer_kv(w, l, "cpu")
+        kb, vb = bits(k), bits(v)
+        t0 = time.perf_counter()
+        o = oracle.quantize_layer(kb, vb, w.img_start, w.image, w.base, w.bits, mask[l],
+                                  int(w.keys_only), w.kivi_group_tokens, w.kivi_group_channels,
+                                  w.kivi_residual)
+        secs += time.perf_counter() - t0
+        nq = o["nq"]
+        code_tok = 128 * w.bits // 8
+        n_prot = int(mask[l].sum())
+        coded_heads_k = (H - n_prot)
+        coded_heads_v = H if w.keys_only else (H - n_prot)
+        meta_k = o["k_meta"][0, 0].nbytes if coded_heads_k else 0
+        meta_v = o["v_meta"][0, 0].nbytes if coded_heads_v else 0
+        written = B * (H * T * 512 - (coded_heads_k + coded_heads_v) * nq * 256
+                       + coded_heads_k * (nq * code_tok + meta_k)
+                       + coded_heads_v * (nq * code_tok + meta_v))
+        nbytes += B * H * T * 512 + written
+        outs.append(o)
+    app_k = [[] for _ in range(n_layers)]
+    app_v = [[] for _ in range(n_layers)]
+    for s in range(n_steps):
+        kn, vn = wl.step_new_kv(w, s, "cpu", n_layers)
+        q = wl.step_query(w, s, "cpu", n_layers)
+        knb, vnb, qb = bits(kn), bits(vn), bits(q)
+        for l in range(n_layers):
+            app_k[l].append((knb[l].astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+            app_v[l].append((vnb[l].astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+            K = np.concatenate([outs[l]["k_att"], np.stack(app_k[l], axis=2)], axis=2)
+            V = np.concatenate([outs[l]["v_deq"].astype(np.float64), np.stack(app_v[l], axis=2)],
+                               axis=2)
+            t0 = time.perf_counter()
+            oracle.attention_layer(qb[l], K, V, sigma)
+            secs += time.perf_counter() - t0
+            Tt = K.shape[2]
+            # same per-token bytes as the packed cache the GPU reads
+            nbytes += _decode_bytes_layer(w, mask[l], outs[l]["nq"], Tt - T) + 2 * B * w.q_heads * 256
+    threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    return nbytes, secs, threads
+
+
+def _decode_bytes_layer(w, mask_row, nq, appended):
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    code_tok = 128 * w.bits // 8
+    kmeta = (128 * 8 // 32) if w.base == 1 else 8
+    vmeta = 32 if w.base == 1 else 8
+    tot = 0
+    for h in range(H):
+        prot = bool(mask_row[h])
+        if prot and not w.keys_only:
+            tot += (T + appended) * 512
+        elif prot:
+            tot += (T - nq + appended) * 512 + nq * (256 + code_tok + vmeta)
+        else:
+            tot += (T - nq + appended) * 512 + nq * (2 * code_tok + kmeta + vmeta)
+    return B * tot
+
+
+def cpu_sample_plan(w):
+    """Bounded sample sizes: about 10-30 s of oracle work."""
+    per_layer_tokens = w.batch * w.kv_heads * w.seq_len
+    if per_layer_tokens <= 10000:
+        return min(w.layers, 28), min(w.decode_steps, 8)
+    return 1, 2
+
+
+def run_reference(args):
+    from paper_2609_35800_gb300 import workloads as wl
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    w = wl.WORKLOADS[args.workload]
+    n_layers, n_steps = cpu_sample_plan(w)
+    vals = []
+    tot_s = 0.0
+    for i in range(args.warmup + args.steps):
+        nb, secs, threads = oracle_sample(w, n_layers, n_steps)
+        if i >= args.warmup:
+            vals.append(nb / secs / 1e9)
+            tot_s += secs
+    value = statistics.median(vals)
+    sample = ("%s: oracle quantize of %d layer(s) then %d decode step(s) of fp64 attention over "
+              "them; timed oracle calls only" % (w.name, n_layers, n_steps))
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 4), "unit": "GB/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1000 * tot_s / max(1, args.steps), 3), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "fp32/fp64", "data": "synthetic",
+        "config": {"workload": w.name, "sample": sample},
+        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
+                         "kind": "oracle", "sample": sample},
+        "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_gpu(args):
+    import torch
+
+    import paper_2609_35800_gb300 as hg
+    from paper_2609_35800_gb300 import build, workloads as wl
+    from paper_2609_35800_gb300.runner import CacheRunner
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    if rank == 0:
+        build.build()
+    if dist is not None:
+        dist.barrier()
+    hg.library()
+
+    w = wl.WORKLOADS[args.workload]
+    dev = "cuda:%d" % local
+    stream = torch.cuda.current_stream()
+    runner = CacheRunner(w, device=dev)
+    L, S = w.layers, w.decode_steps
+    # resident inputs of one step
+    prefill = [wl.layer_kv(w, l, dev) for l in range(L)]
+    ks = [k for k, _ in prefill]
+    vs = [v for _, v in prefill]
+    qs = [wl.step_query(w, s, dev) for s in range(S)]
+    news = [wl.step_new_kv(w, s, dev) for s in range(S)]
+    out = torch.empty_like(qs[0])
+    flush = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.int32, device=dev)
+    sigma = 0.0
+    quant_b, dec_b, app_b = geometry_bytes(runner)
+    step_bytes = quant_b + sum(dec_b) + S * app_b
+    launches_per_step = (L + 63) // 64 + S * 2 * ((L + 63) // 64)
+
+    def cushion():
+        flush.zero_()
+        torch.cuda._sleep(200000)  # keep the stream busy while the host enqueues the group
+
+    def one_step(record):
+        ev = []
+        cushion()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for l0 in range(0, L, 64):
+            n = min(64, L - l0)
+            hg.hg_quantize_kv(runner.cache, l0, ks[l0:l0 + n], vs[l0:l0 + n], stream)
+        e1.record(stream)
+        ev.append(("quant", e0, e1))
+        for s in range(S):
+            cushion()
+            a0, a1, a2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            a0.record(stream)
+            hg.hg_append_kv(runner.cache, 0, L, news[s][0], news[s][1], stream)
+            a1.record(stream)
+            hg.hg_decode_attention(runner.cache, 0, L, qs[s], out, sigma, runner.ws,
+                                   runner.ws_bytes, stream)
+            a2.record(stream)
+            ev.append(("append", a0, a1))
+            ev.append(("decode", a1, a2))
+        if record is not None:
+            record.append(ev)
+
+    for _ in range(args.warmup):
+        one_step(None)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    records = []
+    with ClockSampler(local) as clk:
+        t_wall = time.perf_counter()
+        for _ in range(args.steps):
+            one_step(records)
+        torch.cuda.synchronize()
+        t_wall = time.perf_counter() - t_wall
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    per = {"quant": [], "append": [], "decode": []}
+    step_ms = []
+    for ev in records:
+        tot = 0.0
+        for kind, a, b in ev:
+            ms = a.elapsed_time(b)
+            per[kind].append(ms)
+            tot += ms
+        step_ms.append(tot)
+    ms_step = sum(step_ms) / len(step_ms)
+    if dist is not None:
+        t = torch.tensor([ms_step], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms_step = float(t.item())
+    value = world * step_bytes / (ms_step * 1e-3) / 1e9
+
+    quant_ms = statistics.mean(per["quant"])
+    dec_ms = statistics.mean(per["decode"])
+    app_ms = statistics.mean(per["append"])
+    dec_bytes_mean = sum(dec_b) / S
+    tok_s = world * w.batch * S / ((sum(per["decode"]) + sum(per["append"])) / args.steps * 1e-3)
+
+    peaks, peak_src = measured_peaks()
+    peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
+    achieved = dec_bytes_mean / (dec_ms * 1e-3) / 1e9
+    traffic = profiled_traffic(w.name)
+
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream)
+
+    line = {
+        "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "fp32", "data": "synthetic",
+        "config": {"workload": w.name, "layers": L, "batch": w.batch,
+                   "q_heads": w.q_heads, "kv_heads": w.kv_heads,
+                   "tokens": "%d text + %d image + %d text" % (w.text_prefix, w.image,
+                                                               w.text_suffix),
+                   "base": ["minmax", "kivi", "akvq"][w.base], "bits": w.bits,
+                   "keys_only": w.keys_only, "protected_heads": int(runner.mask.sum()),
+                   "decode_steps": S, "l2": "flushed (512 MiB write) before every timed launch group",
+                   "launch": "quantize: all layers per launch; decode: append + attention over all layers per step"},
+        "pct_of_8TBps": round(100 * value / NOMINAL_HBM_GBS, 2),
+        "pct_of_measured_hbm": round(100 * value / peak, 2),
+        "decode_tokens_per_s": round(tok_s, 1),
+        "kernels": {
+            "quantize": {"ms": round(quant_ms, 4), "GBps": round(quant_b / quant_ms / 1e6, 1)},
+            "decode_attention": {"ms": round(dec_ms, 4), "GBps": round(achieved, 1)},
+            "append": {"ms": round(app_ms, 4), "GBps": round(app_b / app_ms / 1e6, 1)},
+        },
+        "step_bytes": step_bytes,
+        "wall_s_timed_region": round(t_wall, 4),
+        "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                     "frac": round(achieved / peak, 4), "traffic": traffic,
+                     "kernel": "decode_attention", "peak_source": peak_src + " hbm_gbs (burst copy)"},
+        "clocks": clk.summary(),
+        "gpu_launches": launches_per_step * args.steps,
+    }
+    if e2e is not None:
+        line["e2e"] = e2e
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        n_layers, n_steps = cpu_sample_plan(w)
+        nb, secs, threads = oracle_sample(w, n_layers, n_steps)
+        line["cpu_baseline"] = {
+            "value": round(nb / secs / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
+            "sample": "%s: oracle quantize of %d layer(s) then %d decode step(s) of fp64 attention "
+                      "over them; timed oracle calls only" % (w.name, n_layers, n_steps)}
+    if rank == 0:
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+    return 0
+
+
+def run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream):
+    """Same step driven from pinned host buffers through the C ABI."""
+    import torch
+
+    import paper_2609_35800_gb300 as hg
+    L, S = w.layers, w.decode_steps
+    hk = [k.cpu().pin_memory() for k, _ in prefill]
+    hv = [v.cpu().pin_memory() for _, v in prefill]
+    hq = [q.cpu().pin_memory() for q in qs]
+    hkn = [kn.cpu().pin_memory() for kn, _ in news]
+    hvn = [vn.cpu().pin_memory() for _, vn in news]
+    hout = torch.empty((S,) + tuple(qs[0].shape), dtype=qs[0].dtype).pin_memory()
+    dk = [torch.empty_like(k) for k, _ in prefill]
+    dv = [torch.empty_like(v) for _, v in prefill]
+    dq = torch.empty_like(qs[0])
+    dkn = torch.empty_like(news[0][0])
+    dvn = torch.empty_like(news[0][1])
+    dout = torch.empty_like(qs[0])
+    h2d = sum(t.numel() * 2 for t in hk + hv + hq + hkn + hvn)
+    d2h = hout.numel() * 2
+
+    def step():
+        for l in range(L):
+            dk[l].copy_(hk[l], non_blocking=True)
+            dv[l].copy_(hv[l], non_blocking=True)
+        for l0 in range(0, L, 64):
+            n = min(64, L - l0)
+            hg.hg_quantize_kv(runner.cache, l0, dk[l0:l0 + n], dv[l0:l0 + n], stream)
+        for s in range(S):
+            dq.copy_(hq[s], non_blocking=True)
+            dkn.copy_(hkn[s], non_blocking=True)
+            dvn.copy_(hvn[s], non_blocking=True)
+            hg.hg_append_kv(runner.cache, 0, L, dkn, dvn, stream)
+            hg.hg_decode_attention(runner.cache, 0, L, dq, dout, 0.0, runner.ws, runner.ws_bytes,
+                                   stream)
+            hout[s].copy_(dout, non_blocking=True)
+
+    for _ in range(max(1, args.warmup)):
+        step()
+    torch.cuda.synchronize()
+    times = []
+    for _ in range(args.steps):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        times.append(e0.elapsed_time(e1))
+    ms = statistics.mean(times)
+    return {"value": round(step_bytes / (ms * 1e-3) / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": round(ms, 4)}
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -83,6 +83,21 @@ uint64_t layer_mask_bits(const uint8_t* mask, int layer, int H) {
   return m;
 }
 
+// Every region start and batch-row stride must be a multiple of 16 bytes (the
+// kernels move data with 16-byte vector and asynchronous copies).
+bool geometry_aligned(const Dims& d, const LayerGeom& g) {
+  for (int h = 0; h < d.H; ++h) {
+    const HeadGeom hd = head_geom(d, g, h);
+    const uint64_t offs[] = {hd.kb, hd.vb, hd.kq, hd.kqm, hd.vq, hd.vqm, hd.kimg};
+    for (uint64_t o : offs)
+      if (o != kNone && (o & 15u)) return false;
+    const uint64_t strides[] = {hd.kb_bs, hd.kq_bs, hd.kqm_bs, hd.vq_bs, hd.vqm_bs, hd.kimg_bs};
+    for (uint64_t s : strides)
+      if (s & 15u) return false;
+  }
+  return true;
+}
+
 // Arena layout: layer blocks back to back, each 256-byte aligned.
 size_t compute_layout(const Dims& d, const uint8_t* mask, std::vector<uint64_t>* bases,
                       std::vector<uint64_t>* masks) {
@@ -90,6 +105,7 @@ size_t compute_layout(const Dims& d, const uint8_t* mask, std::vector<uint64_t>*
   for (int l = 0; l < d.L; ++l) {
     const uint64_t m = layer_mask_bits(mask, l, d.H);
     const LayerGeom g = layer_geom(d, m);
+    if (!geometry_aligned(d, g)) return 0;
     if (bases) bases->push_back(off);
     if (masks) masks->push_back(m);
     off += g.size;
@@ -151,7 +167,9 @@ hg_status hg_cache_layout(const hg_shape* shape, const hg_quant_config* config,
   const hg_status st = validate(shape, config, head_mask, &d);
   if (st != HG_OK) return st;
   if (!arena_bytes) return HG_ERR_INVALID_ARG;
-  *arena_bytes = compute_layout(d, head_mask, nullptr, nullptr);
+  const size_t n = compute_layout(d, head_mask, nullptr, nullptr);
+  if (n == 0) return HG_ERR_UNSUPPORTED;
+  *arena_bytes = n;
   return HG_OK;
 }
 
@@ -169,6 +187,10 @@ hg_status hg_cache_create(const hg_shape* shape, const hg_quant_config* config,
   c->cfg = *config;
   c->d = d;
   c->needed_bytes = compute_layout(d, head_mask, &c->layer_base, &c->layer_mask);
+  if (c->needed_bytes == 0) {
+    delete c;
+    return HG_ERR_UNSUPPORTED;
+  }
   if (arena_bytes < c->needed_bytes) {
     delete c;
     return HG_ERR_ARENA_TOO_SMALL;

@@ -67,6 +67,28 @@ __device__ __forceinline__ void fwht128_warp(float (&x)[4], int lane) {
   for (int i = 0; i < 4; ++i) x[i] = __fmul_rn(x[i], c);
 }
 
+// code = clamp(rint_even(fl32(d / scale)), 0, levels) computed without a
+// division in almost every case.  With r = fl32(1 / scale) and q' = fl32(d r),
+// q' = (d / scale)(1 + e1)(1 + e2) with |e1|, |e2| <= 2^-24, and the correctly
+// rounded quotient q = fl32(d / scale) is within 2^-24 relative of d / scale,
+// so |q' - q| <= 3 * 2^-24 * (d / scale) <= 3e-6 for d / scale <= 16.  When q'
+// is farther than 2^-17 from every half-integer, q lies strictly on the same
+// side of it and rint(q) == rint(q'); otherwise (a near-tie, about 1.5e-5 of
+// the values) the IEEE division decides.  Valid while r is a normal finite
+// number (scale >= 2^-125); the caller passes fast = false otherwise.
+__device__ __forceinline__ uint32_t code_of(float d, float scale, float r, float levels, bool fast) {
+  float rq;
+  if (fast) {
+    const float q = __fmul_rn(d, r);
+    rq = rintf(q);
+    if (0.5f - fabsf(__fsub_rn(q, rq)) < 7.62939453125e-6f) rq = rintf(__fdiv_rn(d, scale));
+  } else {
+    rq = rintf(__fdiv_rn(d, scale));
+  }
+  rq = fminf(fmaxf(rq, 0.0f), levels);
+  return (uint32_t)rq;
+}
+
 // Group quantizer over a group spread across GL consecutive lanes (aligned),
 // 4 values per lane.  min / max by butterflies (exact), signed zeros folded to
 // +0, scale = (max - min) / (2^bits - 1), code = round-half-even((x - min) /
@@ -86,17 +108,11 @@ __device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, u
   const float levels = (float)((1 << bits) - 1);
   scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   zero = mn;
+  const bool fast = scale >= 2.3509887e-38f;  // 2^-125
+  const float r = __frcp_rn(fast ? scale : 1.0f);
 #pragma unroll
-  for (int i = 0; i < 4; ++i) {
-    if (scale == 0.0f) {
-      code[i] = 0u;
-    } else {
-      const float q = __fdiv_rn(__fsub_rn(x[i], mn), scale);
-      float r = rintf(q);
-      r = fminf(fmaxf(r, 0.0f), levels);
-      code[i] = (uint32_t)r;
-    }
-  }
+  for (int i = 0; i < 4; ++i)
+    code[i] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[i], mn), scale, r, levels, fast);
 }
 
 // Reconstruction fl32(fl32(code * scale) + zero).

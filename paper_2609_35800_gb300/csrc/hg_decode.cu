@@ -1,83 +1,731 @@
-// Split-K decode attention over the mixed-precision cache.
+// Split-K decode attention over the mixed-precision cache (tensor cores).
 //
-// One CTA per work item = one chunk of one (layer, batch row, KV head): either
-// a run of BF16 tokens (text, image tokens not coded, protected heads,
-// appended tokens) or a run of coded image tokens (codes + fp32 scale/zero for
-// K and V, or BF16 K + coded V for keys-only protected heads).  The segment
-// type is uniform inside a CTA, so the only branch on the mask or the image
-// span is taken once per CTA.  Each warp streams 32-token tiles into shared
-// memory, computes the G query heads' scores (lane = token), keeps an online
-// softmax, and accumulates P.V (lane = 4 channels).  Warps are combined in
-// shared memory; a CTA that is not alone on its head writes its (m, l, o)
-// partial to the workspace and the last CTA to arrive (atomic ticket, no
-// waiting) merges them and writes the BF16 output.
+// One CTA per work item = one chunk of one (layer, batch row, KV head).  A
+// chunk is uniform: a run of BF16 tokens (text, uncoded image tokens,
+// protected heads, appended tokens), a run of coded image tokens (packed
+// codes + fp32 scale/zero for K and V), or, for keys-only protected heads, BF16
+// keys with coded values.  The only branch on the mask or the image span is
+// therefore taken once per CTA.
 //
-// AKVQ-style keys are coded in the rotated domain; since the normalised
-// Hadamard matrix is symmetric and orthonormal, <q, H k'> = <H q, k'>, so the
-// query is rotated once per CTA instead of inverse-rotating every key.
+// Tiles of the chunk stream through a 3-stage cp.async pipeline in shared
+// memory.  Each warp owns 16-token slices and computes, with mma.sync
+// m16n8k16 (BF16 in, fp32 accumulate):
+//   S^T[token][query] = K . q     A = keys (BF16 via ldmatrix, or codes
+//                                 expanded exactly to BF16 in registers),
+//                                 B = the G queries of the KV head (padded to 8)
+//   O^T[chan][query] += V^T . P^T A = values (ldmatrix.trans, or codes),
+//                                 B = P^T, transposed from the score fragment
+//                                 with movmatrix.
+// Coded keys are contracted in the code domain: with per-token groups
+// k^_d = s c_d + z, so q.k^ = s (q.c) + z sum(q); KIVI-style per-channel
+// groups fold the channel scale into the query (q~_d = q_d s_d, split into a
+// BF16 hi + lo pair) and add sum_d q_d z_d.  Values fold the token scale into
+// P (p s) and add sum_t p_t z_t.  AKVQ-style keys are coded in the rotated
+// domain; since the normalised Hadamard matrix is symmetric and orthonormal,
+// <q, H k'> = <H q, k'>, so the query is rotated once per CTA (hi + lo split).
+//
+// The online softmax rescales its accumulators only when a running maximum
+// grows by more than 2^8 (probabilities stay <= 256 before normalisation).
+// Warps are combined in shared memory; a CTA that is not alone on its head
+// writes an (m, l, o) partial to the workspace and the last CTA to arrive
+// (atomic ticket, no waiting) merges them and writes the BF16 output.
 #include <cuda_runtime.h>
 
 #include "hg_common.cuh"
 #include "hg_internal.h"
+#include "hg_mma.cuh"
 
 namespace hg {
 
 namespace {
 
 constexpr int kThreads = 128;
-constexpr int kWarps = kThreads / 32;
-constexpr int kTile = 32;
-constexpr int kKRowHalves = kD + 8;                       // padded BF16 key row (272 bytes)
-constexpr int kWarpTileBytes = kTile * kKRowHalves * 2 + kTile * kD * 2;  // K + V BF16 tiles
+constexpr int kWarps = 4;
+constexpr int kStages = 3;
+constexpr int kStageBytes = 32768;
+constexpr int kBf16Tile = 64;      // tokens per tile of BF16 rows (K 16 KB + V 16 KB)
+constexpr int kMixTile = 64;       // tokens per tile of BF16 keys + coded values
 constexpr int kPartialStride = kD + 2;
+constexpr int kQOff = 0;                      // float q[16][128]
+constexpr int kZsumOff = kMaxG * kD * 4;      // float sum(q)[16]
+constexpr int kStageOff = kZsumOff + 256;
+constexpr int kSmemBytes = kStageOff + kStages * kStageBytes;
+constexpr unsigned kFull = 0xffffffffu;
 
-template <int MAXG>
-struct Smem {
-  static constexpr int q_off = 0;                                   // float [MAXG][128]
-  static constexpr int qr_off = q_off + MAXG * kD * 4;              // float [MAXG][128] rotated
-  static constexpr int p_off = qr_off + MAXG * kD * 4;              // float [warps][32][MAXG]
-  static constexpr int tile_off = p_off + kWarps * kTile * MAXG * 4;
-  static constexpr int bytes = tile_off + kWarps * kWarpTileBytes;
+enum KMode { K_BF16 = 0, K_TOKEN = 1, K_KIVI = 2 };
+enum VMode { V_BF16 = 0, V_TOKEN = 1, V_KIVI = 2 };
+
+template <int VM>
+struct NZOf {
+  static constexpr int value = VM == V_TOKEN ? 1 : (VM == V_KIVI ? 4 : 1);
 };
 
-__device__ __forceinline__ void warp_copy16(void* dst, const void* src, int nbytes, int lane) {
-  for (int off = lane * 16; off < nbytes; off += 32 * 16)
-    *reinterpret_cast<uint4*>(static_cast<char*>(dst) + off) =
-        __ldg(reinterpret_cast<const uint4*>(static_cast<const char*>(src) + off));
+// Tokens per tile of coded K + coded V (multiple of 64, divides 512).
+__host__ __device__ constexpr int coded_tile(int bits) { return bits == 2 ? 256 : 128; }
+
+struct Seg {
+  const char* k;   // BF16 key rows (K_BF16)
+  const char* v;   // BF16 value rows (V_BF16)
+  const char* kc;  // key codes
+  const char* km;  // key metadata
+  const char* vc;  // value codes
+  const char* vm;  // value metadata
+};
+
+__device__ __forceinline__ void copy_linear(uint32_t dst, const char* src, int slot_bytes,
+                                            int valid_bytes, int tid) {
+  for (int off = tid * 16; off < slot_bytes; off += kThreads * 16) {
+    int n = valid_bytes - off;
+    n = n < 0 ? 0 : (n > 16 ? 16 : n);
+    cp_async16(dst + off, n > 0 ? src + off : src, n);
+  }
 }
-__device__ __forceinline__ void warp_copy8(void* dst, const void* src, int nbytes, int lane) {
-  for (int off = lane * 8; off < nbytes; off += 32 * 8)
-    *reinterpret_cast<uint2*>(static_cast<char*>(dst) + off) =
-        __ldg(reinterpret_cast<const uint2*>(static_cast<const char*>(src) + off));
-}
-// nt rows of 256 bytes into a tile with row pitch `pitch` bytes.
-__device__ __forceinline__ void warp_copy_rows(char* dst, int pitch, const char* src, int nt, int lane) {
-  for (int idx = lane; idx < nt * 16; idx += 32) {
-    const int row = idx >> 4, col = idx & 15;
-    *reinterpret_cast<uint4*>(dst + row * pitch + col * 16) =
-        __ldg(reinterpret_cast<const uint4*>(src + row * 256 + col * 16));
+
+// nvalid BF16 rows (256 B each) into a 64-row tile, 16-byte chunks swizzled by
+// (row & 7) so that ldmatrix reads are conflict free; missing rows are zero.
+__device__ __forceinline__ void copy_rows_swizzled(uint32_t dst, const char* src, int nvalid,
+                                                   int tid) {
+  for (int q = tid; q < 64 * 16; q += kThreads) {
+    const int r = q >> 4, c = q & 15;
+    const bool ok = r < nvalid;
+    cp_async16(dst + r * 256 + ((c ^ (r & 7)) << 4), ok ? src + r * 256 + c * 16 : src,
+               ok ? 16 : 0);
   }
 }
 
 template <int BITS>
-__device__ __forceinline__ void codes4(const uint32_t* row, int c4, uint32_t (&c)[4]) {
-  // codes of channels 4*c4 .. 4*c4+3 from a packed 128-code row
-  if (BITS == 2) {
-    const uint32_t byte = (row[c4 >> 2] >> (8 * (c4 & 3))) & 0xffu;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) c[i] = (byte >> (2 * i)) & 3u;
+__device__ __forceinline__ uint32_t pair2(uint32_t x) {  // codes at bits [0,b) and [16,16+b)
+  return codes_bf16x2(x & (BITS == 2 ? 0x00030003u : 0x000F000Fu));
+}
+
+template <int NT, int NZ>
+struct WarpState {
+  float o[NT][8][4];
+  float m[NT][2];
+  float l[NT][2];
+  float z[NT][2][NZ];
+};
+
+template <int BITS, int KM, int VM>
+struct Tile {
+  static constexpr int tokens = (KM == K_BF16 && VM == V_BF16) ? kBf16Tile
+                                : (KM == K_BF16 ? kMixTile : coded_tile(BITS));
+  static constexpr int kc_bytes = (KM == K_BF16) ? tokens * 256 : tokens * 16 * BITS;
+  static constexpr int km_bytes = (KM == K_TOKEN) ? tokens * 8 : (KM == K_KIVI ? tokens * 32 : 0);
+  static constexpr int vc_bytes = (VM == V_BF16) ? tokens * 256 : tokens * 16 * BITS;
+  static constexpr int vm_bytes = (VM == V_TOKEN) ? tokens * 8 : (VM == V_KIVI ? tokens * 32 : 0);
+  static constexpr int kc_off = 0;
+  static constexpr int km_off = kc_off + kc_bytes;
+  static constexpr int vc_off = km_off + km_bytes;
+  static constexpr int vm_off = vc_off + vc_bytes;
+  static_assert(vm_off + vm_bytes <= kStageBytes, "tile does not fit a stage");
+};
+
+template <int BITS, int KM, int VM>
+__device__ __forceinline__ void issue_tile(uint32_t st, const Seg& sg, int t0, int nvalid, int tid) {
+  using TL = Tile<BITS, KM, VM>;
+  if (KM == K_BF16) {
+    copy_rows_swizzled(st + TL::kc_off, sg.k + (size_t)t0 * 256, nvalid, tid);
   } else {
-    const uint32_t half = (row[c4 >> 1] >> (16 * (c4 & 1))) & 0xffffu;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) c[i] = (half >> (4 * i)) & 15u;
+    copy_linear(st + TL::kc_off, sg.kc + (size_t)t0 * 16 * BITS, TL::kc_bytes, nvalid * 16 * BITS, tid);
+    // KIVI-style key metadata: one (scale, zero) per channel per 32 tokens = 32 B per token
+    constexpr int kmb = (KM == K_TOKEN) ? 8 : 32;
+    copy_linear(st + TL::km_off, sg.km + (size_t)t0 * kmb, TL::km_bytes, nvalid * kmb, tid);
+  }
+  if (VM == V_BF16) {
+    copy_rows_swizzled(st + TL::vc_off, sg.v + (size_t)t0 * 256, nvalid, tid);
+  } else {
+    copy_linear(st + TL::vc_off, sg.vc + (size_t)t0 * 16 * BITS, TL::vc_bytes, nvalid * 16 * BITS, tid);
+    constexpr int vmb = (VM == V_TOKEN) ? 8 : 32;
+    copy_linear(st + TL::vm_off, sg.vm + (size_t)t0 * vmb, TL::vm_bytes, nvalid * vmb, tid);
   }
 }
 
-template <int MAXG, int BITS>
-__global__ void __launch_bounds__(kThreads)
+// ---------------------------------------------------------------------------
+// Query fragments
+// ---------------------------------------------------------------------------
+// hi + lo BF16 split of an fp32 pair (x = hi + lo to ~16 significant bits)
+__device__ __forceinline__ void split_pair(float x0, float x1, uint32_t& hi, uint32_t& lo) {
+  hi = pack_bf16x2(x0, x1);
+  const float h0 = __uint_as_float(hi << 16), h1 = __uint_as_float(hi & 0xffff0000u);
+  lo = pack_bf16x2(x0 - h0, x1 - h1);
+}
+
+// Natural channel order (BF16 keys): k-step j covers channels 16j..16j+15.
+template <int NT>
+__device__ __forceinline__ void qfrag_natural(uint32_t (&qb)[NT][8][2], const float* q_s, int g, int tq) {
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    const float* qr = q_s + (nt * 8 + g) * kD;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      qb[nt][j][0] = pack_bf16x2(qr[16 * j + 2 * tq], qr[16 * j + 2 * tq + 1]);
+      qb[nt][j][1] = pack_bf16x2(qr[16 * j + 2 * tq + 8], qr[16 * j + 2 * tq + 9]);
+    }
+  }
+}
+
+// Channels matching the in-register expansion of a packed token row.
+// 2-bit: thread tq reads words 2tq and 2tq+1; k-step j takes code pair
+// (j, j+8) of each.  4-bit: thread tq reads words 4tq..4tq+3; k-step j takes
+// pairs (i, i+4) and (i+1, i+5), i = 2 (j & 1), of word 4tq + j/2.
+template <int BITS>
+__device__ __forceinline__ void token_channels(int tq, int j, int (&c)[4]) {
+  if (BITS == 2) {
+    c[0] = 32 * tq + j;
+    c[1] = 32 * tq + j + 8;
+    c[2] = 32 * tq + 16 + j;
+    c[3] = 32 * tq + 24 + j;
+  } else {
+    const int w = 4 * tq + (j >> 1), i = 2 * (j & 1);
+    c[0] = 8 * w + i;
+    c[1] = 8 * w + i + 4;
+    c[2] = 8 * w + i + 1;
+    c[3] = 8 * w + i + 5;
+  }
+}
+
+template <int BITS, int NT, bool ROT>
+__device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (&ql)[NT][8][2],
+                                            const float* q_s, int g, int tq) {
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+    const float* qr = q_s + (nt * 8 + g) * kD;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      int c[4];
+      token_channels<BITS>(tq, j, c);
+      if (ROT) {
+        split_pair(qr[c[0]], qr[c[1]], qb[nt][j][0], ql[nt][j][0]);
+        split_pair(qr[c[2]], qr[c[3]], qb[nt][j][1], ql[nt][j][1]);
+      } else {
+        qb[nt][j][0] = pack_bf16x2(qr[c[0]], qr[c[1]]);
+        qb[nt][j][1] = pack_bf16x2(qr[c[2]], qr[c[3]]);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Softmax update of one 16-token slice
+// ---------------------------------------------------------------------------
+template <int NT, int NZ>
+__device__ __forceinline__ void softmax_update(WarpState<NT, NZ>& ws, float (&sc)[NT][4], float (&p)[NT][4]) {
+  float mx[NT][2];
+  bool need = false;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      float v = fmaxf(sc[nt][e], sc[nt][2 + e]);
+      v = fmaxf(v, __shfl_xor_sync(kFull, v, 4));
+      v = fmaxf(v, __shfl_xor_sync(kFull, v, 8));
+      v = fmaxf(v, __shfl_xor_sync(kFull, v, 16));
+      mx[nt][e] = v;
+      need |= v > ws.m[nt][e] + 8.0f;
+    }
+  }
+  if (__any_sync(kFull, need)) {
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 2; ++e) {
+        const float mn = fmaxf(ws.m[nt][e], mx[nt][e]);
+        const float a = (ws.m[nt][e] == -INFINITY) ? 0.f : exp2f(ws.m[nt][e] - mn);
+        ws.m[nt][e] = mn;
+        ws.l[nt][e] *= a;
+#pragma unroll
+        for (int zz = 0; zz < NZ; ++zz) ws.z[nt][e][zz] *= a;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          ws.o[nt][mt][e] *= a;
+          ws.o[nt][mt][2 + e] *= a;
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) p[nt][i] = exp2f(sc[nt][i] - ws.m[nt][i & 1]);
+#pragma unroll
+    for (int e = 0; e < 2; ++e) ws.l[nt][e] += p[nt][e] + p[nt][2 + e];
+  }
+}
+
+// B fragments of P^T (rows scaled by fg for token g, fg8 for token g+8), as a
+// BF16 hi + lo pair: b[0..1] hi, b[2..3] lo, so that P is carried to ~16 bits.
+__device__ __forceinline__ void pfrag(const float (&p)[4], float fg, float fg8, uint32_t (&b)[4]) {
+  uint32_t h0, l0, h1, l1;
+  split_pair(p[0] * fg, p[1] * fg, h0, l0);
+  split_pair(p[2] * fg8, p[3] * fg8, h1, l1);
+  b[0] = movtrans(h0);
+  b[1] = movtrans(h1);
+  b[2] = movtrans(l0);
+  b[3] = movtrans(l1);
+}
+
+// O^T m-tile += A * P^T (hi and lo parts)
+__device__ __forceinline__ void mma_pv(float (&o)[4], const uint32_t (&a)[4], const uint32_t (&b)[4]) {
+  mma_bf16(o, a, b[0], b[1]);
+  mma_bf16(o, a, b[2], b[3]);
+}
+
+// ---------------------------------------------------------------------------
+// One tile: every warp processes its 16-token slices
+// ---------------------------------------------------------------------------
+template <int BITS, int NT, int KM, int VM, bool ROT>
+__device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws, const char* st,
+                                             int nvalid, const uint32_t (&qb)[NT][8][2],
+                                             const uint32_t (&ql)[NT][8][2], const float* q_s,
+                                             const float* zsum_s, float scale_log2, int warp,
+                                             int lane) {
+  using TL = Tile<BITS, KM, VM>;
+  constexpr int NZ = NZOf<VM>::value;
+  const int g = lane >> 2, tq = lane & 3;
+  const uint32_t st_u32 = smem_u32(st);
+  const uint32_t* kc32 = reinterpret_cast<const uint32_t*>(st + TL::kc_off);
+  const float2* km2 = reinterpret_cast<const float2*>(st + TL::km_off);
+  const uint32_t* vc32 = reinterpret_cast<const uint32_t*>(st + TL::vc_off);
+  const float2* vm2 = reinterpret_cast<const float2*>(st + TL::vm_off);
+
+  // KIVI-style keys: a warp takes whole 32-token groups (two slices) so the
+  // group's scaled query fragments are built once.
+  constexpr int SPU = (KM == K_KIVI) ? 2 : 1;  // slices per unit
+  constexpr int UNITS = TL::tokens / (16 * SPU);
+  for (int u = warp; u < UNITS; u += kWarps) {
+    if (u * 16 * SPU >= nvalid) break;
+    float acc[SPU][NT][4];
+#pragma unroll
+    for (int s = 0; s < SPU; ++s)
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[s][nt][i] = 0.f;
+    float zk[NT][2];  // KIVI-style: sum_c q_c z_c of the group, per query column
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) zk[nt][0] = zk[nt][1] = 0.f;
+
+    // ---------------- scores ----------------
+    if (KM == K_BF16) {
+      const int tok0 = u * 16;
+      const int mat = lane >> 3, r = lane & 7;
+      const int row = tok0 + r + 8 * (mat & 1);
+      const uint32_t rbase = st_u32 + TL::kc_off + row * 256;
+      const int rsw = row & 7, ch = mat >> 1;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        uint32_t a[4];
+        ldsm_x4(a, rbase + (((2 * j + ch) ^ rsw) << 4));
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
+      }
+    } else if (KM == K_TOKEN) {
+      const int tok0 = u * 16;
+      if (BITS == 2) {
+        const uint2 ka = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g) * 8 + 2 * tq);
+        const uint2 kb = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g + 8) * 8 + 2 * tq);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          uint32_t a[4];
+          a[0] = pair2<2>(ka.x >> (2 * j));
+          a[1] = pair2<2>(kb.x >> (2 * j));
+          a[2] = pair2<2>(ka.y >> (2 * j));
+          a[3] = pair2<2>(kb.y >> (2 * j));
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
+            if (ROT) mma_bf16(acc[0][nt], a, ql[nt][j][0], ql[nt][j][1]);
+          }
+        }
+      } else {
+        const uint4 ka = *reinterpret_cast<const uint4*>(kc32 + (tok0 + g) * 16 + 4 * tq);
+        const uint4 kb = *reinterpret_cast<const uint4*>(kc32 + (tok0 + g + 8) * 16 + 4 * tq);
+        const uint32_t wa[4] = {ka.x, ka.y, ka.z, ka.w};
+        const uint32_t wb[4] = {kb.x, kb.y, kb.z, kb.w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int wi = j >> 1, i = 2 * (j & 1);
+          uint32_t a[4];
+          a[0] = pair2<4>(wa[wi] >> (4 * i));
+          a[1] = pair2<4>(wb[wi] >> (4 * i));
+          a[2] = pair2<4>(wa[wi] >> (4 * i + 4));
+          a[3] = pair2<4>(wb[wi] >> (4 * i + 4));
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
+            if (ROT) mma_bf16(acc[0][nt], a, ql[nt][j][0], ql[nt][j][1]);
+          }
+        }
+      }
+    } else {  // K_KIVI: group u of the tile; channel c has (scale, zero) = meta[u][c]
+      const float2* gm = km2 + u * kD;
+      uint32_t qh[NT][8][2], qlo[NT][8][2];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt) {
+        const float* qr = q_s + (nt * 8 + g) * kD;
+        float zpart = 0.f;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          // k-slots 2tq, 2tq+1, 2tq+8, 2tq+9 of k-step j <-> channels 32tq + 4j + 0..3
+          const int c0 = 32 * tq + 4 * j;
+          const float4 m01 = *reinterpret_cast<const float4*>(gm + c0);
+          const float4 m23 = *reinterpret_cast<const float4*>(gm + c0 + 2);
+          const float4 qv = *reinterpret_cast<const float4*>(qr + c0);
+          split_pair(qv.x * m01.x, qv.y * m01.z, qh[nt][j][0], qlo[nt][j][0]);
+          split_pair(qv.z * m23.x, qv.w * m23.z, qh[nt][j][1], qlo[nt][j][1]);
+          zpart = fmaf(qv.x, m01.y, zpart);
+          zpart = fmaf(qv.y, m01.w, zpart);
+          zpart = fmaf(qv.z, m23.y, zpart);
+          zpart = fmaf(qv.w, m23.w, zpart);
+        }
+        // sum over the four tq lanes of query g, then fetch the columns' values
+        zpart += __shfl_xor_sync(kFull, zpart, 1);
+        zpart += __shfl_xor_sync(kFull, zpart, 2);
+        zk[nt][0] = __shfl_sync(kFull, zpart, (2 * tq) << 2);
+        zk[nt][1] = __shfl_sync(kFull, zpart, (2 * tq + 1) << 2);
+      }
+      const uint32_t* gc = kc32 + u * kD * BITS;  // [128 channels][BITS words], token order
+      // byte selector: byte (g/2) of a -> byte 0, byte (g/2) of b -> byte 2
+      const uint32_t sel4 = (uint32_t)(g >> 1) | ((uint32_t)(4 + (g >> 1)) << 8);
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int c0 = 32 * tq + 4 * j;
+        uint32_t w[4][4];
+#pragma unroll
+        for (int cc = 0; cc < 4; ++cc) {
+          if (BITS == 2) {
+            const uint2 t2 = *reinterpret_cast<const uint2*>(gc + (c0 + cc) * 2);
+            w[cc][0] = t2.x;
+            w[cc][1] = t2.y;
+            w[cc][2] = w[cc][3] = 0u;
+          } else {
+            const uint4 t4 = *reinterpret_cast<const uint4*>(gc + (c0 + cc) * 4);
+            w[cc][0] = t4.x;
+            w[cc][1] = t4.y;
+            w[cc][2] = t4.z;
+            w[cc][3] = t4.w;
+          }
+        }
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+          uint32_t a[4];
+          if (BITS == 2) {
+            // word s of a channel: tokens 16s..16s+15; its low half holds the first 8
+            a[0] = pair2<2>(prmt(w[0][s], w[1][s], 0x5410) >> (2 * g));
+            a[1] = pair2<2>(prmt(w[0][s], w[1][s], 0x7632) >> (2 * g));
+            a[2] = pair2<2>(prmt(w[2][s], w[3][s], 0x5410) >> (2 * g));
+            a[3] = pair2<2>(prmt(w[2][s], w[3][s], 0x7632) >> (2 * g));
+          } else {
+            // words 2s, 2s+1 of a channel: tokens 16s..16s+7 and 16s+8..16s+15
+            const int sh = 4 * (g & 1);
+            a[0] = pair2<4>(prmt(w[0][2 * s], w[1][2 * s], sel4) >> sh);
+            a[1] = pair2<4>(prmt(w[0][2 * s + 1], w[1][2 * s + 1], sel4) >> sh);
+            a[2] = pair2<4>(prmt(w[2][2 * s], w[3][2 * s], sel4) >> sh);
+            a[3] = pair2<4>(prmt(w[2][2 * s + 1], w[3][2 * s + 1], sel4) >> sh);
+          }
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) {
+            mma_bf16(acc[s][nt], a, qh[nt][j][0], qh[nt][j][1]);
+            mma_bf16(acc[s][nt], a, qlo[nt][j][0], qlo[nt][j][1]);
+          }
+        }
+      }
+    }
+
+    // ---------------- per slice: softmax, then P.V ----------------
+#pragma unroll
+    for (int s = 0; s < SPU; ++s) {
+      const int tok0 = (u * SPU + s) * 16;
+      if (tok0 >= nvalid) break;
+      float sc[NT][4];
+      if (KM == K_TOKEN) {
+        const float2 mg = km2[tok0 + g], mg8 = km2[tok0 + g + 8];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+          for (int e = 0; e < 2; ++e) {
+            const float zq = zsum_s[nt * 8 + 2 * tq + e];
+            sc[nt][e] = fmaf(mg.x, acc[s][nt][e], mg.y * zq) * scale_log2;
+            sc[nt][2 + e] = fmaf(mg8.x, acc[s][nt][2 + e], mg8.y * zq) * scale_log2;
+          }
+        }
+      } else if (KM == K_KIVI) {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) sc[nt][i] = (acc[s][nt][i] + zk[nt][i & 1]) * scale_log2;
+      } else {
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+          for (int i = 0; i < 4; ++i) sc[nt][i] = acc[s][nt][i] * scale_log2;
+      }
+      if (tok0 + 16 > nvalid) {
+        const bool vg0 = tok0 + g < nvalid, vg8 = tok0 + g + 8 < nvalid;
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          if (!vg0) sc[nt][0] = sc[nt][1] = -INFINITY;
+          if (!vg8) sc[nt][2] = sc[nt][3] = -INFINITY;
+        }
+      }
+      float p[NT][4];
+      softmax_update<NT, NZ>(ws, sc, p);
+
+      if (VM == V_BF16) {
+        uint32_t b[NT][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) pfrag(p[nt], 1.f, 1.f, b[nt]);
+        const int mat = lane >> 3, r = lane & 7;
+        const int row = tok0 + r + 8 * (mat >> 1);
+        const uint32_t rbase = st_u32 + TL::vc_off + row * 256;
+        const int rsw = row & 7, ch = mat & 1;
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          uint32_t a[4];
+          ldsm_x4_trans(a, rbase + (((2 * mt + ch) ^ rsw) << 4));
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
+        }
+      } else if (VM == V_TOKEN) {
+        const float2 vg = vm2[tok0 + g], vg8 = vm2[tok0 + g + 8];
+        uint32_t b[NT][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+          pfrag(p[nt], vg.x, vg8.x, b[nt]);
+#pragma unroll
+          for (int e = 0; e < 2; ++e) ws.z[nt][e][0] += p[nt][e] * vg.y + p[nt][2 + e] * vg8.y;
+        }
+        const int t0 = tok0 + 2 * tq;
+        if (BITS == 2) {
+          // word g of a token row holds channels 16g..16g+15
+          const uint32_t w0 = vc32[t0 * 8 + g], w1 = vc32[(t0 + 1) * 8 + g];
+          const uint32_t w8 = vc32[(t0 + 8) * 8 + g], w9 = vc32[(t0 + 9) * 8 + g];
+          const uint32_t x01 = prmt(w0, w1, 0x5410), y01 = prmt(w0, w1, 0x7632);
+          const uint32_t x89 = prmt(w8, w9, 0x5410), y89 = prmt(w8, w9, 0x7632);
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt) {
+            uint32_t a[4];
+            a[0] = pair2<2>(x01 >> (2 * mt));
+            a[1] = pair2<2>(y01 >> (2 * mt));
+            a[2] = pair2<2>(x89 >> (2 * mt));
+            a[3] = pair2<2>(y89 >> (2 * mt));
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
+          }
+        } else {
+          // word 2g holds channels 16g..16g+7 (codes 0-3 low half, 4-7 high), 2g+1 the next 8
+          const uint2 v0 = *reinterpret_cast<const uint2*>(vc32 + t0 * 16 + 2 * g);
+          const uint2 v1 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 1) * 16 + 2 * g);
+          const uint2 v8 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 8) * 16 + 2 * g);
+          const uint2 v9 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 9) * 16 + 2 * g);
+          const uint32_t xa = prmt(v0.x, v1.x, 0x5410), ya = prmt(v0.x, v1.x, 0x7632);
+          const uint32_t xb = prmt(v0.y, v1.y, 0x5410), yb = prmt(v0.y, v1.y, 0x7632);
+          const uint32_t xc = prmt(v8.x, v9.x, 0x5410), yc = prmt(v8.x, v9.x, 0x7632);
+          const uint32_t xd = prmt(v8.y, v9.y, 0x5410), yd = prmt(v8.y, v9.y, 0x7632);
+#pragma unroll
+          for (int mt = 0; mt < 8; ++mt) {
+            const int sh = 4 * (mt & 3);
+            uint32_t a[4];
+            a[0] = pair2<4>((mt < 4 ? xa : ya) >> sh);
+            a[1] = pair2<4>((mt < 4 ? xb : yb) >> sh);
+            a[2] = pair2<4>((mt < 4 ? xc : yc) >> sh);
+            a[3] = pair2<4>((mt < 4 ? xd : yd) >> sh);
+#pragma unroll
+            for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
+          }
+        }
+      } else {  // V_KIVI: 4 value groups of 32 channels; m-tile mt = channels 16mt..16mt+15
+        const float4* vrow_g = reinterpret_cast<const float4*>(vm2 + (tok0 + g) * 4);
+        const float4* vrow_g8 = reinterpret_cast<const float4*>(vm2 + (tok0 + g + 8) * 4);
+        float sv_g[4], zv_g[4], sv_g8[4], zv_g8[4];
+        {
+          const float4 a0 = vrow_g[0], a1 = vrow_g[1], b0 = vrow_g8[0], b1 = vrow_g8[1];
+          sv_g[0] = a0.x; zv_g[0] = a0.y; sv_g[1] = a0.z; zv_g[1] = a0.w;
+          sv_g[2] = a1.x; zv_g[2] = a1.y; sv_g[3] = a1.z; zv_g[3] = a1.w;
+          sv_g8[0] = b0.x; zv_g8[0] = b0.y; sv_g8[1] = b0.z; zv_g8[1] = b0.w;
+          sv_g8[2] = b1.x; zv_g8[2] = b1.y; sv_g8[3] = b1.z; zv_g8[3] = b1.w;
+        }
+        uint32_t b[NT][4][4];
+#pragma unroll
+        for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+          for (int jg = 0; jg < 4; ++jg) {
+            pfrag(p[nt], sv_g[jg], sv_g8[jg], b[nt][jg]);
+#pragma unroll
+            for (int e = 0; e < 2; ++e)
+              ws.z[nt][e][jg % NZ] += p[nt][e] * zv_g[jg] + p[nt][2 + e] * zv_g8[jg];
+          }
+        }
+        const int t0 = tok0 + 2 * tq;
+        constexpr int W = 4 * BITS;  // words per token
+        const uint32_t sel4 = (uint32_t)(g >> 1) | ((uint32_t)(4 + (g >> 1)) << 8);
+#pragma unroll
+        for (int mt = 0; mt < 8; ++mt) {
+          uint32_t a[4];
+          if (BITS == 2) {
+            const uint32_t w0 = vc32[t0 * W + mt], w1 = vc32[(t0 + 1) * W + mt];
+            const uint32_t w8 = vc32[(t0 + 8) * W + mt], w9 = vc32[(t0 + 9) * W + mt];
+            a[0] = pair2<2>(prmt(w0, w1, 0x5410) >> (2 * g));
+            a[1] = pair2<2>(prmt(w0, w1, 0x7632) >> (2 * g));
+            a[2] = pair2<2>(prmt(w8, w9, 0x5410) >> (2 * g));
+            a[3] = pair2<2>(prmt(w8, w9, 0x7632) >> (2 * g));
+          } else {
+            const uint2 u0 = *reinterpret_cast<const uint2*>(vc32 + t0 * W + 2 * mt);
+            const uint2 u1 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 1) * W + 2 * mt);
+            const uint2 u8 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 8) * W + 2 * mt);
+            const uint2 u9 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 9) * W + 2 * mt);
+            const int sh = 4 * (g & 1);
+            a[0] = pair2<4>(prmt(u0.x, u1.x, sel4) >> sh);
+            a[1] = pair2<4>(prmt(u0.y, u1.y, sel4) >> sh);
+            a[2] = pair2<4>(prmt(u8.x, u9.x, sel4) >> sh);
+            a[3] = pair2<4>(prmt(u8.y, u9.y, sel4) >> sh);
+          }
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt][mt >> 1]);
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// One work item with a given key / value mode: pipeline, then per-warp results
+// into shared memory (m, l, o[q][channel]).
+// ---------------------------------------------------------------------------
+template <int BITS, int NT, int KM, int VM, bool ROT>
+__device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int te, float scale_log2,
+                                         const uint16_t* qg, int G, float* red_m, float* red_l,
+                                         float* red_o) {
+  using TL = Tile<BITS, KM, VM>;
+  constexpr int NZ = NZOf<VM>::value;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int g = lane >> 2, tq = lane & 3;
+  float* q_s = reinterpret_cast<float*>(smem + kQOff);
+  float* zsum_s = reinterpret_cast<float*>(smem + kZsumOff);
+  char* stages = smem + kStageOff;
+
+  // First tiles in flight before anything else.
+  const int n_tiles = (te - tb + TL::tokens - 1) / TL::tokens;
+  const uint32_t st0 = smem_u32(stages);
+#pragma unroll
+  for (int s = 0; s < kStages - 1; ++s) {
+    if (s < n_tiles)
+      issue_tile<BITS, KM, VM>(st0 + s * kStageBytes, sg, tb + s * TL::tokens,
+                               min(TL::tokens, te - tb - s * TL::tokens), tid);
+    cp_async_commit();
+  }
+
+  // Queries of this KV head's group (fp32, rows >= G zero), rotated for
+  // AKVQ-style coded keys, and their channel sums.
+  for (int i = tid; i < NT * 8 * kD; i += kThreads) q_s[i] = (i < G * kD) ? bf16_to_f32(qg[i]) : 0.f;
+  __syncthreads();
+  if (ROT) {
+    for (int j = warp; j < G; j += kWarps) {
+      float x[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) x[i] = q_s[j * kD + lane * 4 + i];
+      fwht128_warp(x, lane);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) q_s[j * kD + lane * 4 + i] = x[i];
+    }
+    __syncthreads();
+  }
+  for (int j = warp; j < NT * 8; j += kWarps) {
+    float sum = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) sum += q_s[j * kD + lane * 4 + i];
+    sum = warp_sum(sum);
+    if (lane == 0) zsum_s[j] = sum;
+  }
+  __syncthreads();
+
+  uint32_t qb[NT][8][2], ql[NT][8][2];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+    for (int j = 0; j < 8; ++j) qb[nt][j][0] = qb[nt][j][1] = ql[nt][j][0] = ql[nt][j][1] = 0u;
+  if (KM == K_BF16) qfrag_natural<NT>(qb, q_s, g, tq);
+  if (KM == K_TOKEN) qfrag_token<BITS, NT, ROT>(qb, ql, q_s, g, tq);
+
+  WarpState<NT, NZ> ws;
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      ws.m[nt][e] = -INFINITY;
+      ws.l[nt][e] = 0.f;
+#pragma unroll
+      for (int zz = 0; zz < NZ; ++zz) ws.z[nt][e][zz] = 0.f;
+    }
+#pragma unroll
+    for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ws.o[nt][mt][i] = 0.f;
+  }
+
+  for (int it = 0; it < n_tiles; ++it) {
+    cp_async_wait<kStages - 2>();
+    __syncthreads();
+    const int nx = it + kStages - 1;
+    if (nx < n_tiles)
+      issue_tile<BITS, KM, VM>(st0 + (nx % kStages) * kStageBytes, sg, tb + nx * TL::tokens,
+                               min(TL::tokens, te - tb - nx * TL::tokens), tid);
+    cp_async_commit();
+    compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + (it % kStages) * kStageBytes,
+                                        min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s,
+                                        zsum_s, scale_log2, warp, lane);
+  }
+  cp_async_wait<0>();
+  __syncthreads();  // stage buffers are reused for the reduction below
+
+  // ---- per-warp results: reduce l and the value-zero terms over the 8 rows g ----
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      float l = ws.l[nt][e];
+      l += __shfl_xor_sync(kFull, l, 4);
+      l += __shfl_xor_sync(kFull, l, 8);
+      l += __shfl_xor_sync(kFull, l, 16);
+#pragma unroll
+      for (int zz = 0; zz < NZ; ++zz) {
+        float z = ws.z[nt][e][zz];
+        z += __shfl_xor_sync(kFull, z, 4);
+        z += __shfl_xor_sync(kFull, z, 8);
+        z += __shfl_xor_sync(kFull, z, 16);
+        ws.z[nt][e][zz] = z;
+      }
+      const int q = nt * 8 + 2 * tq + e;
+      if (g == 0) {
+        red_m[warp * kMaxG + q] = ws.m[nt][e];
+        red_l[warp * kMaxG + q] = l;
+      }
+      float* orow = red_o + (warp * kMaxG + q) * kD;
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt) {
+        int c_lo, c_hi;  // channels of rows g and g+8 of m-tile mt
+        float zlo = 0.f, zhi = 0.f;
+        if (VM == V_TOKEN) {
+          c_lo = 16 * g + mt;
+          c_hi = 16 * g + 8 + mt;
+          zlo = zhi = ws.z[nt][e][0];
+        } else {
+          c_lo = 16 * mt + g;
+          c_hi = 16 * mt + 8 + g;
+          if (VM == V_KIVI) zlo = zhi = ws.z[nt][e][(mt >> 1) % NZ];
+        }
+        orow[c_lo] = ws.o[nt][mt][e] + zlo;
+        orow[c_hi] = ws.o[nt][mt][2 + e] + zhi;
+      }
+    }
+  }
+}
+
+template <int BITS, int NT, int BASE>
+__global__ void __launch_bounds__(kThreads, 2)
 decode_kernel(const __grid_constant__ DecodeParams p) {
-  extern __shared__ __align__(16) char smem[];
-  using S = Smem<MAXG>;
+  extern __shared__ __align__(128) char smem[];
   const Dims& d = p.d;
   const int li = blockIdx.y;
   const int ipr = p.items_per_row[li];
@@ -93,8 +741,8 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     if (r < ni) break;
     r -= ni;
   }
-  const LayerGeom g = layer_geom(d, mask);
-  const HeadGeom hd = head_geom(d, g, h);
+  const LayerGeom lg = layer_geom(d, mask);
+  const HeadGeom hd = head_geom(d, lg, h);
   const char* Lb = p.arena + p.lt.base[li];
   const int G = d.G;
   const bool coded = r >= nb;
@@ -106,238 +754,61 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     tb = (r - nb) * p.cq;
     te = min(tb + p.cq, d.nq);
   }
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  constexpr int W = kD * BITS / 32;  // code words per token
-
-  float* q_s = reinterpret_cast<float*>(smem + S::q_off);
-  float* qr_s = reinterpret_cast<float*>(smem + S::qr_off);
-  float* p_s = reinterpret_cast<float*>(smem + S::p_off) + warp * kTile * MAXG;
-  char* tile = smem + S::tile_off + warp * kWarpTileBytes;
-
-  // Queries of this KV head's group, as fp32.
+  const int tid = threadIdx.x;
   const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
-  for (int i = threadIdx.x; i < G * kD; i += kThreads) q_s[i] = bf16_to_f32(qg[i]);
-  const bool rot = coded && d.base == kAkvq && hd.cls == kQuantized;
-  __syncthreads();
-  if (rot) {
-    for (int j = warp; j < G; j += kWarps) {
-      float x[4];
-#pragma unroll
-      for (int i = 0; i < 4; ++i) x[i] = q_s[j * kD + lane * 4 + i];
-      fwht128_warp(x, lane);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) qr_s[j * kD + lane * 4 + i] = x[i];
-    }
-    __syncthreads();
-  }
-  const float* qk_s = rot ? qr_s : q_s;  // queries used against this item's keys
 
-  float m_run[MAXG], l_run[MAXG], o_acc[MAXG][4];
-#pragma unroll
-  for (int j = 0; j < MAXG; ++j) {
-    m_run[j] = -INFINITY;
-    l_run[j] = 0.f;
-#pragma unroll
-    for (int e = 0; e < 4; ++e) o_acc[j][e] = 0.f;
-  }
-
-  const bool k_bf16 = !coded || hd.cls == kKeysOnly;
-  const bool kivi_k = coded && !k_bf16 && d.base == kKivi;
-  const int vg = vgroups(d);
-  // Tile buffer of a warp: [0, 8704) BF16 key rows (pitch 272 B) or key codes
-  // (at 0, <= 2 KB) + key metadata (at 4096, <= 1 KB); [8704, 16896) BF16
-  // value rows or value codes (at 8704) + value metadata (at 8704 + 4096).
-  char* Ks = tile;
-  char* Vs = tile + kTile * kKRowHalves * 2;
-  uint32_t* Kcode = reinterpret_cast<uint32_t*>(tile);
-  float2* Kmeta = reinterpret_cast<float2*>(tile + 4096);
-  uint32_t* Vcode = reinterpret_cast<uint32_t*>(Vs);
-  float2* Vmeta = reinterpret_cast<float2*>(Vs + 4096);
-
-  const int n_tiles = (te - tb + kTile - 1) / kTile;
-  for (int tt = warp; tt < n_tiles; tt += kWarps) {
-    const int t0 = tb + tt * kTile;
-    const int nt = min(kTile, te - t0);
-    // ---- stage the tile ----
-    if (!coded) {
-      warp_copy_rows(Ks, kKRowHalves * 2, Lb + hd.kb + b * hd.kb_bs + (size_t)t0 * 256, nt, lane);
-      warp_copy_rows(Vs, kD * 2, Lb + hd.vb + b * hd.kb_bs + (size_t)t0 * 256, nt, lane);
-    } else {
-      if (k_bf16) {
-        warp_copy_rows(Ks, kKRowHalves * 2, Lb + hd.kimg + b * hd.kimg_bs + (size_t)t0 * 256, nt, lane);
-      } else if (kivi_k) {
-        const size_t grp = (size_t)t0 / kKiviGroup;
-        warp_copy16(Kcode, Lb + hd.kq + b * hd.kq_bs + grp * kD * BITS * 4, kD * BITS * 4, lane);
-        warp_copy16(Kmeta, Lb + hd.kqm + b * hd.kqm_bs + grp * kD * 8, kD * 8, lane);
-      } else {
-        warp_copy16(Kcode, Lb + hd.kq + b * hd.kq_bs + (size_t)t0 * W * 4, nt * W * 4, lane);
-        warp_copy8(Kmeta, Lb + hd.kqm + b * hd.kqm_bs + (size_t)t0 * 8, nt * 8, lane);
-      }
-      warp_copy16(Vcode, Lb + hd.vq + b * hd.vq_bs + (size_t)t0 * W * 4, nt * W * 4, lane);
-      warp_copy8(Vmeta, Lb + hd.vqm + b * hd.vqm_bs + (size_t)t0 * vg * 8, nt * vg * 8, lane);
-    }
-    __syncwarp();
-
-    // ---- scores: lane = token ----
-    float acc[MAXG];
-#pragma unroll
-    for (int j = 0; j < MAXG; ++j) acc[j] = 0.f;
-    if (lane < nt) {
-      if (k_bf16) {
-        const char* krow = Ks + lane * kKRowHalves * 2;
-#pragma unroll 2
-        for (int c8 = 0; c8 < 16; ++c8) {
-          const uint4 w = *reinterpret_cast<const uint4*>(krow + c8 * 16);
-          float k[8];
-          bf16x2_to_f32(w.x, k[0], k[1]);
-          bf16x2_to_f32(w.y, k[2], k[3]);
-          bf16x2_to_f32(w.z, k[4], k[5]);
-          bf16x2_to_f32(w.w, k[6], k[7]);
-#pragma unroll
-          for (int j = 0; j < MAXG; ++j) {
-            if (j < G) {
-              const float4 qa = *reinterpret_cast<const float4*>(qk_s + j * kD + c8 * 8);
-              const float4 qb = *reinterpret_cast<const float4*>(qk_s + j * kD + c8 * 8 + 4);
-              float a = acc[j];
-              a = fmaf(qa.x, k[0], a); a = fmaf(qa.y, k[1], a);
-              a = fmaf(qa.z, k[2], a); a = fmaf(qa.w, k[3], a);
-              a = fmaf(qb.x, k[4], a); a = fmaf(qb.y, k[5], a);
-              a = fmaf(qb.z, k[6], a); a = fmaf(qb.w, k[7], a);
-              acc[j] = a;
-            }
-          }
-        }
-      } else if (kivi_k) {
-        // lane = token e of the 32-token group; channel c has its own (scale, zero)
-        constexpr int per = 32 / BITS;
-        const int e = lane;
-#pragma unroll 4
-        for (int c = 0; c < kD; ++c) {
-          const uint32_t word = Kcode[c * BITS + e / per];
-          const uint32_t code = (word >> (BITS * (e % per))) & ((1u << BITS) - 1u);
-          const float2 m = Kmeta[c];
-          const float x = dequant1(code, m.x, m.y);
-#pragma unroll
-          for (int j = 0; j < MAXG; ++j)
-            if (j < G) acc[j] = fmaf(qk_s[j * kD + c], x, acc[j]);
-        }
-      } else {
-        const uint32_t* crow = Kcode + lane * W;
-        const float2 m = Kmeta[lane];
-#pragma unroll 4
-        for (int c4 = 0; c4 < kD / 4; ++c4) {
-          uint32_t cc[4];
-          codes4<BITS>(crow, c4, cc);
-          float x[4];
-#pragma unroll
-          for (int i = 0; i < 4; ++i) x[i] = dequant1(cc[i], m.x, m.y);
-#pragma unroll
-          for (int j = 0; j < MAXG; ++j) {
-            if (j < G) {
-              const float4 qa = *reinterpret_cast<const float4*>(qk_s + j * kD + c4 * 4);
-              float a = acc[j];
-              a = fmaf(qa.x, x[0], a); a = fmaf(qa.y, x[1], a);
-              a = fmaf(qa.z, x[2], a); a = fmaf(qa.w, x[3], a);
-              acc[j] = a;
-            }
-          }
-        }
-      }
-    }
-
-    // ---- online softmax (log2 domain) ----
-#pragma unroll
-    for (int j = 0; j < MAXG; ++j) {
-      if (j < G) {
-        const float s = (lane < nt) ? acc[j] * p.scale_log2 : -INFINITY;
-        const float mt = warp_max(s);
-        const float mnew = fmaxf(m_run[j], mt);
-        const float alpha = exp2f(m_run[j] - mnew);
-        const float pj = exp2f(s - mnew);
-        l_run[j] = l_run[j] * alpha + pj;
-#pragma unroll
-        for (int e = 0; e < 4; ++e) o_acc[j][e] *= alpha;
-        m_run[j] = mnew;
-        p_s[lane * MAXG + j] = pj;
-      }
-    }
-    __syncwarp();
-
-    // ---- P.V: lane = channels 4*lane .. 4*lane+3 ----
-    for (int i = 0; i < nt; ++i) {
-      float v[4];
-      if (!coded) {
-        const uint2 w = *reinterpret_cast<const uint2*>(Vs + i * kD * 2 + lane * 8);
-        bf16x2_to_f32(w.x, v[0], v[1]);
-        bf16x2_to_f32(w.y, v[2], v[3]);
-      } else {
-        uint32_t cc[4];
-        codes4<BITS>(Vcode + i * W, lane, cc);
-        const float2 m = Vmeta[i * vg + (vg > 1 ? (lane >> 3) : 0)];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) v[e] = dequant1(cc[e], m.x, m.y);
-      }
-#pragma unroll
-      for (int j = 0; j < MAXG; ++j) {
-        if (j < G) {
-          const float pj = p_s[i * MAXG + j];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) o_acc[j][e] = fmaf(pj, v[e], o_acc[j][e]);
-        }
-      }
-    }
-    __syncwarp();
-  }
-
-  // ---- combine the warps of this CTA ----
-  __syncthreads();  // every warp is done with its tile buffers
-  float* red_m = reinterpret_cast<float*>(smem + S::tile_off);  // [warps][MAXG]
-  float* red_l = red_m + kWarps * MAXG;                          // [warps][MAXG]
-  float* red_o = red_l + kWarps * MAXG;                          // [warps][MAXG][128]
-#pragma unroll
-  for (int j = 0; j < MAXG; ++j) {
-    if (j < G) {
-      const float lt = warp_sum(l_run[j]);
-      if (lane == 0) {
-        red_m[warp * MAXG + j] = m_run[j];
-        red_l[warp * MAXG + j] = lt;
-      }
-#pragma unroll
-      for (int e = 0; e < 4; ++e) red_o[(warp * MAXG + j) * kD + lane * 4 + e] = o_acc[j][e];
-    }
+  float* red_m = reinterpret_cast<float*>(smem + kStageOff);  // [warps][16]
+  float* red_l = red_m + kWarps * kMaxG;                        // [warps][16]
+  float* red_o = red_l + kWarps * kMaxG;                        // [warps][16][128]
+  Seg sg;
+  sg.k = sg.v = sg.kc = sg.km = sg.vc = sg.vm = nullptr;
+  if (!coded) {
+    sg.k = Lb + hd.kb + b * hd.kb_bs;
+    sg.v = Lb + hd.vb + b * hd.kb_bs;
+    run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+  } else if (hd.cls == kKeysOnly) {
+    sg.k = Lb + hd.kimg + b * hd.kimg_bs;
+    sg.vc = Lb + hd.vq + b * hd.vq_bs;
+    sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
+    if (BASE == kKivi)
+      run_item<BITS, NT, K_BF16, V_KIVI, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+    else
+      run_item<BITS, NT, K_BF16, V_TOKEN, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+  } else {
+    sg.kc = Lb + hd.kq + b * hd.kq_bs;
+    sg.km = Lb + hd.kqm + b * hd.kqm_bs;
+    sg.vc = Lb + hd.vq + b * hd.vq_bs;
+    sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
+    if (BASE == kKivi)
+      run_item<BITS, NT, K_KIVI, V_KIVI, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+    else if (BASE == kAkvq)
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, true>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+    else
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
   }
   __syncthreads();
 
-  const int c = threadIdx.x;  // channel
+  // ---- combine the warps: thread = channel ----
+  const int c = tid;
   const size_t out_row = ((size_t)li * d.B + b) * d.Hq + (size_t)h * G;
-  if (ni == 1) {
-    for (int j = 0; j < G; ++j) {
-      float M = -INFINITY;
-      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * MAXG + j]);
-      float O = 0.f, Ls = 0.f;
-      for (int w = 0; w < kWarps; ++w) {
-        const float f = exp2f(red_m[w * MAXG + j] - M);
-        O += f * red_o[(w * MAXG + j) * kD + c];
-        Ls += f * red_l[w * MAXG + j];
-      }
-      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / Ls);
-    }
-    return;
-  }
-
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
   float* part = p.partials + (head_lin * p.max_items) * (size_t)G * kPartialStride;
-  {
-    float* mine = part + (size_t)r * G * kPartialStride;
-    for (int j = 0; j < G; ++j) {
-      float M = -INFINITY;
-      for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * MAXG + j]);
-      float O = 0.f, Ls = 0.f;
-      for (int w = 0; w < kWarps; ++w) {
-        const float f = exp2f(red_m[w * MAXG + j] - M);
-        O += f * red_o[(w * MAXG + j) * kD + c];
-        Ls += f * red_l[w * MAXG + j];
-      }
+  float* mine = part + (size_t)r * G * kPartialStride;
+  for (int j = 0; j < G; ++j) {
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * kMaxG + j]);
+    float O = 0.f, Ls = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const float mw = red_m[w * kMaxG + j];
+      const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
+      O += f * red_o[(w * kMaxG + j) * kD + c];
+      Ls += f * red_l[w * kMaxG + j];
+    }
+    if (ni == 1) {
+      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / Ls);
+    } else {
       mine[j * kPartialStride + 2 + c] = O;
       if (c == 0) {
         mine[j * kPartialStride + 0] = M;
@@ -345,10 +816,12 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
       }
     }
   }
+  if (ni == 1) return;
+
   __threadfence();
   __syncthreads();
   __shared__ int s_last;
-  if (threadIdx.x == 0) {
+  if (tid == 0) {
     const unsigned prev = atomicAdd(p.counters + head_lin, 1u);
     s_last = (prev == (unsigned)(ni - 1));
   }
@@ -362,46 +835,47 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     float O = 0.f, Ls = 0.f;
     for (int sidx = 0; sidx < ni; ++sidx) {
       const float* ps = part + ((size_t)sidx * G + j) * kPartialStride;
-      const float f = exp2f(__ldcg(ps) - M);
+      const float ms = __ldcg(ps);
+      const float f = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
       O += f * __ldcg(ps + 2 + c);
       Ls += f * __ldcg(ps + 1);
     }
     p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / Ls);
   }
-  if (threadIdx.x == 0) atomicExch(p.counters + head_lin, 0u);
+  if (tid == 0) atomicExch(p.counters + head_lin, 0u);
 }
 
-template <int MAXG, int BITS>
-cudaError_t launch_decode_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
-  constexpr int smem = Smem<MAXG>::bytes;
+template <int BITS, int NT, int BASE>
+cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
   static bool configured[64] = {};
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
   if (dev < 64 && !configured[dev]) {
-    e = cudaFuncSetAttribute(decode_kernel<MAXG, BITS>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             kSmemBytes);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   dim3 grid(grid_x, p.n_layers, 1);
-  decode_kernel<MAXG, BITS><<<grid, kThreads, smem, s>>>(p);
+  decode_kernel<BITS, NT, BASE><<<grid, kThreads, kSmemBytes, s>>>(p);
   return cudaGetLastError();
 }
 
-template <int BITS>
-cudaError_t launch_decode_bits(const DecodeParams& p, int grid_x, cudaStream_t s) {
-  const int G = p.d.G;
-  if (G <= 1) return launch_decode_t<1, BITS>(p, grid_x, s);
-  if (G <= 2) return launch_decode_t<2, BITS>(p, grid_x, s);
-  if (G <= 4) return launch_decode_t<4, BITS>(p, grid_x, s);
-  if (G <= 8) return launch_decode_t<8, BITS>(p, grid_x, s);
-  return launch_decode_t<16, BITS>(p, grid_x, s);
+template <int BITS, int NT>
+cudaError_t launch_base(const DecodeParams& p, int grid_x, cudaStream_t s) {
+  switch (p.d.base) {
+    case kKivi: return launch_t<BITS, NT, kKivi>(p, grid_x, s);
+    case kAkvq: return launch_t<BITS, NT, kAkvq>(p, grid_x, s);
+    default: return launch_t<BITS, NT, kMinMax>(p, grid_x, s);
+  }
 }
 
 }  // namespace
 
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s) {
-  return p.d.bits == 2 ? launch_decode_bits<2>(p, grid_x, s) : launch_decode_bits<4>(p, grid_x, s);
+  if (p.d.bits == 2) return p.d.G <= 8 ? launch_base<2, 1>(p, grid_x, s) : launch_base<2, 2>(p, grid_x, s);
+  return p.d.G <= 8 ? launch_base<4, 1>(p, grid_x, s) : launch_base<4, 2>(p, grid_x, s);
 }
 
 }  // namespace hg

@@ -54,12 +54,19 @@ HG_HD int quantized_count(int T, int s, int n, int base, int residual) {
 
 // Bytes per token of one head's packed codes (128 codes).
 HG_HD uint64_t code_bytes_per_token(const Dims& d) { return (uint64_t)kD * d.bits / 8; }
-// Key metadata bytes for nq tokens of one batch row of one head.
+HG_HD uint64_t align16(uint64_t x) { return (x + 15) & ~15ull; }
+// Key metadata bytes for nq tokens of one batch row of one head (payload).
 HG_HD uint64_t kmeta_bytes(const Dims& d) {
   return d.base == kKivi ? (uint64_t)(d.nq / kKiviGroup) * kD * 8 : (uint64_t)d.nq * 8;
 }
 // Value metadata groups per token.
 HG_HD int vgroups(const Dims& d) { return d.base == kKivi ? kD / kKiviGroup : 1; }
+HG_HD uint64_t vmeta_bytes(const Dims& d) { return (uint64_t)d.nq * vgroups(d) * 8; }
+// Batch-row strides of the metadata arrays: padded to 16 bytes so that every
+// row (and every head's block of rows) starts on a 16-byte boundary, as the
+// 16-byte asynchronous copies of the decode kernel require.
+HG_HD uint64_t kmeta_stride(const Dims& d) { return align16(kmeta_bytes(d)); }
+HG_HD uint64_t vmeta_stride(const Dims& d) { return align16(vmeta_bytes(d)); }
 
 struct LayerGeom {
   uint64_t mask;
@@ -85,9 +92,9 @@ HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
   g.kb = off; off += g.bf16_bytes;
   g.vb = off; off += g.bf16_bytes;
   g.kq = off; off += align_up((uint64_t)g.n_U * B * nq * code_bytes_per_token(d));
-  g.kqm = off; off += align_up((uint64_t)g.n_U * B * kmeta_bytes(d));
+  g.kqm = off; off += align_up((uint64_t)g.n_U * B * kmeta_stride(d));
   g.vq = off; off += align_up((uint64_t)g.n_VQ * B * nq * code_bytes_per_token(d));
-  g.vqm = off; off += align_up((uint64_t)g.n_VQ * B * nq * vgroups(d) * 8);
+  g.vqm = off; off += align_up((uint64_t)g.n_VQ * B * vmeta_stride(d));
   g.kimg = off; off += align_up((uint64_t)g.n_PK * B * nq * kD * 2);
   g.size = off;
   return g;
@@ -122,9 +129,9 @@ HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
   r.kb = g.kb + B * tok_before * kD * 2;
   r.vb = g.vb + B * tok_before * kD * 2;
   r.kq_bs = nq * code_bytes_per_token(d);
-  r.kqm_bs = kmeta_bytes(d);
+  r.kqm_bs = kmeta_stride(d);
   r.vq_bs = nq * code_bytes_per_token(d);
-  r.vqm_bs = nq * vgroups(d) * 8;
+  r.vqm_bs = vmeta_stride(d);
   r.kimg_bs = nq * kD * 2;
   r.kq = r.kqm = r.vq = r.vqm = r.kimg = kNone;
   if (r.cls == kQuantized) {

@@ -71,16 +71,11 @@ __device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGrou
   const float levels = (float)((1 << bits) - 1);
   scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   zero = mn;
+  const bool fast = scale >= 2.3509887e-38f;  // 2^-125
+  const float r = __frcp_rn(fast ? scale : 1.0f);
 #pragma unroll
-  for (int e = 0; e < kKiviGroup; ++e) {
-    if (scale == 0.0f) {
-      code[e] = 0u;
-    } else {
-      float r = rintf(__fdiv_rn(__fsub_rn(x[e], mn), scale));
-      r = fminf(fmaxf(r, 0.0f), levels);
-      code[e] = (uint32_t)r;
-    }
-  }
+  for (int e = 0; e < kKiviGroup; ++e)
+    code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], mn), scale, r, levels, fast);
 }
 
 __global__ void __launch_bounds__(kThreads)

@@ -61,12 +61,12 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
             assert np.array_equal(vb, v_bits[b, h, toks]), (layer, h, b, "vb")
             if cls == hg.HG_HEAD_QUANTIZED and nq:
                 kw = _slice(arena, r.kq + b * r.kq_bstride, nq * W * 4, np.uint32)
-                km = _slice(arena, r.kqm + b * r.kqm_bstride, r.kqm_bstride, np.uint32)
+                km = _slice(arena, r.kqm + b * r.kqm_bstride, o["k_meta"][b, h].nbytes, np.uint32)
                 assert np.array_equal(kw, o["k_words"][b, h]), (layer, h, b, "kq")
                 assert np.array_equal(km, o["k_meta"][b, h].view(np.uint32)), (layer, h, b, "kqm")
             if cls != hg.HG_HEAD_PROTECTED and nq:
                 vw = _slice(arena, r.vq + b * r.vq_bstride, nq * W * 4, np.uint32)
-                vm = _slice(arena, r.vqm + b * r.vqm_bstride, r.vqm_bstride, np.uint32)
+                vm = _slice(arena, r.vqm + b * r.vqm_bstride, o["v_meta"][b, h].nbytes, np.uint32)
                 assert np.array_equal(vw, o["v_words"][b, h]), (layer, h, b, "vq")
                 assert np.array_equal(vm, o["v_meta"][b, h].view(np.uint32)), (layer, h, b, "vqm")
             if cls == hg.HG_HEAD_KEYS_ONLY and nq:

@@ -93,9 +93,14 @@ def test_create_checks_arena(lib):
     assert e.value.status == 2
 
 
-@pytest.mark.parametrize("name", list(wl.WORKLOADS))
+ODD = {"odd_nq_minmax": wl.custom("odd", 3, 3, 16, 4, 64, 333, 17, wl.BASE_MINMAX, 4, 0),
+       "odd_nq_konly": wl.custom("odd2", 2, 5, 8, 8, 7, 77, 3, wl.BASE_AKVQ, 2, 1),
+       "kivi_odd_rows": wl.custom("odd3", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 2, 1)}
+
+
+@pytest.mark.parametrize("name", list(wl.WORKLOADS) + list(ODD))
 def test_regions_tile_the_arena_without_overlap(lib, name):
-    w = wl.WORKLOADS[name]
+    w = wl.WORKLOADS[name] if name in wl.WORKLOADS else ODD[name]
     cache, n, mask = _fake_cache(w)
     base = 1 << 40
     spans = []
@@ -117,9 +122,12 @@ def test_regions_tile_the_arena_without_overlap(lib, name):
                 spans.append((r.vqm, B * r.vqm_bstride))
             if r.kimg != hg.NONE_OFFSET:
                 spans.append((r.kimg, B * r.kimg_bstride))
-            for off in (r.kb, r.vb, r.kq, r.vq, r.kimg):
+            for off in (r.kb, r.vb, r.kq, r.kqm, r.vq, r.vqm, r.kimg):
                 if off != hg.NONE_OFFSET:
                     assert off % 16 == 0
+            for st in (r.kb_bstride, r.kq_bstride, r.kqm_bstride, r.vq_bstride, r.vqm_bstride,
+                       r.kimg_bstride):
+                assert st % 16 == 0
     spans = sorted(s for s in spans if s[1] > 0)
     for (a, la), (b, _) in zip(spans, spans[1:]):
         assert a + la <= b, (a, la, b)
