@@ -17,9 +17,11 @@
  *
  * Conventions shared by every entry point
  *   Memory     The caller owns every byte.  The library never allocates device
- *              memory; the cache lives in a caller-provided device "arena",
- *              and decode attention uses a caller-provided workspace.  The
- *              only host allocation is the hg_cache descriptor itself.
+ *              memory at run time; the cache lives in a caller-provided device
+ *              "arena", and decode attention uses a caller-provided workspace
+ *              (hg_decode_attention_noalloc instead uses a static 32 MiB array
+ *              the library holds on every GPU that loads it).  The only host
+ *              allocation is the hg_cache descriptor itself.
  *   Tensors    Device tensors are dense row-major BF16 (uint16 bit patterns)
  *              unless stated otherwise, head_dim = 128, and must be 16-byte
  *              aligned.
@@ -203,6 +205,29 @@ hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
 hg_status hg_decode_attention(const hg_cache *cache, int32_t layer_begin, int32_t layer_count,
                               const void *q, void *out, float softmax_scale,
                               void *workspace, size_t workspace_bytes, hg_stream_t stream);
+
+/* Decode attention that allocates nothing: the same computation and arguments
+ * as hg_decode_attention, minus the workspace.  For callers that may not
+ * allocate device memory themselves -- an operator inside an inference
+ * runtime whose plugin interface hands over only inputs and outputs, code
+ * running while another framework owns the whole device memory pool, or a
+ * decode loop that cannot afford cudaMalloc's implicit device
+ * synchronisation.  (This entry point has no counterpart in the paper.)
+ *   Scratch   the split-K workspace is one static device array of 32 MiB
+ *             inside this library; every GPU that loads the library holds it
+ *             until the process exits.  A launch whose workspace
+ *             (hg_decode_workspace_size) exceeds 32 MiB is rejected with
+ *             HG_ERR_WORKSPACE_TOO_SMALL before anything is enqueued.
+ *   Set-up    the first call on a device (with that device current) looks up
+ *             the array's device address with cudaGetSymbolAddress; make that
+ *             first call before any stream capture.
+ *   Sharing   every call uses the same array and clears the part it needs
+ *             (cudaMemsetAsync) before launching; calls that overlap on the
+ *             GPU (different streams, or threads on the same device) race.
+ * No cudaMalloc, cudaFree or other allocating routine is called. */
+hg_status hg_decode_attention_noalloc(const hg_cache *cache, int32_t layer_begin,
+                                      int32_t layer_count, const void *q, void *out,
+                                      float softmax_scale, hg_stream_t stream);
 
 /* Sec. 5.4 storage accounting of the arena's image-token regions: bits per
  * image K/V element actually stored (codes + 64-bit metadata + BF16 entries). */

@@ -19,7 +19,8 @@ __all__ = [
     "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
     "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
     "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_decode_attention",
-    "hg_cache_image_bits_per_elem", "hg_status_string", "library", "library_path",
+    "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem", "hg_status_string",
+    "library", "library_path",
 ]
 
 HG_BASE_MINMAX_TOKEN = 0
@@ -96,6 +97,7 @@ def library():
         "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
         "hg_workspace_clear": ([P, sz, P], st),
         "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
+        "hg_decode_attention_noalloc": ([P, i32, i32, P, P, ctypes.c_float, P], st),
         "hg_cache_image_bits_per_elem": ([P, ctypes.POINTER(ctypes.c_double)], st),
         "hg_status_string": ([st], ctypes.c_char_p),
     }
@@ -238,6 +240,14 @@ def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, 
                                          _ptr(out), float(softmax_scale), _ptr(workspace),
                                          workspace_bytes, _stream(stream)),
            "hg_decode_attention")
+
+
+def hg_decode_attention_noalloc(cache, layer_begin, layer_count, q, out, softmax_scale,
+                                stream=None):
+    """Decode attention with the library's static 32 MiB scratch as workspace (no allocation)."""
+    _check(library().hg_decode_attention_noalloc(cache.handle, layer_begin, layer_count, _ptr(q),
+                                                 _ptr(out), float(softmax_scale), _stream(stream)),
+           "hg_decode_attention_noalloc")
 
 
 def hg_cache_image_bits_per_elem(cache):
