@@ -5,8 +5,9 @@ One step = the whole path over one synthetic cache: quantize-pack every layer
 from its BF16 prefill (one launch per 64 layers), then `decode_steps` decode
 steps, each appending one token per (layer, row, KV head) and running decode
 attention over all layers (one launch each).  Inputs are resident in HBM when
-timing starts; L2 is flushed (a 512 MiB write) before every timed launch
-group, and every group is timed with CUDA events on the launching stream.
+timing starts; L2 is flushed (a 512 MiB write, then a read of it so the
+evicted lines are clean) before every timed launch group, and every group is
+timed with CUDA events on the launching stream.
 
 value     = algorithmic bytes of a step / summed device time of the step (GB/s)
 roofline  = decode attention (the dominant kernel): its algorithmic bytes per
@@ -341,10 +342,11 @@ def run_gpu(args):
     sigma = 0.0
     quant_b, dec_b, app_b = geometry_bytes(runner)
     step_bytes = quant_b + sum(dec_b) + S * app_b
-    launches_per_step = (L + 63) // 64 + S * 2 * ((L + 63) // 64)
+    launches_per_step = (L + 63) // 64 + S * ((L + 63) // 64)
 
     def cushion():
-        flush.zero_()
+        flush.zero_()            # evict L2 (write a buffer larger than L2) ...
+        flush.sum()              # ... and read it back so the evicted lines are clean
         torch.cuda._sleep(200000)  # keep the stream busy while the host enqueues the group
 
     def one_step(record):
@@ -357,17 +359,15 @@ def run_gpu(args):
             hg.hg_quantize_kv(runner.cache, l0, ks[l0:l0 + n], vs[l0:l0 + n], stream)
         e1.record(stream)
         ev.append(("quant", e0, e1))
+        hg.hg_cache_reset_appended(runner.cache)
         for s in range(S):
             cushion()
-            a0, a1, a2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            a0, a1 = (torch.cuda.Event(enable_timing=True) for _ in range(2))
             a0.record(stream)
-            hg.hg_append_kv(runner.cache, 0, L, news[s][0], news[s][1], stream)
+            hg.hg_decode_step(runner.cache, 0, L, qs[s], news[s][0], news[s][1], out, sigma,
+                              runner.ws, runner.ws_bytes, stream)
             a1.record(stream)
-            hg.hg_decode_attention(runner.cache, 0, L, qs[s], out, sigma, runner.ws,
-                                   runner.ws_bytes, stream)
-            a2.record(stream)
-            ev.append(("append", a0, a1))
-            ev.append(("decode", a1, a2))
+            ev.append(("decode", a0, a1))
         if record is not None:
             record.append(ev)
 
@@ -388,7 +388,7 @@ def run_gpu(args):
         dist.barrier()
     torch.cuda.synchronize()
 
-    per = {"quant": [], "append": [], "decode": []}
+    per = {"quant": [], "decode": []}
     step_ms = []
     for ev in records:
         tot = 0.0
@@ -406,9 +406,8 @@ def run_gpu(args):
 
     quant_ms = statistics.mean(per["quant"])
     dec_ms = statistics.mean(per["decode"])
-    app_ms = statistics.mean(per["append"])
-    dec_bytes_mean = sum(dec_b) / S
-    tok_s = world * w.batch * S / ((sum(per["decode"]) + sum(per["append"])) / args.steps * 1e-3)
+    dec_bytes_mean = (sum(dec_b) + S * app_b) / S
+    tok_s = world * w.batch * S / (sum(per["decode"]) / args.steps * 1e-3)
 
     peaks, peak_src = measured_peaks()
     peak = float(peaks.get("hbm_gbs", FALLBACK_HBM_GBS))
@@ -430,21 +429,23 @@ def run_gpu(args):
                                                                w.text_suffix),
                    "base": ["minmax", "kivi", "akvq"][w.base], "bits": w.bits,
                    "keys_only": w.keys_only, "protected_heads": int(runner.mask.sum()),
-                   "decode_steps": S, "l2": "flushed (512 MiB write) before every timed launch group",
-                   "launch": "quantize: all layers per launch; decode: append + attention over all layers per step"},
+                   "decode_steps": S, "l2": "flushed (512 MiB write + read) before every timed launch group",
+                   "launch": "quantize: all layers per launch; each decode step: one launch appending the "
+                             "new K/V and attending over all layers"},
         "pct_of_8TBps": round(100 * value / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_hbm": round(100 * value / peak, 2),
         "decode_tokens_per_s": round(tok_s, 1),
         "kernels": {
             "quantize": {"ms": round(quant_ms, 4), "GBps": round(quant_b / quant_ms / 1e6, 1)},
-            "decode_attention": {"ms": round(dec_ms, 4), "GBps": round(achieved, 1)},
-            "append": {"ms": round(app_ms, 4), "GBps": round(app_b / app_ms / 1e6, 1)},
+            "decode_step (append + attention, one launch)": {"ms": round(dec_ms, 4),
+                                                               "GBps": round(achieved, 1)},
         },
         "step_bytes": step_bytes,
         "wall_s_timed_region": round(t_wall, 4),
         "roofline": {"bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
                      "frac": round(achieved / peak, 4), "traffic": traffic,
-                     "kernel": "decode_attention", "peak_source": peak_src + " hbm_gbs (burst copy)"},
+                     "kernel": "decode_kernel (hg_decode_step)",
+                     "peak_source": peak_src + " hbm_gbs (burst copy)"},
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
     }
@@ -496,9 +497,8 @@ def run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream):
             dq.copy_(hq[s], non_blocking=True)
             dkn.copy_(hkn[s], non_blocking=True)
             dvn.copy_(hvn[s], non_blocking=True)
-            hg.hg_append_kv(runner.cache, 0, L, dkn, dvn, stream)
-            hg.hg_decode_attention(runner.cache, 0, L, dq, dout, 0.0, runner.ws, runner.ws_bytes,
-                                   stream)
+            hg.hg_decode_step(runner.cache, 0, L, dq, dkn, dvn, dout, 0.0, runner.ws, runner.ws_bytes,
+                              stream)
             hout[s].copy_(dout, non_blocking=True)
 
     for _ in range(max(1, args.warmup)):

@@ -206,6 +206,18 @@ hg_status hg_decode_attention(const hg_cache *cache, int32_t layer_begin, int32_
                               const void *q, void *out, float softmax_scale,
                               void *workspace, size_t workspace_bytes, hg_stream_t stream);
 
+/* One decode step in one launch: append the step's K/V (as hg_append_kv) and
+ * run grouped-query decode attention over every token including the new one
+ * (as hg_decode_attention).  k_new / v_new: device BF16
+ * [layer_count][batch][num_kv_heads][128]; the other arguments as for
+ * hg_decode_attention.  The work item that holds the new position reads it
+ * from k_new / v_new and also stores it into the cache.  Returns
+ * HG_ERR_CAPACITY if a layer already holds max_new_tokens appended tokens;
+ * advances the host-side count on success. */
+hg_status hg_decode_step(hg_cache *cache, int32_t layer_begin, int32_t layer_count, const void *q,
+                         const void *k_new, const void *v_new, void *out, float softmax_scale,
+                         void *workspace, size_t workspace_bytes, hg_stream_t stream);
+
 /* Decode attention that allocates nothing: the same computation and arguments
  * as hg_decode_attention, minus the workspace.  For callers that may not
  * allocate device memory themselves -- an operator inside an inference

@@ -19,7 +19,8 @@ __all__ = [
     "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
     "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
     "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_decode_attention",
-    "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem", "hg_status_string",
+    "hg_decode_step", "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem",
+    "hg_status_string",
     "library", "library_path",
 ]
 
@@ -97,6 +98,7 @@ def library():
         "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
         "hg_workspace_clear": ([P, sz, P], st),
         "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
+        "hg_decode_step": ([P, i32, i32, P, P, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_attention_noalloc": ([P, i32, i32, P, P, ctypes.c_float, P], st),
         "hg_cache_image_bits_per_elem": ([P, ctypes.POINTER(ctypes.c_double)], st),
         "hg_status_string": ([st], ctypes.c_char_p),
@@ -240,6 +242,16 @@ def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, 
                                          _ptr(out), float(softmax_scale), _ptr(workspace),
                                          workspace_bytes, _stream(stream)),
            "hg_decode_attention")
+
+
+def hg_decode_step(cache, layer_begin, layer_count, q, k_new, v_new, out, softmax_scale, workspace,
+                   workspace_bytes=None, stream=None):
+    """Append the step's K/V and run decode attention including it, in one launch."""
+    if workspace_bytes is None:
+        workspace_bytes = workspace.numel() * workspace.element_size()
+    _check(library().hg_decode_step(cache.handle, layer_begin, layer_count, _ptr(q), _ptr(k_new),
+                                    _ptr(v_new), _ptr(out), float(softmax_scale), _ptr(workspace),
+                                    workspace_bytes, _stream(stream)), "hg_decode_step")
 
 
 def hg_decode_attention_noalloc(cache, layer_begin, layer_count, q, out, softmax_scale,

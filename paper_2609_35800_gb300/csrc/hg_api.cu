@@ -31,7 +31,6 @@ struct hg_cache {
 
 namespace {
 
-constexpr int kTargetItems = 1024;  // decode work items per launch (~6.7 per SM on 152 SMs)
 
 bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -117,21 +116,97 @@ bool range_ok(const hg_cache* c, int32_t begin, int32_t count) {
   return c && count >= 1 && begin >= 0 && (int64_t)begin + count <= c->d.L;
 }
 
-// Chunk scale k: BF16 chunks of 128k tokens, coded chunks of 512k tokens.
-// The largest k that still gives kTargetItems items (appended = 0) wins.
-int chunk_scale(const hg_cache* c, int begin, int count) {
-  const Dims& d = c->d;
-  for (int k = 32; k > 1; k >>= 1) {
-    int64_t items = 0;
-    for (int l = begin; l < begin + count; ++l)
-      items += (int64_t)d.B * layer_items_per_row(d, c->layer_mask[l], 0, 128 * k, 512 * k);
-    if (items >= kTargetItems) return k;
-  }
-  return 1;
+// Decode work plan.  Chunk sizes are chosen so that a launch has about
+// kTargetItems work items of similar byte size: three resident CTAs on each of
+// the 152 SMs, i.e. one wave.  Chunk sizes are multiples of the kernel's tile
+// (64 tokens for BF16 rows, the coded tile for codes) and depend only on the
+// layer range, so the workspace bound holds for every appended count.
+constexpr int kTargetItems = 3 * 152;
+
+int round_up_to(int x, int g) { return ((x + g - 1) / g) * g; }
+
+// Split a segment of len tokens of bpt bytes each into pieces of about
+// item_bytes; returns the chunk size in tokens (a multiple of granule).
+int chunk_tokens(int len, double bpt, double item_bytes, int granule) {
+  if (len <= 0) return granule;
+  long long n = (long long)(len * bpt / item_bytes + 0.5);
+  if (n < 1) n = 1;
+  const int per = (int)((len + n - 1) / n);
+  return round_up_to(per < 1 ? 1 : per, granule);
 }
 
-size_t ws_size_for(const hg_cache* c, int count, int k) {
-  return (size_t)ws_bytes(c->d, count, 128 * k, 512 * k);
+// Cost per token of each segment kind, in byte-equivalents: the bytes a chunk
+// streams plus about 8 bytes per warp-instruction its tokens cost (measured
+// instruction counts of the decode kernel: ~5 per BF16 token, ~10 / 13 per
+// 2 / 4-bit coded token, ~22 for KIVI-style keys, ~8 for keys-only heads).
+// Balancing cost rather than bytes keeps compute-heavy coded chunks short.
+struct SegBytes {
+  double bf16, coded_u, coded_k;
+};
+
+SegBytes seg_bytes(const Dims& d) {
+  SegBytes b;
+  const double codes = 16.0 * d.bits;  // 128 codes
+  const double kmeta = d.base == kKivi ? 32.0 : 8.0;
+  const double vmeta = 8.0 * vgroups(d);
+  const double instr_u = d.base == kKivi ? (d.bits == 2 ? 22.0 : 26.0) : (d.bits == 2 ? 10.0 : 13.5);
+  b.bf16 = 512.0 + 8.0 * 5.0;
+  b.coded_u = 2.0 * codes + kmeta + vmeta + 8.0 * instr_u;
+  b.coded_k = 256.0 + codes + vmeta + 8.0 * 8.0;
+  return b;
+}
+
+int max_items_of(const Dims& d, const DecodePlan& p);
+
+DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
+  const Dims& d = c->d;
+  const SegBytes sb = seg_bytes(d);
+  double total = 0.0;
+  for (int l = begin; l < begin + count; ++l) {
+    for (int h = 0; h < d.H; ++h) {
+      const int cls = head_class(d, c->layer_mask[l], h);
+      if (cls == kProtected) {
+        total += d.T * sb.bf16;
+      } else {
+        total += (d.T - d.nq) * sb.bf16 + d.nq * (cls == kKeysOnly ? sb.coded_k : sb.coded_u);
+      }
+    }
+  }
+  total *= d.B;
+  double item = total / kTargetItems;
+  if (item < 16384.0) item = 16384.0;
+  const int tile = decode_coded_tile(d.bits);
+  DecodePlan p;
+  p.cbU = chunk_tokens(d.T - d.nq, sb.bf16, item, 64);
+  p.cqU = chunk_tokens(d.nq, sb.coded_u, item, tile);
+  p.cqK = chunk_tokens(d.nq, sb.coded_k, item, 64);
+  p.cbP = chunk_tokens(d.T, sb.bf16, item, 64);
+  // The merging CTA stages (m, l) of all splits of a head in the kernel's
+  // 8 KB query buffer: at most 2 * splits * G + 2 * G floats.
+  while ((long long)max_items_of(d, p) * d.G * 2 + 2LL * d.G > (long long)kMaxG * kD) {
+    p.cbU *= 2;
+    p.cqU *= 2;
+    p.cqK *= 2;
+    p.cbP *= 2;
+  }
+  return p;
+}
+
+ChunkCounts counts_of(const Dims& d, int appended, const DecodePlan& p) {
+  return chunk_counts(d, appended, p.cbU, p.cqU, p.cqK, p.cbP);
+}
+
+// Split slots per (layer, row, head): the most chunks any head can have.
+int max_items_of(const Dims& d, const DecodePlan& p) {
+  const ChunkCounts c = counts_of(d, d.S_new, p);
+  int nb, m = head_chunks(kQuantized, c, &nb);
+  const int prot = head_chunks(d.keys_only ? kKeysOnly : kProtected, c, &nb);
+  return m > prot ? m : prot;
+}
+
+size_t ws_size_for(const hg_cache* c, int begin, int count) {
+  const DecodePlan p = plan_decode(c, begin, count);
+  return (size_t)ws_bytes(c->d, count, max_items_of(c->d, p));
 }
 
 hg_status cuda_status(cudaError_t e) { return e == cudaSuccess ? HG_OK : HG_ERR_CUDA; }
@@ -315,11 +390,14 @@ hg_status hg_append_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count, co
 
 hg_status hg_decode_workspace_size(const hg_cache* c, int32_t layer_count, size_t* bytes) {
   if (!c || !bytes || layer_count < 1 || layer_count > c->d.L) return HG_ERR_INVALID_ARG;
-  // a launch over more than kMaxLayersPerLaunch layers reuses the workspace per group
-  const int per = std::min<int>(layer_count, kMaxLayersPerLaunch);
-  int kmin = 32;
-  for (int b = 0; b + per <= c->d.L; ++b) kmin = std::min(kmin, chunk_scale(c, b, per));
-  *bytes = ws_size_for(c, per, kmin);
+  // A launch over more than kMaxLayersPerLaunch layers reuses the workspace for
+  // each group of layers; the bound is the largest over every placement.
+  size_t need = 0;
+  for (int b = 0; b < c->d.L; ++b) {
+    const int n = std::min<int>(std::min<int>(layer_count, kMaxLayersPerLaunch), c->d.L - b);
+    need = std::max(need, ws_size_for(c, b, n));
+  }
+  *bytes = need;
   return HG_OK;
 }
 
@@ -328,49 +406,100 @@ hg_status hg_workspace_clear(void* ws, size_t bytes, hg_stream_t stream) {
   return cuda_status(cudaMemsetAsync(ws, 0, bytes, reinterpret_cast<cudaStream_t>(stream)));
 }
 
-hg_status hg_decode_attention(const hg_cache* c, int32_t layer_begin, int32_t layer_count,
-                              const void* q, void* out, float softmax_scale, void* ws,
-                              size_t ws_bytes_given, hg_stream_t stream) {
-  if (!range_ok(c, layer_begin, layer_count) || !q || !out || !ws) return HG_ERR_INVALID_ARG;
-  if (!aligned16(q) || !aligned16(out) || !aligned16(ws)) return HG_ERR_ALIGNMENT;
-  if (!(softmax_scale == softmax_scale)) return HG_ERR_INVALID_ARG;  // NaN
+}  // extern "C"
+
+namespace {
+
+// Decode attention over layers [layer_begin, +layer_count); with k_new / v_new
+// the step's new tokens (already counted in the cache's appended state) are
+// read from the inputs and stored into the arena by the same launch.
+hg_status decode_launch(const hg_cache* c, int32_t layer_begin, int32_t layer_count, const void* q,
+                        const void* k_new, const void* v_new, void* out, float softmax_scale,
+                        void* ws, size_t ws_bytes_given, hg_stream_t stream) {
   const Dims& d = c->d;
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)kD);
   const size_t layer_elems = (size_t)d.B * d.Hq * kD;
-  // validate every group before launching any
+  const size_t kv_elems = (size_t)d.B * d.H * kD;
   for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
     const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
-    const int k = chunk_scale(c, layer_begin + done, n);
-    if (ws_bytes_given < ws_size_for(c, n, k)) return HG_ERR_WORKSPACE_TOO_SMALL;
-  }
-  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
-    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
-    const int k = chunk_scale(c, layer_begin + done, n);
     DecodeParams p;
     std::memset(&p, 0, sizeof p);
     p.d = d;
     p.arena = c->arena;
     p.n_layers = n;
-    p.cb = 128 * k;
-    p.cq = 512 * k;
-    p.max_items = max_head_items(d, p.cb, p.cq);
+    p.plan = plan_decode(c, layer_begin + done, n);
+    p.max_items = max_items_of(d, p.plan);
     p.scale_log2 = scale * 1.4426950408889634f;
     p.q = static_cast<const uint16_t*>(q) + (size_t)done * layer_elems;
     p.out = static_cast<uint16_t*>(out) + (size_t)done * layer_elems;
+    if (k_new) {
+      p.k_new = static_cast<const uint16_t*>(k_new) + (size_t)done * kv_elems;
+      p.v_new = static_cast<const uint16_t*>(v_new) + (size_t)done * kv_elems;
+    }
     p.counters = static_cast<uint32_t*>(ws);
     p.partials = reinterpret_cast<float*>(static_cast<char*>(ws) + ws_counter_bytes(d, n));
     fill_table(c, layer_begin + done, n, &p.lt);
-    int grid_x = 0;
+    int total = 0;
     for (int i = 0; i < n; ++i) {
       const int l = layer_begin + done + i;
-      p.appended[i] = c->appended[l];
-      p.items_per_row[i] = layer_items_per_row(d, c->layer_mask[l], c->appended[l], p.cb, p.cq);
-      grid_x = std::max(grid_x, p.items_per_row[i] * d.B);
+      const ChunkCounts cc = counts_of(d, c->appended[l], p.plan);
+      DecodeLayer& dl = p.layer[i];
+      dl.appended = c->appended[l];
+      dl.nbU = cc.nbU;
+      dl.nqU = cc.nqU;
+      dl.nqK = cc.nqK;
+      dl.nbP = cc.nbP;
+      dl.items_per_row = row_chunks(d, c->layer_mask[l], cc);
+      dl.item_base = total;
+      total += dl.items_per_row * d.B;
     }
-    const hg_status st = cuda_status(launch_decode(p, grid_x, reinterpret_cast<cudaStream_t>(stream)));
+    p.total_items = total;
+    const hg_status st = cuda_status(launch_decode(p, total, reinterpret_cast<cudaStream_t>(stream)));
     if (st != HG_OK) return st;
   }
   return HG_OK;
+}
+
+hg_status decode_checks(const hg_cache* c, int32_t layer_begin, int32_t layer_count, const void* q,
+                        void* out, float softmax_scale, void* ws, size_t ws_bytes_given) {
+  if (!range_ok(c, layer_begin, layer_count) || !q || !out || !ws) return HG_ERR_INVALID_ARG;
+  if (!aligned16(q) || !aligned16(out) || !aligned16(ws)) return HG_ERR_ALIGNMENT;
+  if (!(softmax_scale == softmax_scale)) return HG_ERR_INVALID_ARG;  // NaN
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    if (ws_bytes_given < ws_size_for(c, layer_begin + done, n)) return HG_ERR_WORKSPACE_TOO_SMALL;
+  }
+  return HG_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+hg_status hg_decode_attention(const hg_cache* c, int32_t layer_begin, int32_t layer_count,
+                              const void* q, void* out, float softmax_scale, void* ws,
+                              size_t ws_bytes_given, hg_stream_t stream) {
+  const hg_status st = decode_checks(c, layer_begin, layer_count, q, out, softmax_scale, ws, ws_bytes_given);
+  if (st != HG_OK) return st;
+  return decode_launch(c, layer_begin, layer_count, q, nullptr, nullptr, out, softmax_scale, ws,
+                       ws_bytes_given, stream);
+}
+
+hg_status hg_decode_step(hg_cache* c, int32_t layer_begin, int32_t layer_count, const void* q,
+                         const void* k_new, const void* v_new, void* out, float softmax_scale,
+                         void* ws, size_t ws_bytes_given, hg_stream_t stream) {
+  hg_status st = decode_checks(c, layer_begin, layer_count, q, out, softmax_scale, ws, ws_bytes_given);
+  if (st != HG_OK) return st;
+  if (!k_new || !v_new) return HG_ERR_INVALID_ARG;
+  if (!aligned16(k_new) || !aligned16(v_new)) return HG_ERR_ALIGNMENT;
+  for (int i = 0; i < layer_count; ++i)
+    if (c->appended[layer_begin + i] >= c->d.S_new) return HG_ERR_CAPACITY;
+  for (int i = 0; i < layer_count; ++i) c->appended[layer_begin + i] += 1;
+  st = decode_launch(c, layer_begin, layer_count, q, k_new, v_new, out, softmax_scale, ws,
+                     ws_bytes_given, stream);
+  if (st != HG_OK)
+    for (int i = 0; i < layer_count; ++i) c->appended[layer_begin + i] -= 1;
+  return st;
 }
 
 hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {

@@ -7,8 +7,8 @@
 // keys with coded values.  The only branch on the mask or the image span is
 // therefore taken once per CTA.
 //
-// Tiles of the chunk stream through a 3-stage cp.async pipeline in shared
-// memory.  Each warp owns 16-token slices and computes, with mma.sync
+// Tiles of the chunk stream through a cp.async pipeline in a 64 KB shared
+// buffer (two to four stages depending on the tile size).  Each warp owns 16-token slices and computes, with mma.sync
 // m16n8k16 (BF16 in, fp32 accumulate):
 //   S^T[token][query] = K . q     A = keys (BF16 via ldmatrix, or codes
 //                                 expanded exactly to BF16 in registers),
@@ -17,7 +17,9 @@
 //                                 B = P^T, transposed from the score fragment
 //                                 with movmatrix.
 // Coded keys are contracted in the code domain: with per-token groups
-// k^_d = s c_d + z, so q.k^ = s (q.c) + z sum(q); KIVI-style per-channel
+// k^_d = s c_d + z, so q.k^ = s (q.c) + z sum(q); the key codes enter the MMA
+// as the exact BF16 values 128 + c (no subtraction), and the 128 sum(q) offset
+// is removed in the fp32 epilogue; KIVI-style per-channel
 // groups fold the channel scale into the query (q~_d = q_d s_d, split into a
 // BF16 hi + lo pair) and add sum_d q_d z_d.  Values fold the token scale into
 // P (p s) and add sum_t p_t z_t.  AKVQ-style keys are coded in the rotated
@@ -41,15 +43,14 @@ namespace {
 
 constexpr int kThreads = 128;
 constexpr int kWarps = 4;
-constexpr int kStages = 3;
-constexpr int kStageBytes = 32768;
+constexpr int kBufBytes = 65536;   // pipeline buffer (stages of one tile each)
 constexpr int kBf16Tile = 64;      // tokens per tile of BF16 rows (K 16 KB + V 16 KB)
 constexpr int kMixTile = 64;       // tokens per tile of BF16 keys + coded values
-constexpr int kPartialStride = kD + 2;
+constexpr int kPartialStride = kD + 4;  // m, l, 2 pad, o[128]: rows of 528 bytes (16-byte multiple)
 constexpr int kQOff = 0;                      // float q[16][128]
 constexpr int kZsumOff = kMaxG * kD * 4;      // float sum(q)[16]
 constexpr int kStageOff = kZsumOff + 256;
-constexpr int kSmemBytes = kStageOff + kStages * kStageBytes;
+constexpr int kSmemBytes = kStageOff + kBufBytes;
 constexpr unsigned kFull = 0xffffffffu;
 
 enum KMode { K_BF16 = 0, K_TOKEN = 1, K_KIVI = 2 };
@@ -70,27 +71,52 @@ struct Seg {
   const char* km;  // key metadata
   const char* vc;  // value codes
   const char* vm;  // value metadata
+  // Fused append: BF16 row new_pos of this segment comes from these input
+  // rows instead of the arena (new_pos < 0: none).
+  int new_pos;
+  const char* k_new;
+  const char* v_new;
 };
 
-__device__ __forceinline__ void copy_linear(uint32_t dst, const char* src, int slot_bytes,
-                                            int valid_bytes, int tid) {
-  for (int off = tid * 16; off < slot_bytes; off += kThreads * 16) {
-    int n = valid_bytes - off;
-    n = n < 0 ? 0 : (n > 16 ? 16 : n);
-    cp_async16(dst + off, n > 0 ? src + off : src, n);
+// SLOT bytes from src into a linear slot; only the first valid_bytes are read,
+// the rest of the slot is zero-filled.
+template <int SLOT>
+__device__ __forceinline__ void copy_linear(uint32_t dst, const char* src, int valid_bytes, int tid) {
+#pragma unroll
+  for (int off = tid * 16, i = 0; i < (SLOT + kThreads * 16 - 1) / (kThreads * 16); ++i, off += kThreads * 16) {
+    if (off < SLOT) {
+      int n = valid_bytes - off;
+      n = n < 0 ? 0 : (n > 16 ? 16 : n);
+      cp_async16(dst + off, n > 0 ? src + off : src, n);
+    }
   }
 }
 
 // nvalid BF16 rows (256 B each) into a 64-row tile, 16-byte chunks swizzled by
 // (row & 7) so that ldmatrix reads are conflict free; missing rows are zero.
+// Thread t always moves chunk (t & 15) of rows (t >> 4) + 8 i.
+// Row sub_row (if >= 0) is read from sub instead (a new decode token).
 __device__ __forceinline__ void copy_rows_swizzled(uint32_t dst, const char* src, int nvalid,
-                                                   int tid) {
-  for (int q = tid; q < 64 * 16; q += kThreads) {
-    const int r = q >> 4, c = q & 15;
+                                                   int tid, int sub_row, const char* sub) {
+  const int r0 = tid >> 4, c = tid & 15;
+  const uint32_t d0 = dst + r0 * 256 + ((c ^ (r0 & 7)) << 4);
+  const char* s0 = src + r0 * 256 + c * 16;
+#pragma unroll
+  for (int i = 0; i < 64 / (kThreads / 16); ++i) {
+    const int r = r0 + (kThreads / 16) * i;
     const bool ok = r < nvalid;
-    cp_async16(dst + r * 256 + ((c ^ (r & 7)) << 4), ok ? src + r * 256 + c * 16 : src,
-               ok ? 16 : 0);
+    const char* from = (r == sub_row) ? sub + c * 16 : s0 + i * (kThreads / 16) * 256;
+    cp_async16(d0 + i * (kThreads / 16) * 256, ok ? from : src, ok ? 16 : 0);
   }
+}
+
+// cp.async.wait_group with a run-time count in [0, S).
+template <int S>
+__device__ __forceinline__ void cp_async_wait_pending(int n) {
+  if (S > 3 && n >= 3) { cp_async_wait<3>(); return; }
+  if (S > 2 && n == 2) { cp_async_wait<2>(); return; }
+  if (n == 1) { cp_async_wait<1>(); return; }
+  cp_async_wait<0>();
 }
 
 template <int BITS>
@@ -98,13 +124,37 @@ __device__ __forceinline__ uint32_t pair2(uint32_t x) {  // codes at bits [0,b) 
   return codes_bf16x2(x & (BITS == 2 ? 0x00030003u : 0x000F000Fu));
 }
 
+// The same pair as the BF16 values (128 + code): exact, without the subtraction.
+template <int BITS>
+__device__ __forceinline__ uint32_t pair2_off(uint32_t x) {
+  return (x & (BITS == 2 ? 0x00030003u : 0x000F000Fu)) | 0x43004300u;
+}
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
+  return y;
+}
+
 template <int NT, int NZ>
 struct WarpState {
   float o[NT][8][4];
+  float corr[NT][4];  // 128 * sum_t P^T[t][q] for value codes carried as 128 + c
   float m[NT][2];
   float l[NT][2];
   float z[NT][2][NZ];
 };
+
+// 2-bit codes of one word sit in pairs (j, j + 8) at bits (2j, 2j + 16).  Pair j
+// is taken from (w >> 6 * (j / 3)) masked at bit 2 * (j % 3): that yields
+// 4^(j % 3) * code, which stays inside the 7-bit BF16 mantissa of 128 + x, and
+// costs one shift per three pairs.  The factor is removed where it is exact
+// (a power of two on the other MMA operand or on the accumulator).
+__device__ __forceinline__ int pos3(int j) { return 2 * (j % 3); }
+__device__ __forceinline__ uint32_t pair2_scaled(uint32_t w, uint32_t w6, uint32_t w12, int j) {
+  const uint32_t src = j < 3 ? w : (j < 6 ? w6 : w12);
+  return (src & (0x00030003u << pos3(j))) | 0x43004300u;
+}
 
 template <int BITS, int KM, int VM>
 struct Tile {
@@ -118,26 +168,28 @@ struct Tile {
   static constexpr int km_off = kc_off + kc_bytes;
   static constexpr int vc_off = km_off + km_bytes;
   static constexpr int vm_off = vc_off + vc_bytes;
-  static_assert(vm_off + vm_bytes <= kStageBytes, "tile does not fit a stage");
+  static constexpr int stage_bytes = ((vm_off + vm_bytes + 127) / 128) * 128;
+  static constexpr int stages = (kBufBytes / stage_bytes) > 4 ? 4 : (kBufBytes / stage_bytes);
+  static_assert(stages >= 2, "a tile must fit twice in the pipeline buffer");
 };
 
 template <int BITS, int KM, int VM>
 __device__ __forceinline__ void issue_tile(uint32_t st, const Seg& sg, int t0, int nvalid, int tid) {
   using TL = Tile<BITS, KM, VM>;
   if (KM == K_BF16) {
-    copy_rows_swizzled(st + TL::kc_off, sg.k + (size_t)t0 * 256, nvalid, tid);
+    copy_rows_swizzled(st + TL::kc_off, sg.k + (size_t)t0 * 256, nvalid, tid, sg.new_pos - t0, sg.k_new);
   } else {
-    copy_linear(st + TL::kc_off, sg.kc + (size_t)t0 * 16 * BITS, TL::kc_bytes, nvalid * 16 * BITS, tid);
+    copy_linear<TL::kc_bytes>(st + TL::kc_off, sg.kc + (size_t)t0 * 16 * BITS, nvalid * 16 * BITS, tid);
     // KIVI-style key metadata: one (scale, zero) per channel per 32 tokens = 32 B per token
     constexpr int kmb = (KM == K_TOKEN) ? 8 : 32;
-    copy_linear(st + TL::km_off, sg.km + (size_t)t0 * kmb, TL::km_bytes, nvalid * kmb, tid);
+    copy_linear<TL::km_bytes>(st + TL::km_off, sg.km + (size_t)t0 * kmb, nvalid * kmb, tid);
   }
   if (VM == V_BF16) {
-    copy_rows_swizzled(st + TL::vc_off, sg.v + (size_t)t0 * 256, nvalid, tid);
+    copy_rows_swizzled(st + TL::vc_off, sg.v + (size_t)t0 * 256, nvalid, tid, sg.new_pos - t0, sg.v_new);
   } else {
-    copy_linear(st + TL::vc_off, sg.vc + (size_t)t0 * 16 * BITS, TL::vc_bytes, nvalid * 16 * BITS, tid);
+    copy_linear<TL::vc_bytes>(st + TL::vc_off, sg.vc + (size_t)t0 * 16 * BITS, nvalid * 16 * BITS, tid);
     constexpr int vmb = (VM == V_TOKEN) ? 8 : 32;
-    copy_linear(st + TL::vm_off, sg.vm + (size_t)t0 * vmb, TL::vm_bytes, nvalid * vmb, tid);
+    copy_linear<TL::vm_bytes>(st + TL::vm_off, sg.vm + (size_t)t0 * vmb, nvalid * vmb, tid);
   }
 }
 
@@ -185,23 +237,51 @@ __device__ __forceinline__ void token_channels(int tq, int j, int (&c)[4]) {
   }
 }
 
+// Query fragments for coded per-token keys.  2-bit: k-step j carries q / 4^(j % 3)
+// to match the scaled key pairs.  Also returns, per query column of this
+// thread, s1 = sum of the fragment values as the MMA sees them (for removing
+// the 128 offset of the key codes) and s0 = sum of the unscaled queries.
 template <int BITS, int NT, bool ROT>
 __device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (&ql)[NT][8][2],
+                                            float (&s1)[NT][2], float (&s0)[NT][2],
                                             const float* q_s, int g, int tq) {
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
     const float* qr = q_s + (nt * 8 + g) * kD;
+    float a1 = 0.f, a0 = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       int c[4];
       token_channels<BITS>(tq, j, c);
-      if (ROT) {
-        split_pair(qr[c[0]], qr[c[1]], qb[nt][j][0], ql[nt][j][0]);
-        split_pair(qr[c[2]], qr[c[3]], qb[nt][j][1], ql[nt][j][1]);
-      } else {
-        qb[nt][j][0] = pack_bf16x2(qr[c[0]], qr[c[1]]);
-        qb[nt][j][1] = pack_bf16x2(qr[c[2]], qr[c[3]]);
+      const float f = (BITS == 2) ? 1.0f / (float)(1 << pos3(j)) : 1.0f;  // exact
+#pragma unroll
+      for (int hh = 0; hh < 2; ++hh) {
+        const float x0 = qr[c[2 * hh]] * f, x1 = qr[c[2 * hh + 1]] * f;
+        uint32_t hi, lo = 0u;
+        if (ROT) {
+          split_pair(x0, x1, hi, lo);
+        } else {
+          hi = pack_bf16x2(x0, x1);  // exact: the queries are BF16
+        }
+        qb[nt][j][hh] = hi;
+        ql[nt][j][hh] = lo;
+        float h0, h1, l0, l1;
+        bf16x2_to_f32(hi, h0, h1);
+        bf16x2_to_f32(lo, l0, l1);
+        const float part = (h0 + l0) + (h1 + l1);
+        a1 += part;
+        a0 += part * (1.0f / f);
       }
+    }
+    // totals for query g, then the values of this thread's columns 2tq, 2tq+1
+    a1 += __shfl_xor_sync(kFull, a1, 1);
+    a1 += __shfl_xor_sync(kFull, a1, 2);
+    a0 += __shfl_xor_sync(kFull, a0, 1);
+    a0 += __shfl_xor_sync(kFull, a0, 2);
+#pragma unroll
+    for (int e = 0; e < 2; ++e) {
+      s1[nt][e] = __shfl_sync(kFull, a1, (2 * tq + e) << 2);
+      s0[nt][e] = __shfl_sync(kFull, a0, (2 * tq + e) << 2);
     }
   }
 }
@@ -211,27 +291,24 @@ __device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (
 // ---------------------------------------------------------------------------
 template <int NT, int NZ>
 __device__ __forceinline__ void softmax_update(WarpState<NT, NZ>& ws, float (&sc)[NT][4], float (&p)[NT][4]) {
-  float mx[NT][2];
+  // The running maxima are only moved when a score exceeds them by 2^8, so the
+  // exact column maxima are needed only when some lane sees such a score.
   bool need = false;
 #pragma unroll
-  for (int nt = 0; nt < NT; ++nt) {
+  for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-    for (int e = 0; e < 2; ++e) {
-      float v = fmaxf(sc[nt][e], sc[nt][2 + e]);
-      v = fmaxf(v, __shfl_xor_sync(kFull, v, 4));
-      v = fmaxf(v, __shfl_xor_sync(kFull, v, 8));
-      v = fmaxf(v, __shfl_xor_sync(kFull, v, 16));
-      mx[nt][e] = v;
-      need |= v > ws.m[nt][e] + 8.0f;
-    }
-  }
+    for (int e = 0; e < 2; ++e) need |= fmaxf(sc[nt][e], sc[nt][2 + e]) > ws.m[nt][e] + 8.0f;
   if (__any_sync(kFull, need)) {
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
       for (int e = 0; e < 2; ++e) {
-        const float mn = fmaxf(ws.m[nt][e], mx[nt][e]);
-        const float a = (ws.m[nt][e] == -INFINITY) ? 0.f : exp2f(ws.m[nt][e] - mn);
+        float v = fmaxf(sc[nt][e], sc[nt][2 + e]);
+        v = fmaxf(v, __shfl_xor_sync(kFull, v, 4));
+        v = fmaxf(v, __shfl_xor_sync(kFull, v, 8));
+        v = fmaxf(v, __shfl_xor_sync(kFull, v, 16));
+        const float mn = fmaxf(ws.m[nt][e], v);
+        const float a = (ws.m[nt][e] == -INFINITY) ? 0.f : fast_exp2(ws.m[nt][e] - mn);
         ws.m[nt][e] = mn;
         ws.l[nt][e] *= a;
 #pragma unroll
@@ -241,13 +318,15 @@ __device__ __forceinline__ void softmax_update(WarpState<NT, NZ>& ws, float (&sc
           ws.o[nt][mt][e] *= a;
           ws.o[nt][mt][2 + e] *= a;
         }
+        ws.corr[nt][e] *= a;
+        ws.corr[nt][2 + e] *= a;
       }
     }
   }
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) p[nt][i] = exp2f(sc[nt][i] - ws.m[nt][i & 1]);
+    for (int i = 0; i < 4; ++i) p[nt][i] = fast_exp2(sc[nt][i] - ws.m[nt][i & 1]);
 #pragma unroll
     for (int e = 0; e < 2; ++e) ws.l[nt][e] += p[nt][e] + p[nt][2 + e];
   }
@@ -278,8 +357,8 @@ template <int BITS, int NT, int KM, int VM, bool ROT>
 __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws, const char* st,
                                              int nvalid, const uint32_t (&qb)[NT][8][2],
                                              const uint32_t (&ql)[NT][8][2], const float* q_s,
-                                             const float* zsum_s, float scale_log2, int warp,
-                                             int lane) {
+                                             const float (&s1)[NT][2], const float (&s0)[NT][2],
+                                             float scale_log2, int warp, int lane) {
   using TL = Tile<BITS, KM, VM>;
   constexpr int NZ = NZOf<VM>::value;
   const int g = lane >> 2, tq = lane & 3;
@@ -313,29 +392,50 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       const int row = tok0 + r + 8 * (mat & 1);
       const uint32_t rbase = st_u32 + TL::kc_off + row * 256;
       const int rsw = row & 7, ch = mat >> 1;
+      float acc2[NT][4];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc2[nt][i] = 0.f;
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         uint32_t a[4];
         ldsm_x4(a, rbase + (((2 * j + ch) ^ rsw) << 4));
 #pragma unroll
-        for (int nt = 0; nt < NT; ++nt) mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
+        for (int nt = 0; nt < NT; ++nt)
+          mma_bf16((j & 1) ? acc2[nt] : acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
       }
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[0][nt][i] += acc2[nt][i];
     } else if (KM == K_TOKEN) {
       const int tok0 = u * 16;
+      float acc2[NT][4];
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc2[nt][i] = 0.f;
       if (BITS == 2) {
         const uint2 ka = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g) * 8 + 2 * tq);
         const uint2 kb = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g + 8) * 8 + 2 * tq);
+        const uint32_t w[4] = {ka.x, kb.x, ka.y, kb.y};
+        uint32_t w6[4], w12[4];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          w6[k] = w[k] >> 6;
+          w12[k] = w[k] >> 12;
+        }
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
           uint32_t a[4];
-          a[0] = pair2<2>(ka.x >> (2 * j));
-          a[1] = pair2<2>(kb.x >> (2 * j));
-          a[2] = pair2<2>(ka.y >> (2 * j));
-          a[3] = pair2<2>(kb.y >> (2 * j));
+#pragma unroll
+          for (int k = 0; k < 4; ++k) a[k] = pair2_scaled(w[k], w6[k], w12[k], j);
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
-            if (ROT) mma_bf16(acc[0][nt], a, ql[nt][j][0], ql[nt][j][1]);
+            float (&dst)[4] = (j & 1) ? acc2[nt] : acc[0][nt];
+            mma_bf16(dst, a, qb[nt][j][0], qb[nt][j][1]);
+            if (ROT) mma_bf16(dst, a, ql[nt][j][0], ql[nt][j][1]);
           }
         }
       } else {
@@ -347,17 +447,22 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         for (int j = 0; j < 8; ++j) {
           const int wi = j >> 1, i = 2 * (j & 1);
           uint32_t a[4];
-          a[0] = pair2<4>(wa[wi] >> (4 * i));
-          a[1] = pair2<4>(wb[wi] >> (4 * i));
-          a[2] = pair2<4>(wa[wi] >> (4 * i + 4));
-          a[3] = pair2<4>(wb[wi] >> (4 * i + 4));
+          a[0] = pair2_off<4>(wa[wi] >> (4 * i));
+          a[1] = pair2_off<4>(wb[wi] >> (4 * i));
+          a[2] = pair2_off<4>(wa[wi] >> (4 * i + 4));
+          a[3] = pair2_off<4>(wb[wi] >> (4 * i + 4));
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            mma_bf16(acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
-            if (ROT) mma_bf16(acc[0][nt], a, ql[nt][j][0], ql[nt][j][1]);
+            float (&dst)[4] = (j & 1) ? acc2[nt] : acc[0][nt];
+            mma_bf16(dst, a, qb[nt][j][0], qb[nt][j][1]);
+            if (ROT) mma_bf16(dst, a, ql[nt][j][0], ql[nt][j][1]);
           }
         }
       }
+#pragma unroll
+      for (int nt = 0; nt < NT; ++nt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) acc[0][nt][i] += acc2[nt][i];
     } else {  // K_KIVI: group u of the tile; channel c has (scale, zero) = meta[u][c]
       const float2* gm = km2 + u * kD;
       uint32_t qh[NT][8][2], qlo[NT][8][2];
@@ -440,14 +545,16 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       if (tok0 >= nvalid) break;
       float sc[NT][4];
       if (KM == K_TOKEN) {
+        // acc = sum_d (128 + f c_d) (q_d / f) = 128 s1 + q.c, so
+        // score = s (acc - 128 s1) + z s0
         const float2 mg = km2[tok0 + g], mg8 = km2[tok0 + g + 8];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
           for (int e = 0; e < 2; ++e) {
-            const float zq = zsum_s[nt * 8 + 2 * tq + e];
-            sc[nt][e] = fmaf(mg.x, acc[s][nt][e], mg.y * zq) * scale_log2;
-            sc[nt][2 + e] = fmaf(mg8.x, acc[s][nt][2 + e], mg8.y * zq) * scale_log2;
+            const float off = -128.f * s1[nt][e];
+            sc[nt][e] = fmaf(mg.x, acc[s][nt][e] + off, mg.y * s0[nt][e]) * scale_log2;
+            sc[nt][2 + e] = fmaf(mg8.x, acc[s][nt][2 + e] + off, mg8.y * s0[nt][e]) * scale_log2;
           }
         }
       } else if (KM == K_KIVI) {
@@ -496,20 +603,31 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 #pragma unroll
           for (int e = 0; e < 2; ++e) ws.z[nt][e][0] += p[nt][e] * vg.y + p[nt][2 + e] * vg8.y;
         }
+        // value codes enter as 128 + f c; the 128 part is collected in ws.corr by
+        // one MMA on a constant tile and removed at the end (f: see pair2_scaled)
+        {
+          const uint32_t c128[4] = {0x43004300u, 0x43004300u, 0x43004300u, 0x43004300u};
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) mma_pv(ws.corr[nt], c128, b[nt]);
+        }
         const int t0 = tok0 + 2 * tq;
         if (BITS == 2) {
           // word g of a token row holds channels 16g..16g+15
           const uint32_t w0 = vc32[t0 * 8 + g], w1 = vc32[(t0 + 1) * 8 + g];
           const uint32_t w8 = vc32[(t0 + 8) * 8 + g], w9 = vc32[(t0 + 9) * 8 + g];
-          const uint32_t x01 = prmt(w0, w1, 0x5410), y01 = prmt(w0, w1, 0x7632);
-          const uint32_t x89 = prmt(w8, w9, 0x5410), y89 = prmt(w8, w9, 0x7632);
+          const uint32_t x[4] = {prmt(w0, w1, 0x5410), prmt(w0, w1, 0x7632), prmt(w8, w9, 0x5410),
+                                 prmt(w8, w9, 0x7632)};
+          uint32_t x6[4], x12[4];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            x6[k] = x[k] >> 6;
+            x12[k] = x[k] >> 12;
+          }
 #pragma unroll
           for (int mt = 0; mt < 8; ++mt) {
             uint32_t a[4];
-            a[0] = pair2<2>(x01 >> (2 * mt));
-            a[1] = pair2<2>(y01 >> (2 * mt));
-            a[2] = pair2<2>(x89 >> (2 * mt));
-            a[3] = pair2<2>(y89 >> (2 * mt));
+#pragma unroll
+            for (int k = 0; k < 4; ++k) a[k] = pair2_scaled(x[k], x6[k], x12[k], mt);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
           }
@@ -527,10 +645,10 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           for (int mt = 0; mt < 8; ++mt) {
             const int sh = 4 * (mt & 3);
             uint32_t a[4];
-            a[0] = pair2<4>((mt < 4 ? xa : ya) >> sh);
-            a[1] = pair2<4>((mt < 4 ? xb : yb) >> sh);
-            a[2] = pair2<4>((mt < 4 ? xc : yc) >> sh);
-            a[3] = pair2<4>((mt < 4 ? xd : yd) >> sh);
+            a[0] = pair2_off<4>((mt < 4 ? xa : ya) >> sh);
+            a[1] = pair2_off<4>((mt < 4 ? xb : yb) >> sh);
+            a[2] = pair2_off<4>((mt < 4 ? xc : yc) >> sh);
+            a[3] = pair2_off<4>((mt < 4 ? xd : yd) >> sh);
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
           }
@@ -602,23 +720,38 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, tq = lane & 3;
   float* q_s = reinterpret_cast<float*>(smem + kQOff);
-  float* zsum_s = reinterpret_cast<float*>(smem + kZsumOff);
   char* stages = smem + kStageOff;
 
-  // First tiles in flight before anything else.
+  // Every tile that fits the buffer goes in flight before anything else (the
+  // work plan sizes chunks to fit); later tiles, if any, reuse slots as the
+  // ring advances.
+  constexpr int STAGES = TL::stages;
   const int n_tiles = (te - tb + TL::tokens - 1) / TL::tokens;
   const uint32_t st0 = smem_u32(stages);
-#pragma unroll
-  for (int s = 0; s < kStages - 1; ++s) {
-    if (s < n_tiles)
-      issue_tile<BITS, KM, VM>(st0 + s * kStageBytes, sg, tb + s * TL::tokens,
-                               min(TL::tokens, te - tb - s * TL::tokens), tid);
+  int issued = n_tiles < STAGES ? n_tiles : STAGES;
+  for (int s = 0; s < issued; ++s) {
+    issue_tile<BITS, KM, VM>(st0 + s * TL::stage_bytes, sg, tb + s * TL::tokens,
+                             min(TL::tokens, te - tb - s * TL::tokens), tid);
     cp_async_commit();
   }
 
   // Queries of this KV head's group (fp32, rows >= G zero), rotated for
-  // AKVQ-style coded keys, and their channel sums.
-  for (int i = tid; i < NT * 8 * kD; i += kThreads) q_s[i] = (i < G * kD) ? bf16_to_f32(qg[i]) : 0.f;
+  // AKVQ-style coded keys.
+  for (int i = tid; i < NT * 8 * 16; i += kThreads) {
+    float4* dst = reinterpret_cast<float4*>(q_s + i * 8);
+    if (i < G * 16) {
+      const uint4 v = ldg16(qg + i * 8);
+      float f[8];
+      bf16x2_to_f32(v.x, f[0], f[1]);
+      bf16x2_to_f32(v.y, f[2], f[3]);
+      bf16x2_to_f32(v.z, f[4], f[5]);
+      bf16x2_to_f32(v.w, f[6], f[7]);
+      dst[0] = make_float4(f[0], f[1], f[2], f[3]);
+      dst[1] = make_float4(f[4], f[5], f[6], f[7]);
+    } else {
+      dst[0] = dst[1] = make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+  }
   __syncthreads();
   if (ROT) {
     for (int j = warp; j < G; j += kWarps) {
@@ -631,22 +764,16 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
     }
     __syncthreads();
   }
-  for (int j = warp; j < NT * 8; j += kWarps) {
-    float sum = 0.f;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) sum += q_s[j * kD + lane * 4 + i];
-    sum = warp_sum(sum);
-    if (lane == 0) zsum_s[j] = sum;
-  }
-  __syncthreads();
-
   uint32_t qb[NT][8][2], ql[NT][8][2];
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
     for (int j = 0; j < 8; ++j) qb[nt][j][0] = qb[nt][j][1] = ql[nt][j][0] = ql[nt][j][1] = 0u;
+  float s1[NT][2], s0[NT][2];
+#pragma unroll
+  for (int nt = 0; nt < NT; ++nt) s1[nt][0] = s1[nt][1] = s0[nt][0] = s0[nt][1] = 0.f;
   if (KM == K_BF16) qfrag_natural<NT>(qb, q_s, g, tq);
-  if (KM == K_TOKEN) qfrag_token<BITS, NT, ROT>(qb, ql, q_s, g, tq);
+  if (KM == K_TOKEN) qfrag_token<BITS, NT, ROT>(qb, ql, s1, s0, q_s, g, tq);
 
   WarpState<NT, NZ> ws;
 #pragma unroll
@@ -662,19 +789,23 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
     for (int mt = 0; mt < 8; ++mt)
 #pragma unroll
       for (int i = 0; i < 4; ++i) ws.o[nt][mt][i] = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) ws.corr[nt][i] = 0.f;
   }
 
   for (int it = 0; it < n_tiles; ++it) {
-    cp_async_wait<kStages - 2>();
+    // tile `it` has landed once at most issued - it - 1 groups are pending
+    cp_async_wait_pending<STAGES>(issued - it - 1);
     __syncthreads();
-    const int nx = it + kStages - 1;
-    if (nx < n_tiles)
-      issue_tile<BITS, KM, VM>(st0 + (nx % kStages) * kStageBytes, sg, tb + nx * TL::tokens,
-                               min(TL::tokens, te - tb - nx * TL::tokens), tid);
-    cp_async_commit();
-    compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + (it % kStages) * kStageBytes,
+    if (it > 0 && issued < n_tiles) {  // refill the slot of tile it - 1
+      issue_tile<BITS, KM, VM>(st0 + (issued % STAGES) * TL::stage_bytes, sg, tb + issued * TL::tokens,
+                               min(TL::tokens, te - tb - issued * TL::tokens), tid);
+      cp_async_commit();
+      ++issued;
+    }
+    compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + (it % STAGES) * TL::stage_bytes,
                                         min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s,
-                                        zsum_s, scale_log2, warp, lane);
+                                        s1, s0, scale_log2, warp, lane);
   }
   cp_async_wait<0>();
   __syncthreads();  // stage buffers are reused for the reduction below
@@ -705,39 +836,44 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) {
         int c_lo, c_hi;  // channels of rows g and g+8 of m-tile mt
-        float zlo = 0.f, zhi = 0.f;
         if (VM == V_TOKEN) {
+          // remove the 128 offset and the 4^(mt % 3) factor of 2-bit value pairs
           c_lo = 16 * g + mt;
           c_hi = 16 * g + 8 + mt;
-          zlo = zhi = ws.z[nt][e][0];
+          const float f = (BITS == 2) ? 1.0f / (float)(1 << pos3(mt)) : 1.0f;
+          orow[c_lo] = (ws.o[nt][mt][e] - ws.corr[nt][e]) * f + ws.z[nt][e][0];
+          orow[c_hi] = (ws.o[nt][mt][2 + e] - ws.corr[nt][2 + e]) * f + ws.z[nt][e][0];
         } else {
           c_lo = 16 * mt + g;
           c_hi = 16 * mt + 8 + g;
-          if (VM == V_KIVI) zlo = zhi = ws.z[nt][e][(mt >> 1) % NZ];
+          const float z = (VM == V_KIVI) ? ws.z[nt][e][(mt >> 1) % NZ] : 0.f;
+          orow[c_lo] = ws.o[nt][mt][e] + z;
+          orow[c_hi] = ws.o[nt][mt][2 + e] + z;
         }
-        orow[c_lo] = ws.o[nt][mt][e] + zlo;
-        orow[c_hi] = ws.o[nt][mt][2 + e] + zhi;
       }
     }
   }
 }
 
 template <int BITS, int NT, int BASE>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, NT == 1 ? 3 : 2)
 decode_kernel(const __grid_constant__ DecodeParams p) {
   extern __shared__ __align__(128) char smem[];
   const Dims& d = p.d;
-  const int li = blockIdx.y;
-  const int ipr = p.items_per_row[li];
   const int item = blockIdx.x;
-  if (item >= ipr * d.B) return;
-  const int b = item / ipr;
-  int r = item - b * ipr;
+  if (item >= p.total_items) return;
+  int li = 0;
+  while (li + 1 < p.n_layers && p.layer[li + 1].item_base <= item) ++li;
+  const DecodeLayer& L = p.layer[li];
+  const int in_layer = item - L.item_base;
+  const int b = in_layer / L.items_per_row;
+  int r = in_layer - b * L.items_per_row;
   const uint64_t mask = p.lt.mask[li];
-  const int app = p.appended[li];
-  int h = 0, nb = 0, ni = 0;
+  const ChunkCounts cc = {L.nbU, L.nqU, L.nqK, L.nbP};
+  int h = 0, nb = 0, ni = 0, cls = kQuantized;
   for (; h < d.H; ++h) {
-    ni = head_items(d, head_class(d, mask, h), app, p.cb, p.cq, &nb);
+    cls = head_class(d, mask, h);
+    ni = head_chunks(cls, cc, &nb);
     if (r < ni) break;
     r -= ni;
   }
@@ -748,11 +884,13 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   const bool coded = r >= nb;
   int tb, te;
   if (!coded) {
-    tb = r * p.cb;
-    te = min(tb + p.cb, hd.bf16_prefill + app);
+    const int c = (cls == kProtected) ? p.plan.cbP : p.plan.cbU;
+    tb = r * c;
+    te = min(tb + c, hd.bf16_prefill + L.appended);
   } else {
-    tb = (r - nb) * p.cq;
-    te = min(tb + p.cq, d.nq);
+    const int c = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
+    tb = (r - nb) * c;
+    te = min(tb + c, d.nq);
   }
   const int tid = threadIdx.x;
   const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
@@ -762,9 +900,25 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   float* red_o = red_l + kWarps * kMaxG;                        // [warps][16][128]
   Seg sg;
   sg.k = sg.v = sg.kc = sg.km = sg.vc = sg.vm = nullptr;
+  sg.new_pos = -1;
+  sg.k_new = sg.v_new = nullptr;
   if (!coded) {
     sg.k = Lb + hd.kb + b * hd.kb_bs;
     sg.v = Lb + hd.vb + b * hd.kb_bs;
+    const int pos = hd.bf16_prefill + L.appended - 1;  // the step's new token
+    if (p.k_new && pos >= tb && pos < te) {
+      const size_t row = (((size_t)li * d.B + b) * d.H + h) * kD;
+      sg.new_pos = pos;
+      sg.k_new = reinterpret_cast<const char*>(p.k_new + row);
+      sg.v_new = reinterpret_cast<const char*>(p.v_new + row);
+      // this CTA alone owns the position in this launch: store it in the arena
+      if (threadIdx.x < 32) {
+        const int c = threadIdx.x & 15;
+        const char* src = (threadIdx.x < 16) ? sg.k_new : sg.v_new;
+        char* dst = const_cast<char*>((threadIdx.x < 16) ? sg.k : sg.v) + (size_t)pos * 256;
+        *reinterpret_cast<uint4*>(dst + c * 16) = ldg16(src + c * 16);
+      }
+    }
     run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
   } else if (hd.cls == kKeysOnly) {
     sg.k = Lb + hd.kimg + b * hd.kimg_bs;
@@ -788,60 +942,113 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   }
   __syncthreads();
 
-  // ---- combine the warps: thread = channel ----
+  // ---- combine the warps: per query, weights of the four warps, then thread = channel ----
+  float* red_f = red_o + kWarps * kMaxG * kD;  // [warps][16] weights
+  float* red_ML = red_f + kWarps * kMaxG;       // [16][2] max, sum
+  if (tid < G) {
+    const int j = tid;
+    float M = -INFINITY;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * kMaxG + j]);
+    float Ls = 0.f;
+#pragma unroll
+    for (int w = 0; w < kWarps; ++w) {
+      const float mw = red_m[w * kMaxG + j];
+      const float f = (mw == -INFINITY) ? 0.f : fast_exp2(mw - M);
+      red_f[w * kMaxG + j] = f;
+      Ls += f * red_l[w * kMaxG + j];
+    }
+    red_ML[2 * j] = M;
+    red_ML[2 * j + 1] = Ls;
+  }
+  __syncthreads();
   const int c = tid;
   const size_t out_row = ((size_t)li * d.B + b) * d.Hq + (size_t)h * G;
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
   float* part = p.partials + (head_lin * p.max_items) * (size_t)G * kPartialStride;
   float* mine = part + (size_t)r * G * kPartialStride;
   for (int j = 0; j < G; ++j) {
-    float M = -INFINITY;
+    float O = 0.f;
 #pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * kMaxG + j]);
-    float O = 0.f, Ls = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const float mw = red_m[w * kMaxG + j];
-      const float f = (mw == -INFINITY) ? 0.f : exp2f(mw - M);
-      O += f * red_o[(w * kMaxG + j) * kD + c];
-      Ls += f * red_l[w * kMaxG + j];
-    }
+    for (int w = 0; w < kWarps; ++w) O = fmaf(red_f[w * kMaxG + j], red_o[(w * kMaxG + j) * kD + c], O);
     if (ni == 1) {
-      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / Ls);
+      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / red_ML[2 * j + 1]);
     } else {
-      mine[j * kPartialStride + 2 + c] = O;
+      mine[j * kPartialStride + 4 + c] = O;
       if (c == 0) {
-        mine[j * kPartialStride + 0] = M;
-        mine[j * kPartialStride + 1] = Ls;
+        mine[j * kPartialStride + 0] = red_ML[2 * j];
+        mine[j * kPartialStride + 1] = red_ML[2 * j + 1];
       }
     }
   }
   if (ni == 1) return;
 
-  __threadfence();
+  // Publish the partial: the CTA barrier orders every thread's stores before
+  // thread 0's device-scope fence (fences are cumulative), then take a ticket.
   __syncthreads();
   __shared__ int s_last;
   if (tid == 0) {
+    __threadfence();
     const unsigned prev = atomicAdd(p.counters + head_lin, 1u);
     s_last = (prev == (unsigned)(ni - 1));
   }
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int j = 0; j < G; ++j) {
-    float M = -INFINITY;
-    for (int sidx = 0; sidx < ni; ++sidx)
-      M = fmaxf(M, __ldcg(part + ((size_t)sidx * G + j) * kPartialStride));
-    float O = 0.f, Ls = 0.f;
-    for (int sidx = 0; sidx < ni; ++sidx) {
-      const float* ps = part + ((size_t)sidx * G + j) * kPartialStride;
-      const float ms = __ldcg(ps);
-      const float f = (ms == -INFINITY) ? 0.f : exp2f(ms - M);
-      O += f * __ldcg(ps + 2 + c);
-      Ls += f * __ldcg(ps + 1);
-    }
-    p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / Ls);
+
+  // Last CTA of the head: merge every split.  1) (m, l) of all (split, query)
+  // pairs in one round of loads, then per query the maximum, the weights
+  // f = 2^(m - M) (stored over m) and the normaliser L.
+  float* ml = reinterpret_cast<float*>(smem + kQOff);  // [ni][G][2], queries are no longer needed
+  float* MLq = ml + 2 * ni * G;                         // [G][2]
+  for (int i = tid; i < ni * G; i += kThreads) {
+    ml[2 * i] = __ldcg(part + (size_t)i * kPartialStride);
+    ml[2 * i + 1] = __ldcg(part + (size_t)i * kPartialStride + 1);
   }
+  __syncthreads();
+  if (tid < G) {
+    const int j = tid;
+    float M = -INFINITY;
+    for (int sidx = 0; sidx < ni; ++sidx) M = fmaxf(M, ml[2 * (sidx * G + j)]);
+    float Ls = 0.f;
+    for (int sidx = 0; sidx < ni; ++sidx) {
+      const float ms = ml[2 * (sidx * G + j)];
+      const float f = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
+      ml[2 * (sidx * G + j)] = f;
+      Ls += f * ml[2 * (sidx * G + j) + 1];
+    }
+    MLq[2 * j] = M;
+    MLq[2 * j + 1] = Ls;
+  }
+  __syncthreads();
+  // 2) the o rows, batch by batch of splits through the pipeline buffer with
+  //    one asynchronous sweep each (the partials of a head are contiguous).
+  float O[NT * 8];
+#pragma unroll
+  for (int j = 0; j < NT * 8; ++j) O[j] = 0.f;
+  const int split_floats = G * kPartialStride;
+  const int batch = kBufBytes / (split_floats * 4);
+  const uint32_t buf_u32 = smem_u32(smem + kStageOff);
+  const float* buf = reinterpret_cast<const float*>(smem + kStageOff);
+  for (int s0 = 0; s0 < ni; s0 += batch) {
+    const int nbatch = min(batch, ni - s0);
+    const int bytes = nbatch * split_floats * 4;
+    const char* src = reinterpret_cast<const char*>(part + (size_t)s0 * split_floats);
+    for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, src + off, 16);
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
+    for (int sidx = 0; sidx < nbatch; ++sidx) {
+#pragma unroll
+      for (int j = 0; j < NT * 8; ++j)
+        if (j < G)
+          O[j] = fmaf(ml[2 * ((s0 + sidx) * G + j)], buf[(sidx * G + j) * kPartialStride + 4 + c], O[j]);
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int j = 0; j < NT * 8; ++j)
+    if (j < G) p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O[j] / MLq[2 * j + 1]);
   if (tid == 0) atomicExch(p.counters + head_lin, 0u);
 }
 
@@ -857,8 +1064,8 @@ cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
-  dim3 grid(grid_x, p.n_layers, 1);
-  decode_kernel<BITS, NT, BASE><<<grid, kThreads, kSmemBytes, s>>>(p);
+  (void)grid_x;
+  decode_kernel<BITS, NT, BASE><<<p.total_items, kThreads, kSmemBytes, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -872,6 +1079,25 @@ cudaError_t launch_base(const DecodeParams& p, int grid_x, cudaStream_t s) {
 }
 
 }  // namespace
+
+int decode_coded_tile(int bits) { return coded_tile(bits); }
+
+template <int BITS>
+void capacity_t(int base, int* bf16, int* coded, int* keys_only) {
+  *bf16 = Tile<BITS, K_BF16, V_BF16>::stages * Tile<BITS, K_BF16, V_BF16>::tokens;
+  if (base == kKivi) {
+    *coded = Tile<BITS, K_KIVI, V_KIVI>::stages * Tile<BITS, K_KIVI, V_KIVI>::tokens;
+    *keys_only = Tile<BITS, K_BF16, V_KIVI>::stages * Tile<BITS, K_BF16, V_KIVI>::tokens;
+  } else {
+    *coded = Tile<BITS, K_TOKEN, V_TOKEN>::stages * Tile<BITS, K_TOKEN, V_TOKEN>::tokens;
+    *keys_only = Tile<BITS, K_BF16, V_TOKEN>::stages * Tile<BITS, K_BF16, V_TOKEN>::tokens;
+  }
+}
+
+void decode_chunk_capacity(int bits, int base, int* bf16, int* coded, int* keys_only) {
+  if (bits == 2) capacity_t<2>(base, bf16, coded, keys_only);
+  else capacity_t<4>(base, bf16, coded, keys_only);
+}
 
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s) {
   if (p.d.bits == 2) return p.d.G <= 8 ? launch_base<2, 1>(p, grid_x, s) : launch_base<2, 2>(p, grid_x, s);

@@ -47,25 +47,53 @@ struct AppendParams {
   const uint16_t* v_new;
 };
 
+// Decode work plan of one launch.  Each (layer, row, head) segment is cut into
+// chunks of a fixed token count per segment kind; a CTA processes one chunk.
+//   cbU  BF16 tokens of quantized / keys-only heads   (text, uncoded image, appended)
+//   cqU  coded tokens of quantized heads               (codes for K and V)
+//   cqK  coded tokens of keys-only heads               (BF16 K, coded V)
+//   cbP  BF16 tokens of protected K+V heads
+// Per layer, the host passes the resulting chunk counts of each kind.
+struct DecodePlan {
+  int cbU, cqU, cqK, cbP;
+};
+
+struct DecodeLayer {
+  int appended;
+  int nbU, nqU, nqK, nbP;  // chunks per head of each kind
+  int items_per_row;       // chunks of all heads of one batch row
+  int item_base;           // first work item of this layer in the launch
+};
+
 struct DecodeParams {
   Dims d;
   const char* arena;
   int n_layers;
-  int cb, cq;          // chunk sizes (tokens) for BF16 and coded segments
+  DecodePlan plan;
   int max_items;       // split slots per (layer, row, head) in the workspace
   float scale_log2;    // softmax_scale * log2(e)
   const uint16_t* q;   // [n_layers][B][Hq][128]
   uint16_t* out;       // [n_layers][B][Hq][128]
+  // Fused append (or null): the step's new K/V [n_layers][B][H][128], already
+  // counted in `appended`; the chunk that holds the new position reads it from
+  // here and writes it into the arena.
+  const uint16_t* k_new;
+  const uint16_t* v_new;
+  int total_items;
   uint32_t* counters;  // [n_layers][B][H]
-  float* partials;     // [n_layers][B][H][max_items][G][130]
+  float* partials;     // [n_layers][B][H][max_items][G][132]
   LayerTable lt;
-  int appended[kMaxLayersPerLaunch];
-  int items_per_row[kMaxLayersPerLaunch];
+  DecodeLayer layer[kMaxLayersPerLaunch];
 };
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s);
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s);
+// Tokens per pipeline tile of coded K + coded V (chunk sizes are multiples of it).
+int decode_coded_tile(int bits);
+// Largest chunk (tokens) whose tiles all fit the kernel's pipeline buffer at
+// once, for BF16 chunks, coded chunks and keys-only coded chunks.
+void decode_chunk_capacity(int bits, int base, int* bf16, int* coded, int* keys_only);
 
 }  // namespace hg

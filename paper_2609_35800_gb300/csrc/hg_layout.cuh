@@ -160,44 +160,53 @@ HG_HD int bf16_pos(const Dims& d, int cls, int t) {
 }
 
 // ---------------------------------------------------------------------------
-// Decode work decomposition.  Each (layer, batch row, KV head) is split into
-// chunks of at most cb BF16 tokens and cq coded tokens; a work item is one
-// chunk.  Items of one layer are numbered batch-row major, then head, then
-// BF16 chunks before coded chunks.
+// Decode work decomposition.  Each (layer, batch row, KV head) is cut into
+// chunks: BF16 segments of quantized / keys-only heads into chunks of cbU
+// tokens, coded segments into chunks of cqU (quantized heads) or cqK
+// (keys-only heads) tokens, BF16 segments of protected K+V heads into chunks
+// of cbP tokens.  A work item is one chunk.  Items of one (layer, row) are
+// numbered head by head, BF16 chunks before coded chunks.
 // ---------------------------------------------------------------------------
 HG_HD int cdiv(int a, int b) { return (a + b - 1) / b; }
 
-HG_HD int head_items(const Dims& d, int cls, int appended, int cb, int cq, int* n_bf16_items) {
-  const int lb = ((cls == kProtected) ? d.T : d.T - d.nq) + appended;
-  const int nb = cdiv(lb, cb);
-  const int nqi = (cls == kProtected) ? 0 : cdiv(d.nq, cq);
-  if (n_bf16_items) *n_bf16_items = nb;
-  return nb + nqi;
+struct ChunkCounts {
+  int nbU, nqU, nqK, nbP;
+};
+
+HG_HD ChunkCounts chunk_counts(const Dims& d, int appended, int cbU, int cqU, int cqK, int cbP) {
+  ChunkCounts c;
+  c.nbU = cdiv(d.T - d.nq + appended, cbU);
+  c.nqU = cdiv(d.nq, cqU);
+  c.nqK = cdiv(d.nq, cqK);
+  c.nbP = cdiv(d.T + appended, cbP);
+  return c;
 }
 
-HG_HD int layer_items_per_row(const Dims& d, uint64_t mask, int appended, int cb, int cq) {
-  int tot = 0;
-  for (int h = 0; h < d.H; ++h) tot += head_items(d, head_class(d, mask, h), appended, cb, cq, nullptr);
+// Chunks of one head and how many of them are BF16 chunks.
+HG_HD int head_chunks(int cls, const ChunkCounts& c, int* n_bf16) {
+  if (cls == kProtected) {
+    *n_bf16 = c.nbP;
+    return c.nbP;
+  }
+  *n_bf16 = c.nbU;
+  return c.nbU + (cls == kKeysOnly ? c.nqK : c.nqU);
+}
+
+HG_HD int row_chunks(const Dims& d, uint64_t mask, const ChunkCounts& c) {
+  int tot = 0, nb;
+  for (int h = 0; h < d.H; ++h) tot += head_chunks(head_class(d, mask, h), c, &nb);
   return tot;
 }
 
-// Largest number of items any head can have (appended = max_new_tokens).
-HG_HD int max_head_items(const Dims& d, int cb, int cq) {
-  int a = head_items(d, kQuantized, d.S_new, cb, cq, nullptr);
-  int b = head_items(d, d.keys_only ? kKeysOnly : kProtected, d.S_new, cb, cq, nullptr);
-  return a > b ? a : b;
-}
-
 // Decode workspace: a counter per (layer, row, head), then partial results
-// [layer][row][head][split][G][kD + 2] floats (m, l, o[kD]).
+// [layer][row][head][split][G][kD + 4] floats (m, l, two pad, o[kD]).
 HG_HD uint64_t ws_counter_bytes(const Dims& d, int n_layers) {
   return align_up((uint64_t)n_layers * d.B * d.H * 4);
 }
-HG_HD uint64_t ws_partial_floats_per_split(const Dims& d) { return (uint64_t)d.G * (kD + 2); }
-HG_HD uint64_t ws_bytes(const Dims& d, int n_layers, int cb, int cq) {
+HG_HD uint64_t ws_partial_floats_per_split(const Dims& d) { return (uint64_t)d.G * (kD + 4); }
+HG_HD uint64_t ws_bytes(const Dims& d, int n_layers, int max_items) {
   return ws_counter_bytes(d, n_layers) +
-         align_up((uint64_t)n_layers * d.B * d.H * max_head_items(d, cb, cq) *
-                  ws_partial_floats_per_split(d) * 4);
+         align_up((uint64_t)n_layers * d.B * d.H * max_items * ws_partial_floats_per_split(d) * 4);
 }
 
 }  // namespace hg

@@ -3,9 +3,8 @@ create the cache descriptor, quantize the synthetic prefill and drive decode
 steps.  Marshalling only -- every step of the path runs in the library."""
 import torch
 
-from . import (QuantConfig, Shape, hg_append_kv, hg_cache_create, hg_cache_layout,
-               hg_decode_attention, hg_decode_workspace_size, hg_quantize_kv,
-               hg_workspace_clear, workloads)
+from . import (QuantConfig, Shape, hg_cache_create, hg_cache_layout, hg_decode_step,
+               hg_decode_workspace_size, hg_quantize_kv, hg_workspace_clear, workloads)
 
 
 def shape_of(w):
@@ -60,7 +59,8 @@ class CacheRunner:
 
     def decode_step(self, step, layer_begin=0, layer_count=None, q=None, k_new=None, v_new=None,
                     out=None, softmax_scale=0.0):
-        """Append the step's K/V and run decode attention; returns out [layers][B][Hq][128]."""
+        """Append the step's K/V and run decode attention in one launch; returns
+        out [layers][B][Hq][128]."""
         w = self.w
         n = w.layers if layer_count is None else layer_count
         if k_new is None:
@@ -69,7 +69,6 @@ class CacheRunner:
             q = workloads.step_query(w, step, self.device, n)
         if out is None:
             out = torch.empty_like(q)
-        hg_append_kv(self.cache, layer_begin, n, k_new, v_new)
-        hg_decode_attention(self.cache, layer_begin, n, q, out, softmax_scale, self.ws,
-                            self.ws_bytes)
+        hg_decode_step(self.cache, layer_begin, n, q, k_new, v_new, out, softmax_scale, self.ws,
+                       self.ws_bytes)
         return out

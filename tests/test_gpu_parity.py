@@ -56,7 +56,7 @@ def _workload(case):
                      seed=7, protected=prot, residual=R)
 
 
-def _run_and_check(w, layer_batched=True):
+def _run_and_check(w, layer_batched=True, fused=False):
     runner = CacheRunner(w)
     kept = runner.quantize_all(keep=True)
     torch.cuda.synchronize()
@@ -67,18 +67,22 @@ def _run_and_check(w, layer_batched=True):
         o = oracle_layer(runner, l, kb, vb)
         check_arena_layer(runner, l, kb, vb, o, arena=arena)
         outs.append(o)
-    # decode steps (append + attention), compared after every step
+    # decode steps (append + attention, or the fused step), compared after every step
     app_k = [[] for _ in range(w.layers)]
     app_v = [[] for _ in range(w.layers)]
     for step in range(w.decode_steps):
         k_new, v_new = wl.step_new_kv(w, step, "cuda")
         q = wl.step_query(w, step, "cuda")
         out = torch.empty_like(q)
-        hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
-        if layer_batched:
+        if fused:
+            hg.hg_decode_step(runner.cache, 0, w.layers, q, k_new, v_new, out, SIGMA, runner.ws,
+                              runner.ws_bytes)
+        elif layer_batched:
+            hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
             hg.hg_decode_attention(runner.cache, 0, w.layers, q, out, SIGMA, runner.ws,
                                    runner.ws_bytes)
         else:
+            hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
             for l in range(w.layers):
                 hg.hg_decode_attention(runner.cache, l, 1, q[l], out[l], SIGMA, runner.ws,
                                        runner.ws_bytes)
@@ -104,6 +108,45 @@ def test_tiny_workload_parity():
 @pytest.mark.parametrize("case", [CASES[0], CASES[3], CASES[6]], ids=["minmax", "kivi", "akvq"])
 def test_per_layer_launches(case):
     _run_and_check(_workload(case), layer_batched=False)
+
+
+@pytest.mark.parametrize("case", [CASES[0], CASES[2], CASES[3], CASES[6], CASES[12], CASES[13]],
+                         ids=["minmax", "minmax_konly", "kivi", "akvq", "g16", "long"])
+def test_fused_decode_step(case):
+    """hg_decode_step appends and attends in one launch: same attention as the
+    oracle after every step, and the new tokens end up in the cache."""
+    w = _workload(case)
+    runner, kept, outs = _run_and_check(w, fused=True)
+    assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
+    Tt = w.seq_len + w.decode_steps
+    k32 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
+    v32 = torch.empty_like(k32)
+    for l in range(w.layers):
+        hg.hg_dequantize_kv(runner.cache, l, k32, v32, True)
+        torch.cuda.synchronize()
+        for step in range(w.decode_steps):
+            k_new, v_new = wl.step_new_kv(w, step, "cuda")
+            assert np.array_equal(k32[:, :, w.seq_len + step].cpu().numpy(),
+                                  k_new[l].float().cpu().numpy())
+            assert np.array_equal(v32[:, :, w.seq_len + step].cpu().numpy(),
+                                  v_new[l].float().cpu().numpy())
+
+
+def test_decode_step_capacity_and_rollback():
+    w = _workload(CASES[1])
+    runner = CacheRunner(w)
+    runner.quantize_all()
+    q = wl.step_query(w, 0, "cuda")
+    out = torch.empty_like(q)
+    k_new, v_new = wl.step_new_kv(w, 0, "cuda")
+    for _ in range(w.decode_steps):
+        hg.hg_decode_step(runner.cache, 0, w.layers, q, k_new, v_new, out, SIGMA, runner.ws,
+                          runner.ws_bytes)
+    with pytest.raises(hg.HGError) as e:
+        hg.hg_decode_step(runner.cache, 0, w.layers, q, k_new, v_new, out, SIGMA, runner.ws,
+                          runner.ws_bytes)
+    assert e.value.status == 5
+    assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
 
 
 @pytest.mark.parametrize("case", [CASES[1], CASES[2], CASES[4], CASES[5], CASES[7]],
