@@ -191,8 +191,20 @@ hg_status hg_append_kv(hg_cache *cache, int32_t layer_begin, int32_t layer_count
 hg_status hg_decode_workspace_size(const hg_cache *cache, int32_t layer_count, size_t *bytes);
 
 /* Zero a workspace (cudaMemsetAsync).  Required once before its first use;
- * decode attention leaves it zeroed again on completion. */
+ * decode attention leaves it zeroed again on completion.  Layout: a 512-byte
+ * header holding a status word at byte 0, split counters, split partials. */
 hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
+
+/* Health of the decode launches that used a workspace: waits for `stream`,
+ * then copies the workspace's status word to *status (host).  0 = healthy;
+ * bit 0 (1) = a CTA's wait for a tile of its data ran out (about 2^20 polls of
+ * the tile's mbarrier), after which that CTA skipped its remaining work and
+ * let the copies it had issued land before exiting.  Decode CTAs wait with a
+ * bound instead of hanging; after a non-zero status the outputs of the
+ * launches since the last clear are undefined and the workspace must be
+ * cleared (hg_workspace_clear) before it is used again.  (Failure detection
+ * of the kernels; the paper has no counterpart.) */
+hg_status hg_workspace_status(const void *workspace, uint32_t *status, hg_stream_t stream);
 
 /* Grouped-query decode attention of one step over layers
  * [layer_begin, +layer_count), reading packed codes and BF16 entries in one

@@ -18,7 +18,8 @@ __all__ = [
     "HG_HEAD_QUANTIZED", "HG_HEAD_KEYS_ONLY", "HG_HEAD_PROTECTED",
     "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
     "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
-    "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_decode_attention",
+    "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_workspace_status",
+    "hg_decode_attention",
     "hg_decode_step", "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem",
     "hg_status_string",
     "library", "library_path",
@@ -97,6 +98,7 @@ def library():
         "hg_append_kv": ([P, i32, i32, P, P, P], st),
         "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
         "hg_workspace_clear": ([P, sz, P], st),
+        "hg_workspace_status": ([P, ctypes.POINTER(ctypes.c_uint32), P], st),
         "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_step": ([P, i32, i32, P, P, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_attention_noalloc": ([P, i32, i32, P, P, ctypes.c_float, P], st),
@@ -232,6 +234,14 @@ def hg_workspace_clear(workspace, nbytes=None, stream=None):
         nbytes = workspace.numel() * workspace.element_size()
     _check(library().hg_workspace_clear(_ptr(workspace), nbytes, _stream(stream)),
            "hg_workspace_clear")
+
+
+def hg_workspace_status(workspace, stream=None):
+    """Status word of a decode workspace (waits for the stream); 0 = healthy."""
+    out = ctypes.c_uint32(0)
+    _check(library().hg_workspace_status(_ptr(workspace), ctypes.byref(out), _stream(stream)),
+           "hg_workspace_status")
+    return out.value
 
 
 def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, workspace,

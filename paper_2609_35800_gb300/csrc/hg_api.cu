@@ -2,6 +2,8 @@
 // validation, arena layout, decode work decomposition and kernel launches.
 // Every check runs before anything is enqueued; no device memory is
 // allocated here.
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -27,6 +29,10 @@ struct hg_cache {
   char* arena;
   size_t arena_bytes;
   size_t needed_bytes;
+  // The arena as a BF16 tensor [arena_bytes / 256][128] for the decode
+  // kernel's TMA loads; encoded by the first decode call.
+  mutable CUtensorMap arena_map;
+  mutable bool arena_map_ready;
 };
 
 namespace {
@@ -210,6 +216,43 @@ size_t ws_size_for(const hg_cache* c, int begin, int count) {
 }
 
 hg_status cuda_status(cudaError_t e) { return e == cudaSuccess ? HG_OK : HG_ERR_CUDA; }
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link
+// against the driver library).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* f = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &f, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(f);
+  }
+  return fn;
+}
+
+// Every BF16 token row of the arena is a 256-byte row at a 256-byte offset:
+// the arena is viewed as a BF16 tensor of arena_bytes / 256 rows of 128
+// channels, read in boxes of kArenaBoxRows rows x 64 channels (128 bytes, the
+// span of the 128-byte swizzle).
+hg_status arena_tensor_map(const hg_cache* c) {
+  if (c->arena_map_ready) return HG_OK;
+  const uint64_t rows = c->arena_bytes / 256;
+  if (rows == 0 || rows > (uint64_t)INT32_MAX) return HG_ERR_UNSUPPORTED;
+  PFN_cuTensorMapEncodeTiled_v12000 encode = tensor_map_encoder();
+  if (!encode) return HG_ERR_CUDA;
+  const cuuint64_t dims[2] = {(cuuint64_t)kD, (cuuint64_t)rows};
+  const cuuint64_t strides[1] = {256};
+  const cuuint32_t box[2] = {64, (cuuint32_t)kArenaBoxRows};
+  const cuuint32_t estrides[2] = {1, 1};
+  const CUresult r = encode(&c->arena_map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, c->arena, dims, strides, box,
+                            estrides, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+  if (r != CUDA_SUCCESS) return HG_ERR_CUDA;
+  c->arena_map_ready = true;
+  return HG_OK;
+}
 
 void fill_table(const hg_cache* c, int begin, int count, LayerTable* t) {
   for (int i = 0; i < count; ++i) {
@@ -406,6 +449,18 @@ hg_status hg_workspace_clear(void* ws, size_t bytes, hg_stream_t stream) {
   return cuda_status(cudaMemsetAsync(ws, 0, bytes, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+hg_status hg_workspace_status(const void* ws, uint32_t* status, hg_stream_t stream) {
+  if (!ws || !status) return HG_ERR_INVALID_ARG;
+  if (!aligned16(ws)) return HG_ERR_ALIGNMENT;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  uint32_t v = 0;
+  cudaError_t e = cudaMemcpyAsync(&v, ws, sizeof v, cudaMemcpyDeviceToHost, s);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(s);
+  if (e != cudaSuccess) return HG_ERR_CUDA;
+  *status = v;
+  return HG_OK;
+}
+
 }  // extern "C"
 
 namespace {
@@ -417,6 +472,8 @@ hg_status decode_launch(const hg_cache* c, int32_t layer_begin, int32_t layer_co
                         const void* k_new, const void* v_new, void* out, float softmax_scale,
                         void* ws, size_t ws_bytes_given, hg_stream_t stream) {
   const Dims& d = c->d;
+  const hg_status mst = arena_tensor_map(c);
+  if (mst != HG_OK) return mst;
   const float scale = softmax_scale > 0.f ? softmax_scale : 1.0f / std::sqrt((float)kD);
   const size_t layer_elems = (size_t)d.B * d.Hq * kD;
   const size_t kv_elems = (size_t)d.B * d.H * kD;
@@ -436,8 +493,11 @@ hg_status decode_launch(const hg_cache* c, int32_t layer_begin, int32_t layer_co
       p.k_new = static_cast<const uint16_t*>(k_new) + (size_t)done * kv_elems;
       p.v_new = static_cast<const uint16_t*>(v_new) + (size_t)done * kv_elems;
     }
-    p.counters = static_cast<uint32_t*>(ws);
-    p.partials = reinterpret_cast<float*>(static_cast<char*>(ws) + ws_counter_bytes(d, n));
+    char* wsb = static_cast<char*>(ws);
+    p.arena_map = c->arena_map;
+    p.status = reinterpret_cast<uint32_t*>(wsb);
+    p.counters = reinterpret_cast<uint32_t*>(wsb + kWsHeaderBytes);
+    p.partials = reinterpret_cast<float*>(wsb + kWsHeaderBytes + ws_counter_bytes(d, n));
     fill_table(c, layer_begin + done, n, &p.lt);
     int total = 0;
     for (int i = 0; i < n; ++i) {

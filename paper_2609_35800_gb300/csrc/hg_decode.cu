@@ -7,8 +7,11 @@
 // keys with coded values.  The only branch on the mask or the image span is
 // therefore taken once per CTA.
 //
-// Tiles of the chunk stream through a cp.async pipeline in a 64 KB shared
-// buffer (two to four stages depending on the tile size).  Each warp owns 16-token slices and computes, with mma.sync
+// Tiles of the chunk stream through a TMA pipeline in a 64 KB shared buffer
+// (two to four stages depending on the tile size, one mbarrier each): BF16
+// rows arrive as tensor-map boxes with the 128-byte swizzle, packed codes and
+// metadata as one bulk copy per array, all issued by one thread.  Each warp
+// owns 16-token slices and computes, with mma.sync
 // m16n8k16 (BF16 in, fp32 accumulate):
 //   S^T[token][query] = K . q     A = keys (BF16 via ldmatrix, or codes
 //                                 expanded exactly to BF16 in registers),
@@ -47,11 +50,15 @@ constexpr int kBufBytes = 65536;   // pipeline buffer (stages of one tile each)
 constexpr int kBf16Tile = 64;      // tokens per tile of BF16 rows (K 16 KB + V 16 KB)
 constexpr int kMixTile = 64;       // tokens per tile of BF16 keys + coded values
 constexpr int kPartialStride = kD + 4;  // m, l, 2 pad, o[128]: rows of 528 bytes (16-byte multiple)
-constexpr int kQOff = 0;                      // float q[16][128]
-constexpr int kZsumOff = kMaxG * kD * 4;      // float sum(q)[16]
-constexpr int kStageOff = kZsumOff + 256;
-constexpr int kSmemBytes = kStageOff + kBufBytes;
+// Shared memory, from a 1024-byte aligned base (swizzled TMA boxes need it).
+constexpr int kStageOff = 0;                    // pipeline buffer
+constexpr int kQOff = kStageOff + kBufBytes;     // float q[16][128]
+constexpr int kBarOff = kQOff + kMaxG * kD * 4;  // mbarrier per stage (4), abort flag, merge flag
+constexpr int kSmemUsed = kBarOff + 64;
+constexpr int kSmemBytes = kSmemUsed + 1024;     // + alignment slack
+constexpr int kMaxStages = 4;
 constexpr unsigned kFull = 0xffffffffu;
+constexpr uint32_t kSpinLimit = 1u << 20;       // mbarrier polls before a wait is declared stuck
 
 enum KMode { K_BF16 = 0, K_TOKEN = 1, K_KIVI = 2 };
 enum VMode { V_BF16 = 0, V_TOKEN = 1, V_KIVI = 2 };
@@ -67,57 +74,18 @@ __host__ __device__ constexpr int coded_tile(int bits) { return bits == 2 ? 256 
 struct Seg {
   const char* k;   // BF16 key rows (K_BF16)
   const char* v;   // BF16 value rows (V_BF16)
+  int k_row0;      // arena tensor-map row of key token 0 (K_BF16)
+  int v_row0;      // arena tensor-map row of value token 0 (V_BF16)
   const char* kc;  // key codes
   const char* km;  // key metadata
   const char* vc;  // value codes
   const char* vm;  // value metadata
-  // Fused append: BF16 row new_pos of this segment comes from these input
-  // rows instead of the arena (new_pos < 0: none).
+  // Fused append: BF16 row new_pos of this segment is stored from these
+  // input rows into the arena before its tile is loaded (new_pos < 0: none).
   int new_pos;
   const char* k_new;
   const char* v_new;
 };
-
-// SLOT bytes from src into a linear slot; only the first valid_bytes are read,
-// the rest of the slot is zero-filled.
-template <int SLOT>
-__device__ __forceinline__ void copy_linear(uint32_t dst, const char* src, int valid_bytes, int tid) {
-#pragma unroll
-  for (int off = tid * 16, i = 0; i < (SLOT + kThreads * 16 - 1) / (kThreads * 16); ++i, off += kThreads * 16) {
-    if (off < SLOT) {
-      int n = valid_bytes - off;
-      n = n < 0 ? 0 : (n > 16 ? 16 : n);
-      cp_async16(dst + off, n > 0 ? src + off : src, n);
-    }
-  }
-}
-
-// nvalid BF16 rows (256 B each) into a 64-row tile, 16-byte chunks swizzled by
-// (row & 7) so that ldmatrix reads are conflict free; missing rows are zero.
-// Thread t always moves chunk (t & 15) of rows (t >> 4) + 8 i.
-// Row sub_row (if >= 0) is read from sub instead (a new decode token).
-__device__ __forceinline__ void copy_rows_swizzled(uint32_t dst, const char* src, int nvalid,
-                                                   int tid, int sub_row, const char* sub) {
-  const int r0 = tid >> 4, c = tid & 15;
-  const uint32_t d0 = dst + r0 * 256 + ((c ^ (r0 & 7)) << 4);
-  const char* s0 = src + r0 * 256 + c * 16;
-#pragma unroll
-  for (int i = 0; i < 64 / (kThreads / 16); ++i) {
-    const int r = r0 + (kThreads / 16) * i;
-    const bool ok = r < nvalid;
-    const char* from = (r == sub_row) ? sub + c * 16 : s0 + i * (kThreads / 16) * 256;
-    cp_async16(d0 + i * (kThreads / 16) * 256, ok ? from : src, ok ? 16 : 0);
-  }
-}
-
-// cp.async.wait_group with a run-time count in [0, S).
-template <int S>
-__device__ __forceinline__ void cp_async_wait_pending(int n) {
-  if (S > 3 && n >= 3) { cp_async_wait<3>(); return; }
-  if (S > 2 && n == 2) { cp_async_wait<2>(); return; }
-  if (n == 1) { cp_async_wait<1>(); return; }
-  cp_async_wait<0>();
-}
 
 template <int BITS>
 __device__ __forceinline__ uint32_t pair2(uint32_t x) {  // codes at bits [0,b) and [16,16+b)
@@ -168,29 +136,66 @@ struct Tile {
   static constexpr int km_off = kc_off + kc_bytes;
   static constexpr int vc_off = km_off + km_bytes;
   static constexpr int vm_off = vc_off + vc_bytes;
-  static constexpr int stage_bytes = ((vm_off + vm_bytes + 127) / 128) * 128;
-  static constexpr int stages = (kBufBytes / stage_bytes) > 4 ? 4 : (kBufBytes / stage_bytes);
+  // stages start on 1024-byte boundaries (swizzled BF16 boxes)
+  static constexpr int stage_bytes = ((vm_off + vm_bytes + 1023) / 1024) * 1024;
+  static constexpr int stages = (kBufBytes / stage_bytes) > kMaxStages ? kMaxStages : (kBufBytes / stage_bytes);
   static_assert(stages >= 2, "a tile must fit twice in the pipeline buffer");
+  static_assert(tokens % kArenaBoxRows == 0, "BF16 tiles are whole TMA boxes");
+  static_assert(VM != V_BF16 || vc_off % 1024 == 0, "swizzled value boxes start on 1024-byte boundaries");
 };
 
+// One tile into a stage, issued by a single thread: the expected byte count
+// on the stage's mbarrier, then the copies.  A BF16 operand of R rows lands
+// as two column halves of R x 128 bytes (channels 0-63, 64-127), each written
+// by TMA boxes of kArenaBoxRows rows with the 128-byte swizzle (16-byte chunk
+// c of row r at chunk c ^ (r % 8)); rows past the chunk end are loaded too and
+// ignored or zeroed by the consumers.  Packed codes and metadata arrive as one
+// bulk copy per array (metadata rounded up to 16 bytes: the arena pads every
+// metadata row to 16 bytes); bytes past nvalid tokens are left stale.
 template <int BITS, int KM, int VM>
-__device__ __forceinline__ void issue_tile(uint32_t st, const Seg& sg, int t0, int nvalid, int tid) {
+__device__ __forceinline__ void issue_tile(uint32_t st, uint32_t bar, const Seg& sg, int t0, int nvalid,
+                                           const CUtensorMap* map) {
   using TL = Tile<BITS, KM, VM>;
+  constexpr int kmb = (KM == K_TOKEN) ? 8 : 32;
+  constexpr int vmb = (VM == V_TOKEN) ? 8 : 32;
+  constexpr int kBox = kArenaBoxRows * 128;  // bytes of one box
+  const int boxes = (nvalid + kArenaBoxRows - 1) / kArenaBoxRows;
+  const uint32_t kc_bytes = (KM == K_BF16) ? boxes * 2 * kBox : nvalid * 16 * BITS;
+  const uint32_t km_bytes = (KM == K_BF16) ? 0u : (uint32_t)((nvalid * kmb + 15) & ~15);
+  const uint32_t vc_bytes = (VM == V_BF16) ? boxes * 2 * kBox : nvalid * 16 * BITS;
+  const uint32_t vm_bytes = (VM == V_BF16) ? 0u : (uint32_t)((nvalid * vmb + 15) & ~15);
+  mbar_arrive_expect_tx(bar, kc_bytes + km_bytes + vc_bytes + vm_bytes);
   if (KM == K_BF16) {
-    copy_rows_swizzled(st + TL::kc_off, sg.k + (size_t)t0 * 256, nvalid, tid, sg.new_pos - t0, sg.k_new);
+    for (int bx = 0; bx < boxes; ++bx)
+      for (int hf = 0; hf < 2; ++hf)
+        tma_load_2d(st + TL::kc_off + hf * (TL::tokens * 128) + bx * kBox, map, hf * 64,
+                    sg.k_row0 + t0 + bx * kArenaBoxRows, bar);
   } else {
-    copy_linear<TL::kc_bytes>(st + TL::kc_off, sg.kc + (size_t)t0 * 16 * BITS, nvalid * 16 * BITS, tid);
-    // KIVI-style key metadata: one (scale, zero) per channel per 32 tokens = 32 B per token
-    constexpr int kmb = (KM == K_TOKEN) ? 8 : 32;
-    copy_linear<TL::km_bytes>(st + TL::km_off, sg.km + (size_t)t0 * kmb, nvalid * kmb, tid);
+    bulk_g2s(st + TL::kc_off, sg.kc + (size_t)t0 * 16 * BITS, kc_bytes, bar);
+    bulk_g2s(st + TL::km_off, sg.km + (size_t)t0 * kmb, km_bytes, bar);
   }
   if (VM == V_BF16) {
-    copy_rows_swizzled(st + TL::vc_off, sg.v + (size_t)t0 * 256, nvalid, tid, sg.new_pos - t0, sg.v_new);
+    for (int bx = 0; bx < boxes; ++bx)
+      for (int hf = 0; hf < 2; ++hf)
+        tma_load_2d(st + TL::vc_off + hf * (TL::tokens * 128) + bx * kBox, map, hf * 64,
+                    sg.v_row0 + t0 + bx * kArenaBoxRows, bar);
   } else {
-    copy_linear<TL::vc_bytes>(st + TL::vc_off, sg.vc + (size_t)t0 * 16 * BITS, nvalid * 16 * BITS, tid);
-    constexpr int vmb = (VM == V_TOKEN) ? 8 : 32;
-    copy_linear<TL::vm_bytes>(st + TL::vm_off, sg.vm + (size_t)t0 * vmb, nvalid * vmb, tid);
+    bulk_g2s(st + TL::vc_off, sg.vc + (size_t)t0 * 16 * BITS, vc_bytes, bar);
+    bulk_g2s(st + TL::vm_off, sg.vm + (size_t)t0 * vmb, vm_bytes, bar);
   }
+}
+
+// Bounded wait for a phase of a stage's mbarrier.  On timeout, or once another
+// warp gave up, marks the CTA aborted, records the failure in the workspace
+// status word and returns false (the caller skips the tile's work).
+__device__ __forceinline__ bool wait_tile(uint32_t bar, uint32_t parity, volatile int* abort, uint32_t* status) {
+  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if (*abort) return false;
+  }
+  *abort = 1;
+  atomicOr(status, kStatusWaitTimeout);
+  return false;
 }
 
 // ---------------------------------------------------------------------------
@@ -388,10 +393,9 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
     // ---------------- scores ----------------
     if (KM == K_BF16) {
       const int tok0 = u * 16;
-      const int mat = lane >> 3, r = lane & 7;
-      const int row = tok0 + r + 8 * (mat & 1);
-      const uint32_t rbase = st_u32 + TL::kc_off + row * 256;
-      const int rsw = row & 7, ch = mat >> 1;
+      const int row = tok0 + (lane & 7) + 8 * ((lane >> 3) & 1);
+      const uint32_t rbase = st_u32 + TL::kc_off + row * 128;
+      const int rsw = lane & 7, ch = lane >> 4;  // row % 8; second 8 channels of the k-step
       float acc2[NT][4];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt)
@@ -400,7 +404,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         uint32_t a[4];
-        ldsm_x4(a, rbase + (((2 * j + ch) ^ rsw) << 4));
+        ldsm_x4(a, rbase + (j >> 2) * (TL::tokens * 128) + (((2 * (j & 3) + ch) ^ rsw) << 4));
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
           mma_bf16((j & 1) ? acc2[nt] : acc[0][nt], a, qb[nt][j][0], qb[nt][j][1]);
@@ -583,19 +587,32 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         uint32_t b[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) pfrag(p[nt], 1.f, 1.f, b[nt]);
-        const int mat = lane >> 3, r = lane & 7;
-        const int row = tok0 + r + 8 * (mat >> 1);
-        const uint32_t rbase = st_u32 + TL::vc_off + row * 256;
-        const int rsw = row & 7, ch = mat & 1;
+        if (tok0 + 16 > nvalid) {
+          // rows past the end hold whatever follows in the arena: zero them so
+          // that 0 * (non-finite) cannot reach the accumulators
+          for (int i = lane; i < (tok0 + 16 - nvalid) * 16; i += 32) {
+            const int rr = nvalid + (i >> 4), c = i & 15;
+            *reinterpret_cast<uint4*>(const_cast<char*>(st) + TL::vc_off + (c >> 3) * (TL::tokens * 128) +
+                                      rr * 128 + (c & 7) * 16) = make_uint4(0u, 0u, 0u, 0u);
+          }
+          fence_proxy_async_shared();  // the stage is refilled by TMA later
+          __syncwarp();
+        }
+        const int row = tok0 + (lane & 7) + 8 * (lane >> 4);
+        const uint32_t rbase = st_u32 + TL::vc_off + row * 128;
+        const int rsw = lane & 7, ch = (lane >> 3) & 1;
 #pragma unroll
         for (int mt = 0; mt < 8; ++mt) {
           uint32_t a[4];
-          ldsm_x4_trans(a, rbase + (((2 * mt + ch) ^ rsw) << 4));
+          ldsm_x4_trans(a, rbase + (mt >> 2) * (TL::tokens * 128) + (((2 * (mt & 3) + ch) ^ rsw) << 4));
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
         }
       } else if (VM == V_TOKEN) {
-        const float2 vg = vm2[tok0 + g], vg8 = vm2[tok0 + g + 8];
+        // metadata past the end of the tile is stale: its factors are zeroed
+        const bool ok0 = tok0 + g < nvalid, ok8 = tok0 + g + 8 < nvalid;
+        const float2 vg = ok0 ? vm2[tok0 + g] : make_float2(0.f, 0.f);
+        const float2 vg8 = ok8 ? vm2[tok0 + g + 8] : make_float2(0.f, 0.f);
         uint32_t b[NT][4];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -658,7 +675,10 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         const float4* vrow_g8 = reinterpret_cast<const float4*>(vm2 + (tok0 + g + 8) * 4);
         float sv_g[4], zv_g[4], sv_g8[4], zv_g8[4];
         {
-          const float4 a0 = vrow_g[0], a1 = vrow_g[1], b0 = vrow_g8[0], b1 = vrow_g8[1];
+          const float4 zf = make_float4(0.f, 0.f, 0.f, 0.f);  // stale metadata past the end
+          const bool ok0 = tok0 + g < nvalid, ok8 = tok0 + g + 8 < nvalid;
+          const float4 a0 = ok0 ? vrow_g[0] : zf, a1 = ok0 ? vrow_g[1] : zf;
+          const float4 b0 = ok8 ? vrow_g8[0] : zf, b1 = ok8 ? vrow_g8[1] : zf;
           sv_g[0] = a0.x; zv_g[0] = a0.y; sv_g[1] = a0.z; zv_g[1] = a0.w;
           sv_g[2] = a1.x; zv_g[2] = a1.y; sv_g[3] = a1.z; zv_g[3] = a1.w;
           sv_g8[0] = b0.x; zv_g8[0] = b0.y; sv_g8[1] = b0.z; zv_g8[1] = b0.w;
@@ -712,7 +732,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 // into shared memory (m, l, o[q][channel]).
 // ---------------------------------------------------------------------------
 template <int BITS, int NT, int KM, int VM, bool ROT>
-__device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int te, float scale_log2,
+__device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int te, const DecodeParams& p,
                                          const uint16_t* qg, int G, float* red_m, float* red_l,
                                          float* red_o) {
   using TL = Tile<BITS, KM, VM>;
@@ -722,18 +742,20 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   float* q_s = reinterpret_cast<float*>(smem + kQOff);
   char* stages = smem + kStageOff;
 
-  // Every tile that fits the buffer goes in flight before anything else (the
-  // work plan sizes chunks to fit); later tiles, if any, reuse slots as the
-  // ring advances.
+  // Every tile that fits the buffer goes in flight before anything else;
+  // later tiles, if any, reuse stages as the ring advances.  Tile i uses stage
+  // i % STAGES and phase i / STAGES of that stage's mbarrier.
   constexpr int STAGES = TL::stages;
+  const float scale_log2 = p.scale_log2;
   const int n_tiles = (te - tb + TL::tokens - 1) / TL::tokens;
   const uint32_t st0 = smem_u32(stages);
-  int issued = n_tiles < STAGES ? n_tiles : STAGES;
-  for (int s = 0; s < issued; ++s) {
-    issue_tile<BITS, KM, VM>(st0 + s * TL::stage_bytes, sg, tb + s * TL::tokens,
-                             min(TL::tokens, te - tb - s * TL::tokens), tid);
-    cp_async_commit();
-  }
+  const uint32_t bars = smem_u32(smem + kBarOff);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + kBarOff + 8 * kMaxStages);
+  int issued = n_tiles < STAGES ? n_tiles : STAGES;  // meaningful in thread 0
+  if (tid == 0)
+    for (int s = 0; s < issued; ++s)
+      issue_tile<BITS, KM, VM>(st0 + s * TL::stage_bytes, bars + 8 * s, sg, tb + s * TL::tokens,
+                               min(TL::tokens, te - tb - s * TL::tokens), &p.arena_map);
 
   // Queries of this KV head's group (fp32, rows >= G zero), rotated for
   // AKVQ-style coded keys.
@@ -794,20 +816,29 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   }
 
   for (int it = 0; it < n_tiles; ++it) {
-    // tile `it` has landed once at most issued - it - 1 groups are pending
-    cp_async_wait_pending<STAGES>(issued - it - 1);
+    const int st = it % STAGES;
+    const bool ok = __all_sync(kFull, !*abort && wait_tile(bars + 8 * st, (it / STAGES) & 1, abort, p.status));
     __syncthreads();
-    if (it > 0 && issued < n_tiles) {  // refill the slot of tile it - 1
-      issue_tile<BITS, KM, VM>(st0 + (issued % STAGES) * TL::stage_bytes, sg, tb + issued * TL::tokens,
-                               min(TL::tokens, te - tb - issued * TL::tokens), tid);
-      cp_async_commit();
+    if (tid == 0 && it > 0 && issued < n_tiles && !*abort) {  // refill the stage of tile it - 1
+      fence_proxy_async_shared();
+      issue_tile<BITS, KM, VM>(st0 + (issued % STAGES) * TL::stage_bytes, bars + 8 * (issued % STAGES), sg,
+                               tb + issued * TL::tokens, min(TL::tokens, te - tb - issued * TL::tokens),
+                               &p.arena_map);
       ++issued;
     }
-    compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + (it % STAGES) * TL::stage_bytes,
-                                        min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s,
-                                        s1, s0, scale_log2, warp, lane);
+    if (ok)
+      compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + st * TL::stage_bytes,
+                                          min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s,
+                                          s1, s0, scale_log2, warp, lane);
   }
-  cp_async_wait<0>();
+  if (tid == 0 && *abort) {
+    // A stage is refilled only after its previous tile landed, so only the
+    // last STAGES tiles can still be in flight: let them land (bounded)
+    // before the buffer is reused or the CTA exits.
+    for (int t = (issued > STAGES ? issued - STAGES : 0); t < issued; ++t)
+      for (uint32_t i = 0; i < kSpinLimit && !mbar_try_wait(bars + 8 * (t % STAGES), (t / STAGES) & 1); ++i) {
+      }
+  }
   __syncthreads();  // stage buffers are reused for the reduction below
 
   // ---- per-warp results: reduce l and the value-zero terms over the 8 rows g ----
@@ -858,10 +889,19 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
 template <int BITS, int NT, int BASE>
 __global__ void __launch_bounds__(kThreads, NT == 1 ? 3 : 2)
 decode_kernel(const __grid_constant__ DecodeParams p) {
-  extern __shared__ __align__(128) char smem[];
+  extern __shared__ __align__(1024) char smem_raw[];
+  // swizzled TMA boxes need 1024-byte aligned shared addresses
+  char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const Dims& d = p.d;
   const int item = blockIdx.x;
   if (item >= p.total_items) return;
+  if (threadIdx.x == 0) {
+    const uint32_t bars = smem_u32(smem + kBarOff);
+    for (int s = 0; s < kMaxStages; ++s) mbar_init(bars + 8 * s, 1);
+    mbar_init_fence();
+    *reinterpret_cast<volatile int*>(smem + kBarOff + 8 * kMaxStages) = 0;  // abort flag
+    prefetch_tensormap(&p.arena_map);
+  }
   int li = 0;
   while (li + 1 < p.n_layers && p.layer[li + 1].item_base <= item) ++li;
   const DecodeLayer& L = p.layer[li];
@@ -902,43 +942,52 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   sg.k = sg.v = sg.kc = sg.km = sg.vc = sg.vm = nullptr;
   sg.new_pos = -1;
   sg.k_new = sg.v_new = nullptr;
+  sg.k_row0 = sg.v_row0 = 0;
   if (!coded) {
     sg.k = Lb + hd.kb + b * hd.kb_bs;
     sg.v = Lb + hd.vb + b * hd.kb_bs;
+    sg.k_row0 = (int)((p.lt.base[li] + hd.kb + b * hd.kb_bs) >> 8);
+    sg.v_row0 = (int)((p.lt.base[li] + hd.vb + b * hd.kb_bs) >> 8);
     const int pos = hd.bf16_prefill + L.appended - 1;  // the step's new token
     if (p.k_new && pos >= tb && pos < te) {
       const size_t row = (((size_t)li * d.B + b) * d.H + h) * kD;
       sg.new_pos = pos;
       sg.k_new = reinterpret_cast<const char*>(p.k_new + row);
       sg.v_new = reinterpret_cast<const char*>(p.v_new + row);
-      // this CTA alone owns the position in this launch: store it in the arena
+      // this CTA alone owns the position in this launch: store it in the
+      // arena, ordered before the TMA reads of its tile
       if (threadIdx.x < 32) {
         const int c = threadIdx.x & 15;
         const char* src = (threadIdx.x < 16) ? sg.k_new : sg.v_new;
         char* dst = const_cast<char*>((threadIdx.x < 16) ? sg.k : sg.v) + (size_t)pos * 256;
         *reinterpret_cast<uint4*>(dst + c * 16) = ldg16(src + c * 16);
+        fence_proxy_async_global();
       }
     }
-    run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+    __syncthreads();  // barriers initialised, new row stored
+    run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
   } else if (hd.cls == kKeysOnly) {
+    __syncthreads();  // barriers initialised
     sg.k = Lb + hd.kimg + b * hd.kimg_bs;
+    sg.k_row0 = (int)((p.lt.base[li] + hd.kimg + b * hd.kimg_bs) >> 8);
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_BF16, V_KIVI, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_BF16, V_KIVI, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
     else
-      run_item<BITS, NT, K_BF16, V_TOKEN, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_BF16, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
   } else {
+    __syncthreads();  // barriers initialised
     sg.kc = Lb + hd.kq + b * hd.kq_bs;
     sg.km = Lb + hd.kqm + b * hd.kqm_bs;
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_KIVI, V_KIVI, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_KIVI, V_KIVI, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
     else if (BASE == kAkvq)
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, true>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, true>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
     else
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, false>(smem, sg, tb, te, p.scale_log2, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
   }
   __syncthreads();
 
@@ -1061,6 +1110,10 @@ cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
   if (dev < 64 && !configured[dev]) {
     e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              kSmemBytes);
+    if (e != cudaSuccess) return e;
+    // three CTAs of 75 KB share an SM: ask for the full shared-memory carve-out
+    e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                             cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }

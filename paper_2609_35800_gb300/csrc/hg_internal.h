@@ -1,6 +1,7 @@
 // Launch parameter blocks and launcher entry points shared between the host
 // runtime (hg_api.cu) and the kernel translation units.
 #pragma once
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -66,6 +67,10 @@ struct DecodeLayer {
 };
 
 struct DecodeParams {
+  // The arena as a two-dimensional BF16 tensor [arena_bytes / 256][128]: every
+  // BF16 token row of the cache is one row of it.  Boxes of kArenaBoxRows rows
+  // x 64 channels, 128-byte swizzle.
+  CUtensorMap arena_map;
   Dims d;
   const char* arena;
   int n_layers;
@@ -80,11 +85,15 @@ struct DecodeParams {
   const uint16_t* k_new;
   const uint16_t* v_new;
   int total_items;
+  uint32_t* status;    // workspace status word (kStatus* bits; zero while healthy)
   uint32_t* counters;  // [n_layers][B][H]
   float* partials;     // [n_layers][B][H][max_items][G][132]
   LayerTable lt;
   DecodeLayer layer[kMaxLayersPerLaunch];
 };
+
+// BF16 rows per TMA box of the arena tensor map.
+constexpr int kArenaBoxRows = 32;
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s);
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);

@@ -198,14 +198,17 @@ HG_HD int row_chunks(const Dims& d, uint64_t mask, const ChunkCounts& c) {
   return tot;
 }
 
-// Decode workspace: a counter per (layer, row, head), then partial results
+// Decode workspace: a 512-byte header (status word at byte 0), a counter per
+// (layer, row, head), then partial results
 // [layer][row][head][split][G][kD + 4] floats (m, l, two pad, o[kD]).
+constexpr uint64_t kWsHeaderBytes = 512;
+constexpr uint32_t kStatusWaitTimeout = 1u;  // a wait for a tile's data ran out
 HG_HD uint64_t ws_counter_bytes(const Dims& d, int n_layers) {
   return align_up((uint64_t)n_layers * d.B * d.H * 4);
 }
 HG_HD uint64_t ws_partial_floats_per_split(const Dims& d) { return (uint64_t)d.G * (kD + 4); }
 HG_HD uint64_t ws_bytes(const Dims& d, int n_layers, int max_items) {
-  return ws_counter_bytes(d, n_layers) +
+  return kWsHeaderBytes + ws_counter_bytes(d, n_layers) +
          align_up((uint64_t)n_layers * d.B * d.H * max_items * ws_partial_floats_per_split(d) * 4);
 }
 

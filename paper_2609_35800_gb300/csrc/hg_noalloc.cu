@@ -66,8 +66,8 @@ extern "C" hg_status hg_decode_attention_noalloc(const hg_cache* cache, int32_t 
   void* scratch = nullptr;
   st = scratch_address(&scratch);
   if (st != HG_OK) return st;
-  // The array keeps whatever the previous call left; the split counters must
-  // start at zero.
+  // The array keeps whatever the previous call left; the status word and the
+  // split counters must start at zero.
   if (cudaMemsetAsync(scratch, 0, need, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
     return HG_ERR_CUDA;
   return hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, scratch,
