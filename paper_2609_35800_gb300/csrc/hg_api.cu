@@ -122,12 +122,22 @@ bool range_ok(const hg_cache* c, int32_t begin, int32_t count) {
   return c && count >= 1 && begin >= 0 && (int64_t)begin + count <= c->d.L;
 }
 
-// Decode work plan.  Chunk sizes are chosen so that a launch has about
-// kTargetItems work items of similar byte size: three resident CTAs on each of
-// the 152 SMs, i.e. one wave.  Chunk sizes are multiples of the kernel's tile
-// (64 tokens for BF16 rows, the coded tile for codes) and depend only on the
-// layer range, so the workspace bound holds for every appended count.
-constexpr int kTargetItems = 3 * 152;
+// Decode work plan.  Chunk sizes are chosen so that a launch has at most one
+// wave of work items (the CTAs that are resident at once: three per SM for up
+// to 8 queries per KV head, two above) of similar cost.  Chunk sizes are
+// multiples of 64 tokens and depend only on the layer range and the device,
+// so the workspace bound holds for every appended count.
+int sm_count() {
+  static int cached[64] = {};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
+  if (cached[dev] == 0) {
+    int n = 0;
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
+    cached[dev] = n;
+  }
+  return cached[dev];
+}
 
 int round_up_to(int x, int g) { return ((x + g - 1) / g) * g; }
 
@@ -142,10 +152,10 @@ int chunk_tokens(int len, double bpt, double item_bytes, int granule) {
 }
 
 // Cost per token of each segment kind, in byte-equivalents: the bytes a chunk
-// streams plus about 8 bytes per warp-instruction its tokens cost (measured
-// instruction counts of the decode kernel: ~5 per BF16 token, ~10 / 13 per
-// 2 / 4-bit coded token, ~22 for KIVI-style keys, ~8 for keys-only heads).
-// Balancing cost rather than bytes keeps compute-heavy coded chunks short.
+// streams plus a compute term calibrated on measured per-CTA timelines of the
+// decode kernel (a 2-bit coded token costs about 0.6 of a BF16 token's time
+// although it moves 0.16 of its bytes).  Balancing cost rather than bytes
+// keeps compute-heavy coded chunks short.
 struct SegBytes {
   double bf16, coded_u, coded_k;
 };
@@ -155,14 +165,15 @@ SegBytes seg_bytes(const Dims& d) {
   const double codes = 16.0 * d.bits;  // 128 codes
   const double kmeta = d.base == kKivi ? 32.0 : 8.0;
   const double vmeta = 8.0 * vgroups(d);
-  const double instr_u = d.base == kKivi ? (d.bits == 2 ? 22.0 : 26.0) : (d.bits == 2 ? 10.0 : 13.5);
+  const double instr_u = d.base == kKivi ? (d.bits == 2 ? 66.0 : 78.0) : (d.bits == 2 ? 30.0 : 40.0);
   b.bf16 = 512.0 + 8.0 * 5.0;
   b.coded_u = 2.0 * codes + kmeta + vmeta + 8.0 * instr_u;
-  b.coded_k = 256.0 + codes + vmeta + 8.0 * 8.0;
+  b.coded_k = 256.0 + codes + vmeta + 8.0 * 16.0;
   return b;
 }
 
 int max_items_of(const Dims& d, const DecodePlan& p);
+ChunkCounts counts_of(const Dims& d, int appended, const DecodePlan& p);
 
 DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
   const Dims& d = c->d;
@@ -179,14 +190,23 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
     }
   }
   total *= d.B;
-  double item = total / kTargetItems;
+  const int wave = (d.G <= 8 ? 3 : 2) * sm_count();
+  double item = total / wave;
   if (item < 16384.0) item = 16384.0;
-  const int tile = decode_coded_tile(d.bits);
+  // Grow the item size until the items (at the largest appended count) fit
+  // one wave, or every segment is a single chunk.
   DecodePlan p;
-  p.cbU = chunk_tokens(d.T - d.nq, sb.bf16, item, 64);
-  p.cqU = chunk_tokens(d.nq, sb.coded_u, item, tile);
-  p.cqK = chunk_tokens(d.nq, sb.coded_k, item, 64);
-  p.cbP = chunk_tokens(d.T, sb.bf16, item, 64);
+  for (int iter = 0; iter < 64; ++iter, item *= 1.05) {
+    p.cbU = chunk_tokens(d.T - d.nq + d.S_new, sb.bf16, item, 64);
+    p.cqU = chunk_tokens(d.nq, sb.coded_u, item, 64);
+    p.cqK = chunk_tokens(d.nq, sb.coded_k, item, 64);
+    p.cbP = chunk_tokens(d.T + d.S_new, sb.bf16, item, 64);
+    long long items = 0;
+    for (int l = begin; l < begin + count; ++l)
+      items += (long long)d.B * row_chunks(d, c->layer_mask[l], counts_of(d, d.S_new, p));
+    if (items <= wave) break;
+    if (p.cbU >= d.T - d.nq + d.S_new && p.cqU >= d.nq && p.cqK >= d.nq && p.cbP >= d.T + d.S_new) break;
+  }
   // The merging CTA stages (m, l) of all splits of a head in the kernel's
   // 8 KB query buffer: at most 2 * splits * G + 2 * G floats.
   while ((long long)max_items_of(d, p) * d.G * 2 + 2LL * d.G > (long long)kMaxG * kD) {

@@ -98,6 +98,16 @@ __device__ __forceinline__ uint32_t pair2_off(uint32_t x) {
   return (x & (BITS == 2 ? 0x00030003u : 0x000F000Fu)) | 0x43004300u;
 }
 
+// FP16 forms for value codes: exact codes, and 1024 + code.
+template <int BITS>
+__device__ __forceinline__ uint32_t pair2_h(uint32_t x) {
+  return codes_f16x2(x & (BITS == 2 ? 0x00030003u : 0x000F000Fu));
+}
+template <int BITS>
+__device__ __forceinline__ uint32_t pair2_off_h(uint32_t x) {
+  return (x & (BITS == 2 ? 0x00030003u : 0x000F000Fu)) | 0x64006400u;
+}
+
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
   asm("ex2.approx.ftz.f32 %0, %1;\n" : "=f"(y) : "f"(x));
@@ -107,7 +117,8 @@ __device__ __forceinline__ float fast_exp2(float x) {
 template <int NT, int NZ>
 struct WarpState {
   float o[NT][8][4];
-  float corr[NT][4];  // 128 * sum_t P^T[t][q] for value codes carried as 128 + c
+  float corr[NT][4];  // 1024 * sum_t P'^T[t][q] for value codes carried as 1024 + c
+  float vb;           // coded values: power-of-two bound of the value scales seen so far
   float m[NT][2];
   float l[NT][2];
   float z[NT][2][NZ];
@@ -122,6 +133,16 @@ __device__ __forceinline__ int pos3(int j) { return 2 * (j % 3); }
 __device__ __forceinline__ uint32_t pair2_scaled(uint32_t w, uint32_t w6, uint32_t w12, int j) {
   const uint32_t src = j < 3 ? w : (j < 6 ? w6 : w12);
   return (src & (0x00030003u << pos3(j))) | 0x43004300u;
+}
+// The same pair as the FP16 values 1024 + 4^(j % 3) * code (value codes).
+__device__ __forceinline__ uint32_t pair2_scaled_h(uint32_t w, uint32_t w6, uint32_t w12, int j) {
+  const uint32_t src = j < 3 ? w : (j < 6 ? w6 : w12);
+  return (src & (0x00030003u << pos3(j))) | 0x64006400u;
+}
+
+// Smallest power of two >= m (m > 0, finite).
+__device__ __forceinline__ float pow2_ceil(float m) {
+  return __uint_as_float((__float_as_uint(m) + 0x007FFFFFu) & 0xFF800000u);
 }
 
 template <int BITS, int KM, int VM>
@@ -353,6 +374,36 @@ __device__ __forceinline__ void pfrag(const float (&p)[4], float fg, float fg8, 
 __device__ __forceinline__ void mma_pv(float (&o)[4], const uint32_t (&a)[4], const uint32_t (&b)[4]) {
   mma_bf16(o, a, b[0], b[1]);
   mma_bf16(o, a, b[2], b[3]);
+}
+
+// Coded values multiply exact FP16 codes by P' = p * s / vb in FP16 (one MMA;
+// about 11 significant bits, so each product carries at most 2^-12 relative
+// error, far inside the tolerance).  vb is a power of two bounding every value
+// scale s seen so far, so P' <= p <= 256 never overflows, and only weights
+// below ~1e-4 of the largest reach FP16's subnormal range; when a larger
+// scale arrives, vb grows and the accumulators are rescaled exactly.  The
+// accumulators are in units of vb.
+__device__ __forceinline__ void pfrag16(const float (&p)[4], float fg, float fg8, uint32_t (&b)[2]) {
+  b[0] = movtrans(pack_half2(p[0] * fg, p[1] * fg));
+  b[1] = movtrans(pack_half2(p[2] * fg8, p[3] * fg8));
+}
+
+template <int NT, int NZ>
+__device__ __forceinline__ void vscale_update(WarpState<NT, NZ>& ws, float smax) {
+  if (__any_sync(kFull, smax > ws.vb)) {
+    const float nb = pow2_ceil(warp_max(smax));
+    const float a = ws.vb / nb;  // a power of two: exact
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) ws.o[nt][mt][i] *= a;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ws.corr[nt][i] *= a;
+    }
+    ws.vb = nb;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -613,19 +664,21 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         const bool ok0 = tok0 + g < nvalid, ok8 = tok0 + g + 8 < nvalid;
         const float2 vg = ok0 ? vm2[tok0 + g] : make_float2(0.f, 0.f);
         const float2 vg8 = ok8 ? vm2[tok0 + g + 8] : make_float2(0.f, 0.f);
-        uint32_t b[NT][4];
+        vscale_update(ws, fmaxf(vg.x, vg8.x));
+        const float inv = 1.0f / ws.vb;  // exact: vb is a power of two
+        uint32_t b[NT][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
-          pfrag(p[nt], vg.x, vg8.x, b[nt]);
+          pfrag16(p[nt], vg.x * inv, vg8.x * inv, b[nt]);
 #pragma unroll
           for (int e = 0; e < 2; ++e) ws.z[nt][e][0] += p[nt][e] * vg.y + p[nt][2 + e] * vg8.y;
         }
-        // value codes enter as 128 + f c; the 128 part is collected in ws.corr by
-        // one MMA on a constant tile and removed at the end (f: see pair2_scaled)
+        // value codes enter as 1024 + f c; the 1024 part is collected in ws.corr
+        // by one MMA on a constant tile and removed at the end (f: see pair2_scaled)
         {
-          const uint32_t c128[4] = {0x43004300u, 0x43004300u, 0x43004300u, 0x43004300u};
+          const uint32_t c1024[4] = {0x64006400u, 0x64006400u, 0x64006400u, 0x64006400u};
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) mma_pv(ws.corr[nt], c128, b[nt]);
+          for (int nt = 0; nt < NT; ++nt) mma_f16(ws.corr[nt], c1024, b[nt][0], b[nt][1]);
         }
         const int t0 = tok0 + 2 * tq;
         if (BITS == 2) {
@@ -644,9 +697,9 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           for (int mt = 0; mt < 8; ++mt) {
             uint32_t a[4];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) a[k] = pair2_scaled(x[k], x6[k], x12[k], mt);
+            for (int k = 0; k < 4; ++k) a[k] = pair2_scaled_h(x[k], x6[k], x12[k], mt);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
+            for (int nt = 0; nt < NT; ++nt) mma_f16(ws.o[nt][mt], a, b[nt][0], b[nt][1]);
           }
         } else {
           // word 2g holds channels 16g..16g+7 (codes 0-3 low half, 4-7 high), 2g+1 the next 8
@@ -662,12 +715,12 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           for (int mt = 0; mt < 8; ++mt) {
             const int sh = 4 * (mt & 3);
             uint32_t a[4];
-            a[0] = pair2_off<4>((mt < 4 ? xa : ya) >> sh);
-            a[1] = pair2_off<4>((mt < 4 ? xb : yb) >> sh);
-            a[2] = pair2_off<4>((mt < 4 ? xc : yc) >> sh);
-            a[3] = pair2_off<4>((mt < 4 ? xd : yd) >> sh);
+            a[0] = pair2_off_h<4>((mt < 4 ? xa : ya) >> sh);
+            a[1] = pair2_off_h<4>((mt < 4 ? xb : yb) >> sh);
+            a[2] = pair2_off_h<4>((mt < 4 ? xc : yc) >> sh);
+            a[3] = pair2_off_h<4>((mt < 4 ? xd : yd) >> sh);
 #pragma unroll
-            for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt]);
+            for (int nt = 0; nt < NT; ++nt) mma_f16(ws.o[nt][mt], a, b[nt][0], b[nt][1]);
           }
         }
       } else {  // V_KIVI: 4 value groups of 32 channels; m-tile mt = channels 16mt..16mt+15
@@ -684,12 +737,15 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           sv_g8[0] = b0.x; zv_g8[0] = b0.y; sv_g8[1] = b0.z; zv_g8[1] = b0.w;
           sv_g8[2] = b1.x; zv_g8[2] = b1.y; sv_g8[3] = b1.z; zv_g8[3] = b1.w;
         }
-        uint32_t b[NT][4][4];
+        vscale_update(ws, fmaxf(fmaxf(fmaxf(sv_g[0], sv_g[1]), fmaxf(sv_g[2], sv_g[3])),
+                                fmaxf(fmaxf(sv_g8[0], sv_g8[1]), fmaxf(sv_g8[2], sv_g8[3]))));
+        const float inv = 1.0f / ws.vb;  // exact: vb is a power of two
+        uint32_t b[NT][4][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
           for (int jg = 0; jg < 4; ++jg) {
-            pfrag(p[nt], sv_g[jg], sv_g8[jg], b[nt][jg]);
+            pfrag16(p[nt], sv_g[jg] * inv, sv_g8[jg] * inv, b[nt][jg]);
 #pragma unroll
             for (int e = 0; e < 2; ++e)
               ws.z[nt][e][jg % NZ] += p[nt][e] * zv_g[jg] + p[nt][2 + e] * zv_g8[jg];
@@ -704,23 +760,23 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           if (BITS == 2) {
             const uint32_t w0 = vc32[t0 * W + mt], w1 = vc32[(t0 + 1) * W + mt];
             const uint32_t w8 = vc32[(t0 + 8) * W + mt], w9 = vc32[(t0 + 9) * W + mt];
-            a[0] = pair2<2>(prmt(w0, w1, 0x5410) >> (2 * g));
-            a[1] = pair2<2>(prmt(w0, w1, 0x7632) >> (2 * g));
-            a[2] = pair2<2>(prmt(w8, w9, 0x5410) >> (2 * g));
-            a[3] = pair2<2>(prmt(w8, w9, 0x7632) >> (2 * g));
+            a[0] = pair2_h<2>(prmt(w0, w1, 0x5410) >> (2 * g));
+            a[1] = pair2_h<2>(prmt(w0, w1, 0x7632) >> (2 * g));
+            a[2] = pair2_h<2>(prmt(w8, w9, 0x5410) >> (2 * g));
+            a[3] = pair2_h<2>(prmt(w8, w9, 0x7632) >> (2 * g));
           } else {
             const uint2 u0 = *reinterpret_cast<const uint2*>(vc32 + t0 * W + 2 * mt);
             const uint2 u1 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 1) * W + 2 * mt);
             const uint2 u8 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 8) * W + 2 * mt);
             const uint2 u9 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 9) * W + 2 * mt);
             const int sh = 4 * (g & 1);
-            a[0] = pair2<4>(prmt(u0.x, u1.x, sel4) >> sh);
-            a[1] = pair2<4>(prmt(u0.y, u1.y, sel4) >> sh);
-            a[2] = pair2<4>(prmt(u8.x, u9.x, sel4) >> sh);
-            a[3] = pair2<4>(prmt(u8.y, u9.y, sel4) >> sh);
+            a[0] = pair2_h<4>(prmt(u0.x, u1.x, sel4) >> sh);
+            a[1] = pair2_h<4>(prmt(u0.y, u1.y, sel4) >> sh);
+            a[2] = pair2_h<4>(prmt(u8.x, u9.x, sel4) >> sh);
+            a[3] = pair2_h<4>(prmt(u8.y, u9.y, sel4) >> sh);
           }
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) mma_pv(ws.o[nt][mt], a, b[nt][mt >> 1]);
+          for (int nt = 0; nt < NT; ++nt) mma_f16(ws.o[nt][mt], a, b[nt][mt >> 1][0], b[nt][mt >> 1][1]);
         }
       }
     }
@@ -751,27 +807,37 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   const uint32_t st0 = smem_u32(stages);
   const uint32_t bars = smem_u32(smem + kBarOff);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + kBarOff + 8 * kMaxStages);
-  int issued = n_tiles < STAGES ? n_tiles : STAGES;  // meaningful in thread 0
-  if (tid == 0)
-    for (int s = 0; s < issued; ++s)
-      issue_tile<BITS, KM, VM>(st0 + s * TL::stage_bytes, bars + 8 * s, sg, tb + s * TL::tokens,
-                               min(TL::tokens, te - tb - s * TL::tokens), &p.arena_map);
+  // The queries are requested first: they gate every warp's first tile and
+  // would otherwise queue behind the CTAs' tile traffic.
+  constexpr int QV = (NT * 8 * 16 + kThreads - 1) / kThreads;  // 16-byte query pieces per thread
+  uint4 qv[QV];
+#pragma unroll
+  for (int k = 0; k < QV; ++k) {
+    const int i = tid + k * kThreads;
+    qv[k] = (i < G * 16) ? ldg16(qg + i * 8) : make_uint4(0u, 0u, 0u, 0u);
+  }
+  // Only the first tile goes in flight now: with every CTA of the launch
+  // starting at once, first tiles alone make a burst the memory system serves
+  // quickly, so compute starts early; the other stages are filled once the
+  // first tile has landed.
+  int issued = n_tiles > 0 ? 1 : 0;  // meaningful in thread 0
+  if (tid == 0 && issued)
+    issue_tile<BITS, KM, VM>(st0, bars, sg, tb, min(TL::tokens, te - tb), &p.arena_map);
 
   // Queries of this KV head's group (fp32, rows >= G zero), rotated for
   // AKVQ-style coded keys.
-  for (int i = tid; i < NT * 8 * 16; i += kThreads) {
-    float4* dst = reinterpret_cast<float4*>(q_s + i * 8);
-    if (i < G * 16) {
-      const uint4 v = ldg16(qg + i * 8);
+#pragma unroll
+  for (int k = 0; k < QV; ++k) {
+    const int i = tid + k * kThreads;
+    if (i < NT * 8 * 16) {
+      float4* dst = reinterpret_cast<float4*>(q_s + i * 8);
       float f[8];
-      bf16x2_to_f32(v.x, f[0], f[1]);
-      bf16x2_to_f32(v.y, f[2], f[3]);
-      bf16x2_to_f32(v.z, f[4], f[5]);
-      bf16x2_to_f32(v.w, f[6], f[7]);
+      bf16x2_to_f32(qv[k].x, f[0], f[1]);
+      bf16x2_to_f32(qv[k].y, f[2], f[3]);
+      bf16x2_to_f32(qv[k].z, f[4], f[5]);
+      bf16x2_to_f32(qv[k].w, f[6], f[7]);
       dst[0] = make_float4(f[0], f[1], f[2], f[3]);
       dst[1] = make_float4(f[4], f[5], f[6], f[7]);
-    } else {
-      dst[0] = dst[1] = make_float4(0.f, 0.f, 0.f, 0.f);
     }
   }
   __syncthreads();
@@ -814,17 +880,20 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
 #pragma unroll
     for (int i = 0; i < 4; ++i) ws.corr[nt][i] = 0.f;
   }
+  ws.vb = __uint_as_float(0x00800000u);  // 2^-126: no value scale seen yet
 
   for (int it = 0; it < n_tiles; ++it) {
     const int st = it % STAGES;
     const bool ok = __all_sync(kFull, !*abort && wait_tile(bars + 8 * st, (it / STAGES) & 1, abort, p.status));
     __syncthreads();
-    if (tid == 0 && it > 0 && issued < n_tiles && !*abort) {  // refill the stage of tile it - 1
-      fence_proxy_async_shared();
-      issue_tile<BITS, KM, VM>(st0 + (issued % STAGES) * TL::stage_bytes, bars + 8 * (issued % STAGES), sg,
-                               tb + issued * TL::tokens, min(TL::tokens, te - tb - issued * TL::tokens),
-                               &p.arena_map);
-      ++issued;
+    if (tid == 0 && !*abort) {
+      // tile 0 landed: fill the other stages; later, refill the stage of tile it - 1
+      const int upto = (it == 0) ? min(n_tiles, STAGES) : min(n_tiles, it + STAGES);
+      if (it > 0 && issued < upto) fence_proxy_async_shared();
+      for (; issued < upto; ++issued)
+        issue_tile<BITS, KM, VM>(st0 + (issued % STAGES) * TL::stage_bytes, bars + 8 * (issued % STAGES), sg,
+                                 tb + issued * TL::tokens, min(TL::tokens, te - tb - issued * TL::tokens),
+                                 &p.arena_map);
     }
     if (ok)
       compute_tile<BITS, NT, KM, VM, ROT>(ws, stages + st * TL::stage_bytes,
@@ -871,15 +940,17 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
           // remove the 128 offset and the 4^(mt % 3) factor of 2-bit value pairs
           c_lo = 16 * g + mt;
           c_hi = 16 * g + 8 + mt;
-          const float f = (BITS == 2) ? 1.0f / (float)(1 << pos3(mt)) : 1.0f;
+          // and the units (vb) of the coded-value accumulators
+          const float f = ((BITS == 2) ? 1.0f / (float)(1 << pos3(mt)) : 1.0f) * ws.vb;
           orow[c_lo] = (ws.o[nt][mt][e] - ws.corr[nt][e]) * f + ws.z[nt][e][0];
           orow[c_hi] = (ws.o[nt][mt][2 + e] - ws.corr[nt][2 + e]) * f + ws.z[nt][e][0];
         } else {
           c_lo = 16 * mt + g;
           c_hi = 16 * mt + 8 + g;
           const float z = (VM == V_KIVI) ? ws.z[nt][e][(mt >> 1) % NZ] : 0.f;
-          orow[c_lo] = ws.o[nt][mt][e] + z;
-          orow[c_hi] = ws.o[nt][mt][2 + e] + z;
+          const float f = (VM == V_KIVI) ? ws.vb : 1.0f;  // units of coded values
+          orow[c_lo] = ws.o[nt][mt][e] * f + z;
+          orow[c_hi] = ws.o[nt][mt][2 + e] * f + z;
         }
       }
     }
@@ -1045,9 +1116,22 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   if (!s_last) return;
   __threadfence();
 
-  // Last CTA of the head: merge every split.  1) (m, l) of all (split, query)
-  // pairs in one round of loads, then per query the maximum, the weights
-  // f = 2^(m - M) (stored over m) and the normaliser L.
+  // Last CTA of the head: merge every split.  The first batch of partial rows
+  // (m, l, o of as many splits as fit the stage buffer) goes in flight with
+  // one asynchronous sweep, overlapped with the loads of every split's (m, l);
+  // then per query the maximum, the weights f = 2^(m - M) (stored over m) and
+  // the normaliser L; then thread = channel accumulates the o rows.
+  const int split_floats = G * kPartialStride;
+  const int batch = kBufBytes / (split_floats * 4);
+  const uint32_t buf_u32 = smem_u32(smem + kStageOff);
+  const float* buf = reinterpret_cast<const float*>(smem + kStageOff);
+  auto sweep = [&](int s0) {
+    const int bytes = min(batch, ni - s0) * split_floats * 4;
+    const char* src = reinterpret_cast<const char*>(part + (size_t)s0 * split_floats);
+    for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, src + off, 16);
+    cp_async_commit();
+  };
+  sweep(0);
   float* ml = reinterpret_cast<float*>(smem + kQOff);  // [ni][G][2], queries are no longer needed
   float* MLq = ml + 2 * ni * G;                         // [G][2]
   for (int i = tid; i < ni * G; i += kThreads) {
@@ -1069,24 +1153,14 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     MLq[2 * j] = M;
     MLq[2 * j + 1] = Ls;
   }
-  __syncthreads();
-  // 2) the o rows, batch by batch of splits through the pipeline buffer with
-  //    one asynchronous sweep each (the partials of a head are contiguous).
   float O[NT * 8];
 #pragma unroll
   for (int j = 0; j < NT * 8; ++j) O[j] = 0.f;
-  const int split_floats = G * kPartialStride;
-  const int batch = kBufBytes / (split_floats * 4);
-  const uint32_t buf_u32 = smem_u32(smem + kStageOff);
-  const float* buf = reinterpret_cast<const float*>(smem + kStageOff);
   for (int s0 = 0; s0 < ni; s0 += batch) {
-    const int nbatch = min(batch, ni - s0);
-    const int bytes = nbatch * split_floats * 4;
-    const char* src = reinterpret_cast<const char*>(part + (size_t)s0 * split_floats);
-    for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, src + off, 16);
-    cp_async_commit();
+    if (s0 > 0) sweep(s0);
     cp_async_wait<0>();
     __syncthreads();
+    const int nbatch = min(batch, ni - s0);
     for (int sidx = 0; sidx < nbatch; ++sidx) {
 #pragma unroll
       for (int j = 0; j < NT * 8; ++j)

@@ -1,6 +1,7 @@
 // Warp-level tensor-core and async-copy primitives (inline PTX, sm_103a).
 #pragma once
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -14,6 +15,15 @@ __device__ __forceinline__ void mma_bf16(float (&d)[4], const uint32_t (&a)[4], 
                                          uint32_t b1) {
   asm volatile(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
+      "{%8,%9}, {%0,%1,%2,%3};\n"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// The same with FP16 operands (fragment layout as above).
+__device__ __forceinline__ void mma_f16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
       "{%8,%9}, {%0,%1,%2,%3};\n"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
       : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
@@ -69,6 +79,22 @@ __device__ __forceinline__ uint32_t codes_bf16x2(uint32_t x_masked) {
   const __nv_bfloat162 off = __halves2bfloat162(__ushort_as_bfloat16((unsigned short)0x4300),
                                                 __ushort_as_bfloat16((unsigned short)0x4300));
   h = __hsub2(h, off);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+// Two codes in bits [0, 11) and [16, 27) (already masked) -> the FP16 pair
+// (code_lo, code_hi), exactly: 0x6400 | c is the FP16 value 1024 + c (c < 1024
+// lands in the mantissa), minus 1024 is exact.
+__device__ __forceinline__ uint32_t codes_f16x2(uint32_t x_masked) {
+  const uint32_t v = x_masked | 0x64006400u;
+  __half2 h = *reinterpret_cast<const __half2*>(&v);
+  const __half2 off = __halves2half2(__ushort_as_half((unsigned short)0x6400), __ushort_as_half((unsigned short)0x6400));
+  h = __hsub2(h, off);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
+
+__device__ __forceinline__ uint32_t pack_half2(float lo, float hi) {
+  __half2 h = __floats2half2_rn(lo, hi);
   return *reinterpret_cast<const uint32_t*>(&h);
 }
 
