@@ -197,8 +197,8 @@ hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
 
 /* Health of the decode launches that used a workspace: waits for `stream`,
  * then copies the workspace's status word to *status (host).  0 = healthy;
- * bit 0 (1) = a CTA's wait for a tile of its data ran out (about 2^20 polls of
- * the tile's mbarrier), after which that CTA skipped its remaining work and
+ * bit 0 (1) = a CTA's wait for a tile of its data ran out (after about a
+ * second), after which that CTA skipped its remaining work and
  * let the copies it had issued land before exiting.  Decode CTAs wait with a
  * bound instead of hanging; after a non-zero status the outputs of the
  * launches since the last clear are undefined and the workspace must be

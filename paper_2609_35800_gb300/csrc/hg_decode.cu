@@ -58,7 +58,10 @@ constexpr int kSmemUsed = kBarOff + 64;
 constexpr int kSmemBytes = kSmemUsed + 1024;     // + alignment slack
 constexpr int kMaxStages = 4;
 constexpr unsigned kFull = 0xffffffffu;
-constexpr uint32_t kSpinLimit = 1u << 20;       // mbarrier polls before a wait is declared stuck
+// A wait for a tile is declared stuck after kWaitRounds suspensions of up to
+// kWaitSleepNs each (about a second); a healthy wait ends within microseconds.
+constexpr uint32_t kWaitRounds = 20000;
+constexpr uint32_t kWaitSleepNs = 50000;
 
 enum KMode { K_BF16 = 0, K_TOKEN = 1, K_KIVI = 2 };
 enum VMode { V_BF16 = 0, V_TOKEN = 1, V_KIVI = 2 };
@@ -210,8 +213,8 @@ __device__ __forceinline__ void issue_tile(uint32_t st, uint32_t bar, const Seg&
 // warp gave up, marks the CTA aborted, records the failure in the workspace
 // status word and returns false (the caller skips the tile's work).
 __device__ __forceinline__ bool wait_tile(uint32_t bar, uint32_t parity, volatile int* abort, uint32_t* status) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
-    if (mbar_try_wait(bar, parity)) return true;
+  for (uint32_t i = 0; i < kWaitRounds; ++i) {
+    if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
     if (*abort) return false;
   }
   *abort = 1;
@@ -905,7 +908,9 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
     // last STAGES tiles can still be in flight: let them land (bounded)
     // before the buffer is reused or the CTA exits.
     for (int t = (issued > STAGES ? issued - STAGES : 0); t < issued; ++t)
-      for (uint32_t i = 0; i < kSpinLimit && !mbar_try_wait(bars + 8 * (t % STAGES), (t / STAGES) & 1); ++i) {
+      for (uint32_t i = 0; i < kWaitRounds && !mbar_try_wait_sleep(bars + 8 * (t % STAGES), (t / STAGES) & 1,
+                                                                    kWaitSleepNs);
+           ++i) {
       }
   }
   __syncthreads();  // stage buffers are reused for the reduction below
