@@ -1092,6 +1092,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
   float* part = p.partials + (head_lin * p.max_items) * (size_t)G * kPartialStride;
   float* mine = part + (size_t)r * G * kPartialStride;
+#pragma unroll 1
   for (int j = 0; j < G; ++j) {
     float O = 0.f;
 #pragma unroll
@@ -1108,26 +1109,35 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   }
   if (ni == 1) return;
 
-  // Publish the partial: the CTA barrier orders every thread's stores before
-  // thread 0's device-scope fence (fences are cumulative), then take a ticket.
+  // Publish the partial and take a ticket with one acquire-release atomic: the
+  // CTA barrier orders every thread's stores before thread 0's release
+  // (release is cumulative); for the last CTA, the acquire side orders the
+  // other CTAs' partials before its reads (extended to its threads by the
+  // second barrier).  No full device fence is needed.
   __syncthreads();
   __shared__ int s_last;
   if (tid == 0) {
-    __threadfence();
-    const unsigned prev = atomicAdd(p.counters + head_lin, 1u);
+    unsigned prev;
+    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;\n"
+                 : "=r"(prev)
+                 : "l"(p.counters + head_lin)
+                 : "memory");
     s_last = (prev == (unsigned)(ni - 1));
   }
   __syncthreads();
   if (!s_last) return;
-  __threadfence();
 
   // Last CTA of the head: merge every split.  The first batch of partial rows
   // (m, l, o of as many splits as fit the stage buffer) goes in flight with
   // one asynchronous sweep, overlapped with the loads of every split's (m, l);
   // then per query the maximum, the weights f = 2^(m - M) (stored over m) and
   // the normaliser L; then thread = channel accumulates the o rows.
+  // (The merge runs once per head, so its code is cold: loops stay rolled to
+  // keep the instructions fetched small.)  The o sums live in the top of the
+  // stage buffer, one column per thread; batches of partial rows below them.
   const int split_floats = G * kPartialStride;
-  const int batch = kBufBytes / (split_floats * 4);
+  const int batch = (kBufBytes - G * kD * 4) / (split_floats * 4);
+  float* acc_s = reinterpret_cast<float*>(smem + kStageOff + kBufBytes) - G * kD;  // [G][kD]
   const uint32_t buf_u32 = smem_u32(smem + kStageOff);
   const float* buf = reinterpret_cast<const float*>(smem + kStageOff);
   auto sweep = [&](int s0) {
@@ -1139,6 +1149,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   sweep(0);
   float* ml = reinterpret_cast<float*>(smem + kQOff);  // [ni][G][2], queries are no longer needed
   float* MLq = ml + 2 * ni * G;                         // [G][2]
+#pragma unroll 1
   for (int i = tid; i < ni * G; i += kThreads) {
     ml[2 * i] = __ldcg(part + (size_t)i * kPartialStride);
     ml[2 * i + 1] = __ldcg(part + (size_t)i * kPartialStride + 1);
@@ -1147,8 +1158,10 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   if (tid < G) {
     const int j = tid;
     float M = -INFINITY;
+#pragma unroll 1
     for (int sidx = 0; sidx < ni; ++sidx) M = fmaxf(M, ml[2 * (sidx * G + j)]);
     float Ls = 0.f;
+#pragma unroll 1
     for (int sidx = 0; sidx < ni; ++sidx) {
       const float ms = ml[2 * (sidx * G + j)];
       const float f = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
@@ -1158,25 +1171,27 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     MLq[2 * j] = M;
     MLq[2 * j + 1] = Ls;
   }
-  float O[NT * 8];
-#pragma unroll
-  for (int j = 0; j < NT * 8; ++j) O[j] = 0.f;
+#pragma unroll 1
+  for (int j = 0; j < G; ++j) acc_s[j * kD + c] = 0.f;
+#pragma unroll 1
   for (int s0 = 0; s0 < ni; s0 += batch) {
     if (s0 > 0) sweep(s0);
     cp_async_wait<0>();
     __syncthreads();
     const int nbatch = min(batch, ni - s0);
-    for (int sidx = 0; sidx < nbatch; ++sidx) {
-#pragma unroll
-      for (int j = 0; j < NT * 8; ++j)
-        if (j < G)
-          O[j] = fmaf(ml[2 * ((s0 + sidx) * G + j)], buf[(sidx * G + j) * kPartialStride + 4 + c], O[j]);
+#pragma unroll 1
+    for (int j = 0; j < G; ++j) {
+      float O = acc_s[j * kD + c];
+#pragma unroll 1
+      for (int sidx = 0; sidx < nbatch; ++sidx)
+        O = fmaf(ml[2 * ((s0 + sidx) * G + j)], buf[(sidx * G + j) * kPartialStride + 4 + c], O);
+      acc_s[j * kD + c] = O;
     }
     __syncthreads();
   }
-#pragma unroll
-  for (int j = 0; j < NT * 8; ++j)
-    if (j < G) p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O[j] / MLq[2 * j + 1]);
+#pragma unroll 1
+  for (int j = 0; j < G; ++j)
+    p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(acc_s[j * kD + c] / MLq[2 * j + 1]);
   if (tid == 0) atomicExch(p.counters + head_lin, 0u);
 }
 
