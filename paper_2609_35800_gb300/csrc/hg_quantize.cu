@@ -1,6 +1,8 @@
 // Quantize-pack, dequantize and append kernels of the HeadGuard KV cache.
 //
-// Quantize (Sec. 3 "Applying protection" over the Sec. 1 / Sec. 4 bases):
+// Quantize (Sec. 3 "Applying protection" over the Sec. 1 / Sec. 4 bases).
+// Per-token min-max base: quantize_minmax_kernel below, one thread per
+// vector.  KIVI- and AKVQ-style bases: quantize_kernel,
 // one CTA per (32-token tile, batch row, KV head, layer).  The head's class
 // and the image span are resolved once per CTA, so protected heads and text
 // tokens take a uniform BF16 copy path.  A warp owns one token at a time,
@@ -8,6 +10,7 @@
 // max with warp butterflies, KIVI-style value groups (32 channels) with
 // 8-lane butterflies, and KIVI-style key groups (32 tokens of one channel) are
 // quantized by one thread per channel from a shared-memory copy of the tile.
+#include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
 #include "hg_common.cuh"
@@ -191,6 +194,162 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs)[(size_t)grp * kD + c] = make_float2(sc, z);
 }
 
+// ---------------------------------------------------------------------------
+// Per-token min-max base: one thread per (token, K or V) vector.
+//
+// A CTA takes 64 tokens of one (layer, row, KV head): the K and V rows are
+// staged in shared memory with coalesced loads (272-byte row pitch, so that
+// a thread's 16-byte reads of its own row are conflict free), then thread i
+// owns K row i, thread 64 + i V row i.  A coded vector is quantized by its
+// thread alone -- min / max over bf16x2 pairs (exact), then per element
+//   T = RN(d * r + 192), d = fl(x - min), r = RN(1 / scale):
+// T lies in [128, 256), so its low 16 mantissa bits hold d * r to 2^-16 and
+// bits 16.. hold floor(d * r + 0.5) once 0x8000 is added.  Within 2^-16 of
+// a half-integer the exact rule (round-half-even of fl(d / scale)) may differ,
+// so a vector with such an element is redone with IEEE divisions (rare).  The
+// bound: |d r - d / scale| <= 16 * 2^-24 and the FMA and the reference
+// quotient each round by at most 2^-17, so any element whose low bits are not
+// within one unit of 0x8000 rounds the same way as the reference.
+// Uncoded vectors (text, protected heads, keys of keys-only heads) are copied.
+// ---------------------------------------------------------------------------
+constexpr int kQTok = 64;
+constexpr int kQPitch = 272;
+
+template <int BITS>
+__device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, float2* meta) {
+  const uint4* r4 = reinterpret_cast<const uint4*>(row_s);
+  __nv_bfloat162 mn2, mx2;
+  {
+    const uint4 v = r4[0];
+    mn2 = mx2 = *reinterpret_cast<const __nv_bfloat162*>(&v.x);
+  }
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const uint4 v = r4[k];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+      mn2 = __hmin2(mn2, h);
+      mx2 = __hmax2(mx2, h);
+    }
+  }
+  float mn = fminf(__low2float(mn2), __high2float(mn2));
+  float mx = fmaxf(__low2float(mx2), __high2float(mx2));
+  mn = __fadd_rn(mn, 0.0f);  // -0 -> +0
+  mx = __fadd_rn(mx, 0.0f);
+  constexpr uint32_t L = (1u << BITS) - 1u;
+  const float levels = (float)L;
+  const float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  *meta = make_float2(scale, mn);
+  constexpr int W = 4 * BITS;  // code words per token
+  uint32_t word[W];
+#pragma unroll
+  for (int i = 0; i < W; ++i) word[i] = 0u;
+  if (scale == 0.0f) {
+    // constant vector: every code 0
+  } else {
+    const bool fast = scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
+    uint32_t tmin = fast ? 0xFFFFu : 0u;
+    if (fast) {
+      const float r = __frcp_rn(scale);
+#pragma unroll
+      for (int k = 0; k < 16; ++k) {
+        const uint4 v = r4[k];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int e = 8 * k + i;  // channel
+          const uint32_t hw = w[i >> 1];
+          const float x = __uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16));
+          const float t = __fmaf_rn(__fsub_rn(x, mn), r, 192.0f);
+          const uint32_t a = __float_as_uint(t) + 0x8001u;
+          tmin = min(tmin, a & 0xffffu);
+          const uint32_t code = (a >> 16) & L;
+          word[e / (32 / BITS)] |= code << (BITS * (e % (32 / BITS)));
+        }
+      }
+    }
+    if (tmin < 3u) {  // a near-tie somewhere (or a tiny scale): the exact rule for the whole vector
+#pragma unroll 1
+      for (int wi = 0; wi < W; ++wi) {
+        uint32_t acc = 0u;
+#pragma unroll 1
+        for (int j = 0; j < 32 / BITS; ++j) {
+          const int e = wi * (32 / BITS) + j;
+          const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
+          const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
+          float rq = rintf(__fdiv_rn(__fsub_rn(x, mn), scale));
+          rq = fminf(fmaxf(rq, 0.0f), levels);
+          acc |= (uint32_t)rq << (BITS * j);
+        }
+        codes[wi] = acc;
+      }
+      return;
+    }
+  }
+  uint4* c4 = reinterpret_cast<uint4*>(codes);
+#pragma unroll
+  for (int i = 0; i < W / 4; ++i) c4[i] = make_uint4(word[4 * i], word[4 * i + 1], word[4 * i + 2], word[4 * i + 3]);
+}
+
+template <int BITS>
+__global__ void __launch_bounds__(kThreads)
+quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
+  const Dims& d = p.d;
+  const int li = blockIdx.z, bh = blockIdx.y;
+  const int b = bh / d.H, h = bh % d.H;
+  const int t0 = blockIdx.x * kQTok;
+  const int n = min(kQTok, d.T - t0);
+  if (n <= 0) return;
+  const int tid = threadIdx.x;
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+  const HeadGeom hd = head_geom(d, g, h);
+  char* Lb = p.arena + p.lt.base[li];
+  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + t0;
+  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
+  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
+
+  __shared__ __align__(16) char rows[2][kQTok][kQPitch];
+  // coalesced staging: chunk c = 16 bytes of one row
+  for (int c = tid; c < 2 * n * 16; c += kThreads) {
+    const int kv = c / (n * 16), rem = c - kv * (n * 16);
+    const int r = rem >> 4, col = rem & 15;
+    *reinterpret_cast<uint4*>(&rows[kv][r][col * 16]) = ldg16((kv ? src_v : src_k) + (size_t)r * 256 + col * 16);
+  }
+  __syncthreads();
+
+  const int kv = tid >> 6, r = tid & (kQTok - 1);
+  if (r >= n) return;
+  const int t = t0 + r;
+  const bool coded = t >= d.s && t < d.s + d.nq;
+  const int ti = t - d.s;
+  const char* row_s = rows[kv][r];
+  constexpr int W = 4 * BITS;
+  if (kv == 0) {
+    if (coded && hd.cls == kQuantized) {
+      quantize_row_token<BITS>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
+                               reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs) + ti);
+      return;
+    }
+    char* dst = (coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
+                                               : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+      reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+  } else {
+    if (coded && hd.cls != kProtected) {
+      quantize_row_token<BITS>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+                               reinterpret_cast<float2*>(Lb + hd.vqm + b * hd.vqm_bs) + ti);
+      return;
+    }
+    char* dst = Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
+#pragma unroll
+    for (int k = 0; k < 16; ++k)
+      reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+  }
+}
+
 // Reconstruct one layer as floats in original token order (then appended).
 __global__ void __launch_bounds__(kThreads)
 dequantize_kernel(const __grid_constant__ DequantParams p) {
@@ -288,6 +447,12 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 }  // namespace
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
+  if (p.d.base == kMinMax) {  // one thread per vector
+    dim3 grid((p.d.T + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
+    if (p.d.bits == 2) quantize_minmax_kernel<2><<<grid, kThreads, 0, s>>>(p);
+    else quantize_minmax_kernel<4><<<grid, kThreads, 0, s>>>(p);
+    return cudaGetLastError();
+  }
   dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
   quantize_kernel<<<grid, kThreads, 0, s>>>(p);
   return cudaGetLastError();

@@ -206,3 +206,37 @@ def test_capacity_error_leaves_state():
         hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
     assert e.value.status == 5
     assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
+
+
+@pytest.mark.parametrize("bits", [2, 4])
+def test_minmax_quantize_exact_ties(bits):
+    """Vectors built so that (x - min) / scale lands exactly on half-integers:
+    every such element must round half to even, as the oracle does (the
+    kernel's fast multiply-by-reciprocal path has to hand these to the exact
+    division rule)."""
+    w = wl.custom("ties%d" % bits, 1, 2, 8, 4, 5, 96, 7, M, bits, 0, decode_steps=1, seed=3,
+                  protected=[(0, 1)], residual=32)
+    runner = CacheRunner(w)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    gen = torch.Generator().manual_seed(11)
+    L = (1 << bits) - 1
+    # x = (g / 2 + m) * 2^e with g in [0, 2L]: min m 2^e and max (L + m) 2^e are
+    # pinned, so scale = 2^e exactly and (x - min) / scale = g / 2 -- exact in BF16
+    g = torch.randint(0, 2 * L + 1, (2, B, H, T, 128), generator=gen).float()
+    g[..., 0] = 0.0
+    g[..., 1] = 2.0 * L
+    m = torch.randint(-8, 8, (2, B, H, T, 1), generator=gen).float()
+    e = torch.randint(-6, 6, (2, B, H, T, 1), generator=gen).float()
+    x = (g * 0.5 + m) * torch.pow(2.0, e)
+    # a quarter of the vectors random instead (ordinary, tie-free values)
+    rnd = torch.rand((2, B, H, T, 1), generator=gen) < 0.25
+    x = torch.where(rnd, torch.randn((2, B, H, T, 128), generator=gen) * 3.0, x)
+    xb = x.to(torch.bfloat16)
+    assert torch.equal(xb[~rnd.expand_as(x)].float(), x[~rnd.expand_as(x)])  # exact in BF16
+    k = xb[0].contiguous().cuda()
+    v = xb[1].contiguous().cuda()
+    hg.hg_quantize_kv(runner.cache, 0, [k], [v])
+    torch.cuda.synchronize()
+    kb, vb = bits16(k), bits16(v)
+    o = oracle_layer(runner, 0, kb, vb)
+    check_arena_layer(runner, 0, kb, vb, o)
