@@ -206,7 +206,8 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
 // T lies in [128, 256), so its low 16 mantissa bits hold d * r to 2^-16 and
 // bits 16.. hold floor(d * r + 0.5) once 0x8000 is added.  Within 2^-16 of
 // a half-integer the exact rule (round-half-even of fl(d / scale)) may differ,
-// so a vector with such an element is redone with IEEE divisions (rare).  The
+// so such an element takes one IEEE division (BF16 inputs make exact
+// half-integer quotients common, so this is per element, not per vector).  The
 // bound: |d r - d / scale| <= 16 * 2^-24 and the FMA and the reference
 // quotient each round by at most 2^-17, so any element whose low bits are not
 // within one unit of 0x8000 rounds the same way as the reference.
@@ -214,6 +215,11 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
 // ---------------------------------------------------------------------------
 constexpr int kQTok = 64;
 constexpr int kQPitch = 272;
+
+// Round-half-even of fl(d / scale), clamped to the levels (IEEE division).
+__device__ __noinline__ uint32_t exact_code(float d, float scale, float levels) {
+  return (uint32_t)fminf(fmaxf(rintf(__fdiv_rn(d, scale)), 0.0f), levels);
+}
 
 template <int BITS>
 __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, float2* meta) {
@@ -248,45 +254,38 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   for (int i = 0; i < W; ++i) word[i] = 0u;
   if (scale == 0.0f) {
     // constant vector: every code 0
-  } else {
-    const bool fast = scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
-    uint32_t tmin = fast ? 0xFFFFu : 0u;
-    if (fast) {
-      const float r = __frcp_rn(scale);
+  } else if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
+    const float r = __frcp_rn(scale);
 #pragma unroll
-      for (int k = 0; k < 16; ++k) {
-        const uint4 v = r4[k];
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    for (int k = 0; k < 16; ++k) {
+      const uint4 v = r4[k];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int e = 8 * k + i;  // channel
-          const uint32_t hw = w[i >> 1];
-          const float x = __uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16));
-          const float t = __fmaf_rn(__fsub_rn(x, mn), r, 192.0f);
-          const uint32_t a = __float_as_uint(t) + 0x8001u;
-          tmin = min(tmin, a & 0xffffu);
-          const uint32_t code = (a >> 16) & L;
-          word[e / (32 / BITS)] |= code << (BITS * (e % (32 / BITS)));
-        }
+      for (int i = 0; i < 8; ++i) {
+        const int e = 8 * k + i;  // channel
+        const uint32_t hw = w[i >> 1];
+        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
+        const uint32_t a = __float_as_uint(__fmaf_rn(d, r, 192.0f)) + 0x8001u;
+        // BF16 data puts many quotients exactly on half-integers: those (and
+        // anything within a unit of one) take the exact rule
+        const uint32_t code = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : ((a >> 16) & L);
+        word[e / (32 / BITS)] |= code << (BITS * (e % (32 / BITS)));
       }
     }
-    if (tmin < 3u) {  // a near-tie somewhere (or a tiny scale): the exact rule for the whole vector
+  } else {  // tiny scale: the exact rule throughout
 #pragma unroll 1
-      for (int wi = 0; wi < W; ++wi) {
-        uint32_t acc = 0u;
+    for (int wi = 0; wi < W; ++wi) {
+      uint32_t acc = 0u;
 #pragma unroll 1
-        for (int j = 0; j < 32 / BITS; ++j) {
-          const int e = wi * (32 / BITS) + j;
-          const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
-          const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
-          float rq = rintf(__fdiv_rn(__fsub_rn(x, mn), scale));
-          rq = fminf(fmaxf(rq, 0.0f), levels);
-          acc |= (uint32_t)rq << (BITS * j);
-        }
-        codes[wi] = acc;
+      for (int j = 0; j < 32 / BITS; ++j) {
+        const int e = wi * (32 / BITS) + j;
+        const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
+        const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
+        acc |= exact_code(__fsub_rn(x, mn), scale, levels) << (BITS * j);
       }
-      return;
+      codes[wi] = acc;
     }
+    return;
   }
   uint4* c4 = reinterpret_cast<uint4*>(codes);
 #pragma unroll
