@@ -249,47 +249,55 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   const float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   *meta = make_float2(scale, mn);
   constexpr int W = 4 * BITS;  // code words per token
-  uint32_t word[W];
+  if (scale == 0.0f) {  // constant vector: every code 0
 #pragma unroll
-  for (int i = 0; i < W; ++i) word[i] = 0u;
-  if (scale == 0.0f) {
-    // constant vector: every code 0
-  } else if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
+    for (int i = 0; i < W; ++i) codes[i] = 0u;
+    return;
+  }
+  if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
     const float r = __frcp_rn(scale);
-#pragma unroll
+    // chunks of 8 channels (one uint4 of the row): 16 code bits (2-bit) or 32
+    // (4-bit); the loop stays rolled (by two) so the code is small and stays
+    // in the instruction cache
+    uint32_t prev = 0u;
+#pragma unroll 2
     for (int k = 0; k < 16; ++k) {
       const uint4 v = r4[k];
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t chunk = 0u;
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const int e = 8 * k + i;  // channel
         const uint32_t hw = w[i >> 1];
         const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
         const uint32_t a = __float_as_uint(__fmaf_rn(d, r, 192.0f)) + 0x8001u;
         // BF16 data puts many quotients exactly on half-integers: those (and
         // anything within a unit of one) take the exact rule
         const uint32_t code = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : ((a >> 16) & L);
-        word[e / (32 / BITS)] |= code << (BITS * (e % (32 / BITS)));
+        chunk |= code << (BITS * i);
       }
-    }
-  } else {  // tiny scale: the exact rule throughout
-#pragma unroll 1
-    for (int wi = 0; wi < W; ++wi) {
-      uint32_t acc = 0u;
-#pragma unroll 1
-      for (int j = 0; j < 32 / BITS; ++j) {
-        const int e = wi * (32 / BITS) + j;
-        const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
-        const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
-        acc |= exact_code(__fsub_rn(x, mn), scale, levels) << (BITS * j);
+      if (BITS == 4) {
+        codes[k] = chunk;
+      } else if (k & 1) {
+        codes[k >> 1] = prev | (chunk << 16);
+      } else {
+        prev = chunk;
       }
-      codes[wi] = acc;
     }
     return;
   }
-  uint4* c4 = reinterpret_cast<uint4*>(codes);
-#pragma unroll
-  for (int i = 0; i < W / 4; ++i) c4[i] = make_uint4(word[4 * i], word[4 * i + 1], word[4 * i + 2], word[4 * i + 3]);
+  // tiny scale: the exact rule throughout
+#pragma unroll 1
+  for (int wi = 0; wi < W; ++wi) {
+    uint32_t acc = 0u;
+#pragma unroll 1
+    for (int j = 0; j < 32 / BITS; ++j) {
+      const int e = wi * (32 / BITS) + j;
+      const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
+      const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
+      acc |= exact_code(__fsub_rn(x, mn), scale, levels) << (BITS * j);
+    }
+    codes[wi] = acc;
+  }
 }
 
 template <int BITS>
