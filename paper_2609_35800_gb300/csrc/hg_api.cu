@@ -123,7 +123,7 @@ bool range_ok(const hg_cache* c, int32_t begin, int32_t count) {
 }
 
 // Decode work plan.  Chunk sizes are chosen so that a launch has at most one
-// wave of work items (the CTAs that are resident at once: three per SM for up
+// wave of work items (the CTAs that are resident at once: four per SM for up
 // to 8 queries per KV head, two above) of similar cost.  Chunk sizes are
 // multiples of 64 tokens and depend only on the layer range and the device,
 // so the workspace bound holds for every appended count.
@@ -190,7 +190,7 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
     }
   }
   total *= d.B;
-  const int wave = (d.G <= 8 ? 3 : 2) * sm_count();
+  const int wave = (d.G <= 8 ? 4 : 2) * sm_count();
   double item = total / wave;
   if (item < 16384.0) item = 16384.0;
   // Grow the item size until the items (at the largest appended count) fit
@@ -208,8 +208,10 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
     if (p.cbU >= d.T - d.nq + d.S_new && p.cqU >= d.nq && p.cqK >= d.nq && p.cbP >= d.T + d.S_new) break;
   }
   // The merging CTA stages (m, l) of all splits of a head in the kernel's
-  // 8 KB query buffer: at most 2 * splits * G + 2 * G floats.
-  while ((long long)max_items_of(d, p) * d.G * 2 + 2LL * d.G > (long long)kMaxG * kD) {
+  // query buffer (8 or 16 query rows of 128 floats): at most 2 * splits * G +
+  // 2 * G floats.
+  const long long qbuf = (d.G <= 8 ? 8LL : 16LL) * kD;
+  while ((long long)max_items_of(d, p) * d.G * 2 + 2LL * d.G > qbuf) {
     p.cbU *= 2;
     p.cqU *= 2;
     p.cqK *= 2;
@@ -485,6 +487,54 @@ hg_status hg_workspace_status(const void* ws, uint32_t* status, hg_stream_t stre
 
 namespace {
 
+// CTA order of the work items.  Consecutive CTAs land on different SMs and
+// CTA b and b + (number of SMs) mostly on the same one, so the items are
+// sorted by estimated cost (largest first) and dealt out in rounds of one per
+// SM, every other round reversed: each SM gets a mix of large and small items
+// instead of whatever the (layer, row, head) enumeration puts together.
+// Returns the number of ordered CTAs (0: natural order).
+int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, int total,
+                uint16_t* order) {
+  if (total > kMaxOrderedItems || total < 2) return 0;
+  const Dims& d = c->d;
+  const SegBytes sb = seg_bytes(d);
+  std::vector<std::pair<double, int>> cost;
+  cost.reserve(total);
+  int item = 0;
+  for (int i = 0; i < count; ++i) {
+    const DecodeLayer& L = p.layer[i];
+    const ChunkCounts cc = {L.nbU, L.nqU, L.nqK, L.nbP};
+    for (int b = 0; b < d.B; ++b) {
+      for (int h = 0; h < d.H; ++h) {
+        const int cls = head_class(d, c->layer_mask[begin + i], h);
+        int nb;
+        const int ni = head_chunks(cls, cc, &nb);
+        const int blen = (cls == kProtected ? d.T : d.T - d.nq) + L.appended;
+        const int bc = (cls == kProtected) ? p.plan.cbP : p.plan.cbU;
+        const int qc = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
+        const double qb = (cls == kKeysOnly) ? sb.coded_k : sb.coded_u;
+        for (int r = 0; r < ni; ++r) {
+          double w;
+          if (r < nb) w = std::min(bc, blen - r * bc) * sb.bf16;
+          else w = std::min(qc, d.nq - (r - nb) * qc) * qb;
+          cost.emplace_back(w, item++);
+        }
+      }
+    }
+  }
+  if (item != total) return 0;
+  std::stable_sort(cost.begin(), cost.end(),
+                   [](const std::pair<double, int>& a, const std::pair<double, int>& b) { return a.first > b.first; });
+  const int S = sm_count();
+  for (int j = 0; j < total; ++j) {
+    const int r = j / S, s = j % S;
+    const bool full_round = (r + 1) * S <= total;
+    const int blk = r * S + ((r & 1) && full_round ? S - 1 - s : s);
+    order[blk] = (uint16_t)cost[j].second;
+  }
+  return total;
+}
+
 // Decode attention over layers [layer_begin, +layer_count); with k_new / v_new
 // the step's new tokens (already counted in the cache's appended state) are
 // read from the inputs and stored into the arena by the same launch.
@@ -534,6 +584,7 @@ hg_status decode_launch(const hg_cache* c, int32_t layer_begin, int32_t layer_co
       total += dl.items_per_row * d.B;
     }
     p.total_items = total;
+    p.n_order = order_items(c, layer_begin + done, n, p, total, p.order);
     const hg_status st = cuda_status(launch_decode(p, total, reinterpret_cast<cudaStream_t>(stream)));
     if (st != HG_OK) return st;
   }

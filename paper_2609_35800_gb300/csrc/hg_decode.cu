@@ -46,16 +46,19 @@ namespace {
 
 constexpr int kThreads = 128;
 constexpr int kWarps = 4;
-constexpr int kBufBytes = 65536;   // pipeline buffer (stages of one tile each)
-constexpr int kBf16Tile = 64;      // tokens per tile of BF16 rows (K 16 KB + V 16 KB)
-constexpr int kMixTile = 64;       // tokens per tile of BF16 keys + coded values
+constexpr int kBufBytes = 49152;   // pipeline buffer (stages of one tile each)
+constexpr int kBf16Tile = 48;      // tokens per tile of BF16 rows (K 12 KB + V 12 KB)
+constexpr int kMixTile = 48;       // tokens per tile of BF16 keys + coded values
 constexpr int kPartialStride = kD + 4;  // m, l, 2 pad, o[128]: rows of 528 bytes (16-byte multiple)
 // Shared memory, from a 1024-byte aligned base (swizzled TMA boxes need it).
 constexpr int kStageOff = 0;                    // pipeline buffer
-constexpr int kQOff = kStageOff + kBufBytes;     // float q[16][128]
-constexpr int kBarOff = kQOff + kMaxG * kD * 4;  // mbarrier per stage (4), abort flag, merge flag
-constexpr int kSmemUsed = kBarOff + 64;
-constexpr int kSmemBytes = kSmemUsed + 1024;     // + alignment slack
+// Four CTAs per SM for up to 8 queries per KV head (NT = 1), two above.
+template <int NT>
+struct SmemLayout {
+  static constexpr int q = kStageOff + kBufBytes;  // float q[NT * 8][128]
+  static constexpr int bar = q + NT * 8 * kD * 4;  // mbarrier per stage (4), abort flag
+  static constexpr int bytes = bar + 64 + 1024;    // + alignment slack
+};
 constexpr int kMaxStages = 4;
 constexpr unsigned kFull = 0xffffffffu;
 // A wait for a tile is declared stuck after kWaitRounds suspensions of up to
@@ -71,8 +74,9 @@ struct NZOf {
   static constexpr int value = VM == V_TOKEN ? 1 : (VM == V_KIVI ? 4 : 1);
 };
 
-// Tokens per tile of coded K + coded V (multiple of 64, divides 512).
-__host__ __device__ constexpr int coded_tile(int bits) { return bits == 2 ? 256 : 128; }
+// Tokens per tile of coded K + coded V: per-token groups 256 (2-bit) / 128
+// (4-bit); KIVI-style (32 bytes of key metadata per token) 128.
+__host__ __device__ constexpr int coded_tile(int bits, int km) { return (bits == 2 && km != 2) ? 256 : 128; }
 
 struct Seg {
   const char* k;   // BF16 key rows (K_BF16)
@@ -151,7 +155,7 @@ __device__ __forceinline__ float pow2_ceil(float m) {
 template <int BITS, int KM, int VM>
 struct Tile {
   static constexpr int tokens = (KM == K_BF16 && VM == V_BF16) ? kBf16Tile
-                                : (KM == K_BF16 ? kMixTile : coded_tile(BITS));
+                                : (KM == K_BF16 ? kMixTile : coded_tile(BITS, KM));
   static constexpr int kc_bytes = (KM == K_BF16) ? tokens * 256 : tokens * 16 * BITS;
   static constexpr int km_bytes = (KM == K_TOKEN) ? tokens * 8 : (KM == K_KIVI ? tokens * 32 : 0);
   static constexpr int vc_bytes = (VM == V_BF16) ? tokens * 256 : tokens * 16 * BITS;
@@ -798,7 +802,7 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   constexpr int NZ = NZOf<VM>::value;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int g = lane >> 2, tq = lane & 3;
-  float* q_s = reinterpret_cast<float*>(smem + kQOff);
+  float* q_s = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);
   char* stages = smem + kStageOff;
 
   // Every tile that fits the buffer goes in flight before anything else;
@@ -808,8 +812,8 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   const float scale_log2 = p.scale_log2;
   const int n_tiles = (te - tb + TL::tokens - 1) / TL::tokens;
   const uint32_t st0 = smem_u32(stages);
-  const uint32_t bars = smem_u32(smem + kBarOff);
-  volatile int* abort = reinterpret_cast<volatile int*>(smem + kBarOff + 8 * kMaxStages);
+  const uint32_t bars = smem_u32(smem + SmemLayout<NT>::bar);
+  volatile int* abort = reinterpret_cast<volatile int*>(smem + SmemLayout<NT>::bar + 8 * kMaxStages);
   // The queries are requested first: they gate every warp's first tile and
   // would otherwise queue behind the CTAs' tile traffic.
   constexpr int QV = (NT * 8 * 16 + kThreads - 1) / kThreads;  // 16-byte query pieces per thread
@@ -963,19 +967,19 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
 }
 
 template <int BITS, int NT, int BASE>
-__global__ void __launch_bounds__(kThreads, NT == 1 ? 3 : 2)
+__global__ void __launch_bounds__(kThreads, NT == 1 ? 4 : 2)
 decode_kernel(const __grid_constant__ DecodeParams p) {
   extern __shared__ __align__(1024) char smem_raw[];
   // swizzled TMA boxes need 1024-byte aligned shared addresses
   char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const Dims& d = p.d;
-  const int item = blockIdx.x;
-  if (item >= p.total_items) return;
+  if ((int)blockIdx.x >= p.total_items) return;
+  const int item = ((int)blockIdx.x < p.n_order) ? (int)p.order[blockIdx.x] : (int)blockIdx.x;
   if (threadIdx.x == 0) {
-    const uint32_t bars = smem_u32(smem + kBarOff);
+    const uint32_t bars = smem_u32(smem + SmemLayout<NT>::bar);
     for (int s = 0; s < kMaxStages; ++s) mbar_init(bars + 8 * s, 1);
     mbar_init_fence();
-    *reinterpret_cast<volatile int*>(smem + kBarOff + 8 * kMaxStages) = 0;  // abort flag
+    *reinterpret_cast<volatile int*>(smem + SmemLayout<NT>::bar + 8 * kMaxStages) = 0;  // abort flag
     prefetch_tensormap(&p.arena_map);
   }
   int li = 0;
@@ -1147,7 +1151,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     cp_async_commit();
   };
   sweep(0);
-  float* ml = reinterpret_cast<float*>(smem + kQOff);  // [ni][G][2], queries are no longer needed
+  float* ml = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);  // [ni][G][2], queries are no longer needed
   float* MLq = ml + 2 * ni * G;                         // [G][2]
 #pragma unroll 1
   for (int i = tid; i < ni * G; i += kThreads) {
@@ -1203,16 +1207,16 @@ cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   if (dev < 64 && !configured[dev]) {
     e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             kSmemBytes);
+                             SmemLayout<NT>::bytes);
     if (e != cudaSuccess) return e;
-    // three CTAs of 75 KB share an SM: ask for the full shared-memory carve-out
+    // four CTAs of 54 KB share an SM: ask for the full shared-memory carve-out
     e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
     configured[dev] = true;
   }
   (void)grid_x;
-  decode_kernel<BITS, NT, BASE><<<p.total_items, kThreads, kSmemBytes, s>>>(p);
+  decode_kernel<BITS, NT, BASE><<<p.total_items, kThreads, SmemLayout<NT>::bytes, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -1227,7 +1231,7 @@ cudaError_t launch_base(const DecodeParams& p, int grid_x, cudaStream_t s) {
 
 }  // namespace
 
-int decode_coded_tile(int bits) { return coded_tile(bits); }
+int decode_coded_tile(int bits) { return coded_tile(bits, 0); }
 
 template <int BITS>
 void capacity_t(int base, int* bf16, int* coded, int* keys_only) {

@@ -66,6 +66,9 @@ struct DecodeLayer {
   int item_base;           // first work item of this layer in the launch
 };
 
+// Largest launch whose CTAs get a host-chosen item order.
+constexpr int kMaxOrderedItems = 1024;
+
 struct DecodeParams {
   // The arena as a two-dimensional BF16 tensor [arena_bytes / 256][128]: every
   // BF16 token row of the cache is one row of it.  Boxes of kArenaBoxRows rows
@@ -90,10 +93,13 @@ struct DecodeParams {
   float* partials;     // [n_layers][B][H][max_items][G][132]
   LayerTable lt;
   DecodeLayer layer[kMaxLayersPerLaunch];
+  // Work item of each CTA (blockIdx.x < n_order; item = blockIdx.x beyond).
+  int n_order;
+  uint16_t order[kMaxOrderedItems];
 };
 
 // BF16 rows per TMA box of the arena tensor map.
-constexpr int kArenaBoxRows = 32;
+constexpr int kArenaBoxRows = 16;
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s);
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
