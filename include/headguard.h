@@ -206,6 +206,17 @@ hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
  * of the kernels; the paper has no counterpart.) */
 hg_status hg_workspace_status(const void *workspace, uint32_t *status, hg_stream_t stream);
 
+/* Self-check of the bounded wait that guards every decode tile (failure
+ * detection; the paper has no counterpart).  One CTA waits on an mbarrier
+ * phase that has completed and on one that nothing will complete, each with
+ * the decode kernel's wait routine bounded to `rounds` suspensions of up to
+ * 50 us (1 <= rounds <= 100000).  `word`: device, 16-byte aligned, 4 bytes,
+ * zeroed by this call; when the stream reaches the end it holds 3 if the
+ * completed wait succeeded (bit 1) and the other one gave up and flagged the
+ * timeout (bit 0).  Faults and hangs nothing: the wait that cannot succeed
+ * returns after at most rounds * 50 us. */
+hg_status hg_check_bounded_wait(void *word, uint32_t rounds, hg_stream_t stream);
+
 /* Grouped-query decode attention of one step over layers
  * [layer_begin, +layer_count), reading packed codes and BF16 entries in one
  * pass.  q: device BF16 [layer_count][batch][num_q_heads][128]; out: device

@@ -19,6 +19,7 @@ __all__ = [
     "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
     "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
     "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_workspace_status",
+    "hg_check_bounded_wait",
     "hg_decode_attention",
     "hg_decode_step", "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem",
     "hg_status_string",
@@ -99,6 +100,7 @@ def library():
         "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
         "hg_workspace_clear": ([P, sz, P], st),
         "hg_workspace_status": ([P, ctypes.POINTER(ctypes.c_uint32), P], st),
+        "hg_check_bounded_wait": ([P, ctypes.c_uint32, P], st),
         "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_step": ([P, i32, i32, P, P, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_attention_noalloc": ([P, i32, i32, P, P, ctypes.c_float, P], st),
@@ -242,6 +244,12 @@ def hg_workspace_status(workspace, stream=None):
     _check(library().hg_workspace_status(_ptr(workspace), ctypes.byref(out), _stream(stream)),
            "hg_workspace_status")
     return out.value
+
+
+def hg_check_bounded_wait(word, rounds, stream=None):
+    """Run the bounded-wait self-check into the device word `word` (see the header)."""
+    _check(library().hg_check_bounded_wait(_ptr(word), int(rounds), _stream(stream)),
+           "hg_check_bounded_wait")
 
 
 def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, workspace,

@@ -471,6 +471,15 @@ hg_status hg_workspace_clear(void* ws, size_t bytes, hg_stream_t stream) {
   return cuda_status(cudaMemsetAsync(ws, 0, bytes, reinterpret_cast<cudaStream_t>(stream)));
 }
 
+hg_status hg_check_bounded_wait(void* word, uint32_t rounds, hg_stream_t stream) {
+  if (!word || rounds == 0 || rounds > 100000) return HG_ERR_INVALID_ARG;
+  if (!aligned16(word)) return HG_ERR_ALIGNMENT;
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaMemsetAsync(word, 0, sizeof(uint32_t), s);
+  if (e == cudaSuccess) e = launch_wait_probe(static_cast<uint32_t*>(word), rounds, s);
+  return cuda_status(e);
+}
+
 hg_status hg_workspace_status(const void* ws, uint32_t* status, hg_stream_t stream) {
   if (!ws || !status) return HG_ERR_INVALID_ARG;
   if (!aligned16(ws)) return HG_ERR_ALIGNMENT;

@@ -216,8 +216,9 @@ __device__ __forceinline__ void issue_tile(uint32_t st, uint32_t bar, const Seg&
 // Bounded wait for a phase of a stage's mbarrier.  On timeout, or once another
 // warp gave up, marks the CTA aborted, records the failure in the workspace
 // status word and returns false (the caller skips the tile's work).
-__device__ __forceinline__ bool wait_tile(uint32_t bar, uint32_t parity, volatile int* abort, uint32_t* status) {
-  for (uint32_t i = 0; i < kWaitRounds; ++i) {
+__device__ __forceinline__ bool wait_tile(uint32_t bar, uint32_t parity, volatile int* abort, uint32_t* status,
+                                          uint32_t rounds = kWaitRounds) {
+  for (uint32_t i = 0; i < rounds; ++i) {
     if (mbar_try_wait_sleep(bar, parity, kWaitSleepNs)) return true;
     if (*abort) return false;
   }
@@ -1248,6 +1249,31 @@ void capacity_t(int base, int* bf16, int* coded, int* keys_only) {
 void decode_chunk_capacity(int bits, int base, int* bf16, int* coded, int* keys_only) {
   if (bits == 2) capacity_t<2>(base, bf16, coded, keys_only);
   else capacity_t<4>(base, bf16, coded, keys_only);
+}
+
+// Check of the bounded wait that every decode tile wait uses: one mbarrier
+// whose phase is completed (the wait must succeed: bit 1) and one that nothing
+// ever arrives on (the wait must give up after `rounds` suspensions and flag
+// kStatusWaitTimeout: bit 0).  Expected result 3.
+__global__ void wait_probe_kernel(uint32_t* result, uint32_t rounds) {
+  __shared__ __align__(8) uint64_t bars[2];
+  __shared__ int abort_flag;
+  if (threadIdx.x != 0) return;
+  const uint32_t done = smem_u32(&bars[0]), never = smem_u32(&bars[1]);
+  mbar_init(done, 1);
+  mbar_init(never, 1);
+  mbar_init_fence();
+  abort_flag = 0;
+  mbar_arrive_expect_tx(done, 0);  // completes phase 0 of `done`
+  uint32_t r = 0;
+  if (wait_tile(done, 0, &abort_flag, result, rounds)) r |= 2u;
+  wait_tile(never, 0, &abort_flag, result, rounds);  // sets bit 0 of *result on timeout
+  atomicOr(result, r);
+}
+
+cudaError_t launch_wait_probe(uint32_t* result, uint32_t rounds, cudaStream_t s) {
+  wait_probe_kernel<<<1, 32, 0, s>>>(result, rounds);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s) {

@@ -105,6 +105,7 @@ cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s);
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s);
+cudaError_t launch_wait_probe(uint32_t* result, uint32_t rounds, cudaStream_t s);
 // Tokens per pipeline tile of coded K + coded V (chunk sizes are multiples of it).
 int decode_coded_tile(int bits);
 // Largest chunk (tokens) whose tiles all fit the kernel's pipeline buffer at

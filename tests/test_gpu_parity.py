@@ -240,3 +240,18 @@ def test_minmax_quantize_exact_ties(bits):
     kb, vb = bits16(k), bits16(v)
     o = oracle_layer(runner, 0, kb, vb)
     check_arena_layer(runner, 0, kb, vb, o)
+
+
+def test_bounded_wait_gives_up_and_flags():
+    """Failure detection without a fault: the decode kernel's tile wait, run on
+    an mbarrier phase that nothing completes, returns after its bound and sets
+    the timeout bit; on a completed phase it succeeds.  The context stays usable."""
+    import time
+    word = torch.zeros(4, dtype=torch.int32, device="cuda")
+    t0 = time.time()
+    hg.hg_check_bounded_wait(word, 200)  # at most 200 x 50 us
+    torch.cuda.synchronize()
+    assert time.time() - t0 < 30.0
+    assert int(word[0].item()) == 3
+    # the device still works: an ordinary decode afterwards is correct
+    _run_and_check(_workload(CASES[1]))
