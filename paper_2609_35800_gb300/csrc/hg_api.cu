@@ -207,11 +207,8 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
     if (items <= wave) break;
     if (p.cbU >= d.T - d.nq + d.S_new && p.cqU >= d.nq && p.cqK >= d.nq && p.cbP >= d.T + d.S_new) break;
   }
-  // The merging CTA stages (m, l) of all splits of a head in the kernel's
-  // query buffer (8 or 16 query rows of 128 floats): at most 2 * splits * G +
-  // 2 * G floats.
-  const long long qbuf = (d.G <= 8 ? 8LL : 16LL) * kD;
-  while ((long long)max_items_of(d, p) * d.G * 2 + 2LL * d.G > qbuf) {
+  // The merging CTA stages every split's partial of a head in its stage buffer.
+  while (max_items_of(d, p) > decode_max_splits(d.G)) {
     p.cbU *= 2;
     p.cqU *= 2;
     p.cqK *= 2;

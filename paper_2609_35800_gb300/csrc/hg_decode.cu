@@ -792,13 +792,59 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 }
 
 // ---------------------------------------------------------------------------
+// Combine of (m, l, o) partials of the same queries (the four warps of a CTA,
+// or the splits of a head): part s, query j at parts + s * sstride + j * 132
+// (m at +0, l at +1, o at +4).  With M = max_s m_s and f_s = 2^(m_s - M):
+// o = sum_s f_s o_s / L, L = sum_s f_s l_s.  combine_weights leaves f_s in
+// fw[s][j] (s < 16), L in fw[kFwL][j] and M in fw[kFwM][j] (rows of kMaxG).
+// ---------------------------------------------------------------------------
+constexpr int kFwL = 16, kFwM = 17;
+
+__device__ __forceinline__ void combine_weights(const float* parts, int n, int sstride, int G, float* fw,
+                                                int tid) {
+  if (tid < G) {
+    const int j = tid;
+    float M = -INFINITY;
+#pragma unroll 1
+    for (int s = 0; s < n; ++s) M = fmaxf(M, parts[s * sstride + j * kPartialStride]);
+    float Ls = 0.f;
+#pragma unroll 1
+    for (int s = 0; s < n; ++s) {
+      const float ms = parts[s * sstride + j * kPartialStride];
+      const float f = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
+      fw[s * kMaxG + j] = f;
+      Ls = fmaf(f, parts[s * sstride + j * kPartialStride + 1], Ls);
+    }
+    fw[kFwL * kMaxG + j] = Ls;
+    fw[kFwM * kMaxG + j] = M;
+  }
+  __syncthreads();
+}
+
+__device__ __forceinline__ float combine_o(const float* parts, int n, int sstride, const float* fw, int j, int c) {
+  // four independent sums, so that the loads of four parts are in flight together
+  const float* pj = parts + j * kPartialStride + 4 + c;
+  float o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
+  int s = 0;
+#pragma unroll 1
+  for (; s + 4 <= n; s += 4) {
+    o0 = fmaf(fw[s * kMaxG + j], pj[s * sstride], o0);
+    o1 = fmaf(fw[(s + 1) * kMaxG + j], pj[(s + 1) * sstride], o1);
+    o2 = fmaf(fw[(s + 2) * kMaxG + j], pj[(s + 2) * sstride], o2);
+    o3 = fmaf(fw[(s + 3) * kMaxG + j], pj[(s + 3) * sstride], o3);
+  }
+#pragma unroll 1
+  for (; s < n; ++s) o0 = fmaf(fw[s * kMaxG + j], pj[s * sstride], o0);
+  return (o0 + o1) + (o2 + o3);
+}
+
+// ---------------------------------------------------------------------------
 // One work item with a given key / value mode: pipeline, then per-warp results
 // into shared memory (m, l, o[q][channel]).
 // ---------------------------------------------------------------------------
 template <int BITS, int NT, int KM, int VM, bool ROT>
 __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int te, const DecodeParams& p,
-                                         const uint16_t* qg, int G, float* red_m, float* red_l,
-                                         float* red_o) {
+                                         const uint16_t* qg, int G, float* parts) {
   using TL = Tile<BITS, KM, VM>;
   constexpr int NZ = NZOf<VM>::value;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -938,11 +984,12 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
         ws.z[nt][e][zz] = z;
       }
       const int q = nt * 8 + 2 * tq + e;
+      float* prow = parts + (warp * kMaxG + q) * kPartialStride;  // (m, l, -, -, o[128])
       if (g == 0) {
-        red_m[warp * kMaxG + q] = ws.m[nt][e];
-        red_l[warp * kMaxG + q] = l;
+        prow[0] = ws.m[nt][e];
+        prow[1] = l;
       }
-      float* orow = red_o + (warp * kMaxG + q) * kD;
+      float* orow = prow + 4;
 #pragma unroll
       for (int mt = 0; mt < 8; ++mt) {
         int c_lo, c_hi;  // channels of rows g and g+8 of m-tile mt
@@ -1016,9 +1063,9 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   const int tid = threadIdx.x;
   const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
 
-  float* red_m = reinterpret_cast<float*>(smem + kStageOff);  // [warps][16]
-  float* red_l = red_m + kWarps * kMaxG;                        // [warps][16]
-  float* red_o = red_l + kWarps * kMaxG;                        // [warps][16][128]
+  // the warps' (m, l, o) partials [warp][16][132], in the stage buffer once the
+  // tiles are consumed (the same row layout as the split partials)
+  float* parts = reinterpret_cast<float*>(smem + kStageOff);
   Seg sg;
   sg.k = sg.v = sg.kc = sg.km = sg.vc = sg.vm = nullptr;
   sg.new_pos = -1;
@@ -1046,7 +1093,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
       }
     }
     __syncthreads();  // barriers initialised, new row stored
-    run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+    run_item<BITS, NT, K_BF16, V_BF16, false>(smem, sg, tb, te, p, qg, G, parts);
   } else if (hd.cls == kKeysOnly) {
     __syncthreads();  // barriers initialised
     sg.k = Lb + hd.kimg + b * hd.kimg_bs;
@@ -1054,9 +1101,9 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_BF16, V_KIVI, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_BF16, V_KIVI, false>(smem, sg, tb, te, p, qg, G, parts);
     else
-      run_item<BITS, NT, K_BF16, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_BF16, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, parts);
   } else {
     __syncthreads();  // barriers initialised
     sg.kc = Lb + hd.kq + b * hd.kq_bs;
@@ -1064,34 +1111,18 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_KIVI, V_KIVI, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_KIVI, V_KIVI, false>(smem, sg, tb, te, p, qg, G, parts);
     else if (BASE == kAkvq)
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, true>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, true>(smem, sg, tb, te, p, qg, G, parts);
     else
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, red_m, red_l, red_o);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, false>(smem, sg, tb, te, p, qg, G, parts);
   }
   __syncthreads();
 
-  // ---- combine the warps: per query, weights of the four warps, then thread = channel ----
-  float* red_f = red_o + kWarps * kMaxG * kD;  // [warps][16] weights
-  float* red_ML = red_f + kWarps * kMaxG;       // [16][2] max, sum
-  if (tid < G) {
-    const int j = tid;
-    float M = -INFINITY;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) M = fmaxf(M, red_m[w * kMaxG + j]);
-    float Ls = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) {
-      const float mw = red_m[w * kMaxG + j];
-      const float f = (mw == -INFINITY) ? 0.f : fast_exp2(mw - M);
-      red_f[w * kMaxG + j] = f;
-      Ls += f * red_l[w * kMaxG + j];
-    }
-    red_ML[2 * j] = M;
-    red_ML[2 * j + 1] = Ls;
-  }
-  __syncthreads();
+  // ---- combine the warps, then write the output (a head in one chunk) or this
+  // split's partial ----
+  float* fw = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);  // weights; queries no longer needed
+  combine_weights(parts, kWarps, kMaxG * kPartialStride, G, fw, tid);
   const int c = tid;
   const size_t out_row = ((size_t)li * d.B + b) * d.Hq + (size_t)h * G;
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
@@ -1099,16 +1130,14 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   float* mine = part + (size_t)r * G * kPartialStride;
 #pragma unroll 1
   for (int j = 0; j < G; ++j) {
-    float O = 0.f;
-#pragma unroll
-    for (int w = 0; w < kWarps; ++w) O = fmaf(red_f[w * kMaxG + j], red_o[(w * kMaxG + j) * kD + c], O);
+    const float O = combine_o(parts, kWarps, kMaxG * kPartialStride, fw, j, c);
     if (ni == 1) {
-      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / red_ML[2 * j + 1]);
+      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / fw[kFwL * kMaxG + j]);
     } else {
       mine[j * kPartialStride + 4 + c] = O;
       if (c == 0) {
-        mine[j * kPartialStride + 0] = red_ML[2 * j];
-        mine[j * kPartialStride + 1] = red_ML[2 * j + 1];
+        mine[j * kPartialStride + 0] = fw[kFwM * kMaxG + j];
+        mine[j * kPartialStride + 1] = fw[kFwL * kMaxG + j];
       }
     }
   }
@@ -1132,71 +1161,27 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   __syncthreads();
   if (!s_last) return;
 
-  // Last CTA of the head: merge every split.  The first batch of partial rows
-  // (m, l, o of as many splits as fit the stage buffer) goes in flight with
-  // one asynchronous sweep, overlapped with the loads of every split's (m, l);
-  // then per query the maximum, the weights f = 2^(m - M) (stored over m) and
-  // the normaliser L; then thread = channel accumulates the o rows.
-  // (The merge runs once per head, so its code is cold: loops stay rolled to
-  // keep the instructions fetched small.)  The o sums live in the top of the
-  // stage buffer, one column per thread; batches of partial rows below them.
-  const int split_floats = G * kPartialStride;
-  const int batch = (kBufBytes - G * kD * 4) / (split_floats * 4);
-  float* acc_s = reinterpret_cast<float*>(smem + kStageOff + kBufBytes) - G * kD;  // [G][kD]
-  const uint32_t buf_u32 = smem_u32(smem + kStageOff);
-  const float* buf = reinterpret_cast<const float*>(smem + kStageOff);
-  auto sweep = [&](int s0) {
-    const int bytes = min(batch, ni - s0) * split_floats * 4;
-    const char* src = reinterpret_cast<const char*>(part + (size_t)s0 * split_floats);
+  // Last CTA of the head: all ni partials in one asynchronous sweep into the
+  // stage buffer (the plan keeps them within it), then the same combine as
+  // the warps' -- code this CTA has just run, so its instructions are cached
+  // (the merge runs once per head: cold code would cost microseconds).
+  {
+    const int bytes = ni * G * kPartialStride * 4;
+    const uint32_t buf_u32 = smem_u32(smem + kStageOff);
+    const char* src = reinterpret_cast<const char*>(part);
+#pragma unroll 1
     for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, src + off, 16);
     cp_async_commit();
-  };
-  sweep(0);
-  float* ml = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);  // [ni][G][2], queries are no longer needed
-  float* MLq = ml + 2 * ni * G;                         // [G][2]
-#pragma unroll 1
-  for (int i = tid; i < ni * G; i += kThreads) {
-    ml[2 * i] = __ldcg(part + (size_t)i * kPartialStride);
-    ml[2 * i + 1] = __ldcg(part + (size_t)i * kPartialStride + 1);
+    cp_async_wait<0>();
   }
   __syncthreads();
-  if (tid < G) {
-    const int j = tid;
-    float M = -INFINITY;
+  const float* all = reinterpret_cast<const float*>(smem + kStageOff);  // [ni][G][132]
+  combine_weights(all, ni, G * kPartialStride, G, fw, tid);
 #pragma unroll 1
-    for (int sidx = 0; sidx < ni; ++sidx) M = fmaxf(M, ml[2 * (sidx * G + j)]);
-    float Ls = 0.f;
-#pragma unroll 1
-    for (int sidx = 0; sidx < ni; ++sidx) {
-      const float ms = ml[2 * (sidx * G + j)];
-      const float f = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
-      ml[2 * (sidx * G + j)] = f;
-      Ls += f * ml[2 * (sidx * G + j) + 1];
-    }
-    MLq[2 * j] = M;
-    MLq[2 * j + 1] = Ls;
+  for (int j = 0; j < G; ++j) {
+    const float O = combine_o(all, ni, G * kPartialStride, fw, j, c);
+    p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / fw[kFwL * kMaxG + j]);
   }
-#pragma unroll 1
-  for (int j = 0; j < G; ++j) acc_s[j * kD + c] = 0.f;
-#pragma unroll 1
-  for (int s0 = 0; s0 < ni; s0 += batch) {
-    if (s0 > 0) sweep(s0);
-    cp_async_wait<0>();
-    __syncthreads();
-    const int nbatch = min(batch, ni - s0);
-#pragma unroll 1
-    for (int j = 0; j < G; ++j) {
-      float O = acc_s[j * kD + c];
-#pragma unroll 1
-      for (int sidx = 0; sidx < nbatch; ++sidx)
-        O = fmaf(ml[2 * ((s0 + sidx) * G + j)], buf[(sidx * G + j) * kPartialStride + 4 + c], O);
-      acc_s[j * kD + c] = O;
-    }
-    __syncthreads();
-  }
-#pragma unroll 1
-  for (int j = 0; j < G; ++j)
-    p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(acc_s[j * kD + c] / MLq[2 * j + 1]);
   if (tid == 0) atomicExch(p.counters + head_lin, 0u);
 }
 
@@ -1233,6 +1218,13 @@ cudaError_t launch_base(const DecodeParams& p, int grid_x, cudaStream_t s) {
 }  // namespace
 
 int decode_coded_tile(int bits) { return coded_tile(bits, 0); }
+
+// The merging CTA stages every split's partial in its stage buffer and keeps
+// one weight row per split.
+int decode_max_splits(int G) {
+  const int n = kBufBytes / (G * kPartialStride * 4);
+  return n < kFwL ? n : kFwL;
+}
 
 template <int BITS>
 void capacity_t(int base, int* bf16, int* coded, int* keys_only) {
