@@ -268,6 +268,23 @@ hg_status hg_decode_attention_noalloc(const hg_cache *cache, int32_t layer_begin
  * image K/V element actually stored (codes + 64-bit metadata + BF16 entries). */
 hg_status hg_cache_image_bits_per_elem(const hg_cache *cache, double *bits);
 
+/* Protected-head selection from per-query-head sensitivity scores (Sec. 3
+ * "Selecting physical KV heads", Eq. 2): the query-head scores of each GQA
+ * group (query head qh belongs to KV head qh / G, G = num_q_heads /
+ * num_kv_heads) are averaged into per-KV-head scores g_i and o_i; each is
+ * standardised over all num_layers * num_kv_heads KV heads, z(x) = (x - mean)
+ * / std (population std; a constant score gives z = 0); s_i = z(g_i) + z(o_i);
+ * the k heads with the largest s are protected, ties to the lower index i =
+ * layer * num_kv_heads + head.  g_scores, o_scores: host float
+ * [num_layers][num_q_heads], finite; k < 0 selects round(N_KV / 8); k is
+ * clamped to [0, N_KV].  mask_out: host uint8 [num_layers][num_kv_heads], 1 =
+ * protected (the head_mask of hg_cache_layout).  Arithmetic in binary64 on
+ * the host; no device work.  HG_ERR_INVALID_ARG on a null pointer,
+ * non-positive sizes, num_q_heads not a multiple of num_kv_heads, or a
+ * non-finite score. */
+hg_status hg_select_heads(const float *g_scores, const float *o_scores, int32_t num_layers,
+                          int32_t num_q_heads, int32_t num_kv_heads, int32_t k, uint8_t *mask_out);
+
 /* Static description of a status code. */
 const char *hg_status_string(hg_status status);
 

@@ -19,7 +19,7 @@ __all__ = [
     "hg_cache_layout", "hg_cache_create", "hg_cache_destroy", "hg_cache_head_regions",
     "hg_cache_appended", "hg_cache_reset_appended", "hg_quantize_kv", "hg_dequantize_kv",
     "hg_append_kv", "hg_decode_workspace_size", "hg_workspace_clear", "hg_workspace_status",
-    "hg_check_bounded_wait",
+    "hg_check_bounded_wait", "hg_select_heads",
     "hg_decode_attention",
     "hg_decode_step", "hg_decode_attention_noalloc", "hg_cache_image_bits_per_elem",
     "hg_status_string",
@@ -101,6 +101,7 @@ def library():
         "hg_workspace_clear": ([P, sz, P], st),
         "hg_workspace_status": ([P, ctypes.POINTER(ctypes.c_uint32), P], st),
         "hg_check_bounded_wait": ([P, ctypes.c_uint32, P], st),
+        "hg_select_heads": ([P, P, i32, i32, i32, i32, P], st),
         "hg_decode_attention": ([P, i32, i32, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_step": ([P, i32, i32, P, P, P, P, ctypes.c_float, P, sz, P], st),
         "hg_decode_attention_noalloc": ([P, i32, i32, P, P, ctypes.c_float, P], st),
@@ -250,6 +251,19 @@ def hg_check_bounded_wait(word, rounds, stream=None):
     """Run the bounded-wait self-check into the device word `word` (see the header)."""
     _check(library().hg_check_bounded_wait(_ptr(word), int(rounds), _stream(stream)),
            "hg_check_bounded_wait")
+
+
+def hg_select_heads(g_scores, o_scores, num_layers, num_q_heads, num_kv_heads, k=-1):
+    """Protected-head mask (numpy uint8 [num_layers][num_kv_heads]) from host
+    per-query-head scores [num_layers][num_q_heads] (see the header)."""
+    import numpy as np
+    g = np.ascontiguousarray(np.asarray(g_scores, dtype=np.float32))
+    o = np.ascontiguousarray(np.asarray(o_scores, dtype=np.float32))
+    mask = np.zeros((num_layers, num_kv_heads), dtype=np.uint8)
+    _check(library().hg_select_heads(g.ctypes.data_as(ctypes.c_void_p), o.ctypes.data_as(ctypes.c_void_p),
+                                     num_layers, num_q_heads, num_kv_heads, int(k),
+                                     mask.ctypes.data_as(ctypes.c_void_p)), "hg_select_heads")
+    return mask
 
 
 def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, workspace,

@@ -639,6 +639,46 @@ hg_status hg_decode_step(hg_cache* c, int32_t layer_begin, int32_t layer_count, 
   return st;
 }
 
+hg_status hg_select_heads(const float* g_scores, const float* o_scores, int32_t num_layers, int32_t num_q_heads,
+                          int32_t num_kv_heads, int32_t k, uint8_t* mask_out) {
+  if (!g_scores || !o_scores || !mask_out || num_layers <= 0 || num_q_heads <= 0 || num_kv_heads <= 0)
+    return HG_ERR_INVALID_ARG;
+  if (num_q_heads % num_kv_heads != 0) return HG_ERR_INVALID_ARG;
+  const int G = num_q_heads / num_kv_heads;
+  const int n = num_layers * num_kv_heads;
+  for (int64_t i = 0; i < (int64_t)num_layers * num_q_heads; ++i)
+    if (!std::isfinite(g_scores[i]) || !std::isfinite(o_scores[i])) return HG_ERR_INVALID_ARG;
+  // per-KV-head group means, then standardisation over all KV heads
+  std::vector<double> gb(n), ob(n), sc(n, 0.0);
+  for (int l = 0; l < num_layers; ++l)
+    for (int h = 0; h < num_kv_heads; ++h) {
+      double sg = 0.0, so = 0.0;
+      for (int j = 0; j < G; ++j) {
+        sg += g_scores[(size_t)l * num_q_heads + h * G + j];
+        so += o_scores[(size_t)l * num_q_heads + h * G + j];
+      }
+      gb[l * num_kv_heads + h] = sg / G;
+      ob[l * num_kv_heads + h] = so / G;
+    }
+  for (const std::vector<double>* x : {&gb, &ob}) {
+    double mean = 0.0, var = 0.0;
+    for (double v : *x) mean += v;
+    mean /= n;
+    for (double v : *x) var += (v - mean) * (v - mean);
+    const double sd = std::sqrt(var / n);
+    if (sd > 0.0)
+      for (int i = 0; i < n; ++i) sc[i] += ((*x)[i] - mean) / sd;
+  }
+  if (k < 0) k = (int)std::nearbyint(n / 8.0);
+  if (k > n) k = n;
+  std::vector<int> idx(n);
+  for (int i = 0; i < n; ++i) idx[i] = i;
+  std::stable_sort(idx.begin(), idx.end(), [&](int a, int b) { return sc[a] > sc[b]; });
+  for (int i = 0; i < n; ++i) mask_out[i] = 0;
+  for (int i = 0; i < k; ++i) mask_out[idx[i]] = 1;
+  return HG_OK;
+}
+
 hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {
   if (!c || !bits) return HG_ERR_INVALID_ARG;
   const Dims& d = c->d;
