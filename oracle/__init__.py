@@ -37,6 +37,12 @@ def lib():
         L.hgo_bf16_to_f32.restype = ctypes.c_float
         L.hgo_quantize_group.argtypes = [P, i, i, i, P, P, P]
         L.hgo_quantize_group.restype = None
+        L.hgo_quantize_group_m.argtypes = [P, i, i, i, i, P, P, P]
+        L.hgo_quantize_group_m.restype = None
+        L.hgo_f32_to_f16.argtypes = [ctypes.c_float]
+        L.hgo_f32_to_f16.restype = ctypes.c_uint16
+        L.hgo_f16_to_f32.argtypes = [ctypes.c_uint16]
+        L.hgo_f16_to_f32.restype = ctypes.c_float
         L.hgo_dequant.argtypes = [ctypes.c_uint8, ctypes.c_float, ctypes.c_float]
         L.hgo_dequant.restype = ctypes.c_float
         L.hgo_pack.argtypes = [P, i, i, P]
@@ -53,6 +59,8 @@ def lib():
         L.hgo_quantize_head.restype = i
         L.hgo_quantize_layer.argtypes = [P, P, i, i, i, i, i, i, i, P, i, i, i, i] + [P] * 9
         L.hgo_quantize_layer.restype = i
+        L.hgo_quantize_layer_m.argtypes = [P, P, i, i, i, i, i, i, i, i, P, i, i, i, i] + [P] * 9
+        L.hgo_quantize_layer_m.restype = i
         L.hgo_attention_layer.argtypes = [P, P, P, i, i, i, i, ctypes.c_double, P]
         L.hgo_attention_layer.restype = i
         L.hgo_image_bits_per_elem.argtypes = [i, i, i, ctypes.c_double, i]
@@ -79,14 +87,28 @@ def bf16_bits_to_f32(bits):
     return (b.astype(np.uint32) << 16).view(np.float32)
 
 
-def quantize_group(x, bits):
-    """Sec. 1 group quantizer: (codes uint8[n], scale f32, zero f32)."""
+def quantize_group(x, bits, meta16=False):
+    """Sec. 1 group quantizer: (codes uint8[n], scale f32, zero f32).  With
+    meta16 (Sec. 5.4 32-bit metadata, reading R13) scale and zero are the
+    stored binary16 values and the codes are computed against them."""
     x = _c(x, np.float32)
     codes = np.zeros(x.size, np.uint8)
     sc = np.zeros(1, np.float32)
     ze = np.zeros(1, np.float32)
-    lib().hgo_quantize_group(_ptr(x), x.size, 1, bits, _ptr(codes), _ptr(sc), _ptr(ze))
+    if meta16:
+        lib().hgo_quantize_group_m(_ptr(x), x.size, 1, bits, 1, _ptr(codes), _ptr(sc), _ptr(ze))
+    else:
+        lib().hgo_quantize_group(_ptr(x), x.size, 1, bits, _ptr(codes), _ptr(sc), _ptr(ze))
     return codes, np.float32(sc[0]), np.float32(ze[0])
+
+
+def f32_to_f16_bits(x):
+    """binary32 -> binary16 bits, round to nearest even, |x| >= 65504 saturating (R13)."""
+    return np.uint16(lib().hgo_f32_to_f16(float(np.float32(x))))
+
+
+def f16_bits_to_f32(h):
+    return np.float32(lib().hgo_f16_to_f32(int(h)))
 
 
 def dequant(code, scale, zero):
@@ -138,7 +160,7 @@ def image_bits_per_elem(bits, meta_bits, frac_protected, keys_only, head_dim=D):
 # --------------------------------------------------------------------------
 
 def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
-                   group_tokens=32, group_channels=32, residual=32, want_att=True):
+                   group_tokens=32, group_channels=32, residual=32, want_att=True, meta16=False):
     """Quantize one layer.
 
     k_bits, v_bits: uint16 [B][H][T][128] BF16 bit patterns.
@@ -169,7 +191,7 @@ def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
         k_deq=np.zeros((B, H, T, D), np.float32), v_deq=np.zeros((B, H, T, D), np.float32),
         k_att=np.zeros((B, H, T, D), np.float64) if want_att else None,
     )
-    lib().hgo_quantize_layer(_ptr(k_bits), _ptr(v_bits), B, H, T, s, n, base, bits,
+    lib().hgo_quantize_layer_m(_ptr(k_bits), _ptr(v_bits), B, H, T, s, n, base, bits, int(meta16),
                              _ptr(head_mask), int(keys_only), group_tokens, group_channels,
                              residual, _ptr(out["kq"]), _ptr(out["vq"]), _ptr(out["k_words"]),
                              _ptr(out["k_meta"]), _ptr(out["v_words"]), _ptr(out["v_meta"]),

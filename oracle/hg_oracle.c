@@ -37,6 +37,10 @@
  *      qh / G, the decoded token attends to its own appended entry;
  *   R12 signed zeros: the group min and max are canonicalised with "+ 0.0f"
  *      so the stored metadata has one bit pattern.
+ *   R13 32-bit metadata (the Sec. 5.4 storage model, optional): scale and
+ *      zero are stored as binary16 (round to nearest even, magnitudes above
+ *      65504 saturate to 65504), and the codes are computed against the
+ *      stored values, so reconstruction uses exactly what is stored.
  */
 #include <math.h>
 #include <stdint.h>
@@ -74,8 +78,47 @@ float hgo_bf16_to_f32(uint16_t h)
  *            = clamp(rint_even( fl32( fl32(x_i - mn) / scale ) ), 0, 2^b - 1)
  *   zero     = mn
  */
-void hgo_quantize_group(const float *x, int n, int stride, int bits,
-                        uint8_t *codes, float *scale_out, float *zero_out)
+/* IEEE binary16 bits of a binary32 value: round to nearest even; magnitudes
+ * of 65504 and above (and non-finite values) saturate to +-65504 (R13). */
+uint16_t hgo_f32_to_f16(float f)
+{
+    uint32_t u;
+    memcpy(&u, &f, 4);
+    const uint32_t sign = (u >> 16) & 0x8000u;
+    const uint32_t a = u & 0x7fffffffu;
+    if (a >= 0x477fe000u) return (uint16_t)(sign | 0x7bffu);    /* >= 65504 */
+    if (a <= 0x33000000u) return (uint16_t)sign;                 /* <= 2^-25: rounds to 0 */
+    if (a < 0x38800000u) {                                       /* below 2^-14: subnormal */
+        const uint32_t e = a >> 23, m = (a & 0x7fffffu) | 0x800000u;
+        const uint32_t sh = 126u - e;                            /* value / 2^-24 = m / 2^sh */
+        uint32_t q = m >> sh;
+        const uint32_t rem = m & ((1u << sh) - 1u), half = 1u << (sh - 1u);
+        if (rem > half || (rem == half && (q & 1u))) ++q;
+        return (uint16_t)(sign | q);
+    }
+    uint32_t r = (a - 0x38000000u) >> 13;                        /* rebias 127 -> 15, 23 -> 10 bits */
+    const uint32_t rem = a & 0x1fffu;
+    if (rem > 0x1000u || (rem == 0x1000u && (r & 1u))) ++r;
+    return (uint16_t)(sign | r);
+}
+
+float hgo_f16_to_f32(uint16_t h)
+{
+    const uint32_t sign = ((uint32_t)h & 0x8000u) << 16;
+    const uint32_t e = ((uint32_t)h >> 10) & 0x1fu, m = (uint32_t)h & 0x3ffu;
+    float f;
+    if (e == 0) {
+        f = (float)m * 5.9604644775390625e-8f; /* m * 2^-24, exact */
+    } else {
+        const uint32_t u = ((e + 112u) << 23) | (m << 13);
+        memcpy(&f, &u, 4);
+    }
+    return sign ? -f : f;
+}
+
+/* The group quantizer with the metadata width as a parameter (meta16: R13). */
+void hgo_quantize_group_m(const float *x, int n, int stride, int bits, int meta16,
+                          uint8_t *codes, float *scale_out, float *zero_out)
 {
     float mn = x[0], mx = x[0];
     for (int i = 1; i < n; ++i) {
@@ -83,25 +126,35 @@ void hgo_quantize_group(const float *x, int n, int stride, int bits,
         if (xi < mn) mn = xi;
         if (xi > mx) mx = xi;
     }
-    mn = mn + 0.0f; /* R12: -0 becomes +0 */
+    mn = mn + 0.0f; /* R12 */
     mx = mx + 0.0f;
     const float levels = (float)((1 << bits) - 1);
-    const float range = mx - mn;
-    const float scale = range / levels;
+    float scale = (mx - mn) / levels;
+    float zero = mn;
+    if (meta16) {
+        scale = hgo_f16_to_f32(hgo_f32_to_f16(scale));
+        zero = hgo_f16_to_f32(hgo_f32_to_f16(zero));
+    }
     for (int i = 0; i < n; ++i) {
         if (scale == 0.0f) {
             codes[i] = 0;
             continue;
         }
-        float d = x[(long)i * stride] - mn;
+        float d = x[(long)i * stride] - zero;
         float q = d / scale;
-        float r = nearbyintf(q); /* default rounding mode: nearest, ties to even */
+        float r = nearbyintf(q);
         if (r < 0.0f) r = 0.0f;
         if (r > levels) r = levels;
         codes[i] = (uint8_t)r;
     }
     *scale_out = scale;
-    *zero_out = mn;
+    *zero_out = zero;
+}
+
+void hgo_quantize_group(const float *x, int n, int stride, int bits,
+                        uint8_t *codes, float *scale_out, float *zero_out)
+{
+    hgo_quantize_group_m(x, n, stride, bits, 0, codes, scale_out, zero_out);
 }
 
 /* Sec. 4 "reconstructed as floating-point values": x^ = fl32(fl32(code*scale) + zero). */
@@ -223,8 +276,8 @@ int hgo_quantized_count(int T, int s, int n, int base, int group_tokens, int res
  *                                  be NULL
  *   Returns nq.  Metadata pairs are (scale, zero).
  */
-int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
-                      int base, int bits, int protect, int keys_only,
+int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int n,
+                      int base, int bits, int meta16, int protect, int keys_only,
                       int group_tokens, int group_channels, int residual,
                       uint8_t *kq, uint8_t *vq,
                       uint32_t *k_words, float *k_meta,
@@ -263,7 +316,7 @@ int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
                     float scale, zero;
                     for (int e = 0; e < group_tokens; ++e)
                         col[e] = hgo_bf16_to_f32(k[(long)(t0 + e) * D + c]);
-                    hgo_quantize_group(col, group_tokens, 1, bits, codes, &scale, &zero);
+                    hgo_quantize_group_m(col, group_tokens, 1, bits, meta16, codes, &scale, &zero);
                     long row = (long)g * D + c;
                     hgo_pack(codes, group_tokens, bits, k_words + row * (group_tokens * bits / 32));
                     k_meta[row * 2 + 0] = scale;
@@ -281,7 +334,7 @@ int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
                 float scale, zero;
                 for (int c = 0; c < D; ++c) xk[c] = hgo_bf16_to_f32(k[(long)t * D + c]);
                 if (base == HGO_BASE_AKVQ) hgo_fwht128(xk); /* rotate, then per-token RTN */
-                hgo_quantize_group(xk, D, 1, bits, codes, &scale, &zero);
+                hgo_quantize_group_m(xk, D, 1, bits, meta16, codes, &scale, &zero);
                 hgo_pack(codes, D, bits, k_words + (long)i * wpt);
                 k_meta[(long)i * 2 + 0] = scale;
                 k_meta[(long)i * 2 + 1] = zero;
@@ -313,7 +366,7 @@ int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
             for (int c = 0; c < D; ++c) xv[c] = hgo_bf16_to_f32(v[(long)t * D + c]);
             for (int j = 0; j < ngr; ++j) {
                 float scale, zero;
-                hgo_quantize_group(xv + j * gsize, gsize, 1, bits, codes + j * gsize, &scale, &zero);
+                hgo_quantize_group_m(xv + j * gsize, gsize, 1, bits, meta16, codes + j * gsize, &scale, &zero);
                 v_meta[((long)i * ngr + j) * 2 + 0] = scale;
                 v_meta[((long)i * ngr + j) * 2 + 1] = zero;
                 for (int e = 0; e < gsize; ++e)
@@ -336,8 +389,8 @@ int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
  * head_mask[h] is the layer's protection mask.  Parallel over (b, h) when
  * built with OpenMP; every head is computed independently.
  */
-int hgo_quantize_layer(const uint16_t *k, const uint16_t *v, int B, int H, int T,
-                       int s, int n, int base, int bits, const uint8_t *head_mask,
+int hgo_quantize_layer_m(const uint16_t *k, const uint16_t *v, int B, int H, int T,
+                       int s, int n, int base, int bits, int meta16, const uint8_t *head_mask,
                        int keys_only, int group_tokens, int group_channels, int residual,
                        uint8_t *kq, uint8_t *vq,
                        uint32_t *k_words, float *k_meta, uint32_t *v_words, float *v_meta,
@@ -352,12 +405,38 @@ int hgo_quantize_layer(const uint16_t *k, const uint16_t *v, int B, int H, int T
     for (int bh = 0; bh < B * H; ++bh) {
         const int h = bh % H;
         const long tok = (long)bh * T;
-        hgo_quantize_head(k + tok * D, v + tok * D, T, s, n, base, bits, head_mask[h], keys_only,
+        hgo_quantize_head_m(k + tok * D, v + tok * D, T, s, n, base, bits, meta16, head_mask[h], keys_only,
                           group_tokens, group_channels, residual, kq + tok, vq + tok,
                           k_words + bh * kw, k_meta + bh * km, v_words + bh * kw, v_meta + bh * vm,
                           k_deq + tok * D, v_deq + tok * D, k_att ? k_att + tok * D : NULL);
     }
     return nq;
+}
+
+/* The 64-bit-metadata forms (R5). */
+int hgo_quantize_head(const uint16_t *k, const uint16_t *v, int T, int s, int n,
+                      int base, int bits, int protect, int keys_only,
+                      int group_tokens, int group_channels, int residual,
+                      uint8_t *kq, uint8_t *vq,
+                      uint32_t *k_words, float *k_meta,
+                      uint32_t *v_words, float *v_meta,
+                      float *k_deq, float *v_deq, double *k_att)
+{
+    return hgo_quantize_head_m(k, v, T, s, n, base, bits, 0, protect, keys_only, group_tokens,
+                               group_channels, residual, kq, vq, k_words, k_meta, v_words, v_meta,
+                               k_deq, v_deq, k_att);
+}
+
+int hgo_quantize_layer(const uint16_t *k, const uint16_t *v, int B, int H, int T,
+                       int s, int n, int base, int bits, const uint8_t *head_mask,
+                       int keys_only, int group_tokens, int group_channels, int residual,
+                       uint8_t *kq, uint8_t *vq,
+                       uint32_t *k_words, float *k_meta, uint32_t *v_words, float *v_meta,
+                       float *k_deq, float *v_deq, double *k_att)
+{
+    return hgo_quantize_layer_m(k, v, B, H, T, s, n, base, bits, 0, head_mask, keys_only,
+                                group_tokens, group_channels, residual, kq, vq, k_words, k_meta,
+                                v_words, v_meta, k_deq, v_deq, k_att);
 }
 
 /* ------------------------------------------------------------------------ */
