@@ -43,6 +43,8 @@ def parse_args():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="headguard", choices=["headguard", "reference"])
     ap.add_argument("--workload", default="qwen25vl7b")
+    ap.add_argument("--meta-bits", type=int, default=64, choices=[64, 32],
+                    help="metadata per group: fp32 pair (64) or binary16 pair (32, Sec. 5.4)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -208,15 +210,16 @@ def oracle_sample(w, n_layers, n_steps):
         t0 = time.perf_counter()
         o = oracle.quantize_layer(kb, vb, w.img_start, w.image, w.base, w.bits, mask[l],
                                   int(w.keys_only), w.kivi_group_tokens, w.kivi_group_channels,
-                                  w.kivi_residual)
+                                  w.kivi_residual, meta16=w.meta_bits == 32)
         secs += time.perf_counter() - t0
         nq = o["nq"]
         code_tok = 128 * w.bits // 8
         n_prot = int(mask[l].sum())
         coded_heads_k = (H - n_prot)
         coded_heads_v = H if w.keys_only else (H - n_prot)
-        meta_k = o["k_meta"][0, 0].nbytes if coded_heads_k else 0
-        meta_v = o["v_meta"][0, 0].nbytes if coded_heads_v else 0
+        shrink = 2 if w.meta_bits == 32 else 1  # binary16 pairs: half the fp32 pair bytes
+        meta_k = o["k_meta"][0, 0].nbytes // shrink if coded_heads_k else 0
+        meta_v = o["v_meta"][0, 0].nbytes // shrink if coded_heads_v else 0
         written = B * (H * T * 512 - (coded_heads_k + coded_heads_v) * nq * 256
                        + coded_heads_k * (nq * code_tok + meta_k)
                        + coded_heads_v * (nq * code_tok + meta_v))
@@ -247,8 +250,9 @@ def oracle_sample(w, n_layers, n_steps):
 def _decode_bytes_layer(w, mask_row, nq, appended):
     B, H, T = w.batch, w.kv_heads, w.seq_len
     code_tok = 128 * w.bits // 8
-    kmeta = (128 * 8 // 32) if w.base == 1 else 8
-    vmeta = 32 if w.base == 1 else 8
+    pair = 4 if w.meta_bits == 32 else 8  # bytes of one {scale, zero}
+    kmeta = (128 * pair // 32) if w.base == 1 else pair
+    vmeta = 4 * pair if w.base == 1 else pair
     tot = 0
     for h in range(H):
         prot = bool(mask_row[h])
@@ -269,12 +273,21 @@ def cpu_sample_plan(w):
     return 1, 2
 
 
+def _workload(args):
+    import dataclasses
+    from paper_2609_35800_gb300 import workloads as wl
+    w = wl.WORKLOADS[args.workload]
+    if args.meta_bits != w.meta_bits:
+        w = dataclasses.replace(w, meta_bits=args.meta_bits, name=w.name + "_meta%d" % args.meta_bits)
+    return w
+
+
 def run_reference(args):
     from paper_2609_35800_gb300 import workloads as wl
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
-    w = wl.WORKLOADS[args.workload]
+    w = _workload(args)
     n_layers, n_steps = cpu_sample_plan(w)
     vals = []
     tot_s = 0.0
@@ -326,7 +339,7 @@ def run_gpu(args):
         dist.barrier()
     hg.library()
 
-    w = wl.WORKLOADS[args.workload]
+    w = _workload(args)
     dev = "cuda:%d" % local
     stream = torch.cuda.current_stream()
     runner = CacheRunner(w, device=dev)

@@ -87,7 +87,11 @@ typedef struct hg_shape {
 /* Quantizer configuration.  bits in {2, 4}.  keys_only selects K-only protection
  * (Sec. 3: protected heads keep image keys BF16, their image values follow the
  * base).  The KIVI-style group sizes must be 32; kivi_residual >= 0 is the number
- * of trailing prefill tokens kept BF16.  Unused fields are ignored for other bases. */
+ * of trailing prefill tokens kept BF16.  Unused fields are ignored for other bases.
+ * meta_bits: metadata per group, 64 (or 0: the default) = an fp32 {scale, zero}
+ * pair; 32 = a binary16 pair, the Sec. 5.4 storage model (2.25 bits per element
+ * at 2 bits): scale and zero are rounded to nearest-even binary16 (magnitudes
+ * >= 65504 saturate) and the codes are computed against the stored values. */
 typedef struct hg_quant_config {
     int32_t base;
     int32_t bits;
@@ -95,6 +99,7 @@ typedef struct hg_quant_config {
     int32_t kivi_group_tokens;
     int32_t kivi_group_channels;
     int32_t kivi_residual;
+    int32_t meta_bits;
 } hg_quant_config;
 
 /* Opaque host-side descriptor of a cache arena (offsets, mask, appended counts). */

@@ -57,7 +57,7 @@ class Shape(ctypes.Structure):
 class QuantConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "base", "bits", "keys_only", "kivi_group_tokens", "kivi_group_channels",
-        "kivi_residual")]
+        "kivi_residual", "meta_bits")]
 
 
 class HeadRegions(ctypes.Structure):

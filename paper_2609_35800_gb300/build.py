@@ -18,7 +18,7 @@ INCLUDE = os.path.join(ROOT, "include")
 OUT_DIR = os.path.join(HERE, "_build")
 LIB_NAME = "libheadguard.so"
 LIB = os.path.join(OUT_DIR, LIB_NAME)
-SOURCES = ["hg_api.cu", "hg_quantize.cu", "hg_decode.cu", "hg_noalloc.cu"]
+SOURCES = ["hg_api.cu", "hg_quantize.cu", "hg_decode.cu", "hg_decode_m16.cu", "hg_noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
               "-I" + INCLUDE, "-I" + CSRC]

@@ -54,6 +54,7 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
     return HG_ERR_INVALID_ARG;
   if (c->bits != 2 && c->bits != 4) return HG_ERR_UNSUPPORTED;
   if (c->keys_only != 0 && c->keys_only != 1) return HG_ERR_INVALID_ARG;
+  if (c->meta_bits != 0 && c->meta_bits != 32 && c->meta_bits != 64) return HG_ERR_INVALID_ARG;
   if (c->base == HG_BASE_KIVI) {
     if (c->kivi_group_tokens != kKiviGroup || c->kivi_group_channels != kKiviGroup)
       return HG_ERR_UNSUPPORTED;
@@ -77,6 +78,7 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   d->bits = c->bits;
   d->keys_only = c->keys_only;
   d->residual = c->base == HG_BASE_KIVI ? c->kivi_residual : 0;
+  d->meta16 = c->meta_bits == 32 ? 1 : 0;
   d->nq = quantized_count(d->T, d->s, d->n, d->base, d->residual);
   return HG_OK;
 }
@@ -163,8 +165,9 @@ struct SegBytes {
 SegBytes seg_bytes(const Dims& d) {
   SegBytes b;
   const double codes = 16.0 * d.bits;  // 128 codes
-  const double kmeta = d.base == kKivi ? 32.0 : 8.0;
-  const double vmeta = 8.0 * vgroups(d);
+  const double pair = (double)meta_pair_bytes(d);
+  const double kmeta = d.base == kKivi ? 4.0 * pair : pair;
+  const double vmeta = pair * vgroups(d);
   const double instr_u = d.base == kKivi ? (d.bits == 2 ? 66.0 : 78.0) : (d.bits == 2 ? 30.0 : 40.0);
   b.bf16 = 512.0 + 8.0 * 5.0;
   b.coded_u = 2.0 * codes + kmeta + vmeta + 8.0 * instr_u;
@@ -686,8 +689,9 @@ hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {
   // stored bits over all image K/V elements of the cache
   double stored = 0.0;
   const double code_bits = (double)d.bits * kD;                 // per coded token vector
-  const double kmeta_tok = d.base == kKivi ? 64.0 * kD / kKiviGroup : 64.0;
-  const double vmeta_tok = 64.0 * vgroups(d);
+  const double pair = 8.0 * meta_pair_bytes(d);  // bits of one {scale, zero}
+  const double kmeta_tok = d.base == kKivi ? pair * kD / kKiviGroup : pair;
+  const double vmeta_tok = pair * vgroups(d);
   for (int l = 0; l < d.L; ++l) {
     for (int h = 0; h < d.H; ++h) {
       const int cls = head_class(d, c->layer_mask[l], h);

@@ -4,6 +4,7 @@
 // zero, reconstructed values) uses an explicit round-to-nearest intrinsic so
 // that the compiler can neither fuse nor reorder it.
 #pragma once
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -67,6 +68,36 @@ __device__ __forceinline__ void fwht128_warp(float (&x)[4], int lane) {
   for (int i = 0; i < 4; ++i) x[i] = __fmul_rn(x[i], c);
 }
 
+// Metadata pairs {scale, zero}: two fp32 (8 bytes) or, with the 32-bit
+// storage model of Sec. 5.4, two binary16 (4 bytes, scale in the low half).
+// A binary16 value is rounded to nearest even and saturates at +-65504; the
+// codes are then computed against the stored (rounded) scale and zero, so the
+// reconstruction uses exactly what the cache holds.  Since the rounded zero
+// can lie above the group minimum and the rounded scale below the true step,
+// a quotient may fall outside [0, levels]; the clamp of code_of below covers
+// it (only quotients in [0, levels] decide a code, and there its near-tie
+// bound holds).
+__device__ __forceinline__ float half_sat(float x) {
+  return __half2float(__float2half_rn(fminf(fmaxf(x, -65504.0f), 65504.0f)));
+}
+__device__ __forceinline__ void store_meta(char* base, size_t i, float scale, float zero, bool m16) {
+  if (m16) {
+    // scale and zero are binary16 values already: the conversion is exact
+    *reinterpret_cast<__half2*>(base + i * 4) = __floats2half2_rn(scale, zero);
+  } else {
+    reinterpret_cast<float2*>(base)[i] = make_float2(scale, zero);
+  }
+}
+__device__ __forceinline__ float2 half2_bits_to_float2(uint32_t w) {
+  __half2 h;
+  *reinterpret_cast<uint32_t*>(&h) = w;
+  return __half22float2(h);
+}
+__device__ __forceinline__ float2 load_meta(const char* base, size_t i, bool m16) {
+  if (m16) return half2_bits_to_float2(__ldg(reinterpret_cast<const uint32_t*>(base) + i));
+  return __ldg(reinterpret_cast<const float2*>(base) + i);
+}
+
 // code = clamp(rint_even(fl32(d / scale)), 0, levels) computed without a
 // division in almost every case.  With r = fl32(1 / scale) and q' = fl32(d r),
 // q' = (d / scale)(1 + e1)(1 + e2) with |e1|, |e2| <= 2^-24, and the correctly
@@ -92,9 +123,11 @@ __device__ __forceinline__ uint32_t code_of(float d, float scale, float r, float
 // Group quantizer over a group spread across GL consecutive lanes (aligned),
 // 4 values per lane.  min / max by butterflies (exact), signed zeros folded to
 // +0, scale = (max - min) / (2^bits - 1), code = round-half-even((x - min) /
-// scale) clamped to the levels, codes 0 when scale == 0, zero = min.
+// scale) clamped to the levels, codes 0 when scale == 0, zero = min.  With
+// m16 the scale and zero are first rounded to binary16 and the codes taken
+// against the rounded pair.
 template <int GL>
-__device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, uint32_t (&code)[4],
+__device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, bool m16, uint32_t (&code)[4],
                                                 float& scale, float& zero) {
   float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
   float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
@@ -108,11 +141,15 @@ __device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, u
   const float levels = (float)((1 << bits) - 1);
   scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   zero = mn;
+  if (m16) {
+    scale = half_sat(scale);
+    zero = half_sat(zero);
+  }
   const bool fast = scale >= 2.3509887e-38f;  // 2^-125
   const float r = __frcp_rn(fast ? scale : 1.0f);
 #pragma unroll
   for (int i = 0; i < 4; ++i)
-    code[i] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[i], mn), scale, r, levels, fast);
+    code[i] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[i], zero), scale, r, levels, fast);
 }
 
 // Reconstruction fl32(fl32(code * scale) + zero).

@@ -106,12 +106,9 @@ cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s);
 cudaError_t launch_wait_probe(uint32_t* result, uint32_t rounds, cudaStream_t s);
-// Tokens per pipeline tile of coded K + coded V (chunk sizes are multiples of it).
-int decode_coded_tile(int bits);
+// The decode kernels for binary16 metadata pairs (called by launch_decode).
+cudaError_t launch_decode_m16(const DecodeParams& p, int grid_x, cudaStream_t s);
 // Most splits of one head the decode kernel's merge can take.
 int decode_max_splits(int G);
-// Largest chunk (tokens) whose tiles all fit the kernel's pipeline buffer at
-// once, for BF16 chunks, coded chunks and keys-only coded chunks.
-void decode_chunk_capacity(int bits, int base, int* bf16, int* coded, int* keys_only);
 
 }  // namespace hg

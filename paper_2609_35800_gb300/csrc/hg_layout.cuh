@@ -28,6 +28,7 @@ enum HeadClass : int { kQuantized = 0, kKeysOnly = 1, kProtected = 2 };
 struct Dims {
   int B, L, H, Hq, G, T, s, n, nq, S_new;
   int base, bits, keys_only, residual;
+  int meta16;  // metadata pairs as binary16 {scale, zero} (4 bytes) instead of fp32 (8)
 };
 
 HG_HD uint64_t align_up(uint64_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
@@ -55,13 +56,16 @@ HG_HD int quantized_count(int T, int s, int n, int base, int residual) {
 // Bytes per token of one head's packed codes (128 codes).
 HG_HD uint64_t code_bytes_per_token(const Dims& d) { return (uint64_t)kD * d.bits / 8; }
 HG_HD uint64_t align16(uint64_t x) { return (x + 15) & ~15ull; }
+// Bytes of one {scale, zero} metadata pair.
+HG_HD uint64_t meta_pair_bytes(const Dims& d) { return d.meta16 ? 4 : 8; }
 // Key metadata bytes for nq tokens of one batch row of one head (payload).
 HG_HD uint64_t kmeta_bytes(const Dims& d) {
-  return d.base == kKivi ? (uint64_t)(d.nq / kKiviGroup) * kD * 8 : (uint64_t)d.nq * 8;
+  return d.base == kKivi ? (uint64_t)(d.nq / kKiviGroup) * kD * meta_pair_bytes(d)
+                         : (uint64_t)d.nq * meta_pair_bytes(d);
 }
 // Value metadata groups per token.
 HG_HD int vgroups(const Dims& d) { return d.base == kKivi ? kD / kKiviGroup : 1; }
-HG_HD uint64_t vmeta_bytes(const Dims& d) { return (uint64_t)d.nq * vgroups(d) * 8; }
+HG_HD uint64_t vmeta_bytes(const Dims& d) { return (uint64_t)d.nq * vgroups(d) * meta_pair_bytes(d); }
 // Batch-row strides of the metadata arrays: padded to 16 bytes so that every
 // row (and every head's block of rows) starts on a 16-byte boundary, as the
 // 16-byte asynchronous copies of the decode kernel require.

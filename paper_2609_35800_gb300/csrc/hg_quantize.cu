@@ -60,7 +60,7 @@ __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
 }
 
 // One 32-value group held by a single thread (KIVI-style key channel group).
-__device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGroup], int bits,
+__device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGroup], int bits, bool m16,
                                                       uint32_t (&code)[kKiviGroup], float& scale,
                                                       float& zero) {
   float mn = x[0], mx = x[0];
@@ -74,11 +74,15 @@ __device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGrou
   const float levels = (float)((1 << bits) - 1);
   scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   zero = mn;
+  if (m16) {
+    scale = half_sat(scale);
+    zero = half_sat(zero);
+  }
   const bool fast = scale >= 2.3509887e-38f;  // 2^-125
   const float r = __frcp_rn(fast ? scale : 1.0f);
 #pragma unroll
   for (int e = 0; e < kKiviGroup; ++e)
-    code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], mn), scale, r, levels, fast);
+    code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], zero), scale, r, levels, fast);
 }
 
 __global__ void __launch_bounds__(kThreads)
@@ -102,6 +106,7 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   const uint16_t* V = p.v[li] + row0 * kD;
   const int qs = d.s, qe = d.s + d.nq;
   const int W = kD * d.bits / 32;  // code words per token
+  const bool m16 = d.meta16 != 0;
   // A whole KIVI-style key group of a quantized head: tokens [t0, t0 + 32).
   const bool kivi_k_tile = (d.base == kKivi) && (hd.cls == kQuantized) && t0 >= qs && t1 <= qe;
 
@@ -135,11 +140,10 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
         if (d.base == kAkvq) fwht128_warp(x, lane);  // rotate, then per-token RTN
         uint32_t c[4];
         float sc, z;
-        quantize_group4<32>(x, d.bits, c, sc, z);
+        quantize_group4<32>(x, d.bits, m16, c, sc, z);
         uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W;
         store_token_codes(crow, c, d.bits, lane);
-        if (lane == 0)
-          reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs)[ti] = make_float2(sc, z);
+        if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ti, sc, z, m16);
       }
     } else if (coded && hd.cls == kKeysOnly) {
       *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) =
@@ -156,13 +160,14 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
       bf16x4_to_f32(vr[i], x);
       uint32_t c[4];
       float sc, z;
-      float2* meta = reinterpret_cast<float2*>(Lb + hd.vqm + b * hd.vqm_bs) + (size_t)ti * vgroups(d);
+      char* meta = Lb + hd.vqm + b * hd.vqm_bs;
+      const size_t mi = (size_t)ti * vgroups(d);
       if (d.base == kKivi) {
-        quantize_group4<8>(x, d.bits, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
-        if ((lane & 7) == 0) meta[lane >> 3] = make_float2(sc, z);
+        quantize_group4<8>(x, d.bits, m16, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
+        if ((lane & 7) == 0) store_meta(meta, mi + (lane >> 3), sc, z, m16);
       } else {
-        quantize_group4<32>(x, d.bits, c, sc, z);
-        if (lane == 0) meta[0] = make_float2(sc, z);
+        quantize_group4<32>(x, d.bits, m16, c, sc, z);
+        if (lane == 0) store_meta(meta, mi, sc, z, m16);
       }
       uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W;
       store_token_codes(crow, c, d.bits, lane);
@@ -182,7 +187,7 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   for (int e = 0; e < kKiviGroup; ++e) x[e] = bf16_to_f32(ktile[e][c]);
   uint32_t code[kKiviGroup];
   float sc, z;
-  quantize_group_serial(x, d.bits, code, sc, z);
+  quantize_group_serial(x, d.bits, m16, code, sc, z);
   const int grp = (t0 - qs) / kKiviGroup;
   uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * d.bits;
   const int per = 32 / d.bits;
@@ -191,7 +196,7 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
     for (int e = 0; e < per; ++e) word |= code[w * per + e] << (d.bits * e);
     dst[w] = word;
   }
-  reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs)[(size_t)grp * kD + c] = make_float2(sc, z);
+  store_meta(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + c, sc, z, m16);
 }
 
 // ---------------------------------------------------------------------------
@@ -221,8 +226,8 @@ __device__ __noinline__ uint32_t exact_code(float d, float scale, float levels) 
   return (uint32_t)fminf(fmaxf(rintf(__fdiv_rn(d, scale)), 0.0f), levels);
 }
 
-template <int BITS>
-__device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, float2* meta) {
+template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
   const uint4* r4 = reinterpret_cast<const uint4*>(row_s);
   __nv_bfloat162 mn2, mx2;
   {
@@ -246,12 +251,51 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   mx = __fadd_rn(mx, 0.0f);
   constexpr uint32_t L = (1u << BITS) - 1u;
   const float levels = (float)L;
-  const float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
-  *meta = make_float2(scale, mn);
+  float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  if (M16) {  // binary16 metadata: codes against the stored pair
+    scale = half_sat(scale);
+    mn = half_sat(mn);
+  }
+  store_meta(meta, mi, scale, mn, M16);
   constexpr int W = 4 * BITS;  // code words per token
-  if (scale == 0.0f) {  // constant vector: every code 0
+  if (scale == 0.0f) {  // constant vector (or a step below binary16 range): every code 0
 #pragma unroll
     for (int i = 0; i < W; ++i) codes[i] = 0u;
+    return;
+  }
+  if (M16) {
+    // A binary16 scale is at least 2^-24, so r is finite.  The rounded zero
+    // and scale can put a quotient outside [0, levels]: q = d r is clamped to
+    // [-1, levels + 1] (which decides no code differently), then T =
+    // RN(q + 192) lies in [191, 193 + levels] and bits 16.. of T + 0x8001,
+    // less 0x4340, are the unclamped code.  The two roundings (q, then T) keep
+    // T within 2^-16 of fl(d / scale) + 192 for quotients that can decide a
+    // code, so the near-tie test is the same as below.
+    const float r = __frcp_rn(scale);
+    uint32_t prev = 0u;
+#pragma unroll 2
+    for (int k = 0; k < 16; ++k) {
+      const uint4 v = r4[k];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t chunk = 0u;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint32_t hw = w[i >> 1];
+        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
+        const float q = fminf(fmaxf(__fmul_rn(d, r), -1.0f), levels + 1.0f);
+        const uint32_t a = __float_as_uint(__fadd_rn(q, 192.0f)) + 0x8001u;
+        const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
+        const uint32_t code = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
+        chunk |= code << (BITS * i);
+      }
+      if (BITS == 4) {
+        codes[k] = chunk;
+      } else if (k & 1) {
+        codes[k >> 1] = prev | (chunk << 16);
+      } else {
+        prev = chunk;
+      }
+    }
     return;
   }
   if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
@@ -300,7 +344,7 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   }
 }
 
-template <int BITS>
+template <int BITS, bool M16>
 __global__ void __launch_bounds__(kThreads)
 quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
   const Dims& d = p.d;
@@ -335,8 +379,8 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
   constexpr int W = 4 * BITS;
   if (kv == 0) {
     if (coded && hd.cls == kQuantized) {
-      quantize_row_token<BITS>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
-                               reinterpret_cast<float2*>(Lb + hd.kqm + b * hd.kqm_bs) + ti);
+      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
+                                    Lb + hd.kqm + b * hd.kqm_bs, ti);
       return;
     }
     char* dst = (coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
@@ -346,8 +390,8 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
       reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
   } else {
     if (coded && hd.cls != kProtected) {
-      quantize_row_token<BITS>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
-                               reinterpret_cast<float2*>(Lb + hd.vqm + b * hd.vqm_bs) + ti);
+      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+                                    Lb + hd.vqm + b * hd.vqm_bs, ti);
       return;
     }
     char* dst = Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
@@ -370,6 +414,7 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
   const char* Lb = p.arena + p.layer_base;
   const int qs = d.s, qe = d.s + d.nq;
   const int W = kD * d.bits / 32;
+  const bool m16 = d.meta16 != 0;
 
   for (int t = blockIdx.x * kTile + warp; t < min(Tt, (int)(blockIdx.x + 1) * kTile); t += 4) {
     const bool coded = (t >= qs) && (t < qe);
@@ -382,19 +427,19 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
         const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
         const int per = 32 / d.bits;
         const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs);
-        const float2* meta = reinterpret_cast<const float2*>(Lb + hd.kqm + b * hd.kqm_bs);
+        const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const size_t row = (size_t)grp * kD + lane * 4 + i;
           const uint32_t w = __ldg(codes + row * d.bits + e / per);
           const uint32_t code = (w >> (d.bits * (e % per))) & ((1u << d.bits) - 1u);
-          const float2 m = __ldg(meta + row);
+          const float2 m = load_meta(meta, row, m16);
           xk[i] = dequant1(code, m.x, m.y);
         }
       } else {
         load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
                          d.bits, lane, c);
-        const float2 m = __ldg(reinterpret_cast<const float2*>(Lb + hd.kqm + b * hd.kqm_bs) + ti);
+        const float2 m = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ti, m16);
 #pragma unroll
         for (int i = 0; i < 4; ++i) xk[i] = dequant1(c[i], m.x, m.y);
         if (d.base == kAkvq) fwht128_warp(xk, lane);  // inverse rotation (H is self-inverse)
@@ -408,9 +453,8 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
       uint32_t c[4];
       load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
                        d.bits, lane, c);
-      const float2* meta = reinterpret_cast<const float2*>(Lb + hd.vqm + b * hd.vqm_bs) +
-                           (size_t)ti * vgroups(d);
-      const float2 m = __ldg(meta + (d.base == kKivi ? (lane >> 3) : 0));
+      const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
+                                 (size_t)ti * vgroups(d) + (d.base == kKivi ? (lane >> 3) : 0), m16);
 #pragma unroll
       for (int i = 0; i < 4; ++i) xv[i] = dequant1(c[i], m.x, m.y);
     } else {
@@ -456,8 +500,14 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
   if (p.d.base == kMinMax) {  // one thread per vector
     dim3 grid((p.d.T + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
-    if (p.d.bits == 2) quantize_minmax_kernel<2><<<grid, kThreads, 0, s>>>(p);
-    else quantize_minmax_kernel<4><<<grid, kThreads, 0, s>>>(p);
+    const bool m16 = p.d.meta16 != 0;
+    if (p.d.bits == 2) {
+      if (m16) quantize_minmax_kernel<2, true><<<grid, kThreads, 0, s>>>(p);
+      else quantize_minmax_kernel<2, false><<<grid, kThreads, 0, s>>>(p);
+    } else {
+      if (m16) quantize_minmax_kernel<4, true><<<grid, kThreads, 0, s>>>(p);
+      else quantize_minmax_kernel<4, false><<<grid, kThreads, 0, s>>>(p);
+    }
     return cudaGetLastError();
   }
   dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);

@@ -28,16 +28,28 @@ def oracle_layer(runner, layer, k_bits, v_bits):
     w = runner.w
     return oracle.quantize_layer(k_bits, v_bits, w.img_start, w.image, w.base, w.bits,
                                  runner.mask[layer], int(w.keys_only), w.kivi_group_tokens,
-                                 w.kivi_group_channels, w.kivi_residual)
+                                 w.kivi_group_channels, w.kivi_residual,
+                                 meta16=w.meta_bits == 32)
 
 
 def _slice(arena, off, nbytes, dtype):
     return arena[off: off + nbytes].view(dtype)
 
 
+def _meta_words(meta, meta16):
+    """Expected arena words of a metadata array: fp32 pairs as stored, or with
+    32-bit metadata the binary16 bits of each value (scale in the low half)."""
+    if meta16:
+        h = meta.astype(np.float16)  # exact: the oracle's values are binary16 values
+        assert np.array_equal(h.astype(np.float32).view(np.uint32), meta.view(np.uint32))
+        return h.view(np.uint16).view(np.uint32)
+    return meta.view(np.uint32)
+
+
 def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, rows=None):
     """Bit-exact comparison of every region of one layer (or the given heads / rows)."""
     w = runner.w
+    m16 = w.meta_bits == 32
     if arena is None:
         arena = runner.arena.cpu().numpy()
     B, H, T = w.batch, w.kv_heads, w.seq_len
@@ -61,14 +73,16 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
             assert np.array_equal(vb, v_bits[b, h, toks]), (layer, h, b, "vb")
             if cls == hg.HG_HEAD_QUANTIZED and nq:
                 kw = _slice(arena, r.kq + b * r.kq_bstride, nq * W * 4, np.uint32)
-                km = _slice(arena, r.kqm + b * r.kqm_bstride, o["k_meta"][b, h].nbytes, np.uint32)
+                ek = _meta_words(o["k_meta"][b, h], m16)
+                km = _slice(arena, r.kqm + b * r.kqm_bstride, ek.nbytes, np.uint32)
                 assert np.array_equal(kw, o["k_words"][b, h]), (layer, h, b, "kq")
-                assert np.array_equal(km, o["k_meta"][b, h].view(np.uint32)), (layer, h, b, "kqm")
+                assert np.array_equal(km, ek), (layer, h, b, "kqm")
             if cls != hg.HG_HEAD_PROTECTED and nq:
                 vw = _slice(arena, r.vq + b * r.vq_bstride, nq * W * 4, np.uint32)
-                vm = _slice(arena, r.vqm + b * r.vqm_bstride, o["v_meta"][b, h].nbytes, np.uint32)
+                ev = _meta_words(o["v_meta"][b, h], m16)
+                vm = _slice(arena, r.vqm + b * r.vqm_bstride, ev.nbytes, np.uint32)
                 assert np.array_equal(vw, o["v_words"][b, h]), (layer, h, b, "vq")
-                assert np.array_equal(vm, o["v_meta"][b, h].view(np.uint32)), (layer, h, b, "vqm")
+                assert np.array_equal(vm, ev), (layer, h, b, "vqm")
             if cls == hg.HG_HEAD_KEYS_ONLY and nq:
                 ki = _slice(arena, r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)
                 assert np.array_equal(ki, k_bits[b, h, s:s + nq]), (layer, h, b, "kimg")

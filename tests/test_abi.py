@@ -65,6 +65,8 @@ def _status(f, *a):
     ({}, dict(base=1, kivi_group_tokens=16), 3),
     ({}, dict(base=1, kivi_residual=-1), 1),
     ({}, dict(keys_only=2), 1),
+    ({}, dict(meta_bits=16), 1),
+    ({}, dict(meta_bits=48), 1),
 ])
 def test_layout_validation(lib, shape_kw, cfg_kw, status):
     mask = np.zeros((3, max(4, shape_kw.get("num_kv_heads", 4))), np.uint8)
@@ -95,7 +97,11 @@ def test_create_checks_arena(lib):
 
 ODD = {"odd_nq_minmax": wl.custom("odd", 3, 3, 16, 4, 64, 333, 17, wl.BASE_MINMAX, 4, 0),
        "odd_nq_konly": wl.custom("odd2", 2, 5, 8, 8, 7, 77, 3, wl.BASE_AKVQ, 2, 1),
-       "kivi_odd_rows": wl.custom("odd3", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 2, 1)}
+       "kivi_odd_rows": wl.custom("odd3", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 2, 1),
+       "meta16_minmax": wl.custom("m16a", 2, 3, 16, 4, 9, 333, 17, wl.BASE_MINMAX, 2, 0,
+                                  meta_bits=32),
+       "meta16_kivi_konly": wl.custom("m16b", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 4, 1,
+                                      meta_bits=32)}
 
 
 @pytest.mark.parametrize("name", list(wl.WORKLOADS) + list(ODD))
@@ -148,6 +154,39 @@ def test_image_storage_matches_paper_storage_model(lib, oracle):
     cache, _, _ = _fake_cache(w)
     assert hg.hg_cache_image_bits_per_elem(cache) == pytest.approx(2.5)
     assert oracle.image_bits_per_elem(2, 64, 0.0, 0) == pytest.approx(2.5)
+
+
+def test_meta16_storage_model(lib, oracle):
+    # 32-bit metadata (binary16 scale and zero): 2-bit codes cost 2.25 bits per
+    # image element (Sec. 5.4), and protection adds what the model says.
+    w = wl.custom("st16", 1, 1, 8, 8, 0, 64, 0, wl.BASE_MINMAX, 2, 0, protected=[], meta_bits=32)
+    cache, _, _ = _fake_cache(w)
+    assert hg.hg_cache_image_bits_per_elem(cache) == pytest.approx(2.25)
+    for keys_only in (0, 1):
+        w = wl.custom("st16", 2, 1, 8, 8, 0, 64, 0, wl.BASE_MINMAX, 2, keys_only,
+                      protected=[(0, 3), (1, 6)], meta_bits=32)
+        cache, _, _ = _fake_cache(w)
+        want = oracle.image_bits_per_elem(2, 32, 0.125, keys_only)
+        assert hg.hg_cache_image_bits_per_elem(cache) == pytest.approx(want, rel=1e-12)
+
+
+@pytest.mark.parametrize("base", [wl.BASE_MINMAX, wl.BASE_KIVI, wl.BASE_AKVQ])
+def test_meta16_halves_metadata_regions(lib, base):
+    # binary16 pairs: 4 bytes per group instead of 8; row strides stay 16-byte padded
+    kw = dict(protected=[(0, 1)])
+    w64 = wl.custom("m64", 1, 2, 8, 4, 16, 256, 8, base, 2, 0, **kw)
+    w32 = wl.custom("m32", 1, 2, 8, 4, 16, 256, 8, base, 2, 0, meta_bits=32, **kw)
+    c64, n64, _ = _fake_cache(w64)
+    c32, n32, _ = _fake_cache(w32)
+    assert n32 < n64
+    r64 = hg.hg_cache_head_regions(c64, 0, 0)
+    r32 = hg.hg_cache_head_regions(c32, 0, 0)
+    assert r64.nq == r32.nq > 0
+    groups_k = (r64.nq // 32) * 128 if base == wl.BASE_KIVI else r64.nq
+    groups_v = r64.nq * (4 if base == wl.BASE_KIVI else 1)
+    pad = lambda x: (x + 15) // 16 * 16
+    assert (r64.kqm_bstride, r32.kqm_bstride) == (pad(8 * groups_k), pad(4 * groups_k))
+    assert (r64.vqm_bstride, r32.vqm_bstride) == (pad(8 * groups_v), pad(4 * groups_v))
 
 
 def test_calls_validate_before_any_launch(lib):

@@ -1,6 +1,7 @@
 """GPU parity of the CUDA path against the CPU oracle, through the C ABI.
 
-Packed codes, fp32 metadata and BF16 copies must be bit-identical; the fp32
+Packed codes, metadata (fp32 pairs, or binary16 pairs with 32-bit metadata)
+and BF16 copies must be bit-identical; the fp32
 reconstruction (hg_dequantize_kv) must be bit-identical; decode attention
 must match the fp64 oracle within |g - r| <= 2e-3 + 1e-2 |r| element-wise.
 """
@@ -50,10 +51,10 @@ CASES = [
 ]
 
 
-def _workload(case):
+def _workload(case, meta_bits=64):
     (name, L, B, Hq, H, pre, img, suf, base, bits, ko, steps, prot, R) = case
     return wl.custom(name, L, B, Hq, H, pre, img, suf, base, bits, ko, decode_steps=steps,
-                     seed=7, protected=prot, residual=R)
+                     seed=7, protected=prot, residual=R, meta_bits=meta_bits)
 
 
 def _run_and_check(w, layer_batched=True, fused=False):
@@ -149,10 +150,26 @@ def test_decode_step_capacity_and_rollback():
     assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
 
 
+META16 = [CASES[i] for i in (0, 1, 2, 3, 4, 6, 7, 12, 13)]
+
+
+@pytest.mark.parametrize("case", META16, ids=[c[0] for c in META16])
+def test_meta16_quantize_and_decode_parity(case):
+    """32-bit metadata (binary16 scale and zero): codes, metadata bits and
+    attention against the oracle with the same storage model."""
+    _run_and_check(_workload(case, meta_bits=32))
+
+
+@pytest.mark.parametrize("case", [CASES[0], CASES[3], CASES[6]], ids=["minmax", "kivi", "akvq"])
+def test_meta16_fused_decode_step(case):
+    _run_and_check(_workload(case, meta_bits=32), fused=True)
+
+
+@pytest.mark.parametrize("meta_bits", [64, 32])
 @pytest.mark.parametrize("case", [CASES[1], CASES[2], CASES[4], CASES[5], CASES[7]],
                          ids=["minmax4", "minmax2_konly", "kivi4", "kivi2", "akvq2"])
-def test_dequantize_bit_exact(case):
-    w = _workload(case)
+def test_dequantize_bit_exact(case, meta_bits):
+    w = _workload(case, meta_bits)
     runner = CacheRunner(w)
     kept = runner.quantize_all(keep=True)
     # append one step so the appended tail is reconstructed too
@@ -208,14 +225,15 @@ def test_capacity_error_leaves_state():
     assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
 
 
+@pytest.mark.parametrize("meta_bits", [64, 32])
 @pytest.mark.parametrize("bits", [2, 4])
-def test_minmax_quantize_exact_ties(bits):
+def test_minmax_quantize_exact_ties(bits, meta_bits):
     """Vectors built so that (x - min) / scale lands exactly on half-integers:
     every such element must round half to even, as the oracle does (the
     kernel's fast multiply-by-reciprocal path has to hand these to the exact
     division rule)."""
     w = wl.custom("ties%d" % bits, 1, 2, 8, 4, 5, 96, 7, M, bits, 0, decode_steps=1, seed=3,
-                  protected=[(0, 1)], residual=32)
+                  protected=[(0, 1)], residual=32, meta_bits=meta_bits)
     runner = CacheRunner(w)
     B, H, T = w.batch, w.kv_heads, w.seq_len
     gen = torch.Generator().manual_seed(11)
@@ -240,6 +258,43 @@ def test_minmax_quantize_exact_ties(bits):
     kb, vb = bits16(k), bits16(v)
     o = oracle_layer(runner, 0, kb, vb)
     check_arena_layer(runner, 0, kb, vb, o)
+
+
+@pytest.mark.parametrize("base,bits", [(M, 2), (M, 4), (K, 2), (A, 4)],
+                         ids=["minmax2", "minmax4", "kivi2", "akvq4"])
+def test_meta16_extreme_ranges(base, bits):
+    """Binary16 metadata at the edges of its range: magnitudes past 65504
+    (the zero saturates), steps below the smallest subnormal (the stored scale
+    is 0), and subnormal offsets whose rounded zero lies above the group
+    minimum (codes clamp at 0 and at the top level).  Arena bits and the fp32 reconstruction
+    must equal the oracle's."""
+    w = wl.custom("x16", 1, 2, 8, 4, 5, 96, 7, base, bits, 0, decode_steps=1, seed=5,
+                  protected=[(0, 1)], residual=32, meta_bits=32)
+    runner = CacheRunner(w)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    gen = torch.Generator().manual_seed(17)
+    shape = (2, B, H, T, 128)
+    kind = torch.randint(0, 5, (2, B, H, T, 1), generator=gen)
+    z = torch.randn(shape, generator=gen)
+    x = torch.where(kind == 0, z * 3e4 - 6e4, z)                       # past -65504
+    x = torch.where(kind == 1, z * 2e4 + 7e4, x)                       # past +65504
+    x = torch.where(kind == 2, z * 1e-8, x)                            # step below 2^-24
+    # tiny offset: a BF16 minimum below 2^-14 rounds to a binary16 subnormal,
+    # which can lie above it (BF16 values in the normal binary16 range convert exactly)
+    x = torch.where(kind == 3, 1e-6 + torch.rand(shape, generator=gen) * 9e-6, x)
+    xb = x.to(torch.bfloat16)
+    k = xb[0].contiguous().cuda()
+    v = xb[1].contiguous().cuda()
+    hg.hg_quantize_kv(runner.cache, 0, [k], [v])
+    k32 = torch.empty(B, H, T, 128, dtype=torch.float32, device="cuda")
+    v32 = torch.empty_like(k32)
+    hg.hg_dequantize_kv(runner.cache, 0, k32, v32, True)
+    torch.cuda.synchronize()
+    kb, vb = bits16(k), bits16(v)
+    o = oracle_layer(runner, 0, kb, vb)
+    check_arena_layer(runner, 0, kb, vb, o)
+    assert np.array_equal(k32.cpu().numpy().view(np.uint32), o["k_deq"].view(np.uint32))
+    assert np.array_equal(v32.cpu().numpy().view(np.uint32), o["v_deq"].view(np.uint32))
 
 
 def test_bounded_wait_gives_up_and_flags():
