@@ -503,12 +503,15 @@ namespace {
 // instead of whatever the (layer, row, head) enumeration puts together.
 // Returns the number of ordered CTAs (0: natural order).
 int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, int total,
-                uint16_t* order) {
+                uint32_t* order) {
   if (total > kMaxOrderedItems || total < 2) return 0;
   const Dims& d = c->d;
+  if (d.B > kOrderMaxRow || p.max_items > kOrderMaxChunk) return 0;
   const SegBytes sb = seg_bytes(d);
   std::vector<std::pair<double, int>> cost;
+  std::vector<uint32_t> rec;
   cost.reserve(total);
+  rec.reserve(total);
   int item = 0;
   for (int i = 0; i < count; ++i) {
     const DecodeLayer& L = p.layer[i];
@@ -527,6 +530,7 @@ int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, 
           if (r < nb) w = std::min(bc, blen - r * bc) * sb.bf16;
           else w = std::min(qc, d.nq - (r - nb) * qc) * qb;
           cost.emplace_back(w, item++);
+          rec.push_back(order_record(i, b, h, r));
         }
       }
     }
@@ -539,7 +543,7 @@ int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, 
     const int r = j / S, s = j % S;
     const bool full_round = (r + 1) * S <= total;
     const int blk = r * S + ((r & 1) && full_round ? S - 1 - s : s);
-    order[blk] = (uint16_t)cost[j].second;
+    order[blk] = rec[cost[j].second];
   }
   return total;
 }

@@ -829,46 +829,58 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 // or the splits of a head): part s, query j at parts + s * sstride + j * 132
 // (m at +0, l at +1, o at +4).  With M = max_s m_s and f_s = 2^(m_s - M):
 // o = sum_s f_s o_s / L, L = sum_s f_s l_s.  combine_weights leaves f_s in
-// fw[s][j] (s < 16), L in fw[kFwL][j] and M in fw[kFwM][j] (rows of kMaxG).
+// fw[s][j] (s < 16), L in fw[kFwL][j], M in fw[kFwM][j] and 1 / L in
+// fw[kFwR][j] (rows of kMaxG).  Both steps are short dependency chains: eight
+// threads per query reduce the weights with shuffles, and each thread then
+// accumulates one channel of every query at once.
 // ---------------------------------------------------------------------------
-constexpr int kFwL = 16, kFwM = 17;
+constexpr int kFwL = 16, kFwM = 17, kFwR = 18;
+static_assert(kThreads == 8 * kMaxG, "eight combine threads per query");
 
 __device__ __forceinline__ void combine_weights(const float* parts, int n, int sstride, int G, float* fw,
                                                 int tid) {
-  if (tid < G) {
-    const int j = tid;
-    float M = -INFINITY;
-#pragma unroll 1
-    for (int s = 0; s < n; ++s) M = fmaxf(M, parts[s * sstride + j * kPartialStride]);
-    float Ls = 0.f;
-#pragma unroll 1
-    for (int s = 0; s < n; ++s) {
-      const float ms = parts[s * sstride + j * kPartialStride];
-      const float f = (ms == -INFINITY) ? 0.f : fast_exp2(ms - M);
-      fw[s * kMaxG + j] = f;
-      Ls = fmaf(f, parts[s * sstride + j * kPartialStride + 1], Ls);
-    }
+  // thread t: query t / 8, parts t % 8 and t % 8 + 8
+  const int j = tid >> 3, sl = tid & 7;
+  const bool h0 = j < G && sl < n, h1 = j < G && sl + 8 < n;
+  const float* pj = parts + j * kPartialStride;
+  const float m0 = h0 ? pj[sl * sstride] : -INFINITY;
+  const float l0 = h0 ? pj[sl * sstride + 1] : 0.f;
+  const float m1 = h1 ? pj[(sl + 8) * sstride] : -INFINITY;
+  const float l1 = h1 ? pj[(sl + 8) * sstride + 1] : 0.f;
+  float M = fmaxf(m0, m1);
+  M = fmaxf(M, __shfl_xor_sync(kFull, M, 1));
+  M = fmaxf(M, __shfl_xor_sync(kFull, M, 2));
+  M = fmaxf(M, __shfl_xor_sync(kFull, M, 4));
+  const float f0 = (m0 == -INFINITY) ? 0.f : fast_exp2(m0 - M);
+  const float f1 = (m1 == -INFINITY) ? 0.f : fast_exp2(m1 - M);
+  float Ls = fmaf(f0, l0, f1 * l1);
+  Ls += __shfl_xor_sync(kFull, Ls, 1);
+  Ls += __shfl_xor_sync(kFull, Ls, 2);
+  Ls += __shfl_xor_sync(kFull, Ls, 4);
+  if (h0) fw[sl * kMaxG + j] = f0;
+  if (h1) fw[(sl + 8) * kMaxG + j] = f1;
+  if (j < G && sl == 0) {
     fw[kFwL * kMaxG + j] = Ls;
     fw[kFwM * kMaxG + j] = M;
+    fw[kFwR * kMaxG + j] = 1.0f / Ls;
   }
   __syncthreads();
 }
 
-__device__ __forceinline__ float combine_o(const float* parts, int n, int sstride, const float* fw, int j, int c) {
-  // four independent sums, so that the loads of four parts are in flight together
-  const float* pj = parts + j * kPartialStride + 4 + c;
-  float o0 = 0.f, o1 = 0.f, o2 = 0.f, o3 = 0.f;
-  int s = 0;
+// Channel c of queries 0..JM-1 (those below G): acc[j] = sum_s f_s o_s[j][c].
+template <int JM>
+__device__ __forceinline__ void combine_out(const float* parts, int n, int sstride, const float* fw, int G, int c,
+                                            float (&acc)[JM]) {
+#pragma unroll
+  for (int j = 0; j < JM; ++j) acc[j] = 0.f;
 #pragma unroll 1
-  for (; s + 4 <= n; s += 4) {
-    o0 = fmaf(fw[s * kMaxG + j], pj[s * sstride], o0);
-    o1 = fmaf(fw[(s + 1) * kMaxG + j], pj[(s + 1) * sstride], o1);
-    o2 = fmaf(fw[(s + 2) * kMaxG + j], pj[(s + 2) * sstride], o2);
-    o3 = fmaf(fw[(s + 3) * kMaxG + j], pj[(s + 3) * sstride], o3);
+  for (int s = 0; s < n; ++s) {
+    const float* ps = parts + s * sstride + 4 + c;
+    const float* fs = fw + s * kMaxG;
+#pragma unroll
+    for (int j = 0; j < JM; ++j)
+      if (j < G) acc[j] = fmaf(fs[j], ps[j * kPartialStride], acc[j]);
   }
-#pragma unroll 1
-  for (; s < n; ++s) o0 = fmaf(fw[s * kMaxG + j], pj[s * sstride], o0);
-  return (o0 + o1) + (o2 + o3);
 }
 
 // ---------------------------------------------------------------------------
@@ -1055,7 +1067,6 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const Dims& d = p.d;
   if ((int)blockIdx.x >= p.total_items) return;
-  const int item = ((int)blockIdx.x < p.n_order) ? (int)p.order[blockIdx.x] : (int)blockIdx.x;
   if (threadIdx.x == 0) {
     const uint32_t bars = smem_u32(smem + SmemLayout<NT>::bar);
     for (int s = 0; s < kMaxStages; ++s) mbar_init(bars + 8 * s, 1);
@@ -1063,21 +1074,36 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     *reinterpret_cast<volatile int*>(smem + SmemLayout<NT>::bar + 8 * kMaxStages) = 0;  // abort flag
     prefetch_tensormap(&p.arena_map);
   }
-  int li = 0;
-  while (li + 1 < p.n_layers && p.layer[li + 1].item_base <= item) ++li;
+  // (layer, batch row, KV head, chunk) of this CTA's item: a packed record
+  // for host-ordered CTAs, else a search of the layer and head tables
+  int li = 0, b, h, r;
+  if ((int)blockIdx.x < p.n_order) {
+    const uint32_t e = p.order[blockIdx.x];
+    li = (int)(e & 63u);
+    h = (int)((e >> 6) & 63u);
+    r = (int)((e >> 12) & 31u);
+    b = (int)(e >> 17);
+  } else {
+    const int item = (int)blockIdx.x;
+    while (li + 1 < p.n_layers && p.layer[li + 1].item_base <= item) ++li;
+    const DecodeLayer& L0 = p.layer[li];
+    const int in_layer = item - L0.item_base;
+    b = in_layer / L0.items_per_row;
+    r = in_layer - b * L0.items_per_row;
+    const ChunkCounts c0 = {L0.nbU, L0.nqU, L0.nqK, L0.nbP};
+    for (h = 0; h < d.H; ++h) {
+      int nb0;
+      const int n0 = head_chunks(head_class(d, p.lt.mask[li], h), c0, &nb0);
+      if (r < n0) break;
+      r -= n0;
+    }
+  }
   const DecodeLayer& L = p.layer[li];
-  const int in_layer = item - L.item_base;
-  const int b = in_layer / L.items_per_row;
-  int r = in_layer - b * L.items_per_row;
   const uint64_t mask = p.lt.mask[li];
   const ChunkCounts cc = {L.nbU, L.nqU, L.nqK, L.nbP};
-  int h = 0, nb = 0, ni = 0, cls = kQuantized;
-  for (; h < d.H; ++h) {
-    cls = head_class(d, mask, h);
-    ni = head_chunks(cls, cc, &nb);
-    if (r < ni) break;
-    r -= ni;
-  }
+  const int cls = head_class(d, mask, h);
+  int nb;
+  const int ni = head_chunks(cls, cc, &nb);
   const LayerGeom lg = layer_geom(d, mask);
   const HeadGeom hd = head_geom(d, lg, h);
   const char* Lb = p.arena + p.lt.base[li];
@@ -1153,69 +1179,73 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   __syncthreads();
 
   // ---- combine the warps, then write the output (a head in one chunk) or this
-  // split's partial ----
+  // split's partial; the last split of a head to finish then runs the same
+  // combine over all splits' partials (a second pass through this code, whose
+  // instructions are cached by then: the merge runs once per head, and cold
+  // code would cost microseconds) ----
   float* fw = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);  // weights; queries no longer needed
-  combine_weights(parts, kWarps, kMaxG * kPartialStride, G, fw, tid);
   const int c = tid;
   const size_t out_row = ((size_t)li * d.B + b) * d.Hq + (size_t)h * G;
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
   float* part = p.partials + (head_lin * p.max_items) * (size_t)G * kPartialStride;
   float* mine = part + (size_t)r * G * kPartialStride;
+  __shared__ int s_last;
+  const float* src = parts;
+  int n = kWarps, sstride = kMaxG * kPartialStride;
+  bool final = ni == 1;
 #pragma unroll 1
-  for (int j = 0; j < G; ++j) {
-    const float O = combine_o(parts, kWarps, kMaxG * kPartialStride, fw, j, c);
-    if (ni == 1) {
-      p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / fw[kFwL * kMaxG + j]);
-    } else {
-      mine[j * kPartialStride + 4 + c] = O;
-      if (c == 0) {
-        mine[j * kPartialStride + 0] = fw[kFwM * kMaxG + j];
-        mine[j * kPartialStride + 1] = fw[kFwL * kMaxG + j];
+  for (;;) {
+    combine_weights(src, n, sstride, G, fw, tid);
+    float acc[NT * 8];
+    combine_out<NT * 8>(src, n, sstride, fw, G, c, acc);
+#pragma unroll
+    for (int j = 0; j < NT * 8; ++j) {
+      if (j >= G) break;
+      if (final) {
+        p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(acc[j] * fw[kFwR * kMaxG + j]);
+      } else {
+        mine[j * kPartialStride + 4 + c] = acc[j];
+        if (c == 0) {
+          mine[j * kPartialStride + 0] = fw[kFwM * kMaxG + j];
+          mine[j * kPartialStride + 1] = fw[kFwL * kMaxG + j];
+        }
       }
     }
-  }
-  if (ni == 1) return;
+    if (final) break;
 
-  // Publish the partial and take a ticket with one acquire-release atomic: the
-  // CTA barrier orders every thread's stores before thread 0's release
-  // (release is cumulative); for the last CTA, the acquire side orders the
-  // other CTAs' partials before its reads (extended to its threads by the
-  // second barrier).  No full device fence is needed.
-  __syncthreads();
-  __shared__ int s_last;
-  if (tid == 0) {
-    unsigned prev;
-    asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;\n"
-                 : "=r"(prev)
-                 : "l"(p.counters + head_lin)
-                 : "memory");
-    s_last = (prev == (unsigned)(ni - 1));
-  }
-  __syncthreads();
-  if (!s_last) return;
+    // Publish the partial and take a ticket with one acquire-release atomic:
+    // the CTA barrier orders every thread's stores before thread 0's release
+    // (release is cumulative); for the last CTA, the acquire side orders the
+    // other CTAs' partials before its reads (extended to its threads by the
+    // second barrier).  No full device fence is needed.
+    __syncthreads();
+    if (tid == 0) {
+      unsigned prev;
+      asm volatile("atom.acq_rel.gpu.global.add.u32 %0, [%1], 1;\n"
+                   : "=r"(prev)
+                   : "l"(p.counters + head_lin)
+                   : "memory");
+      s_last = (prev == (unsigned)(ni - 1));
+    }
+    __syncthreads();
+    if (!s_last) return;
 
-  // Last CTA of the head: all ni partials in one asynchronous sweep into the
-  // stage buffer (the plan keeps them within it), then the same combine as
-  // the warps' -- code this CTA has just run, so its instructions are cached
-  // (the merge runs once per head: cold code would cost microseconds).
-  {
+    // Last CTA of the head: all ni partials in one asynchronous sweep into the
+    // stage buffer (the plan keeps them within it).
     const int bytes = ni * G * kPartialStride * 4;
     const uint32_t buf_u32 = smem_u32(smem + kStageOff);
-    const char* src = reinterpret_cast<const char*>(part);
+    const char* psrc = reinterpret_cast<const char*>(part);
 #pragma unroll 1
-    for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, src + off, 16);
+    for (int off = tid * 16; off < bytes; off += kThreads * 16) cp_async16(buf_u32 + off, psrc + off, 16);
     cp_async_commit();
     cp_async_wait<0>();
+    __syncthreads();
+    src = reinterpret_cast<const float*>(smem + kStageOff);  // [ni][G][132]
+    n = ni;
+    sstride = G * kPartialStride;
+    final = true;
   }
-  __syncthreads();
-  const float* all = reinterpret_cast<const float*>(smem + kStageOff);  // [ni][G][132]
-  combine_weights(all, ni, G * kPartialStride, G, fw, tid);
-#pragma unroll 1
-  for (int j = 0; j < G; ++j) {
-    const float O = combine_o(all, ni, G * kPartialStride, fw, j, c);
-    p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(O / fw[kFwL * kMaxG + j]);
-  }
-  if (tid == 0) atomicExch(p.counters + head_lin, 0u);
+  if (ni > 1 && tid == 0) atomicExch(p.counters + head_lin, 0u);
 }
 
 template <int BITS, int NT, int BASE, int MB>

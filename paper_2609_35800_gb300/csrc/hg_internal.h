@@ -68,6 +68,12 @@ struct DecodeLayer {
 
 // Largest launch whose CTAs get a host-chosen item order.
 constexpr int kMaxOrderedItems = 1024;
+// Packed work item: layer in the launch (6 bits), KV head (6), chunk of the
+// head (5), batch row (15).
+HG_HD uint32_t order_record(int li, int b, int h, int r) {
+  return (uint32_t)li | ((uint32_t)h << 6) | ((uint32_t)r << 12) | ((uint32_t)b << 17);
+}
+constexpr int kOrderMaxRow = 1 << 15, kOrderMaxChunk = 1 << 5;
 
 struct DecodeParams {
   // The arena as a two-dimensional BF16 tensor [arena_bytes / 256][128]: every
@@ -93,9 +99,11 @@ struct DecodeParams {
   float* partials;     // [n_layers][B][H][max_items][G][132]
   LayerTable lt;
   DecodeLayer layer[kMaxLayersPerLaunch];
-  // Work item of each CTA (blockIdx.x < n_order; item = blockIdx.x beyond).
+  // Work item of each CTA below n_order, as a packed record (order_record):
+  // the kernel reads its item's coordinates instead of searching the layer
+  // and head tables.  CTAs from n_order on take item blockIdx.x.
   int n_order;
-  uint16_t order[kMaxOrderedItems];
+  uint32_t order[kMaxOrderedItems];
 };
 
 // BF16 rows per TMA box of the arena tensor map.
