@@ -152,6 +152,9 @@ __device__ __forceinline__ uint32_t pair2_scaled_h(uint32_t w, uint32_t w6, uint
   return (src & (0x00030003u << pos3(j))) | 0x64006400u;
 }
 
+// 1 / x for a power of two x in [2^-126, 2^126], exactly (exponent arithmetic).
+__device__ __forceinline__ float pow2_inv(float x) { return __uint_as_float(0x7F000000u - __float_as_uint(x)); }
+
 // Smallest power of two >= m (m > 0, finite).
 __device__ __forceinline__ float pow2_ceil(float m) {
   return __uint_as_float((__float_as_uint(m) + 0x007FFFFFu) & 0xFF800000u);
@@ -431,7 +434,7 @@ template <int NT, int NZ>
 __device__ __forceinline__ void vscale_update(WarpState<NT, NZ>& ws, float smax) {
   if (__any_sync(kFull, smax > ws.vb)) {
     const float nb = pow2_ceil(warp_max(smax));
-    const float a = ws.vb / nb;  // a power of two: exact
+    const float a = ws.vb * pow2_inv(nb);  // a power of two: exact
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) {
 #pragma unroll
@@ -704,7 +707,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         const float2 vg = ok0 ? meta_pair<MB>(vmp, tok0 + g) : make_float2(0.f, 0.f);
         const float2 vg8 = ok8 ? meta_pair<MB>(vmp, tok0 + g + 8) : make_float2(0.f, 0.f);
         vscale_update(ws, fmaxf(vg.x, vg8.x));
-        const float inv = 1.0f / ws.vb;  // exact: vb is a power of two
+        const float inv = pow2_inv(ws.vb);
         uint32_t b[NT][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -780,7 +783,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         }
         vscale_update(ws, fmaxf(fmaxf(fmaxf(sv_g[0], sv_g[1]), fmaxf(sv_g[2], sv_g[3])),
                                 fmaxf(fmaxf(sv_g8[0], sv_g8[1]), fmaxf(sv_g8[2], sv_g8[3]))));
-        const float inv = 1.0f / ws.vb;  // exact: vb is a power of two
+        const float inv = pow2_inv(ws.vb);
         uint32_t b[NT][4][2];
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt) {
@@ -991,13 +994,13 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
       if (it > 0 && issued < upto) fence_proxy_async_shared();
       for (; issued < upto; ++issued)
         issue_tile<BITS, KM, VM, MB>(st0 + (issued % STAGES) * TL::stage_bytes, bars + 8 * (issued % STAGES), sg,
-                                 tb + issued * TL::tokens, min(TL::tokens, te - tb - issued * TL::tokens),
-                                 &p.arena_map);
+                                     tb + issued * TL::tokens, min(TL::tokens, te - tb - issued * TL::tokens),
+                                     &p.arena_map);
     }
     if (ok)
       compute_tile<BITS, NT, KM, VM, ROT, MB>(ws, stages + st * TL::stage_bytes,
-                                          min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s,
-                                          s1, s0, scale_log2, warp, lane);
+                                              min(TL::tokens, te - tb - it * TL::tokens), qb, ql, q_s, s1, s0,
+                                              scale_log2, warp, lane);
   }
   if (tid == 0 && *abort) {
     // A stage is refilled only after its previous tile landed, so only the
