@@ -61,6 +61,14 @@ def lib():
         L.hgo_quantize_layer.restype = i
         L.hgo_quantize_layer_m.argtypes = [P, P, i, i, i, i, i, i, i, i, P, i, i, i, i] + [P] * 9
         L.hgo_quantize_layer_m.restype = i
+        L.hgo_quantize_layer_s.argtypes = [P, P, i, i, i, i, i, i, i, i, P, i, i, i, i, i] + [P] * 10
+        L.hgo_quantize_layer_s.restype = i
+        L.hgo_key_norm2.argtypes = [P]
+        L.hgo_key_norm2.restype = ctypes.c_float
+        L.hgo_salient_count.argtypes = [i, i]
+        L.hgo_salient_count.restype = i
+        L.hgo_select_salient.argtypes = [P, i, i, P]
+        L.hgo_select_salient.restype = None
         L.hgo_attention_layer.argtypes = [P, P, P, i, i, i, i, ctypes.c_double, P]
         L.hgo_attention_layer.restype = i
         L.hgo_image_bits_per_elem.argtypes = [i, i, i, ctypes.c_double, i]
@@ -159,8 +167,27 @@ def image_bits_per_elem(bits, meta_bits, frac_protected, keys_only, head_dim=D):
 # Layer-level quantization (Sec. 3 protection over a Sec. 4 base)
 # --------------------------------------------------------------------------
 
+def key_norm2(k_row_bits):
+    """R15: squared norm of one BF16 key row, binary32 in the fixed order."""
+    return np.float32(lib().hgo_key_norm2(_ptr(_c(k_row_bits, np.uint16))))
+
+
+def salient_count(n, permille):
+    """R15: salient tokens per head, ceil(n * permille / 1000)."""
+    return lib().hgo_salient_count(int(n), int(permille))
+
+
+def select_salient(score, ns):
+    """R15: indices of the ns largest scores (ties to the lower index), ascending."""
+    score = _c(score, np.float32)
+    idx = np.zeros(max(ns, 1), np.int32)
+    lib().hgo_select_salient(_ptr(score), score.size, int(ns), _ptr(idx))
+    return idx[:ns]
+
+
 def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
-                   group_tokens=32, group_channels=32, residual=32, want_att=True, meta16=False):
+                   group_tokens=32, group_channels=32, residual=32, want_att=True, meta16=False,
+                   n_salient=0):
     """Quantize one layer.
 
     k_bits, v_bits: uint16 [B][H][T][128] BF16 bit patterns.
@@ -168,6 +195,9 @@ def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
     Returns a dict with per-(b,h) arrays:
       nq, kq, vq [B,H,T], k_words [B,H,...], k_meta, v_words, v_meta (shapes as
       documented in hg_oracle.c), k_deq, v_deq [B,H,T,128] fp32, k_att fp64.
+    n_salient > 0 (R15): heads with quantized keys keep that many image tokens
+    BF16 (indices in salient [B,H,n_salient]); their codes and metadata fill
+    the first nq - n_salient token slots.
     """
     k_bits = _c(k_bits, np.uint16)
     v_bits = _c(v_bits, np.uint16)
@@ -190,12 +220,17 @@ def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
         v_words=np.zeros((B, H, kw), np.uint32), v_meta=np.zeros((B, H, vm), np.float32),
         k_deq=np.zeros((B, H, T, D), np.float32), v_deq=np.zeros((B, H, T, D), np.float32),
         k_att=np.zeros((B, H, T, D), np.float64) if want_att else None,
+        salient=np.zeros((B, H, max(n_salient, 0)), np.int32), n_salient=n_salient,
     )
-    lib().hgo_quantize_layer_m(_ptr(k_bits), _ptr(v_bits), B, H, T, s, n, base, bits, int(meta16),
-                             _ptr(head_mask), int(keys_only), group_tokens, group_channels,
-                             residual, _ptr(out["kq"]), _ptr(out["vq"]), _ptr(out["k_words"]),
-                             _ptr(out["k_meta"]), _ptr(out["v_words"]), _ptr(out["v_meta"]),
-                             _ptr(out["k_deq"]), _ptr(out["v_deq"]), _ptr(out["k_att"]))
+    rc = lib().hgo_quantize_layer_s(_ptr(k_bits), _ptr(v_bits), B, H, T, s, n, base, bits,
+                                    int(meta16), _ptr(head_mask), int(keys_only), group_tokens,
+                                    group_channels, residual, int(n_salient), _ptr(out["kq"]),
+                                    _ptr(out["vq"]), _ptr(out["k_words"]), _ptr(out["k_meta"]),
+                                    _ptr(out["v_words"]), _ptr(out["v_meta"]), _ptr(out["k_deq"]),
+                                    _ptr(out["v_deq"]), _ptr(out["k_att"]),
+                                    _ptr(out["salient"]) if n_salient > 0 else None)
+    if rc < 0:
+        raise ValueError("hgo_quantize_layer_s: unsupported salient configuration")
     return out
 
 

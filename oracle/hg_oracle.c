@@ -41,6 +41,15 @@
  *      zero are stored as binary16 (round to nearest even, magnitudes above
  *      65504 saturate to 65504), and the codes are computed against the
  *      stored values, so reconstruction uses exactly what is stored.
+ *   R15 AKVQ-style salient tokens (Sec. 4, optional): in each (batch row, KV
+ *      head) whose image keys are quantized, the keys and values of the ns
+ *      image tokens with the largest squared key norm stay BF16, ties to the
+ *      lower token index; ns = ceil(n * permille / 1000) ("a nominal 2%" is
+ *      permille 20).  The norm is taken on the unrotated BF16 key in binary32
+ *      in the fixed order of hgo_key_norm2, so that both implementations rank
+ *      the same values.  The remaining image tokens are quantized in order and
+ *      stored compacted.  Built for the AKVQ-style base without K-only
+ *      protection.
  */
 #include <math.h>
 #include <stdint.h>
@@ -276,13 +285,23 @@ int hgo_quantized_count(int T, int s, int n, int base, int group_tokens, int res
  *                                  be NULL
  *   Returns nq.  Metadata pairs are (scale, zero).
  */
-int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int n,
-                      int base, int bits, int meta16, int protect, int keys_only,
-                      int group_tokens, int group_channels, int residual,
-                      uint8_t *kq, uint8_t *vq,
-                      uint32_t *k_words, float *k_meta,
-                      uint32_t *v_words, float *v_meta,
-                      float *k_deq, float *v_deq, double *k_att)
+float hgo_key_norm2(const uint16_t *krow);
+void hgo_select_salient(const float *score, int n, int ns, int32_t *idx);
+
+/*
+ * n_salient > 0 (R15; per-token bases without K-only protection): for a head
+ * whose image keys are quantized, the n_salient image tokens of largest key
+ * norm keep BF16 keys and values, their image-relative indices go to
+ * `salient` (ascending), and the other image tokens are quantized in order
+ * into the first nq - n_salient slots of the code and metadata arrays.
+ */
+int hgo_quantize_head_s(const uint16_t *k, const uint16_t *v, int T, int s, int n,
+                        int base, int bits, int meta16, int protect, int keys_only,
+                        int group_tokens, int group_channels, int residual, int n_salient,
+                        uint8_t *kq, uint8_t *vq,
+                        uint32_t *k_words, float *k_meta,
+                        uint32_t *v_words, float *v_meta,
+                        float *k_deq, float *v_deq, double *k_att, int32_t *salient)
 {
     const int D = HGO_D;
     const int nq = hgo_quantized_count(T, s, n, base, group_tokens, residual);
@@ -292,6 +311,16 @@ int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int 
 
     float xk[HGO_D], xv[HGO_D];
     uint8_t codes[HGO_D];
+
+    /* R15: which image tokens stay BF16 (sal[i] for image token s + i) */
+    uint8_t *sal = (uint8_t *)calloc((size_t)(nq > 0 ? nq : 1), 1);
+    if (n_salient > 0 && quant_k && !keys_only && base != HGO_BASE_KIVI && nq > 0) {
+        float *score = (float *)malloc(sizeof(float) * (size_t)nq);
+        for (int i = 0; i < nq; ++i) score[i] = hgo_key_norm2(k + (long)(s + i) * D);
+        hgo_select_salient(score, nq, n_salient, salient);
+        for (int j = 0; j < n_salient; ++j) sal[salient[j]] = 1;
+        free(score);
+    }
 
     /* Start from the BF16 values everywhere; quantized entries are overwritten. */
     for (int t = 0; t < T; ++t) {
@@ -329,15 +358,17 @@ int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int 
                 }
             }
         } else {
-            for (int i = 0; i < nq; ++i) {
+            for (int i = 0, ci = -1; i < nq; ++i) {
                 const int t = s + i;
+                if (sal[i]) continue; /* R15: stays BF16 */
+                ++ci;
                 float scale, zero;
                 for (int c = 0; c < D; ++c) xk[c] = hgo_bf16_to_f32(k[(long)t * D + c]);
                 if (base == HGO_BASE_AKVQ) hgo_fwht128(xk); /* rotate, then per-token RTN */
                 hgo_quantize_group_m(xk, D, 1, bits, meta16, codes, &scale, &zero);
-                hgo_pack(codes, D, bits, k_words + (long)i * wpt);
-                k_meta[(long)i * 2 + 0] = scale;
-                k_meta[(long)i * 2 + 1] = zero;
+                hgo_pack(codes, D, bits, k_words + (long)ci * wpt);
+                k_meta[(long)ci * 2 + 0] = scale;
+                k_meta[(long)ci * 2 + 1] = zero;
                 float r[HGO_D];
                 for (int c = 0; c < D; ++c) r[c] = hgo_dequant(codes[c], scale, zero);
                 if (base == HGO_BASE_AKVQ) {
@@ -354,30 +385,101 @@ int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int 
                 for (int c = 0; c < D; ++c) k_deq[(long)t * D + c] = r[c];
             }
         }
-        for (int i = 0; i < nq; ++i) kq[s + i] = 1;
+        for (int i = 0; i < nq; ++i) kq[s + i] = sal[i] ? 0 : 1;
     }
 
     /* ---- values (never rotated, R9) ---- */
     if (quant_v && nq > 0) {
         const int gsize = (base == HGO_BASE_KIVI) ? group_channels : D;
         const int ngr = D / gsize;
-        for (int i = 0; i < nq; ++i) {
+        for (int i = 0, ci = -1; i < nq; ++i) {
             const int t = s + i;
+            if (sal[i]) continue; /* R15: stays BF16 */
+            ++ci;
             for (int c = 0; c < D; ++c) xv[c] = hgo_bf16_to_f32(v[(long)t * D + c]);
             for (int j = 0; j < ngr; ++j) {
                 float scale, zero;
                 hgo_quantize_group_m(xv + j * gsize, gsize, 1, bits, meta16, codes + j * gsize, &scale, &zero);
-                v_meta[((long)i * ngr + j) * 2 + 0] = scale;
-                v_meta[((long)i * ngr + j) * 2 + 1] = zero;
+                v_meta[((long)ci * ngr + j) * 2 + 0] = scale;
+                v_meta[((long)ci * ngr + j) * 2 + 1] = zero;
                 for (int e = 0; e < gsize; ++e)
                     v_deq[(long)t * D + j * gsize + e] = hgo_dequant(codes[j * gsize + e], scale, zero);
             }
             /* group j's element e is channel j*gsize + e: the channel-order packing */
-            hgo_pack(codes, D, bits, v_words + (long)i * wpt);
+            hgo_pack(codes, D, bits, v_words + (long)ci * wpt);
             vq[t] = 1;
         }
     }
+    free(sal);
     return nq;
+}
+
+int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int n,
+                        int base, int bits, int meta16, int protect, int keys_only,
+                        int group_tokens, int group_channels, int residual,
+                        uint8_t *kq, uint8_t *vq,
+                        uint32_t *k_words, float *k_meta,
+                        uint32_t *v_words, float *v_meta,
+                        float *k_deq, float *v_deq, double *k_att)
+{
+    return hgo_quantize_head_s(k, v, T, s, n, base, bits, meta16, protect, keys_only, group_tokens,
+                               group_channels, residual, 0, kq, vq, k_words, k_meta, v_words, v_meta,
+                               k_deq, v_deq, k_att, NULL);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Sec. 4 AKVQ-style salient tokens (R15).                                    */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * Squared norm of one BF16 key row in binary32, in a fixed order: 32 partial
+ * sums of four consecutive channels each, ((x0^2 + x1^2) + x2^2) + x3^2, then
+ * five pairwise rounds in which partial l becomes partial l + partial (l xor m)
+ * for m = 16, 8, 4, 2, 1; the result is partial 0.
+ */
+float hgo_key_norm2(const uint16_t *krow)
+{
+    float part[32], next[32];
+    for (int l = 0; l < 32; ++l) {
+        float a = 0.0f;
+        for (int j = 0; j < 4; ++j) {
+            const float x = hgo_bf16_to_f32(krow[4 * l + j]);
+            const float sq = x * x;
+            a = (j == 0) ? sq : a + sq;
+        }
+        part[l] = a;
+    }
+    for (int m = 16; m >= 1; m >>= 1) {
+        for (int l = 0; l < 32; ++l) next[l] = part[l] + part[l ^ m];
+        memcpy(part, next, sizeof part);
+    }
+    return part[0];
+}
+
+/* Salient tokens per head for n image tokens at a per-mille rate, rounded up. */
+int hgo_salient_count(int n, int permille)
+{
+    if (permille <= 0 || n <= 0) return 0;
+    return (int)(((long)n * permille + 999) / 1000);
+}
+
+/*
+ * The ns indices in [0, n) with the largest scores (ties: the lower index
+ * first), written in ascending order.
+ */
+void hgo_select_salient(const float *score, int n, int ns, int32_t *idx)
+{
+    uint8_t *taken = (uint8_t *)calloc((size_t)(n > 0 ? n : 1), 1);
+    for (int j = 0; j < ns; ++j) {
+        int best = -1;
+        for (int i = 0; i < n; ++i)
+            if (!taken[i] && (best < 0 || score[i] > score[best])) best = i;
+        if (best >= 0) taken[best] = 1;
+    }
+    int c = 0;
+    for (int i = 0; i < n; ++i)
+        if (taken[i]) idx[c++] = i;
+    free(taken);
 }
 
 /*
@@ -389,15 +491,18 @@ int hgo_quantize_head_m(const uint16_t *k, const uint16_t *v, int T, int s, int 
  * head_mask[h] is the layer's protection mask.  Parallel over (b, h) when
  * built with OpenMP; every head is computed independently.
  */
-int hgo_quantize_layer_m(const uint16_t *k, const uint16_t *v, int B, int H, int T,
-                       int s, int n, int base, int bits, int meta16, const uint8_t *head_mask,
-                       int keys_only, int group_tokens, int group_channels, int residual,
-                       uint8_t *kq, uint8_t *vq,
-                       uint32_t *k_words, float *k_meta, uint32_t *v_words, float *v_meta,
-                       float *k_deq, float *v_deq, double *k_att)
+int hgo_quantize_layer_s(const uint16_t *k, const uint16_t *v, int B, int H, int T,
+                         int s, int n, int base, int bits, int meta16, const uint8_t *head_mask,
+                         int keys_only, int group_tokens, int group_channels, int residual,
+                         int n_salient,
+                         uint8_t *kq, uint8_t *vq,
+                         uint32_t *k_words, float *k_meta, uint32_t *v_words, float *v_meta,
+                         float *k_deq, float *v_deq, double *k_att, int32_t *salient)
 {
     const int D = HGO_D;
     const int nq = hgo_quantized_count(T, s, n, base, group_tokens, residual);
+    if (n_salient < 0 || n_salient > nq) return -1;
+    if (n_salient > 0 && (keys_only || base == HGO_BASE_KIVI)) return -1; /* R15 */
     const long kw = (long)nq * D * bits / 32;
     const long km = (base == HGO_BASE_KIVI) ? (long)(nq / group_tokens) * D * 2 : (long)nq * 2;
     const long vm = (base == HGO_BASE_KIVI) ? (long)nq * (D / group_channels) * 2 : (long)nq * 2;
@@ -405,12 +510,25 @@ int hgo_quantize_layer_m(const uint16_t *k, const uint16_t *v, int B, int H, int
     for (int bh = 0; bh < B * H; ++bh) {
         const int h = bh % H;
         const long tok = (long)bh * T;
-        hgo_quantize_head_m(k + tok * D, v + tok * D, T, s, n, base, bits, meta16, head_mask[h], keys_only,
-                          group_tokens, group_channels, residual, kq + tok, vq + tok,
-                          k_words + bh * kw, k_meta + bh * km, v_words + bh * kw, v_meta + bh * vm,
-                          k_deq + tok * D, v_deq + tok * D, k_att ? k_att + tok * D : NULL);
+        hgo_quantize_head_s(k + tok * D, v + tok * D, T, s, n, base, bits, meta16, head_mask[h], keys_only,
+                            group_tokens, group_channels, residual, n_salient, kq + tok, vq + tok,
+                            k_words + bh * kw, k_meta + bh * km, v_words + bh * kw, v_meta + bh * vm,
+                            k_deq + tok * D, v_deq + tok * D, k_att ? k_att + tok * D : NULL,
+                            salient ? salient + (long)bh * n_salient : NULL);
     }
     return nq;
+}
+
+int hgo_quantize_layer_m(const uint16_t *k, const uint16_t *v, int B, int H, int T,
+                         int s, int n, int base, int bits, int meta16, const uint8_t *head_mask,
+                         int keys_only, int group_tokens, int group_channels, int residual,
+                         uint8_t *kq, uint8_t *vq,
+                         uint32_t *k_words, float *k_meta, uint32_t *v_words, float *v_meta,
+                         float *k_deq, float *v_deq, double *k_att)
+{
+    return hgo_quantize_layer_s(k, v, B, H, T, s, n, base, bits, meta16, head_mask, keys_only,
+                                group_tokens, group_channels, residual, 0, kq, vq, k_words, k_meta,
+                                v_words, v_meta, k_deq, v_deq, k_att, NULL);
 }
 
 /* The 64-bit-metadata forms (R5). */
