@@ -91,7 +91,16 @@ typedef struct hg_shape {
  * meta_bits: metadata per group, 64 (or 0: the default) = an fp32 {scale, zero}
  * pair; 32 = a binary16 pair, the Sec. 5.4 storage model (2.25 bits per element
  * at 2 bits): scale and zero are rounded to nearest-even binary16 (magnitudes
- * >= 65504 saturate) and the codes are computed against the stored values. */
+ * >= 65504 saturate) and the codes are computed against the stored values.
+ * salient_permille (0 = off; AKVQ-style base without keys_only, else
+ * HG_ERR_UNSUPPORTED): Sec. 4's salient tokens.  In every (batch row, KV head)
+ * whose image keys are quantized, ceil(nq * salient_permille / 1000) image
+ * tokens (20: the paper's nominal 2%) with the largest squared norm of the
+ * unrotated BF16 key keep BF16 keys and values; ties go to the lower token
+ * index.  The squared norm is summed in binary32 in a fixed order: 32 partial
+ * sums of channels 4l..4l+3, ((x0^2 + x1^2) + x2^2) + x3^2, then five rounds
+ * in which partial l adds partial (l xor m), m = 16, 8, 4, 2, 1.  The other
+ * image tokens are coded in order, compacted. */
 typedef struct hg_quant_config {
     int32_t base;
     int32_t bits;
@@ -100,6 +109,7 @@ typedef struct hg_quant_config {
     int32_t kivi_group_channels;
     int32_t kivi_residual;
     int32_t meta_bits;
+    int32_t salient_permille;
 } hg_quant_config;
 
 /* Opaque host-side descriptor of a cache arena (offsets, mask, appended counts). */
@@ -117,7 +127,9 @@ typedef enum hg_head_class {
  * between batch rows; an absent region has offset UINT64_MAX.
  *   kb / vb   BF16 [batch][bf16_capacity][128]: the head's BF16 tokens in
  *             prefill order (text, image tokens not quantized), then appended
- *             tokens.  bf16_prefill of them come from the prefill.
+ *             tokens.  bf16_prefill of them come from the prefill.  With
+ *             salient tokens: leading text, the salient image tokens in token
+ *             order, trailing text, appended tokens.
  *   kq / kqm  key codes / metadata (quantized class only).  Per-token bases:
  *             codes uint32 [batch][nq][4*bits] (128 codes, channel order, packed
  *             LSB-first, 32/bits per word), metadata float2 {scale, zero}
@@ -128,9 +140,15 @@ typedef enum hg_head_class {
  *             [batch][nq][groups], groups = 1 (per token) or 4 (KIVI-style,
  *             channels 32j..32j+31).
  *   kimg      BF16 [batch][nq][128] image keys of a keys-only protected head.
+ *   sal       salient-token map of a quantized head (salient tokens only):
+ *             per batch row uint32 [ceil(nq/32)] (bit j of word w: image
+ *             token 32w + j is salient), then int32 [ceil(nq/32)] (salient
+ *             tokens before block w), row stride sal_bstride.
  * Quantized image tokens are [img_start, img_start + nq); nq equals img_len
  * except for KIVI-style, where only whole 32-token groups inside
- * [img_start, min(img_start + img_len, seq_len - kivi_residual)) are coded. */
+ * [img_start, min(img_start + img_len, seq_len - kivi_residual)) are coded.
+ * The code and metadata arrays hold n_coded tokens (nq less the n_salient
+ * salient tokens of a quantized head), in token order. */
 typedef struct hg_head_regions {
     int32_t head_class;
     int32_t nq;
@@ -138,6 +156,8 @@ typedef struct hg_head_regions {
     int32_t bf16_capacity;
     uint64_t kb, vb, kq, kqm, vq, vqm, kimg;
     uint64_t kb_bstride, kq_bstride, kqm_bstride, vq_bstride, vqm_bstride, kimg_bstride;
+    uint64_t sal, sal_bstride;
+    int32_t n_coded, n_salient;
 } hg_head_regions;
 
 /* Bytes of device arena a cache of this shape / config / mask needs.

@@ -57,7 +57,7 @@ class Shape(ctypes.Structure):
 class QuantConfig(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "base", "bits", "keys_only", "kivi_group_tokens", "kivi_group_channels",
-        "kivi_residual", "meta_bits")]
+        "kivi_residual", "meta_bits", "salient_permille")]
 
 
 class HeadRegions(ctypes.Structure):
@@ -65,7 +65,9 @@ class HeadRegions(ctypes.Structure):
                                                 "bf16_capacity")] +
                 [(n, ctypes.c_uint64) for n in ("kb", "vb", "kq", "kqm", "vq", "vqm", "kimg",
                                                  "kb_bstride", "kq_bstride", "kqm_bstride",
-                                                 "vq_bstride", "vqm_bstride", "kimg_bstride")])
+                                                 "vq_bstride", "vqm_bstride", "kimg_bstride",
+                                                 "sal", "sal_bstride")] +
+                [(n, ctypes.c_int32) for n in ("n_coded", "n_salient")])
 
 
 _lib = None

@@ -55,6 +55,11 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   if (c->bits != 2 && c->bits != 4) return HG_ERR_UNSUPPORTED;
   if (c->keys_only != 0 && c->keys_only != 1) return HG_ERR_INVALID_ARG;
   if (c->meta_bits != 0 && c->meta_bits != 32 && c->meta_bits != 64) return HG_ERR_INVALID_ARG;
+  if (c->salient_permille < 0 || c->salient_permille > 1000) return HG_ERR_INVALID_ARG;
+  // salient tokens (Sec. 4) belong to the AKVQ-style base; K-only protection
+  // would keep salient values of protected heads BF16 too, which is not built
+  if (c->salient_permille > 0 && (c->base != HG_BASE_AKVQ_HADAMARD || c->keys_only))
+    return HG_ERR_UNSUPPORTED;
   if (c->base == HG_BASE_KIVI) {
     if (c->kivi_group_tokens != kKiviGroup || c->kivi_group_channels != kKiviGroup)
       return HG_ERR_UNSUPPORTED;
@@ -80,6 +85,9 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   d->residual = c->base == HG_BASE_KIVI ? c->kivi_residual : 0;
   d->meta16 = c->meta_bits == 32 ? 1 : 0;
   d->nq = quantized_count(d->T, d->s, d->n, d->base, d->residual);
+  d->ns = c->salient_permille > 0 ? (int)(((int64_t)d->nq * c->salient_permille + 999) / 1000) : 0;
+  // the salient selection keeps one score per image token in shared memory
+  if (d->ns > 0 && salient_smem_bytes(*d) > kMaxSalientSmem) return HG_ERR_UNSUPPORTED;
   return HG_OK;
 }
 
@@ -95,7 +103,7 @@ uint64_t layer_mask_bits(const uint8_t* mask, int layer, int H) {
 bool geometry_aligned(const Dims& d, const LayerGeom& g) {
   for (int h = 0; h < d.H; ++h) {
     const HeadGeom hd = head_geom(d, g, h);
-    const uint64_t offs[] = {hd.kb, hd.vb, hd.kq, hd.kqm, hd.vq, hd.vqm, hd.kimg};
+    const uint64_t offs[] = {hd.kb, hd.vb, hd.kq, hd.kqm, hd.vq, hd.vqm, hd.kimg, hd.sal};
     for (uint64_t o : offs)
       if (o != kNone && (o & 15u)) return false;
     const uint64_t strides[] = {hd.kb_bs, hd.kq_bs, hd.kqm_bs, hd.vq_bs, hd.vqm_bs, hd.kimg_bs};
@@ -188,7 +196,8 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
       if (cls == kProtected) {
         total += d.T * sb.bf16;
       } else {
-        total += (d.T - d.nq) * sb.bf16 + d.nq * (cls == kKeysOnly ? sb.coded_k : sb.coded_u);
+        const int nc = cls == kKeysOnly ? d.nq : ncoded(d);
+        total += (d.T - nc) * sb.bf16 + nc * (cls == kKeysOnly ? sb.coded_k : sb.coded_u);
       }
     }
   }
@@ -200,15 +209,16 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
   // one wave, or every segment is a single chunk.
   DecodePlan p;
   for (int iter = 0; iter < 64; ++iter, item *= 1.05) {
-    p.cbU = chunk_tokens(d.T - d.nq + d.S_new, sb.bf16, item, 64);
-    p.cqU = chunk_tokens(d.nq, sb.coded_u, item, 64);
+    p.cbU = chunk_tokens(d.T - ncoded(d) + d.S_new, sb.bf16, item, 64);
+    p.cqU = chunk_tokens(ncoded(d), sb.coded_u, item, 64);
     p.cqK = chunk_tokens(d.nq, sb.coded_k, item, 64);
     p.cbP = chunk_tokens(d.T + d.S_new, sb.bf16, item, 64);
     long long items = 0;
     for (int l = begin; l < begin + count; ++l)
       items += (long long)d.B * row_chunks(d, c->layer_mask[l], counts_of(d, d.S_new, p));
     if (items <= wave) break;
-    if (p.cbU >= d.T - d.nq + d.S_new && p.cqU >= d.nq && p.cqK >= d.nq && p.cbP >= d.T + d.S_new) break;
+    if (p.cbU >= d.T - ncoded(d) + d.S_new && p.cqU >= ncoded(d) && p.cqK >= d.nq && p.cbP >= d.T + d.S_new)
+      break;
   }
   // The merging CTA stages every split's partial of a head in its stage buffer.
   while (max_items_of(d, p) > decode_max_splits(d.G)) {
@@ -367,6 +377,10 @@ hg_status hg_cache_head_regions(const hg_cache* c, int32_t layer, int32_t head, 
   out->vq_bstride = hd.vq_bs;
   out->vqm_bstride = hd.vqm_bs;
   out->kimg_bstride = hd.kimg_bs;
+  out->sal = abs(hd.sal);
+  out->sal_bstride = hd.sal_bs;
+  out->n_coded = hd.cls == kProtected ? 0 : (hd.cls == kKeysOnly ? c->d.nq : ncoded(c->d));
+  out->n_salient = hd.cls == kQuantized ? c->d.ns : 0;
   return HG_OK;
 }
 
@@ -402,6 +416,10 @@ hg_status hg_quantize_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count,
     for (int i = 0; i < n; ++i) {
       p.k[i] = static_cast<const uint16_t*>(k[done + i]);
       p.v[i] = static_cast<const uint16_t*>(v[done + i]);
+    }
+    if (d.ns > 0) {  // the salient-token maps first: the quantizer reads them
+      const hg_status st = cuda_status(launch_salient(p, reinterpret_cast<cudaStream_t>(stream)));
+      if (st != HG_OK) return st;
     }
     const hg_status st = cuda_status(launch_quantize(p, reinterpret_cast<cudaStream_t>(stream)));
     if (st != HG_OK) return st;
@@ -521,14 +539,15 @@ int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, 
         const int cls = head_class(d, c->layer_mask[begin + i], h);
         int nb;
         const int ni = head_chunks(cls, cc, &nb);
-        const int blen = (cls == kProtected ? d.T : d.T - d.nq) + L.appended;
+        const int blen = (cls == kProtected ? d.T : d.T - d.nq + d.ns) + L.appended;
+        const int clen = cls == kKeysOnly ? d.nq : ncoded(d);
         const int bc = (cls == kProtected) ? p.plan.cbP : p.plan.cbU;
         const int qc = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
         const double qb = (cls == kKeysOnly) ? sb.coded_k : sb.coded_u;
         for (int r = 0; r < ni; ++r) {
           double w;
           if (r < nb) w = std::min(bc, blen - r * bc) * sb.bf16;
-          else w = std::min(qc, d.nq - (r - nb) * qc) * qb;
+          else w = std::min(qc, clen - (r - nb) * qc) * qb;
           cost.emplace_back(w, item++);
           rec.push_back(order_record(i, b, h, r));
         }
@@ -699,7 +718,9 @@ hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {
   for (int l = 0; l < d.L; ++l) {
     for (int h = 0; h < d.H; ++h) {
       const int cls = head_class(d, c->layer_mask[l], h);
-      const double coded = d.nq, bf16 = d.n - d.nq;
+      // salient image tokens (quantized heads only) are BF16 like the
+      // image tokens outside the eligible span
+      const double coded = cls == kKeysOnly ? d.nq : ncoded(d), bf16 = d.n - coded;
       double kb = 0, vb = 0;
       if (cls == kQuantized) {
         kb = coded * (code_bits + kmeta_tok) + bf16 * 16.0 * kD;

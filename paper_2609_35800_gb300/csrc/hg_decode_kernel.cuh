@@ -1120,7 +1120,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   } else {
     const int c = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
     tb = (r - nb) * c;
-    te = min(tb + c, d.nq);
+    te = min(tb + c, cls == kKeysOnly ? d.nq : ncoded(d));
   }
   const int tid = threadIdx.x;
   const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;

@@ -110,6 +110,13 @@ struct DecodeParams {
 constexpr int kArenaBoxRows = 16;
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s);
+// Salient-token maps (AKVQ-style, Sec. 4) of every quantized head of the
+// launch's layers, from the prefill keys; run before launch_quantize.
+cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s);
+// Shared memory of the salient selection: a score per image token plus a
+// bit per image token.
+inline size_t salient_smem_bytes(const Dims& d) { return (size_t)d.nq * 4 + (size_t)sal_blocks(d) * 4; }
+constexpr size_t kMaxSalientSmem = 200 * 1024;
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s);

@@ -29,6 +29,7 @@ struct Dims {
   int B, L, H, Hq, G, T, s, n, nq, S_new;
   int base, bits, keys_only, residual;
   int meta16;  // metadata pairs as binary16 {scale, zero} (4 bytes) instead of fp32 (8)
+  int ns;      // salient image tokens kept BF16 per quantized head (AKVQ-style, Sec. 4)
 };
 
 HG_HD uint64_t align_up(uint64_t x) { return (x + kAlign - 1) & ~(kAlign - 1); }
@@ -53,6 +54,15 @@ HG_HD int quantized_count(int T, int s, int n, int base, int residual) {
   return (span / kKiviGroup) * kKiviGroup;
 }
 
+// Image tokens stored coded per head with coded values: the eligible span less
+// the salient tokens (heads whose keys are quantized; no salient tokens exist
+// together with keys-only heads).
+HG_HD int ncoded(const Dims& d) { return d.nq - d.ns; }
+// Salient-token map of one (batch row, quantized head): a bit per image token
+// in 32-token blocks (uint32 [nblk]), then the number of salient tokens before
+// each block (int32 [nblk]); rows padded to 16 bytes.
+HG_HD int sal_blocks(const Dims& d) { return (d.nq + 31) / 32; }
+
 // Bytes per token of one head's packed codes (128 codes).
 HG_HD uint64_t code_bytes_per_token(const Dims& d) { return (uint64_t)kD * d.bits / 8; }
 HG_HD uint64_t align16(uint64_t x) { return (x + 15) & ~15ull; }
@@ -61,25 +71,26 @@ HG_HD uint64_t meta_pair_bytes(const Dims& d) { return d.meta16 ? 4 : 8; }
 // Key metadata bytes for nq tokens of one batch row of one head (payload).
 HG_HD uint64_t kmeta_bytes(const Dims& d) {
   return d.base == kKivi ? (uint64_t)(d.nq / kKiviGroup) * kD * meta_pair_bytes(d)
-                         : (uint64_t)d.nq * meta_pair_bytes(d);
+                         : (uint64_t)ncoded(d) * meta_pair_bytes(d);
 }
 // Value metadata groups per token.
 HG_HD int vgroups(const Dims& d) { return d.base == kKivi ? kD / kKiviGroup : 1; }
-HG_HD uint64_t vmeta_bytes(const Dims& d) { return (uint64_t)d.nq * vgroups(d) * meta_pair_bytes(d); }
+HG_HD uint64_t vmeta_bytes(const Dims& d) { return (uint64_t)ncoded(d) * vgroups(d) * meta_pair_bytes(d); }
 // Batch-row strides of the metadata arrays: padded to 16 bytes so that every
 // row (and every head's block of rows) starts on a 16-byte boundary, as the
 // 16-byte asynchronous copies of the decode kernel require.
 HG_HD uint64_t kmeta_stride(const Dims& d) { return align16(kmeta_bytes(d)); }
 HG_HD uint64_t vmeta_stride(const Dims& d) { return align16(vmeta_bytes(d)); }
+HG_HD uint64_t sal_stride(const Dims& d) { return d.ns > 0 ? align16((uint64_t)sal_blocks(d) * 8) : 0; }
 
 struct LayerGeom {
   uint64_t mask;
   int n_prot, n_U, n_PK, n_PKV, n_VQ;
-  uint64_t kb, vb, kq, kqm, vq, vqm, kimg, size;  // region offsets relative to the layer base
+  uint64_t kb, vb, kq, kqm, vq, vqm, kimg, sal, size;  // region offsets relative to the layer base
   uint64_t bf16_bytes;                             // size of the kb (and vb) region
 };
 
-HG_HD int cap_unprot(const Dims& d) { return d.T - d.nq + d.S_new; }
+HG_HD int cap_unprot(const Dims& d) { return d.T - d.nq + d.ns + d.S_new; }
 
 HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
   LayerGeom g;
@@ -90,16 +101,18 @@ HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
   g.n_PKV = d.keys_only ? 0 : g.n_prot;
   g.n_VQ = g.n_U + g.n_PK;
   const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
-  const uint64_t tok_bf16 = (uint64_t)d.H * cap_unprot(d) + (uint64_t)g.n_PKV * nq;
+  const uint64_t nc = (uint64_t)ncoded(d);
+  const uint64_t tok_bf16 = (uint64_t)d.H * cap_unprot(d) + (uint64_t)g.n_PKV * nc;
   g.bf16_bytes = align_up(B * tok_bf16 * kD * 2);
   uint64_t off = 0;
   g.kb = off; off += g.bf16_bytes;
   g.vb = off; off += g.bf16_bytes;
-  g.kq = off; off += align_up((uint64_t)g.n_U * B * nq * code_bytes_per_token(d));
+  g.kq = off; off += align_up((uint64_t)g.n_U * B * nc * code_bytes_per_token(d));
   g.kqm = off; off += align_up((uint64_t)g.n_U * B * kmeta_stride(d));
-  g.vq = off; off += align_up((uint64_t)g.n_VQ * B * nq * code_bytes_per_token(d));
+  g.vq = off; off += align_up((uint64_t)g.n_VQ * B * nc * code_bytes_per_token(d));
   g.vqm = off; off += align_up((uint64_t)g.n_VQ * B * vmeta_stride(d));
   g.kimg = off; off += align_up((uint64_t)g.n_PK * B * nq * kD * 2);
+  g.sal = off; off += align_up((uint64_t)g.n_U * B * sal_stride(d));
   g.size = off;
   return g;
 }
@@ -115,8 +128,8 @@ struct HeadGeom {
   int cls;
   int bf16_prefill;  // BF16 tokens that come from the prefill
   int cap;           // BF16 capacity (prefill + max_new_tokens)
-  uint64_t kb, vb, kq, kqm, vq, vqm, kimg;
-  uint64_t kb_bs, kq_bs, kqm_bs, vq_bs, vqm_bs, kimg_bs;
+  uint64_t kb, vb, kq, kqm, vq, vqm, kimg, sal;
+  uint64_t kb_bs, kq_bs, kqm_bs, vq_bs, vqm_bs, kimg_bs, sal_bs;
 };
 
 HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
@@ -125,23 +138,27 @@ HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
   const int prot_below = popc64(below);
   const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
   r.cls = head_class(d, g.mask, h);
-  r.bf16_prefill = (r.cls == kProtected) ? d.T : d.T - d.nq;
+  r.bf16_prefill = (r.cls == kProtected) ? d.T : d.T - d.nq + d.ns;
   r.cap = r.bf16_prefill + d.S_new;
   const uint64_t pkv_below = d.keys_only ? 0ull : (uint64_t)prot_below;
-  const uint64_t tok_before = (uint64_t)h * cap_unprot(d) + pkv_below * nq;
+  // a protected K+V head holds ncoded(d) more BF16 tokens than the others
+  const uint64_t tok_before = (uint64_t)h * cap_unprot(d) + pkv_below * (uint64_t)ncoded(d);
   r.kb_bs = (uint64_t)r.cap * kD * 2;
   r.kb = g.kb + B * tok_before * kD * 2;
   r.vb = g.vb + B * tok_before * kD * 2;
-  r.kq_bs = nq * code_bytes_per_token(d);
+  const uint64_t nc = (uint64_t)ncoded(d);
+  r.kq_bs = nc * code_bytes_per_token(d);
   r.kqm_bs = kmeta_stride(d);
-  r.vq_bs = nq * code_bytes_per_token(d);
+  r.vq_bs = nc * code_bytes_per_token(d);
   r.vqm_bs = vmeta_stride(d);
   r.kimg_bs = nq * kD * 2;
-  r.kq = r.kqm = r.vq = r.vqm = r.kimg = kNone;
+  r.sal_bs = sal_stride(d);
+  r.kq = r.kqm = r.vq = r.vqm = r.kimg = r.sal = kNone;
   if (r.cls == kQuantized) {
     const uint64_t u = (uint64_t)(h - prot_below);
     r.kq = g.kq + u * B * r.kq_bs;
     r.kqm = g.kqm + u * B * r.kqm_bs;
+    if (d.ns > 0) r.sal = g.sal + u * B * r.sal_bs;
   }
   if (r.cls != kProtected) {
     const uint64_t vr = d.keys_only ? (uint64_t)h : (uint64_t)(h - prot_below);
@@ -155,12 +172,15 @@ HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
 }
 
 // Position of prefill token t in a head's BF16 region, or -1 when the token is
-// stored in the quantized (or keys-only image) regions.
+// an image token of a head whose image tokens are coded (the salient ones of
+// a quantized head sit at d.s + their rank among the salient tokens; the
+// kernels place them).  Region order: leading text, salient image tokens,
+// trailing text, appended tokens.
 HG_HD int bf16_pos(const Dims& d, int cls, int t) {
   if (cls == kProtected) return t;
   if (t < d.s) return t;
   if (t < d.s + d.nq) return -1;
-  return t - d.nq;
+  return t - d.nq + d.ns;
 }
 
 // ---------------------------------------------------------------------------
@@ -179,8 +199,8 @@ struct ChunkCounts {
 
 HG_HD ChunkCounts chunk_counts(const Dims& d, int appended, int cbU, int cqU, int cqK, int cbP) {
   ChunkCounts c;
-  c.nbU = cdiv(d.T - d.nq + appended, cbU);
-  c.nqU = cdiv(d.nq, cqU);
+  c.nbU = cdiv(d.T - d.nq + d.ns + appended, cbU);
+  c.nqU = cdiv(ncoded(d), cqU);
   c.nqK = cdiv(d.nq, cqK);
   c.nbP = cdiv(d.T + appended, cbP);
   return c;

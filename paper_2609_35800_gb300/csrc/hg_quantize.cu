@@ -10,6 +10,8 @@
 // max with warp butterflies, KIVI-style value groups (32 channels) with
 // 8-lane butterflies, and KIVI-style key groups (32 tokens of one channel) are
 // quantized by one thread per channel from a shared-memory copy of the tile.
+#include <climits>
+
 #include <cuda_bf16.h>
 #include <cuda_runtime.h>
 
@@ -112,6 +114,21 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
 
   __shared__ __align__(16) uint16_t ktile[kTile][kD];
 
+  // AKVQ-style salient tokens (Sec. 4): the map of this tile's image tokens.
+  // Image tiles start on the image's 32-token blocks, so one map word covers
+  // the tile: a salient token goes to BF16 position qs + (its rank among the
+  // salient tokens), every other image token to coded slot ti - (the salient
+  // tokens before it).
+  uint32_t sbits = 0u;
+  int srank = 0;
+  const bool sal_tile = d.ns > 0 && hd.cls == kQuantized && t0 >= qs && t0 < qe;
+  if (sal_tile) {
+    const char* sm = Lb + hd.sal + b * hd.sal_bs;
+    const int w = (t0 - qs) >> 5;
+    sbits = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
+    srank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w);
+  }
+
   // Issue every load of this warp's tokens first (8 tokens x (K, V) x 8 bytes / lane).
   uint2 kr[kTile / 4], vr[kTile / 4];
 #pragma unroll
@@ -129,9 +146,18 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
     if (t >= t1) break;
     const bool coded = (t >= qs) && (t < qe);
     const int ti = t - qs;
+    int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token
+    bool sal = false;
+    if (sal_tile && coded) {
+      const int j = t - t0;
+      const int rank = srank + __popc(sbits & ((1u << j) - 1u));
+      sal = (sbits >> j) & 1u;
+      ci = ti - rank;
+      spos = qs + rank;
+    }
 
     // ---- key ----
-    if (coded && hd.cls == kQuantized) {
+    if (coded && hd.cls == kQuantized && !sal) {
       if (d.base == kKivi) {
         *reinterpret_cast<uint2*>(&ktile[t - t0][lane * 4]) = kr[i];
       } else {
@@ -141,27 +167,27 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
         uint32_t c[4];
         float sc, z;
         quantize_group4<32>(x, d.bits, m16, c, sc, z);
-        uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W;
+        uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
         store_token_codes(crow, c, d.bits, lane);
-        if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ti, sc, z, m16);
+        if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, sc, z, m16);
       }
     } else if (coded && hd.cls == kKeysOnly) {
       *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) =
           kr[i];
     } else {
-      const int pos = bf16_pos(d, hd.cls, t);
+      const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
       *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
           kr[i];
     }
 
     // ---- value (never rotated) ----
-    if (coded && hd.cls != kProtected) {
+    if (coded && hd.cls != kProtected && !sal) {
       float x[4];
       bf16x4_to_f32(vr[i], x);
       uint32_t c[4];
       float sc, z;
       char* meta = Lb + hd.vqm + b * hd.vqm_bs;
-      const size_t mi = (size_t)ti * vgroups(d);
+      const size_t mi = (size_t)ci * vgroups(d);
       if (d.base == kKivi) {
         quantize_group4<8>(x, d.bits, m16, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
         if ((lane & 7) == 0) store_meta(meta, mi + (lane >> 3), sc, z, m16);
@@ -169,10 +195,10 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
         quantize_group4<32>(x, d.bits, m16, c, sc, z);
         if (lane == 0) store_meta(meta, mi, sc, z, m16);
       }
-      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W;
+      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W;
       store_token_codes(crow, c, d.bits, lane);
     } else {
-      const int pos = bf16_pos(d, hd.cls, t);
+      const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
       *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
           vr[i];
     }
@@ -401,6 +427,99 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
   }
 }
 
+// ---------------------------------------------------------------------------
+// AKVQ-style salient tokens (Sec. 4): one CTA per (batch row, KV head, layer);
+// heads whose image keys are not quantized return.  Squared key norms of the
+// image tokens in the fixed binary32 order (a warp per token: lane l sums
+// channels 4l..4l+3, then five butterfly rounds of pairwise sums), ns rounds
+// of a CTA-wide arg-max (largest score, ties to the lower index), then the
+// map: a bit per image token and the salient count before each 32-token block.
+// ---------------------------------------------------------------------------
+constexpr int kSalThreads = 256;
+
+__global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_constant__ QuantizeParams p) {
+  const Dims& d = p.d;
+  const int bh = blockIdx.x, li = blockIdx.y;
+  const int b = bh / d.H, h = bh % d.H;
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+  const HeadGeom hd = head_geom(d, g, h);
+  if (hd.cls != kQuantized || d.ns <= 0) return;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int nq = d.nq, nblk = sal_blocks(d);
+  extern __shared__ __align__(16) float sal_smem[];
+  float* score = sal_smem;                                     // [nq]
+  uint32_t* bits = reinterpret_cast<uint32_t*>(sal_smem + nq);  // [nblk]
+  __shared__ float red_v[kSalThreads / 32];
+  __shared__ int red_i[kSalThreads / 32];
+
+  const uint16_t* K = p.k[li] + (((size_t)b * d.H + h) * d.T + d.s) * kD;
+  for (int i = warp; i < nq; i += kSalThreads / 32) {
+    float x[4];
+    bf16x4_to_f32(ldg8(K + (size_t)i * kD + lane * 4), x);
+    float a = __fmul_rn(x[0], x[0]);
+    a = __fadd_rn(a, __fmul_rn(x[1], x[1]));
+    a = __fadd_rn(a, __fmul_rn(x[2], x[2]));
+    a = __fadd_rn(a, __fmul_rn(x[3], x[3]));
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1) a = __fadd_rn(a, __shfl_xor_sync(kFull, a, m));
+    if (lane == 0) score[i] = a;
+  }
+  for (int w = tid; w < nblk; w += kSalThreads) bits[w] = 0u;
+  __syncthreads();
+
+#pragma unroll 1
+  for (int r = 0; r < d.ns; ++r) {
+    // a thread scans increasing indices, so a strict > keeps the lower index
+    float bv = -INFINITY;
+    int bi = INT_MAX;
+    for (int i = tid; i < nq; i += kSalThreads) {
+      const float v = score[i];
+      if (v > bv) {
+        bv = v;
+        bi = i;
+      }
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float ov = __shfl_xor_sync(kFull, bv, o);
+      const int oi = __shfl_xor_sync(kFull, bi, o);
+      if (ov > bv || (ov == bv && oi < bi)) {
+        bv = ov;
+        bi = oi;
+      }
+    }
+    if (lane == 0) {
+      red_v[warp] = bv;
+      red_i[warp] = bi;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      for (int w = 1; w < kSalThreads / 32; ++w)
+        if (red_v[w] > bv || (red_v[w] == bv && red_i[w] < bi)) {
+          bv = red_v[w];
+          bi = red_i[w];
+        }
+      if (bi < nq) {  // taken tokens drop out of later rounds
+        score[bi] = -INFINITY;
+        bits[bi >> 5] |= 1u << (bi & 31);
+      }
+    }
+    __syncthreads();
+  }
+
+  char* dst = p.arena + p.lt.base[li] + hd.sal + b * hd.sal_bs;
+  uint32_t* out_bits = reinterpret_cast<uint32_t*>(dst);
+  int* out_rank = reinterpret_cast<int*>(dst + (size_t)nblk * 4);
+  for (int w = tid; w < nblk; w += kSalThreads) out_bits[w] = bits[w];
+  if (tid == 0) {
+    int acc = 0;
+    for (int w = 0; w < nblk; ++w) {
+      out_rank[w] = acc;
+      acc += __popc(bits[w]);
+    }
+  }
+}
+
 // Reconstruct one layer as floats in original token order (then appended).
 __global__ void __launch_bounds__(kThreads)
 dequantize_kernel(const __grid_constant__ DequantParams p) {
@@ -419,9 +538,21 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
   for (int t = blockIdx.x * kTile + warp; t < min(Tt, (int)(blockIdx.x + 1) * kTile); t += 4) {
     const bool coded = (t >= qs) && (t < qe);
     const int ti = t - qs;
-    const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : bf16_pos(d, hd.cls, t);
+    int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token (Sec. 4)
+    bool sal = false;
+    if (coded && d.ns > 0 && hd.cls == kQuantized) {
+      const char* sm = Lb + hd.sal + b * hd.sal_bs;
+      const int w = ti >> 5, j = ti & 31;
+      const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
+      const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
+                       __popc(sb & ((1u << j) - 1u));
+      sal = (sb >> j) & 1u;
+      ci = ti - rank;
+      spos = qs + rank;
+    }
+    const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
     float xk[4], xv[4];
-    if (coded && hd.cls == kQuantized) {
+    if (coded && hd.cls == kQuantized && !sal) {
       uint32_t c[4];
       if (d.base == kKivi) {
         const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
@@ -437,9 +568,9 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
           xk[i] = dequant1(code, m.x, m.y);
         }
       } else {
-        load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
+        load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W,
                          d.bits, lane, c);
-        const float2 m = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ti, m16);
+        const float2 m = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, m16);
 #pragma unroll
         for (int i = 0; i < 4; ++i) xk[i] = dequant1(c[i], m.x, m.y);
         if (d.base == kAkvq) fwht128_warp(xk, lane);  // inverse rotation (H is self-inverse)
@@ -449,12 +580,12 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
     } else {
       bf16x4_to_f32(ldg8(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2), xk);
     }
-    if (coded && hd.cls != kProtected) {
+    if (coded && hd.cls != kProtected && !sal) {
       uint32_t c[4];
-      load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+      load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
                        d.bits, lane, c);
       const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
-                                 (size_t)ti * vgroups(d) + (d.base == kKivi ? (lane >> 3) : 0), m16);
+                                 (size_t)ci * vgroups(d) + (d.base == kKivi ? (lane >> 3) : 0), m16);
 #pragma unroll
       for (int i = 0; i < 4; ++i) xv[i] = dequant1(c[i], m.x, m.y);
     } else {
@@ -512,6 +643,18 @@ cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
   }
   dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
   quantize_kernel<<<grid, kThreads, 0, s>>>(p);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s) {
+  const size_t smem = salient_smem_bytes(p.d);
+  if (smem > 48 * 1024) {
+    const cudaError_t e =
+        cudaFuncSetAttribute(salient_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+  }
+  dim3 grid(p.d.B * p.d.H, p.n_layers, 1);
+  salient_kernel<<<grid, kSalThreads, smem, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -17,7 +17,8 @@ def config_of(w):
     return QuantConfig(base=w.base, bits=w.bits, keys_only=int(w.keys_only),
                        kivi_group_tokens=w.kivi_group_tokens,
                        kivi_group_channels=w.kivi_group_channels,
-                       kivi_residual=w.kivi_residual, meta_bits=w.meta_bits)
+                       kivi_residual=w.kivi_residual, meta_bits=w.meta_bits,
+                       salient_permille=w.salient_permille)
 
 
 class CacheRunner:

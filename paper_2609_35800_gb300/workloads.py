@@ -48,6 +48,7 @@ class Workload:
     kivi_group_channels: int = 32
     kivi_residual: int = 32
     meta_bits: int = 64             # 64: fp32 {scale, zero}; 32: binary16 pair (Sec. 5.4)
+    salient_permille: int = 0       # AKVQ-style salient tokens kept BF16 (Sec. 4; 20 = 2%)
 
     @property
     def seq_len(self):
@@ -158,10 +159,11 @@ def step_new_kv(w, step, device, layers=None):
 
 def custom(name, layers, batch, q_heads, kv_heads, text_prefix, image, text_suffix, base, bits,
            keys_only, decode_steps=2, seed=0, protected=None, residual=32, n_outliers=4,
-           meta_bits=64):
+           meta_bits=64, salient_permille=0):
     """A small workload for tests: `protected` lists (layer, head) pairs (empty = none),
     None draws round(N_KV / 8) of them."""
     return Workload(name, layers, batch, q_heads, kv_heads, text_prefix, image, text_suffix, base,
                     bits, bool(keys_only), decode_steps, seed,
                     fixed_protected=None if protected is None else tuple(protected),
-                    n_outliers=n_outliers, kivi_residual=residual, meta_bits=meta_bits)
+                    n_outliers=n_outliers, kivi_residual=residual, meta_bits=meta_bits,
+                    salient_permille=salient_permille)

@@ -24,12 +24,17 @@ def bf16_rne(x):
     return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
 
 
+def n_salient(w):
+    """Salient tokens per quantized head (Sec. 4, reading R15) of a workload."""
+    return oracle.salient_count(w.image, w.salient_permille) if w.salient_permille else 0
+
+
 def oracle_layer(runner, layer, k_bits, v_bits):
     w = runner.w
     return oracle.quantize_layer(k_bits, v_bits, w.img_start, w.image, w.base, w.bits,
                                  runner.mask[layer], int(w.keys_only), w.kivi_group_tokens,
                                  w.kivi_group_channels, w.kivi_residual,
-                                 meta16=w.meta_bits == 32)
+                                 meta16=w.meta_bits == 32, n_salient=n_salient(w))
 
 
 def _slice(arena, off, nbytes, dtype):
@@ -57,31 +62,49 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
     W = 128 * w.bits // 32
     heads = range(H) if heads is None else heads
     rows = range(B) if rows is None else rows
+    ns = o["n_salient"]
     for h in heads:
         r = hg.hg_cache_head_regions(runner.cache, layer, h)
         assert r.nq == nq
         cls = r.head_class
-        if cls == hg.HG_HEAD_PROTECTED:
-            toks = np.arange(T)
-        else:
-            toks = np.concatenate([np.arange(0, s), np.arange(s + nq, T)])
-        assert r.bf16_prefill == toks.size
+        assert r.n_salient == (ns if cls == hg.HG_HEAD_QUANTIZED else 0)
+        nc = 0 if cls == hg.HG_HEAD_PROTECTED else nq - r.n_salient
+        assert r.n_coded == nc
         for b in rows:
+            if cls == hg.HG_HEAD_PROTECTED:
+                toks = np.arange(T)
+            elif r.n_salient:
+                # leading text, salient image tokens in order, trailing text
+                sal = o["salient"][b, h]
+                toks = np.concatenate([np.arange(0, s), s + sal, np.arange(s + nq, T)])
+                nblk = (nq + 31) // 32
+                words = _slice(arena, r.sal + b * r.sal_bstride, nblk * 8, np.uint32)
+                want = np.zeros(nblk, np.uint32)
+                for i in sal:
+                    want[i >> 5] |= np.uint32(1 << (i & 31))
+                ranks = np.concatenate([[0], np.cumsum([bin(int(x)).count("1") for x in want])[:-1]])
+                assert np.array_equal(words[:nblk], want), (layer, h, b, "salient bits")
+                assert np.array_equal(words[nblk:].view(np.int32), ranks), (layer, h, b, "ranks")
+            else:
+                toks = np.concatenate([np.arange(0, s), np.arange(s + nq, T)])
+            assert r.bf16_prefill == toks.size
             kb = _slice(arena, r.kb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
             vb = _slice(arena, r.vb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
             assert np.array_equal(kb, k_bits[b, h, toks]), (layer, h, b, "kb")
             assert np.array_equal(vb, v_bits[b, h, toks]), (layer, h, b, "vb")
-            if cls == hg.HG_HEAD_QUANTIZED and nq:
-                kw = _slice(arena, r.kq + b * r.kq_bstride, nq * W * 4, np.uint32)
-                ek = _meta_words(o["k_meta"][b, h], m16)
+            kmeta_n = o["k_meta"][b, h].size if w.base == 1 else 2 * nc
+            vmeta_n = o["v_meta"][b, h].size * nc // max(nq, 1)
+            if cls == hg.HG_HEAD_QUANTIZED and nc:
+                kw = _slice(arena, r.kq + b * r.kq_bstride, nc * W * 4, np.uint32)
+                ek = _meta_words(o["k_meta"][b, h][:kmeta_n], m16)
                 km = _slice(arena, r.kqm + b * r.kqm_bstride, ek.nbytes, np.uint32)
-                assert np.array_equal(kw, o["k_words"][b, h]), (layer, h, b, "kq")
+                assert np.array_equal(kw, o["k_words"][b, h][:nc * W]), (layer, h, b, "kq")
                 assert np.array_equal(km, ek), (layer, h, b, "kqm")
-            if cls != hg.HG_HEAD_PROTECTED and nq:
-                vw = _slice(arena, r.vq + b * r.vq_bstride, nq * W * 4, np.uint32)
-                ev = _meta_words(o["v_meta"][b, h], m16)
+            if cls != hg.HG_HEAD_PROTECTED and nc:
+                vw = _slice(arena, r.vq + b * r.vq_bstride, nc * W * 4, np.uint32)
+                ev = _meta_words(o["v_meta"][b, h][:vmeta_n], m16)
                 vm = _slice(arena, r.vqm + b * r.vqm_bstride, ev.nbytes, np.uint32)
-                assert np.array_equal(vw, o["v_words"][b, h]), (layer, h, b, "vq")
+                assert np.array_equal(vw, o["v_words"][b, h][:nc * W]), (layer, h, b, "vq")
                 assert np.array_equal(vm, ev), (layer, h, b, "vqm")
             if cls == hg.HG_HEAD_KEYS_ONLY and nq:
                 ki = _slice(arena, r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)

@@ -67,6 +67,11 @@ def _status(f, *a):
     ({}, dict(keys_only=2), 1),
     ({}, dict(meta_bits=16), 1),
     ({}, dict(meta_bits=48), 1),
+    ({}, dict(base=2, salient_permille=-1), 1),
+    ({}, dict(base=2, salient_permille=1001), 1),
+    ({}, dict(base=0, salient_permille=20), 3),
+    ({}, dict(base=1, salient_permille=20), 3),
+    ({}, dict(base=2, keys_only=1, salient_permille=20), 3),
 ])
 def test_layout_validation(lib, shape_kw, cfg_kw, status):
     mask = np.zeros((3, max(4, shape_kw.get("num_kv_heads", 4))), np.uint8)
@@ -101,7 +106,11 @@ ODD = {"odd_nq_minmax": wl.custom("odd", 3, 3, 16, 4, 64, 333, 17, wl.BASE_MINMA
        "meta16_minmax": wl.custom("m16a", 2, 3, 16, 4, 9, 333, 17, wl.BASE_MINMAX, 2, 0,
                                   meta_bits=32),
        "meta16_kivi_konly": wl.custom("m16b", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 4, 1,
-                                      meta_bits=32)}
+                                      meta_bits=32),
+       "salient_akvq": wl.custom("sal", 3, 2, 16, 4, 9, 333, 17, wl.BASE_AKVQ, 4, 0,
+                                 salient_permille=20),
+       "salient_all": wl.custom("sal2", 2, 3, 8, 8, 5, 70, 9, wl.BASE_AKVQ, 2, 0,
+                                salient_permille=1000)}
 
 
 @pytest.mark.parametrize("name", list(wl.WORKLOADS) + list(ODD))
@@ -120,7 +129,7 @@ def test_regions_tile_the_arena_without_overlap(lib, name):
             spans.append((r.vb, B * r.kb_bstride))
             assert r.kb_bstride == r.bf16_capacity * 256
             if r.kq != hg.NONE_OFFSET:
-                assert r.kq_bstride == r.nq * W
+                assert r.kq_bstride == r.n_coded * W
                 spans.append((r.kq, B * r.kq_bstride))
                 spans.append((r.kqm, B * r.kqm_bstride))
             if r.vq != hg.NONE_OFFSET:
@@ -128,7 +137,10 @@ def test_regions_tile_the_arena_without_overlap(lib, name):
                 spans.append((r.vqm, B * r.vqm_bstride))
             if r.kimg != hg.NONE_OFFSET:
                 spans.append((r.kimg, B * r.kimg_bstride))
-            for off in (r.kb, r.vb, r.kq, r.kqm, r.vq, r.vqm, r.kimg):
+            if r.sal != hg.NONE_OFFSET:
+                assert r.n_salient > 0 and r.sal_bstride >= (r.nq + 31) // 32 * 8
+                spans.append((r.sal, B * r.sal_bstride))
+            for off in (r.kb, r.vb, r.kq, r.kqm, r.vq, r.vqm, r.kimg, r.sal):
                 if off != hg.NONE_OFFSET:
                     assert off % 16 == 0
             for st in (r.kb_bstride, r.kq_bstride, r.kqm_bstride, r.vq_bstride, r.vqm_bstride,
@@ -187,6 +199,31 @@ def test_meta16_halves_metadata_regions(lib, base):
     pad = lambda x: (x + 15) // 16 * 16
     assert (r64.kqm_bstride, r32.kqm_bstride) == (pad(8 * groups_k), pad(4 * groups_k))
     assert (r64.vqm_bstride, r32.vqm_bstride) == (pad(8 * groups_v), pad(4 * groups_v))
+
+
+def test_salient_layout(lib):
+    # AKVQ-style salient tokens (Sec. 4): quantized heads hold ceil(2% of n) image
+    # tokens in BF16 and the rest coded; protected heads are unchanged
+    w = wl.custom("s", 1, 2, 8, 4, 16, 1296, 8, wl.BASE_AKVQ, 2, 0, protected=[(0, 1)],
+                  salient_permille=20)
+    w0 = wl.custom("s0", 1, 2, 8, 4, 16, 1296, 8, wl.BASE_AKVQ, 2, 0, protected=[(0, 1)])
+    c, _, _ = _fake_cache(w)
+    c0, _, _ = _fake_cache(w0)
+    for h in range(4):
+        r, r0 = hg.hg_cache_head_regions(c, 0, h), hg.hg_cache_head_regions(c0, 0, h)
+        if h == 1:
+            assert (r.n_salient, r.n_coded, r.bf16_prefill) == (0, 0, r0.bf16_prefill)
+            assert r.sal == hg.NONE_OFFSET
+        else:
+            assert (r.n_salient, r.n_coded) == (26, 1270)
+            assert r.bf16_prefill == r0.bf16_prefill + 26
+            assert r.bf16_capacity == r0.bf16_capacity + 26
+            assert r.kq_bstride == 1270 * 32 and r.kqm_bstride == 1270 * 8
+    # stored bits: 26 of 1296 image tokens of each quantized head in BF16
+    got = hg.hg_cache_image_bits_per_elem(c)
+    q = (1270 * (2 * 128 + 64) + 26 * 16 * 128) / (1296 * 128)
+    want = (3 * q + 1 * 16) / 4
+    assert got == pytest.approx(want, rel=1e-12)
 
 
 def test_calls_validate_before_any_launch(lib):

@@ -51,10 +51,11 @@ CASES = [
 ]
 
 
-def _workload(case, meta_bits=64):
+def _workload(case, meta_bits=64, salient_permille=0):
     (name, L, B, Hq, H, pre, img, suf, base, bits, ko, steps, prot, R) = case
     return wl.custom(name, L, B, Hq, H, pre, img, suf, base, bits, ko, decode_steps=steps,
-                     seed=7, protected=prot, residual=R, meta_bits=meta_bits)
+                     seed=7, protected=prot, residual=R, meta_bits=meta_bits,
+                     salient_permille=salient_permille)
 
 
 def _run_and_check(w, layer_batched=True, fused=False):
@@ -165,11 +166,57 @@ def test_meta16_fused_decode_step(case):
     _run_and_check(_workload(case, meta_bits=32), fused=True)
 
 
+# AKVQ-style salient tokens (Sec. 4): (case, permille)
+SALIENT = [
+    (("akvq4_sal", 2, 2, 16, 4, 64, 333, 17, A, 4, 0, 3, [(0, 3), (1, 0)], 32), 20),
+    (("akvq2_sal_unaligned", 1, 3, 8, 4, 13, 250, 30, A, 2, 0, 2, [(0, 1)], 32), 20),
+    (("akvq2_sal_heavy", 1, 1, 28, 4, 20, 300, 10, A, 2, 0, 2, [(0, 0)], 32), 150),
+    (("akvq4_sal_all", 1, 2, 8, 2, 5, 70, 9, A, 4, 0, 2, [], 32), 1000),
+    (("akvq2_sal_g16", 1, 1, 32, 2, 16, 200, 16, A, 2, 0, 2, [(0, 1)], 32), 20),
+    (("akvq2_sal_long", 1, 1, 28, 4, 50, 3000, 50, A, 2, 0, 2, [(0, 0)], 32), 20),
+]
+
+
+@pytest.mark.parametrize("case,permille", SALIENT, ids=[c[0][0] for c in SALIENT])
+def test_salient_quantize_and_decode_parity(case, permille):
+    """Salient tokens: maps, BF16 rows, compacted codes bit-exact; attention
+    within tolerance (plain and fused decode)."""
+    _run_and_check(_workload(case, salient_permille=permille))
+    _run_and_check(_workload(case, salient_permille=permille), fused=True)
+
+
+def test_salient_ties_and_meta16():
+    """Integer-valued keys give many equal norms: the selection must keep the
+    lower token index on ties, exactly as the oracle; with binary16 metadata."""
+    w = wl.custom("sal_ties", 1, 2, 8, 4, 7, 160, 9, A, 4, 0, decode_steps=1, seed=3,
+                  protected=[(0, 2)], meta_bits=32, salient_permille=50)
+    runner = CacheRunner(w)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    gen = torch.Generator().manual_seed(21)
+    k = torch.randint(-2, 3, (B, H, T, 128), generator=gen).float().to(torch.bfloat16)
+    v = torch.randn((B, H, T, 128), generator=gen).to(torch.bfloat16)
+    k, v = k.contiguous().cuda(), v.contiguous().cuda()
+    hg.hg_quantize_kv(runner.cache, 0, [k], [v])
+    torch.cuda.synchronize()
+    kb, vb = bits16(k), bits16(v)
+    o = oracle_layer(runner, 0, kb, vb)
+    check_arena_layer(runner, 0, kb, vb, o)
+
+
 @pytest.mark.parametrize("meta_bits", [64, 32])
 @pytest.mark.parametrize("case", [CASES[1], CASES[2], CASES[4], CASES[5], CASES[7]],
                          ids=["minmax4", "minmax2_konly", "kivi4", "kivi2", "akvq2"])
 def test_dequantize_bit_exact(case, meta_bits):
-    w = _workload(case, meta_bits)
+    _dequantize_bit_exact(_workload(case, meta_bits))
+
+
+@pytest.mark.parametrize("case,permille", [SALIENT[0], SALIENT[1], SALIENT[3]],
+                         ids=["akvq4", "akvq2_unaligned", "all"])
+def test_salient_dequantize_bit_exact(case, permille):
+    _dequantize_bit_exact(_workload(case, salient_permille=permille))
+
+
+def _dequantize_bit_exact(w):
     runner = CacheRunner(w)
     kept = runner.quantize_all(keep=True)
     # append one step so the appended tail is reconstructed too
