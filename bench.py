@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--workload", default="qwen25vl7b")
     ap.add_argument("--meta-bits", type=int, default=64, choices=[64, 32],
                     help="metadata per group: fp32 pair (64) or binary16 pair (32, Sec. 5.4)")
+    ap.add_argument("--salient-permille", type=int, default=0,
+                    help="AKVQ-style salient tokens kept BF16 per head (Sec. 4; 20 = 2%%)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     return ap.parse_args()
@@ -68,10 +70,11 @@ def geometry_bytes(runner):
     for l in range(w.layers):
         for h in range(H):
             r = hg.hg_cache_head_regions(runner.cache, l, h)
-            nq = r.nq
+            nq = r.n_coded  # coded tokens (image tokens less any salient ones)
             per_b_write = r.bf16_prefill * 512
             per_b_read_dec = r.bf16_prefill * 512
             if r.head_class == hg.HG_HEAD_QUANTIZED:
+                per_b_write += r.sal_bstride  # salient-token map (zero without salient tokens)
                 per_b_write += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
                 per_b_read_dec += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
             elif r.head_class == hg.HG_HEAD_KEYS_ONLY:
@@ -197,6 +200,7 @@ def oracle_sample(w, n_layers, n_steps):
     mask = wl.protection_mask(w).numpy()
     B, H, T = w.batch, w.kv_heads, w.seq_len
     sigma = float(np.float32(1.0 / np.sqrt(128.0)))
+    ns = oracle.salient_count(w.image, w.salient_permille) if w.salient_permille else 0
 
     def bits(t):
         return t.contiguous().view(torch.int16).numpy().view(np.uint16)
@@ -210,16 +214,17 @@ def oracle_sample(w, n_layers, n_steps):
         t0 = time.perf_counter()
         o = oracle.quantize_layer(kb, vb, w.img_start, w.image, w.base, w.bits, mask[l],
                                   int(w.keys_only), w.kivi_group_tokens, w.kivi_group_channels,
-                                  w.kivi_residual, meta16=w.meta_bits == 32)
+                                  w.kivi_residual, meta16=w.meta_bits == 32, n_salient=ns)
         secs += time.perf_counter() - t0
-        nq = o["nq"]
+        nq = o["nq"] - ns  # coded tokens per quantized head
         code_tok = 128 * w.bits // 8
         n_prot = int(mask[l].sum())
         coded_heads_k = (H - n_prot)
         coded_heads_v = H if w.keys_only else (H - n_prot)
         shrink = 2 if w.meta_bits == 32 else 1  # binary16 pairs: half the fp32 pair bytes
-        meta_k = o["k_meta"][0, 0].nbytes // shrink if coded_heads_k else 0
-        meta_v = o["v_meta"][0, 0].nbytes // shrink if coded_heads_v else 0
+        part = nq / max(o["nq"], 1)  # metadata of the coded tokens only
+        meta_k = int(o["k_meta"][0, 0].nbytes * part) // shrink if coded_heads_k else 0
+        meta_v = int(o["v_meta"][0, 0].nbytes * part) // shrink if coded_heads_v else 0
         written = B * (H * T * 512 - (coded_heads_k + coded_heads_v) * nq * 256
                        + coded_heads_k * (nq * code_tok + meta_k)
                        + coded_heads_v * (nq * code_tok + meta_v))
@@ -242,12 +247,12 @@ def oracle_sample(w, n_layers, n_steps):
             secs += time.perf_counter() - t0
             Tt = K.shape[2]
             # same per-token bytes as the packed cache the GPU reads
-            nbytes += _decode_bytes_layer(w, mask[l], outs[l]["nq"], Tt - T) + 2 * B * w.q_heads * 256
+            nbytes += _decode_bytes_layer(w, mask[l], outs[l]["nq"], Tt - T, ns) + 2 * B * w.q_heads * 256
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
     return nbytes, secs, threads
 
 
-def _decode_bytes_layer(w, mask_row, nq, appended):
+def _decode_bytes_layer(w, mask_row, nq, appended, ns=0):
     B, H, T = w.batch, w.kv_heads, w.seq_len
     code_tok = 128 * w.bits // 8
     pair = 4 if w.meta_bits == 32 else 8  # bytes of one {scale, zero}
@@ -261,7 +266,7 @@ def _decode_bytes_layer(w, mask_row, nq, appended):
         elif prot:
             tot += (T - nq + appended) * 512 + nq * (256 + code_tok + vmeta)
         else:
-            tot += (T - nq + appended) * 512 + nq * (2 * code_tok + kmeta + vmeta)
+            tot += (T - nq + ns + appended) * 512 + (nq - ns) * (2 * code_tok + kmeta + vmeta)
     return B * tot
 
 
@@ -279,6 +284,9 @@ def _workload(args):
     w = wl.WORKLOADS[args.workload]
     if args.meta_bits != w.meta_bits:
         w = dataclasses.replace(w, meta_bits=args.meta_bits, name=w.name + "_meta%d" % args.meta_bits)
+    if args.salient_permille != w.salient_permille:
+        w = dataclasses.replace(w, salient_permille=args.salient_permille,
+                                name=w.name + "_salient%d" % args.salient_permille)
     return w
 
 
