@@ -87,6 +87,7 @@ __device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGrou
     code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], zero), scale, r, levels, fast);
 }
 
+template <int BASE>
 __global__ void __launch_bounds__(kThreads)
 quantize_kernel(const __grid_constant__ QuantizeParams p) {
   const Dims& d = p.d;
@@ -110,7 +111,7 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   const int W = kD * d.bits / 32;  // code words per token
   const bool m16 = d.meta16 != 0;
   // A whole KIVI-style key group of a quantized head: tokens [t0, t0 + 32).
-  const bool kivi_k_tile = (d.base == kKivi) && (hd.cls == kQuantized) && t0 >= qs && t1 <= qe;
+  const bool kivi_k_tile = (BASE == kKivi) && (hd.cls == kQuantized) && t0 >= qs && t1 <= qe;
 
   __shared__ __align__(16) uint16_t ktile[kTile][kD];
 
@@ -129,21 +130,21 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
     srank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w);
   }
 
-  // Issue every load of this warp's tokens first (8 tokens x (K, V) x 8 bytes / lane).
-  uint2 kr[kTile / 4], vr[kTile / 4];
-#pragma unroll
-  for (int i = 0; i < kTile / 4; ++i) {
-    const int t = t0 + warp + 4 * i;
-    if (t < t1) {
-      kr[i] = ldg8(K + (size_t)t * kD + lane * 4);
-      vr[i] = ldg8(V + (size_t)t * kD + lane * 4);
-    }
+  // The warp's tokens t0 + warp + 4i, one at a time, the next token's K and V
+  // loaded while this one is processed.  The loop stays rolled: the token
+  // body is long, and eight unrolled copies of it thrash the instruction cache.
+  uint2 kn = make_uint2(0u, 0u), vn = make_uint2(0u, 0u);
+  if (t0 + warp < t1) {
+    kn = ldg8(K + (size_t)(t0 + warp) * kD + lane * 4);
+    vn = ldg8(V + (size_t)(t0 + warp) * kD + lane * 4);
   }
-
-#pragma unroll
-  for (int i = 0; i < kTile / 4; ++i) {
-    const int t = t0 + warp + 4 * i;
-    if (t >= t1) break;
+#pragma unroll 1
+  for (int t = t0 + warp; t < t1; t += 4) {
+    const uint2 kri = kn, vri = vn;
+    if (t + 4 < t1) {
+      kn = ldg8(K + (size_t)(t + 4) * kD + lane * 4);
+      vn = ldg8(V + (size_t)(t + 4) * kD + lane * 4);
+    }
     const bool coded = (t >= qs) && (t < qe);
     const int ti = t - qs;
     int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token
@@ -158,12 +159,12 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
 
     // ---- key ----
     if (coded && hd.cls == kQuantized && !sal) {
-      if (d.base == kKivi) {
-        *reinterpret_cast<uint2*>(&ktile[t - t0][lane * 4]) = kr[i];
+      if (BASE == kKivi) {
+        *reinterpret_cast<uint2*>(&ktile[t - t0][lane * 4]) = kri;
       } else {
         float x[4];
-        bf16x4_to_f32(kr[i], x);
-        if (d.base == kAkvq) fwht128_warp(x, lane);  // rotate, then per-token RTN
+        bf16x4_to_f32(kri, x);
+        if (BASE == kAkvq) fwht128_warp(x, lane);  // rotate, then per-token RTN
         uint32_t c[4];
         float sc, z;
         quantize_group4<32>(x, d.bits, m16, c, sc, z);
@@ -172,23 +173,21 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
         if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, sc, z, m16);
       }
     } else if (coded && hd.cls == kKeysOnly) {
-      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) =
-          kr[i];
+      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) = kri;
     } else {
       const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
-      *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
-          kr[i];
+      *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) = kri;
     }
 
     // ---- value (never rotated) ----
     if (coded && hd.cls != kProtected && !sal) {
       float x[4];
-      bf16x4_to_f32(vr[i], x);
+      bf16x4_to_f32(vri, x);
       uint32_t c[4];
       float sc, z;
       char* meta = Lb + hd.vqm + b * hd.vqm_bs;
       const size_t mi = (size_t)ci * vgroups(d);
-      if (d.base == kKivi) {
+      if (BASE == kKivi) {
         quantize_group4<8>(x, d.bits, m16, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
         if ((lane & 7) == 0) store_meta(meta, mi + (lane >> 3), sc, z, m16);
       } else {
@@ -199,8 +198,7 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
       store_token_codes(crow, c, d.bits, lane);
     } else {
       const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
-      *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) =
-          vr[i];
+      *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) = vri;
     }
   }
 
@@ -642,7 +640,8 @@ cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
     return cudaGetLastError();
   }
   dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
-  quantize_kernel<<<grid, kThreads, 0, s>>>(p);
+  if (p.d.base == kKivi) quantize_kernel<kKivi><<<grid, kThreads, 0, s>>>(p);
+  else quantize_kernel<kAkvq><<<grid, kThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 
