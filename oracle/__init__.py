@@ -49,6 +49,10 @@ def lib():
         L.hgo_pack.restype = None
         L.hgo_unpack.argtypes = [P, i, i]
         L.hgo_unpack.restype = ctypes.c_uint8
+        L.hgo_unpack_group.argtypes = [P, i, i, i]
+        L.hgo_unpack_group.restype = ctypes.c_uint8
+        L.hgo_plane_pos.argtypes = [i]
+        L.hgo_plane_pos.restype = i
         L.hgo_fwht128.argtypes = [P]
         L.hgo_fwht128.restype = None
         L.hgo_fwht128_f64.argtypes = [P]
@@ -125,16 +129,21 @@ def dequant(code, scale, zero):
 
 
 def pack(codes, bits):
+    """Canonical packing (R16 for 3 bits: a 2-bit low part, then a bit-2 plane)."""
     codes = _c(codes, np.uint8)
-    per = 32 // bits
-    words = np.zeros((codes.size + per - 1) // per, np.uint32)
+    if bits == 3:
+        assert codes.size % 32 == 0
+        words = np.zeros(codes.size * 3 // 32, np.uint32)
+    else:
+        per = 32 // bits
+        words = np.zeros((codes.size + per - 1) // per, np.uint32)
     lib().hgo_pack(_ptr(codes), codes.size, bits, _ptr(words))
     return words
 
 
 def unpack(words, n, bits):
     words = _c(words, np.uint32)
-    return np.array([lib().hgo_unpack(_ptr(words), e, bits) for e in range(n)], np.uint8)
+    return np.array([lib().hgo_unpack_group(_ptr(words), n, e, bits) for e in range(n)], np.uint8)
 
 
 def fwht128(x):

@@ -50,6 +50,13 @@
  *      the same values.  The remaining image tokens are quantized in order and
  *      stored compacted.  Built for the AKVQ-style base without K-only
  *      protection.
+ *   R16 3-bit codes (the paper's 3-bit setting, Sec. 4 / Tab. 1): a group of
+ *      n codes (n a multiple of 32) is stored as n/16 words holding bits 0-1
+ *      of every code in the 2-bit packing, then n/32 words holding bit 2 of
+ *      every code, one bit per code: element e at word e / 32, bit position
+ *      (e mod 32) with its index bits 3 and 4 exchanged.  3 bits per code,
+ *      and the bit-2 plane of two codes that share a 2-bit word at a 16-bit
+ *      distance sits at a 16-bit distance too.
  */
 #include <math.h>
 #include <stdint.h>
@@ -173,12 +180,30 @@ float hgo_dequant(uint8_t code, float scale, float zero)
     return prod + zero;
 }
 
+/* R16: bit position of element e's bit 2 inside its 32-element plane word. */
+int hgo_plane_pos(int e)
+{
+    const int r = e % 32;
+    return (r & 7) | (((r >> 4) & 1) << 3) | (((r >> 3) & 1) << 4);
+}
+
 /*
  * Canonical bit packing: element e of a group goes to word e / (32/b), bit
- * offset b * (e mod 32/b), least significant bits first.
+ * offset b * (e mod 32/b), least significant bits first (b = 2, 4).  For
+ * b = 3 (R16) the low two bits of every code are packed as for b = 2 into the
+ * first n/16 words and bit 2 into n/32 plane words after them.
  */
 void hgo_pack(const uint8_t *codes, int n, int bits, uint32_t *words)
 {
+    if (bits == 3) {
+        const int nlo = n / 16, nhi = n / 32;
+        for (int w = 0; w < nlo + nhi; ++w) words[w] = 0u;
+        for (int e = 0; e < n; ++e) {
+            words[e / 16] |= ((uint32_t)(codes[e] & 3u)) << (2 * (e % 16));
+            words[nlo + e / 32] |= ((uint32_t)(codes[e] >> 2) & 1u) << hgo_plane_pos(e);
+        }
+        return;
+    }
     const int per_word = 32 / bits;
     const int nwords = (n + per_word - 1) / per_word;
     for (int w = 0; w < nwords; ++w) words[w] = 0u;
@@ -186,10 +211,21 @@ void hgo_pack(const uint8_t *codes, int n, int bits, uint32_t *words)
         words[e / per_word] |= ((uint32_t)codes[e]) << (bits * (e % per_word));
 }
 
-uint8_t hgo_unpack(const uint32_t *words, int e, int bits)
+/* Element e of a packed group of n codes. */
+uint8_t hgo_unpack_group(const uint32_t *words, int n, int e, int bits)
 {
+    if (bits == 3) {
+        const uint32_t lo = (words[e / 16] >> (2 * (e % 16))) & 3u;
+        const uint32_t hi = (words[n / 16 + e / 32] >> hgo_plane_pos(e)) & 1u;
+        return (uint8_t)(lo | (hi << 2));
+    }
     const int per_word = 32 / bits;
     return (uint8_t)((words[e / per_word] >> (bits * (e % per_word))) & ((1u << bits) - 1u));
+}
+
+uint8_t hgo_unpack(const uint32_t *words, int e, int bits)
+{
+    return hgo_unpack_group(words, 0, e, bits == 3 ? 2 : bits);
 }
 
 /* ------------------------------------------------------------------------ */

@@ -78,22 +78,24 @@ def test_text_and_protected_entries_are_exact(oracle, base, keys_only):
             assert o["kq"][:, h, s:s + nq].all() and o["vq"][:, h, s:s + nq].all()
 
 
-def test_minmax_is_per_token_group(oracle):
-    k, v, o = _layer(oracle, 0, 2, [0, 0, 0, 0], 0)
+@pytest.mark.parametrize("bits", [2, 3])
+def test_minmax_is_per_token_group(oracle, bits):
+    k, v, o = _layer(oracle, 0, bits, [0, 0, 0, 0], 0)
     s, nq = 10, o["nq"]
+    W = 4 * bits
     for b in range(k.shape[0]):
         for h in range(k.shape[1]):
-            kw = o["k_words"][b, h].reshape(nq, 8)
+            kw = o["k_words"][b, h].reshape(nq, W)
             km = o["k_meta"][b, h].reshape(nq, 2)
-            vw = o["v_words"][b, h].reshape(nq, 8)
+            vw = o["v_words"][b, h].reshape(nq, W)
             for i in (0, 1, nq // 2, nq - 1):
-                c, sc, z = oracle.quantize_group(_f32(k[b, h, s + i]), 2)
-                assert np.array_equal(kw[i], oracle.pack(c, 2)) and km[i, 0] == sc and km[i, 1] == z
-                c, sc, z = oracle.quantize_group(_f32(v[b, h, s + i]), 2)
-                assert np.array_equal(vw[i], oracle.pack(c, 2))
+                c, sc, z = oracle.quantize_group(_f32(k[b, h, s + i]), bits)
+                assert np.array_equal(kw[i], oracle.pack(c, bits)) and km[i, 0] == sc and km[i, 1] == z
+                c, sc, z = oracle.quantize_group(_f32(v[b, h, s + i]), bits)
+                assert np.array_equal(vw[i], oracle.pack(c, bits))
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_kivi_key_groups_are_channel_slices(oracle, bits):
     k, v, o = _layer(oracle, 1, bits, [0, 1, 0, 0], 1, T=130, s=5, n=100, R=20)
     s, nq = 5, o["nq"]
@@ -124,7 +126,7 @@ def test_kivi_key_groups_are_channel_slices(oracle, bits):
     assert o["vq"][:, 1, s:s + nq].all() and not o["vq"][:, 1, s + nq:].any()
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_akvq_rotates_keys_only(oracle, bits):
     k, v, o = _layer(oracle, 2, bits, [0, 0, 1, 0], 0)
     s, nq = 10, o["nq"]

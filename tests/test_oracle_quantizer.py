@@ -53,7 +53,7 @@ def _groups(rng, n, count):
     return out
 
 
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 @pytest.mark.parametrize("n", [4, 32, 128])
 def test_invariants_and_nearest_level(oracle, bits, n):
     """codes in [0, L]; min -> 0, max -> L; each code is a nearest level in exact arithmetic."""
@@ -130,3 +130,40 @@ def test_pack_roundtrip(oracle, bits):
     bitsarr = np.unpackbits(w.view(np.uint8), bitorder="little").reshape(-1, bits)
     vals = (bitsarr * (1 << np.arange(bits))).sum(1)
     assert (vals == c).all()
+
+
+def test_pack3_hand_examples(oracle):
+    """R16: bits 0-1 in the 2-bit packing, then a bit-2 plane whose element e
+    sits at e mod 32 with index bits 3 and 4 exchanged."""
+    c = np.zeros(32, np.uint8)
+    assert list(oracle.pack(c, 3)) == [0, 0, 0]
+    c[:] = 4
+    assert list(oracle.pack(c, 3)) == [0, 0, 0xFFFFFFFF]
+    c[:] = 0
+    c[8] = 7    # low bits 3 at word 0 bits 16-17; plane position 16
+    c[16] = 4   # low bits 0; plane position 8
+    c[23] = 5   # low bits 1 at word 1 bits 14-15; plane position 15
+    c[31] = 6   # low bits 2 at word 1 bits 30-31; plane position 31
+    assert list(oracle.pack(c, 3)) == [0x00030000, 0x80004000, 0x80018100]
+    assert [oracle.lib().hgo_plane_pos(e) for e in (0, 7, 8, 15, 16, 23, 24, 31, 40)] == \
+        [0, 7, 16, 23, 8, 15, 24, 31, 16]
+
+
+def test_pack3_roundtrip_and_pairing(oracle):
+    rng = np.random.default_rng(33)
+    for n in (32, 128):
+        c = rng.integers(0, 8, n).astype(np.uint8)
+        w = oracle.pack(c, 3)
+        assert w.size == n * 3 // 32
+        assert (oracle.unpack(w, n, 3) == c).all()
+        # low part: numpy's bit view of the first n/16 words as 2-bit fields
+        lo = np.unpackbits(w[:n // 16].view(np.uint8), bitorder="little").reshape(-1, 2)
+        assert ((lo * [1, 2]).sum(1) == (c & 3)).all()
+        # plane: each code's bit 2 exactly once
+        hi = np.unpackbits(w[n // 16:].view(np.uint8), bitorder="little")
+        assert hi.sum() == int((c >> 2).sum())
+    # codes e and e + 8 of one 16-code word: low bits 16 apart, and so are their plane bits
+    for e in range(128):
+        if e % 16 < 8:
+            pe, pf = oracle.lib().hgo_plane_pos(e), oracle.lib().hgo_plane_pos(e + 8)
+            assert pf - pe == 16 and (e // 32) == ((e + 8) // 32)
