@@ -84,7 +84,10 @@ typedef struct hg_shape {
     int32_t max_new_tokens;
 } hg_shape;
 
-/* Quantizer configuration.  bits in {2, 4}.  keys_only selects K-only protection
+/* Quantizer configuration.  bits in {2, 3, 4} (3 bits: each group stores bits
+ * 0-1 of its codes as in the 2-bit packing, then bit 2 as a plane of one bit
+ * per code, element e at plane word e / 32, bit e mod 32 with index bits 3
+ * and 4 exchanged).  keys_only selects K-only protection
  * (Sec. 3: protected heads keep image keys BF16, their image values follow the
  * base).  The KIVI-style group sizes must be 32; kivi_residual >= 0 is the number
  * of trailing prefill tokens kept BF16.  Unused fields are ignored for other bases.
@@ -132,7 +135,7 @@ typedef enum hg_head_class {
  *             order, trailing text, appended tokens.
  *   kq / kqm  key codes / metadata (quantized class only).  Per-token bases:
  *             codes uint32 [batch][nq][4*bits] (128 codes, channel order, packed
- *             LSB-first, 32/bits per word), metadata float2 {scale, zero}
+ *             LSB-first, 32/bits per word; 3 bits: 8 words + 4 plane words), metadata float2 {scale, zero}
  *             [batch][nq].  KIVI-style: codes [batch][nq/32][128][bits] (one
  *             32-token group of one channel, token order), metadata
  *             [batch][nq/32][128].

@@ -52,7 +52,7 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   if (sh->num_q_heads / sh->num_kv_heads > kMaxG) return HG_ERR_UNSUPPORTED;
   if (c->base != HG_BASE_MINMAX_TOKEN && c->base != HG_BASE_KIVI && c->base != HG_BASE_AKVQ_HADAMARD)
     return HG_ERR_INVALID_ARG;
-  if (c->bits != 2 && c->bits != 4) return HG_ERR_UNSUPPORTED;
+  if (c->bits != 2 && c->bits != 3 && c->bits != 4) return HG_ERR_UNSUPPORTED;
   if (c->keys_only != 0 && c->keys_only != 1) return HG_ERR_INVALID_ARG;
   if (c->meta_bits != 0 && c->meta_bits != 32 && c->meta_bits != 64) return HG_ERR_INVALID_ARG;
   if (c->salient_permille < 0 || c->salient_permille > 1000) return HG_ERR_INVALID_ARG;
@@ -176,7 +176,9 @@ SegBytes seg_bytes(const Dims& d) {
   const double pair = (double)meta_pair_bytes(d);
   const double kmeta = d.base == kKivi ? 4.0 * pair : pair;
   const double vmeta = pair * vgroups(d);
-  const double instr_u = d.base == kKivi ? (d.bits == 2 ? 66.0 : 78.0) : (d.bits == 2 ? 30.0 : 40.0);
+  // compute term per coded token (3-bit: the 2-bit expansion plus its bit-2 plane)
+  const double instr_u = d.base == kKivi ? (d.bits == 2 ? 66.0 : (d.bits == 3 ? 76.0 : 78.0))
+                                         : (d.bits == 2 ? 30.0 : (d.bits == 3 ? 38.0 : 40.0));
   b.bf16 = 512.0 + 8.0 * 5.0;
   b.coded_u = 2.0 * codes + kmeta + vmeta + 8.0 * instr_u;
   b.coded_k = 256.0 + codes + vmeta + 8.0 * 16.0;

@@ -99,25 +99,29 @@ struct Seg {
   const char* v_new;
 };
 
+// Mask of a code pair at bits [0, b) and [16, 16 + b).
+template <int BITS>
+__host__ __device__ constexpr uint32_t pair_mask() { return ((1u << BITS) - 1u) * 0x00010001u; }
+
 template <int BITS>
 __device__ __forceinline__ uint32_t pair2(uint32_t x) {  // codes at bits [0,b) and [16,16+b)
-  return codes_bf16x2(x & (BITS == 2 ? 0x00030003u : 0x000F000Fu));
+  return codes_bf16x2(x & pair_mask<BITS>());
 }
 
 // The same pair as the BF16 values (128 + code): exact, without the subtraction.
 template <int BITS>
 __device__ __forceinline__ uint32_t pair2_off(uint32_t x) {
-  return (x & (BITS == 2 ? 0x00030003u : 0x000F000Fu)) | 0x43004300u;
+  return (x & pair_mask<BITS>()) | 0x43004300u;
 }
 
 // FP16 forms for value codes: exact codes, and 1024 + code.
 template <int BITS>
 __device__ __forceinline__ uint32_t pair2_h(uint32_t x) {
-  return codes_f16x2(x & (BITS == 2 ? 0x00030003u : 0x000F000Fu));
+  return codes_f16x2(x & pair_mask<BITS>());
 }
 template <int BITS>
 __device__ __forceinline__ uint32_t pair2_off_h(uint32_t x) {
-  return (x & (BITS == 2 ? 0x00030003u : 0x000F000Fu)) | 0x64006400u;
+  return (x & pair_mask<BITS>()) | 0x64006400u;
 }
 
 __device__ __forceinline__ float fast_exp2(float x) {
@@ -154,6 +158,23 @@ __device__ __forceinline__ uint32_t pair2_scaled_h(uint32_t w, uint32_t w6, uint
 
 // 1 / x for a power of two x in [2^-126, 2^126], exactly (exponent arithmetic).
 __device__ __forceinline__ float pow2_inv(float x) { return __uint_as_float(0x7F000000u - __float_as_uint(x)); }
+
+// 3-bit codes keep bits 0-1 in the 2-bit packing and bit 2 in a plane word
+// per 32 codes (element e at bit e mod 32 with index bits 3 and 4 exchanged),
+// so the bit-2 pair of two codes 8 apart in one 2-bit word sits 16 bits apart
+// too.  plane_pair moves such a pair from bits (i, i + 16) of a plane-derived
+// register to bits (p + 2, p + 18), on top of the 2-bit pair extracted at
+// bits (p, p + 16); i and p are compile-time after unrolling.
+__device__ __forceinline__ uint32_t plane_pair(uint32_t pl, int i, int p) {
+  const int d = i - (p + 2);
+  const uint32_t x = d >= 0 ? (pl >> d) : (pl << (-d));
+  return x & (0x00010001u << (p + 2));
+}
+// prmt selector: byte bs of a into bytes 0-1 of the result, byte bs of b into
+// bytes 2-3 (the plane bytes of two tokens or two channels, side by side).
+__device__ __forceinline__ uint32_t plane_sel(int bs) {
+  return (uint32_t)(bs | (bs << 4) | ((4 + bs) << 8) | ((4 + bs) << 12));
+}
 
 // Smallest power of two >= m (m > 0, finite).
 __device__ __forceinline__ float pow2_ceil(float m) {
@@ -291,7 +312,7 @@ __device__ __forceinline__ void qfrag_natural(uint32_t (&qb)[NT][8][2], const fl
 // pairs (i, i+4) and (i+1, i+5), i = 2 (j & 1), of word 4tq + j/2.
 template <int BITS>
 __device__ __forceinline__ void token_channels(int tq, int j, int (&c)[4]) {
-  if (BITS == 2) {
+  if (BITS != 4) {  // 2 bits, and the 2-bit part of 3-bit codes
     c[0] = 32 * tq + j;
     c[1] = 32 * tq + j + 8;
     c[2] = 32 * tq + 16 + j;
@@ -321,7 +342,7 @@ __device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (
     for (int j = 0; j < 8; ++j) {
       int c[4];
       token_channels<BITS>(tq, j, c);
-      const float f = (BITS == 2) ? 1.0f / (float)(1 << pos3(j)) : 1.0f;  // exact
+      const float f = (BITS != 4) ? 1.0f / (float)(1 << pos3(j)) : 1.0f;  // exact
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh) {
         const float x0 = qr[c[2 * hh]] * f, x1 = qr[c[2 * hh + 1]] * f;
@@ -513,10 +534,21 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc2[nt][i] = 0.f;
-      if (BITS == 2) {
-        const uint2 ka = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g) * 8 + 2 * tq);
-        const uint2 kb = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g + 8) * 8 + 2 * tq);
+      if (BITS != 4) {
+        constexpr int RW = 4 * BITS;  // words per token row
+        const uint2 ka = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g) * RW + 2 * tq);
+        const uint2 kb = *reinterpret_cast<const uint2*>(kc32 + (tok0 + g + 8) * RW + 2 * tq);
         const uint32_t w[4] = {ka.x, kb.x, ka.y, kb.y};
+        // 3 bits: plane word tq holds bit 2 of words 2tq (pairs at j, j + 16)
+        // and 2tq + 1 (at j + 8, j + 24)
+        uint32_t pl[4] = {0u, 0u, 0u, 0u};
+        if (BITS == 3) {
+          const uint32_t pa = kc32[(tok0 + g) * RW + 8 + tq], pb = kc32[(tok0 + g + 8) * RW + 8 + tq];
+          pl[0] = pa;
+          pl[1] = pb;
+          pl[2] = pa >> 8;
+          pl[3] = pb >> 8;
+        }
         uint32_t w6[4], w12[4];
 #pragma unroll
         for (int k = 0; k < 4; ++k) {
@@ -527,7 +559,10 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         for (int j = 0; j < 8; ++j) {
           uint32_t a[4];
 #pragma unroll
-          for (int k = 0; k < 4; ++k) a[k] = pair2_scaled(w[k], w6[k], w12[k], j);
+          for (int k = 0; k < 4; ++k) {
+            a[k] = pair2_scaled(w[k], w6[k], w12[k], j);
+            if (BITS == 3) a[k] |= plane_pair(pl[k], j, pos3(j));
+          }
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
             float (&dst)[4] = (j & 1) ? acc2[nt] : acc[0][nt];
@@ -601,6 +636,11 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
             w[cc][0] = t2.x;
             w[cc][1] = t2.y;
             w[cc][2] = w[cc][3] = 0u;
+          } else if (BITS == 3) {  // two 2-bit words, then the bit-2 plane of the 32 tokens
+            w[cc][0] = gc[(c0 + cc) * 3];
+            w[cc][1] = gc[(c0 + cc) * 3 + 1];
+            w[cc][2] = gc[(c0 + cc) * 3 + 2];
+            w[cc][3] = 0u;
           } else {
             const uint4 t4 = *reinterpret_cast<const uint4*>(gc + (c0 + cc) * 4);
             w[cc][0] = t4.x;
@@ -618,6 +658,20 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
             a[1] = pair2<2>(prmt(w[0][s], w[1][s], 0x7632) >> (2 * g));
             a[2] = pair2<2>(prmt(w[2][s], w[3][s], 0x5410) >> (2 * g));
             a[3] = pair2<2>(prmt(w[2][s], w[3][s], 0x7632) >> (2 * g));
+          } else if (BITS == 3) {
+            // bit 2 of token 16s + i: plane byte s (i < 8) or 2 + s (i >= 8), bit i % 8
+            const uint32_t lo0 = prmt(w[0][s], w[1][s], 0x5410) >> (2 * g);
+            const uint32_t lo1 = prmt(w[0][s], w[1][s], 0x7632) >> (2 * g);
+            const uint32_t lo2 = prmt(w[2][s], w[3][s], 0x5410) >> (2 * g);
+            const uint32_t lo3 = prmt(w[2][s], w[3][s], 0x7632) >> (2 * g);
+            const uint32_t h0 = prmt(w[0][2], w[1][2], plane_sel(s)) >> g;
+            const uint32_t h1 = prmt(w[0][2], w[1][2], plane_sel(2 + s)) >> g;
+            const uint32_t h2 = prmt(w[2][2], w[3][2], plane_sel(s)) >> g;
+            const uint32_t h3 = prmt(w[2][2], w[3][2], plane_sel(2 + s)) >> g;
+            a[0] = pair2<3>((lo0 & 0x00030003u) | ((h0 & 0x00010001u) << 2));
+            a[1] = pair2<3>((lo1 & 0x00030003u) | ((h1 & 0x00010001u) << 2));
+            a[2] = pair2<3>((lo2 & 0x00030003u) | ((h2 & 0x00010001u) << 2));
+            a[3] = pair2<3>((lo3 & 0x00030003u) | ((h3 & 0x00010001u) << 2));
           } else {
             // words 2s, 2s+1 of a channel: tokens 16s..16s+7 and 16s+8..16s+15
             const int sh = 4 * (g & 1);
@@ -723,12 +777,25 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           for (int nt = 0; nt < NT; ++nt) mma_f16(ws.corr[nt], c1024, b[nt][0], b[nt][1]);
         }
         const int t0 = tok0 + 2 * tq;
-        if (BITS == 2) {
+        if (BITS != 4) {
           // word g of a token row holds channels 16g..16g+15
-          const uint32_t w0 = vc32[t0 * 8 + g], w1 = vc32[(t0 + 1) * 8 + g];
-          const uint32_t w8 = vc32[(t0 + 8) * 8 + g], w9 = vc32[(t0 + 9) * 8 + g];
+          constexpr int RW = 4 * BITS;  // words per token row
+          const uint32_t w0 = vc32[t0 * RW + g], w1 = vc32[(t0 + 1) * RW + g];
+          const uint32_t w8 = vc32[(t0 + 8) * RW + g], w9 = vc32[(t0 + 9) * RW + g];
           const uint32_t x[4] = {prmt(w0, w1, 0x5410), prmt(w0, w1, 0x7632), prmt(w8, w9, 0x5410),
                                  prmt(w8, w9, 0x7632)};
+          // 3 bits: bit 2 of word g's codes 0-7 is byte g % 2 of plane word
+          // 8 + g / 2, codes 8-15 byte 2 + g % 2; two tokens side by side
+          uint32_t hp[4] = {0u, 0u, 0u, 0u};
+          if (BITS == 3) {
+            const int pw = 8 + (g >> 1), bs = g & 1;
+            const uint32_t p0 = vc32[t0 * RW + pw], p1 = vc32[(t0 + 1) * RW + pw];
+            const uint32_t p8 = vc32[(t0 + 8) * RW + pw], p9 = vc32[(t0 + 9) * RW + pw];
+            hp[0] = prmt(p0, p1, plane_sel(bs));
+            hp[1] = prmt(p0, p1, plane_sel(2 + bs));
+            hp[2] = prmt(p8, p9, plane_sel(bs));
+            hp[3] = prmt(p8, p9, plane_sel(2 + bs));
+          }
           uint32_t x6[4], x12[4];
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
@@ -739,7 +806,10 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           for (int mt = 0; mt < 8; ++mt) {
             uint32_t a[4];
 #pragma unroll
-            for (int k = 0; k < 4; ++k) a[k] = pair2_scaled_h(x[k], x6[k], x12[k], mt);
+            for (int k = 0; k < 4; ++k) {
+              a[k] = pair2_scaled_h(x[k], x6[k], x12[k], mt);
+              if (BITS == 3) a[k] |= plane_pair(hp[k], mt, pos3(mt));
+            }
 #pragma unroll
             for (int nt = 0; nt < NT; ++nt) mma_f16(ws.o[nt][mt], a, b[nt][0], b[nt][1]);
           }
@@ -808,6 +878,20 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
             a[1] = pair2_h<2>(prmt(w0, w1, 0x7632) >> (2 * g));
             a[2] = pair2_h<2>(prmt(w8, w9, 0x5410) >> (2 * g));
             a[3] = pair2_h<2>(prmt(w8, w9, 0x7632) >> (2 * g));
+          } else if (BITS == 3) {
+            // channels 16mt + g and 16mt + 8 + g: bit 2 in byte mt % 2 and
+            // 2 + mt % 2 of plane word 8 + mt / 2, bit g
+            const uint32_t w0 = vc32[t0 * W + mt], w1 = vc32[(t0 + 1) * W + mt];
+            const uint32_t w8 = vc32[(t0 + 8) * W + mt], w9 = vc32[(t0 + 9) * W + mt];
+            const int pw = 8 + (mt >> 1), bs = mt & 1;
+            const uint32_t p0 = vc32[t0 * W + pw], p1 = vc32[(t0 + 1) * W + pw];
+            const uint32_t p8 = vc32[(t0 + 8) * W + pw], p9 = vc32[(t0 + 9) * W + pw];
+            const uint32_t h0 = prmt(p0, p1, plane_sel(bs)) >> g, h1 = prmt(p0, p1, plane_sel(2 + bs)) >> g;
+            const uint32_t h2 = prmt(p8, p9, plane_sel(bs)) >> g, h3 = prmt(p8, p9, plane_sel(2 + bs)) >> g;
+            a[0] = pair2_h<3>(((prmt(w0, w1, 0x5410) >> (2 * g)) & 0x00030003u) | ((h0 & 0x00010001u) << 2));
+            a[1] = pair2_h<3>(((prmt(w0, w1, 0x7632) >> (2 * g)) & 0x00030003u) | ((h1 & 0x00010001u) << 2));
+            a[2] = pair2_h<3>(((prmt(w8, w9, 0x5410) >> (2 * g)) & 0x00030003u) | ((h2 & 0x00010001u) << 2));
+            a[3] = pair2_h<3>(((prmt(w8, w9, 0x7632) >> (2 * g)) & 0x00030003u) | ((h3 & 0x00010001u) << 2));
           } else {
             const uint2 u0 = *reinterpret_cast<const uint2*>(vc32 + t0 * W + 2 * mt);
             const uint2 u1 = *reinterpret_cast<const uint2*>(vc32 + (t0 + 1) * W + 2 * mt);
@@ -1046,7 +1130,7 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
           c_lo = 16 * g + mt;
           c_hi = 16 * g + 8 + mt;
           // and the units (vb) of the coded-value accumulators
-          const float f = ((BITS == 2) ? 1.0f / (float)(1 << pos3(mt)) : 1.0f) * ws.vb;
+          const float f = ((BITS != 4) ? 1.0f / (float)(1 << pos3(mt)) : 1.0f) * ws.vb;
           orow[c_lo] = (ws.o[nt][mt][e] - ws.corr[nt][e]) * f + ws.z[nt][e][0];
           orow[c_hi] = (ws.o[nt][mt][2 + e] - ws.corr[nt][2 + e]) * f + ws.z[nt][e][0];
         } else {
@@ -1286,6 +1370,8 @@ template <int MB>
 cudaError_t launch_decode_mb(const DecodeParams& p, int grid_x, cudaStream_t s) {
   if (p.d.bits == 2)
     return p.d.G <= 8 ? launch_base<2, 1, MB>(p, grid_x, s) : launch_base<2, 2, MB>(p, grid_x, s);
+  if (p.d.bits == 3)
+    return p.d.G <= 8 ? launch_base<3, 1, MB>(p, grid_x, s) : launch_base<3, 2, MB>(p, grid_x, s);
   return p.d.G <= 8 ? launch_base<4, 1, MB>(p, grid_x, s) : launch_base<4, 2, MB>(p, grid_x, s);
 }
 

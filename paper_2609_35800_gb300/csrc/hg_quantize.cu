@@ -26,15 +26,32 @@ constexpr int kThreads = 128;
 constexpr int kTile = 32;
 constexpr unsigned kFull = 0xffffffffu;
 
+// 3-bit codes (the 2-bit low part, then the bit-2 plane): bit position, in
+// plane word l / 8, of the bit 2 of channel 4l (channels 4l..4l+3 follow it).
+// Channel e sits at e mod 32 with index bits 3 and 4 exchanged.
+__device__ __forceinline__ int plane_base(int lane) {
+  return 4 * (lane & 1) + 8 * ((lane >> 2) & 1) + 16 * ((lane >> 1) & 1);
+}
+
 // Pack one token's 128 codes (lane l holds channels 4l..4l+3) in channel order,
-// LSB-first, and store its 4*bits words.
+// LSB-first, and store its 4*bits words (3 bits: 8 words of bits 0-1, then 4
+// plane words of bit 2).
 __device__ __forceinline__ void store_token_codes(uint32_t* row, const uint32_t (&c)[4], int bits,
                                                   int lane) {
-  if (bits == 2) {
-    uint32_t x = (c[0] | (c[1] << 2) | (c[2] << 4) | (c[3] << 6)) << (8 * (lane & 3));
+  if (bits == 2 || bits == 3) {
+    uint32_t x = ((c[0] & 3u) | ((c[1] & 3u) << 2) | ((c[2] & 3u) << 4) | ((c[3] & 3u) << 6)) << (8 * (lane & 3));
     x |= __shfl_xor_sync(kFull, x, 1);
     x |= __shfl_xor_sync(kFull, x, 2);
     if ((lane & 3) == 0) row[lane >> 2] = x;
+    if (bits == 3) {
+      uint32_t hp = (((c[0] >> 2) & 1u) | (((c[1] >> 2) & 1u) << 1) | (((c[2] >> 2) & 1u) << 2) |
+                     (((c[3] >> 2) & 1u) << 3))
+                    << plane_base(lane);
+      hp |= __shfl_xor_sync(kFull, hp, 1);
+      hp |= __shfl_xor_sync(kFull, hp, 2);
+      hp |= __shfl_xor_sync(kFull, hp, 4);
+      if ((lane & 7) == 0) row[8 + (lane >> 3)] = hp;
+    }
   } else {
     uint32_t x = (c[0] | (c[1] << 4) | (c[2] << 8) | (c[3] << 12)) << (16 * (lane & 1));
     x |= __shfl_xor_sync(kFull, x, 1);
@@ -45,10 +62,15 @@ __device__ __forceinline__ void store_token_codes(uint32_t* row, const uint32_t 
 // Codes of channels 4l..4l+3 of one token from its packed row.
 __device__ __forceinline__ void load_token_codes(const uint32_t* row, int bits, int lane,
                                                  uint32_t (&c)[4]) {
-  if (bits == 2) {
+  if (bits == 2 || bits == 3) {
     const uint32_t byte = (__ldg(row + (lane >> 2)) >> (8 * (lane & 3))) & 0xffu;
 #pragma unroll
     for (int i = 0; i < 4; ++i) c[i] = (byte >> (2 * i)) & 3u;
+    if (bits == 3) {
+      const uint32_t hp = __ldg(row + 8 + (lane >> 3)) >> plane_base(lane);
+#pragma unroll
+      for (int i = 0; i < 4; ++i) c[i] |= ((hp >> i) & 1u) << 2;
+    }
   } else {
     const uint32_t half = (__ldg(row + (lane >> 1)) >> (16 * (lane & 1))) & 0xffffu;
 #pragma unroll
@@ -214,11 +236,26 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   quantize_group_serial(x, d.bits, m16, code, sc, z);
   const int grp = (t0 - qs) / kKiviGroup;
   uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * d.bits;
-  const int per = 32 / d.bits;
-  for (int w = 0; w < d.bits; ++w) {
-    uint32_t word = 0;
-    for (int e = 0; e < per; ++e) word |= code[w * per + e] << (d.bits * e);
-    dst[w] = word;
+  if (d.bits == 3) {  // two words of bits 0-1 (16 tokens each), then the bit-2 plane
+    uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      lo0 |= (code[e] & 3u) << (2 * e);
+      lo1 |= (code[16 + e] & 3u) << (2 * e);
+    }
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
+    dst[0] = lo0;
+    dst[1] = lo1;
+    dst[2] = hp;
+  } else {
+    const int per = 32 / d.bits;
+    for (int w = 0; w < d.bits; ++w) {
+      uint32_t word = 0;
+      for (int e = 0; e < per; ++e) word |= code[w * per + e] << (d.bits * e);
+      dst[w] = word;
+    }
   }
   store_meta(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + c, sc, z, m16);
 }
@@ -248,6 +285,37 @@ constexpr int kQPitch = 272;
 // Round-half-even of fl(d / scale), clamped to the levels (IEEE division).
 __device__ __noinline__ uint32_t exact_code(float d, float scale, float levels) {
   return (uint32_t)fminf(fmaxf(rintf(__fdiv_rn(d, scale)), 0.0f), levels);
+}
+
+// Eight codes of channels 8k..8k+7 into the packed row: 4 bits -> word k;
+// 2 bits -> half of word k/2; 3 bits -> the same 2-bit half plus one byte of
+// plane word 8 + k/4 (byte ((k >> 1) & 1) | ((k & 1) << 1): channel index bits
+// 3 and 4 exchanged), each word stored once complete.
+template <int BITS>
+__device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32_t* codes, uint32_t& prev,
+                                           uint32_t& plane) {
+  if (BITS == 4) {
+    uint32_t w = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) w |= c[i] << (4 * i);
+    codes[k] = w;
+    return;
+  }
+  uint32_t lo = 0u;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) lo |= (c[i] & 3u) << (2 * i);
+  if (k & 1) codes[k >> 1] = prev | (lo << 16);
+  else prev = lo;
+  if (BITS == 3) {
+    uint32_t hb = 0u;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) hb |= ((c[i] >> 2) & 1u) << i;
+    plane |= hb << (8 * (((k >> 1) & 1) | ((k & 1) << 1)));
+    if ((k & 3) == 3) {
+      codes[8 + (k >> 2)] = plane;
+      plane = 0u;
+    }
+  }
 }
 
 template <int BITS, bool M16>
@@ -296,12 +364,12 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
     // T within 2^-16 of fl(d / scale) + 192 for quotients that can decide a
     // code, so the near-tie test is the same as below.
     const float r = __frcp_rn(scale);
-    uint32_t prev = 0u;
+    uint32_t prev = 0u, plane = 0u;
 #pragma unroll 2
     for (int k = 0; k < 16; ++k) {
       const uint4 v = r4[k];
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint32_t chunk = 0u;
+      uint32_t c8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const uint32_t hw = w[i >> 1];
@@ -309,16 +377,9 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
         const float q = fminf(fmaxf(__fmul_rn(d, r), -1.0f), levels + 1.0f);
         const uint32_t a = __float_as_uint(__fadd_rn(q, 192.0f)) + 0x8001u;
         const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
-        const uint32_t code = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
-        chunk |= code << (BITS * i);
+        c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
       }
-      if (BITS == 4) {
-        codes[k] = chunk;
-      } else if (k & 1) {
-        codes[k >> 1] = prev | (chunk << 16);
-      } else {
-        prev = chunk;
-      }
+      emit_chunk<BITS>(k, c8, codes, prev, plane);
     }
     return;
   }
@@ -327,12 +388,12 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
     // chunks of 8 channels (one uint4 of the row): 16 code bits (2-bit) or 32
     // (4-bit); the loop stays rolled (by two) so the code is small and stays
     // in the instruction cache
-    uint32_t prev = 0u;
+    uint32_t prev = 0u, plane = 0u;
 #pragma unroll 2
     for (int k = 0; k < 16; ++k) {
       const uint4 v = r4[k];
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint32_t chunk = 0u;
+      uint32_t c8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
         const uint32_t hw = w[i >> 1];
@@ -340,31 +401,25 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
         const uint32_t a = __float_as_uint(__fmaf_rn(d, r, 192.0f)) + 0x8001u;
         // BF16 data puts many quotients exactly on half-integers: those (and
         // anything within a unit of one) take the exact rule
-        const uint32_t code = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : ((a >> 16) & L);
-        chunk |= code << (BITS * i);
+        c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : ((a >> 16) & L);
       }
-      if (BITS == 4) {
-        codes[k] = chunk;
-      } else if (k & 1) {
-        codes[k >> 1] = prev | (chunk << 16);
-      } else {
-        prev = chunk;
-      }
+      emit_chunk<BITS>(k, c8, codes, prev, plane);
     }
     return;
   }
   // tiny scale: the exact rule throughout
+  uint32_t prev = 0u, plane = 0u;
 #pragma unroll 1
-  for (int wi = 0; wi < W; ++wi) {
-    uint32_t acc = 0u;
-#pragma unroll 1
-    for (int j = 0; j < 32 / BITS; ++j) {
-      const int e = wi * (32 / BITS) + j;
+  for (int k = 0; k < 16; ++k) {
+    uint32_t c8[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int e = 8 * k + i;
       const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
       const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
-      acc |= exact_code(__fsub_rn(x, mn), scale, levels) << (BITS * j);
+      c8[i] = exact_code(__fsub_rn(x, mn), scale, levels);
     }
-    codes[wi] = acc;
+    emit_chunk<BITS>(k, c8, codes, prev, plane);
   }
 }
 
@@ -560,8 +615,15 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
           const size_t row = (size_t)grp * kD + lane * 4 + i;
-          const uint32_t w = __ldg(codes + row * d.bits + e / per);
-          const uint32_t code = (w >> (d.bits * (e % per))) & ((1u << d.bits) - 1u);
+          uint32_t code;
+          if (d.bits == 3) {
+            const uint32_t lo = (__ldg(codes + row * 3 + e / 16) >> (2 * (e % 16))) & 3u;
+            const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
+            code = lo | (((__ldg(codes + row * 3 + 2) >> pp) & 1u) << 2);
+          } else {
+            const uint32_t w = __ldg(codes + row * d.bits + e / per);
+            code = (w >> (d.bits * (e % per))) & ((1u << d.bits) - 1u);
+          }
           const float2 m = load_meta(meta, row, m16);
           xk[i] = dequant1(code, m.x, m.y);
         }
@@ -633,6 +695,9 @@ cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
     if (p.d.bits == 2) {
       if (m16) quantize_minmax_kernel<2, true><<<grid, kThreads, 0, s>>>(p);
       else quantize_minmax_kernel<2, false><<<grid, kThreads, 0, s>>>(p);
+    } else if (p.d.bits == 3) {
+      if (m16) quantize_minmax_kernel<3, true><<<grid, kThreads, 0, s>>>(p);
+      else quantize_minmax_kernel<3, false><<<grid, kThreads, 0, s>>>(p);
     } else {
       if (m16) quantize_minmax_kernel<4, true><<<grid, kThreads, 0, s>>>(p);
       else quantize_minmax_kernel<4, false><<<grid, kThreads, 0, s>>>(p);

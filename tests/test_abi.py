@@ -60,7 +60,8 @@ def _status(f, *a):
     (dict(num_kv_heads=1, num_q_heads=17), {}, 3),
     (dict(seq_len=0, img_len=0, img_start=0), {}, 1),
     (dict(batch=0), {}, 1),
-    ({}, dict(bits=3), 3),
+    ({}, dict(bits=5), 3),
+    ({}, dict(bits=1), 3),
     ({}, dict(base=7), 1),
     ({}, dict(base=1, kivi_group_tokens=16), 3),
     ({}, dict(base=1, kivi_residual=-1), 1),
@@ -107,6 +108,8 @@ ODD = {"odd_nq_minmax": wl.custom("odd", 3, 3, 16, 4, 64, 333, 17, wl.BASE_MINMA
                                   meta_bits=32),
        "meta16_kivi_konly": wl.custom("m16b", 2, 3, 8, 8, 5, 131, 40, wl.BASE_KIVI, 4, 1,
                                       meta_bits=32),
+       "three_bit_minmax": wl.custom("b3", 2, 3, 16, 4, 9, 333, 17, wl.BASE_MINMAX, 3, 0),
+       "three_bit_kivi_konly": wl.custom("b3k", 2, 2, 8, 8, 5, 131, 40, wl.BASE_KIVI, 3, 1),
        "salient_akvq": wl.custom("sal", 3, 2, 16, 4, 9, 333, 17, wl.BASE_AKVQ, 4, 0,
                                  salient_permille=20),
        "salient_all": wl.custom("sal2", 2, 3, 8, 8, 5, 70, 9, wl.BASE_AKVQ, 2, 0,

@@ -166,6 +166,39 @@ def test_meta16_fused_decode_step(case):
     _run_and_check(_workload(case, meta_bits=32), fused=True)
 
 
+# 3-bit codes (reading R16: a 2-bit low part and a bit-2 plane)
+CASES3 = [
+    ("minmax3_gqa7", 2, 1, 28, 4, 32, 256, 32, M, 3, 0, 2, [(0, 1), (1, 3)], 32),
+    ("minmax3_konly_b2", 2, 2, 8, 4, 7, 200, 9, M, 3, 1, 2, [(0, 2), (1, 0), (1, 1)], 32),
+    ("kivi3_konly_mha", 1, 2, 4, 4, 3, 100, 40, K, 3, 1, 2, [(0, 1)], 32),
+    ("kivi3_unaligned", 2, 1, 4, 4, 13, 130, 45, K, 3, 0, 2, [(1, 2)], 32),
+    ("akvq3_g4_b3", 1, 3, 16, 4, 64, 333, 17, A, 3, 0, 2, [(0, 3)], 32),
+    ("akvq3_konly", 1, 2, 8, 4, 20, 150, 30, A, 3, 1, 2, [(0, 0), (0, 2)], 32),
+    ("minmax3_g16", 1, 1, 32, 2, 16, 200, 16, M, 3, 0, 2, [(0, 1)], 32),
+    ("minmax3_long", 1, 1, 28, 4, 50, 3000, 50, M, 3, 0, 2, [(0, 0)], 32),
+]
+
+
+@pytest.mark.parametrize("case", CASES3, ids=[c[0] for c in CASES3])
+def test_three_bit_parity(case):
+    _run_and_check(_workload(case))
+
+
+@pytest.mark.parametrize("case", [CASES3[0], CASES3[2], CASES3[4]], ids=["minmax", "kivi", "akvq"])
+def test_three_bit_fused_meta16_salient(case):
+    """3-bit codes with the fused decode step, binary16 metadata, and (AKVQ)
+    salient tokens."""
+    _run_and_check(_workload(case, meta_bits=32), fused=True)
+    if case[8] == A:
+        _run_and_check(_workload(case, salient_permille=20), fused=True)
+
+
+@pytest.mark.parametrize("case", [CASES3[1], CASES3[2], CASES3[3], CASES3[5]],
+                         ids=["minmax_konly", "kivi_konly", "kivi", "akvq_konly"])
+def test_three_bit_dequantize_bit_exact(case):
+    _dequantize_bit_exact(_workload(case))
+
+
 # AKVQ-style salient tokens (Sec. 4): (case, permille)
 SALIENT = [
     (("akvq4_sal", 2, 2, 16, 4, 64, 333, 17, A, 4, 0, 3, [(0, 3), (1, 0)], 32), 20),
@@ -273,7 +306,7 @@ def test_capacity_error_leaves_state():
 
 
 @pytest.mark.parametrize("meta_bits", [64, 32])
-@pytest.mark.parametrize("bits", [2, 4])
+@pytest.mark.parametrize("bits", [2, 3, 4])
 def test_minmax_quantize_exact_ties(bits, meta_bits):
     """Vectors built so that (x - min) / scale lands exactly on half-integers:
     every such element must round half to even, as the oracle does (the
