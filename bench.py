@@ -45,6 +45,8 @@ def parse_args():
     ap.add_argument("--workload", default="qwen25vl7b")
     ap.add_argument("--meta-bits", type=int, default=64, choices=[64, 32],
                     help="metadata per group: fp32 pair (64) or binary16 pair (32, Sec. 5.4)")
+    ap.add_argument("--bits", type=int, default=0, choices=[0, 2, 3, 4],
+                    help="code width override (0: the workload's own)")
     ap.add_argument("--salient-permille", type=int, default=0,
                     help="AKVQ-style salient tokens kept BF16 per head (Sec. 4; 20 = 2%%)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -284,6 +286,8 @@ def _workload(args):
     w = wl.WORKLOADS[args.workload]
     if args.meta_bits != w.meta_bits:
         w = dataclasses.replace(w, meta_bits=args.meta_bits, name=w.name + "_meta%d" % args.meta_bits)
+    if args.bits and args.bits != w.bits:
+        w = dataclasses.replace(w, bits=args.bits, name=w.name + "_%dbit" % args.bits)
     if args.salient_permille != w.salient_permille:
         w = dataclasses.replace(w, salient_permille=args.salient_permille,
                                 name=w.name + "_salient%d" % args.salient_permille)
