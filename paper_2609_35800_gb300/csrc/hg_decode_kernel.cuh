@@ -970,6 +970,32 @@ __device__ __forceinline__ void combine_out(const float* parts, int n, int sstri
   }
 }
 
+// One combine pass: the weights, then channel `tid` of every query, written
+// as the final BF16 output rows (out: row 0 of this head's queries) or as this
+// split's partial (mine).  Not inlined: the warp combine and the split merge
+// run the same instructions, so the merge -- once per head, at the end of the
+// launch -- executes from cached code.
+template <int JM>
+__device__ __noinline__ void combine_pass(const float* src, int n, int sstride, float* fw, int G, int tid,
+                                          bool final, uint16_t* out, float* mine) {
+  combine_weights(src, n, sstride, G, fw, tid);
+  float acc[JM];
+  combine_out<JM>(src, n, sstride, fw, G, tid, acc);
+#pragma unroll
+  for (int j = 0; j < JM; ++j) {
+    if (j >= G) break;
+    if (final) {
+      out[(size_t)j * kD + tid] = (uint16_t)f32_to_bf16_rn(acc[j] * fw[kFwR * kMaxG + j]);
+    } else {
+      mine[j * kPartialStride + 4 + tid] = acc[j];
+      if (tid == 0) {
+        mine[j * kPartialStride + 0] = fw[kFwM * kMaxG + j];
+        mine[j * kPartialStride + 1] = fw[kFwL * kMaxG + j];
+      }
+    }
+  }
+}
+
 // ---------------------------------------------------------------------------
 // One work item with a given key / value mode: pipeline, then per-warp results
 // into shared memory (m, l, o[q][channel]).
@@ -1267,11 +1293,8 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
 
   // ---- combine the warps, then write the output (a head in one chunk) or this
   // split's partial; the last split of a head to finish then runs the same
-  // combine over all splits' partials (a second pass through this code, whose
-  // instructions are cached by then: the merge runs once per head, and cold
-  // code would cost microseconds) ----
+  // combine over all splits' partials ----
   float* fw = reinterpret_cast<float*>(smem + SmemLayout<NT>::q);  // weights; queries no longer needed
-  const int c = tid;
   const size_t out_row = ((size_t)li * d.B + b) * d.Hq + (size_t)h * G;
   const size_t head_lin = ((size_t)li * d.B + b) * d.H + h;
   float* part = p.partials + (head_lin * p.max_items) * (size_t)G * kPartialStride;
@@ -1282,22 +1305,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   bool final = ni == 1;
 #pragma unroll 1
   for (;;) {
-    combine_weights(src, n, sstride, G, fw, tid);
-    float acc[NT * 8];
-    combine_out<NT * 8>(src, n, sstride, fw, G, c, acc);
-#pragma unroll
-    for (int j = 0; j < NT * 8; ++j) {
-      if (j >= G) break;
-      if (final) {
-        p.out[(out_row + j) * kD + c] = (uint16_t)f32_to_bf16_rn(acc[j] * fw[kFwR * kMaxG + j]);
-      } else {
-        mine[j * kPartialStride + 4 + c] = acc[j];
-        if (c == 0) {
-          mine[j * kPartialStride + 0] = fw[kFwM * kMaxG + j];
-          mine[j * kPartialStride + 1] = fw[kFwL * kMaxG + j];
-        }
-      }
-    }
+    combine_pass<NT * 8>(src, n, sstride, fw, G, tid, final, p.out + out_row * kD, mine);
     if (final) break;
 
     // Publish the partial and take a ticket with one acquire-release atomic:
