@@ -37,6 +37,10 @@ L2_FLUSH_BYTES = 512 << 20
 
 
 def parse_args():
+    return parse_args_from(None)
+
+
+def parse_args_from(argv):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=5)
@@ -51,7 +55,7 @@ def parse_args():
                     help="AKVQ-style salient tokens kept BF16 per head (Sec. 4; 20 = 2%%)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
-    return ap.parse_args()
+    return ap.parse_args(argv)
 
 
 # ---------------------------------------------------------------------------
@@ -152,6 +156,24 @@ class ClockSampler:
 # ---------------------------------------------------------------------------
 # roofline inputs
 # ---------------------------------------------------------------------------
+
+def max_over_ranks(value, dist, device):
+    """The slowest rank's value (the timing rule for N > 1 ranks: max over
+    ranks after a barrier); `dist` is torch.distributed or None for one rank."""
+    if dist is None:
+        return value
+    import torch
+    t = torch.tensor([float(value)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_gbs(world, step_bytes, ms_step):
+    """Whole-job throughput: every rank streams its own replica's step bytes
+    (weak scaling; the path has no cross-rank exchange) in the slowest rank's
+    time."""
+    return world * step_bytes / (ms_step * 1e-3) / 1e9
+
 
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
@@ -422,12 +444,8 @@ def run_gpu(args):
             per[kind].append(ms)
             tot += ms
         step_ms.append(tot)
-    ms_step = sum(step_ms) / len(step_ms)
-    if dist is not None:
-        t = torch.tensor([ms_step], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms_step = float(t.item())
-    value = world * step_bytes / (ms_step * 1e-3) / 1e9
+    ms_step = max_over_ranks(sum(step_ms) / len(step_ms), dist, dev)
+    value = whole_job_gbs(world, step_bytes, ms_step)
 
     quant_ms = statistics.mean(per["quant"])
     dec_ms = statistics.mean(per["decode"])
