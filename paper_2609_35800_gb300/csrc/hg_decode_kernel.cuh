@@ -58,10 +58,18 @@ constexpr int kPartialStride = kD + 4;  // m, l, 2 pad, o[128]: rows of 528 byte
 // Shared memory, from a 1024-byte aligned base (swizzled TMA boxes need it).
 constexpr int kStageOff = 0;                    // pipeline buffer
 // Four CTAs per SM for up to 8 queries per KV head (NT = 1), two above.
+// Staged queries: row r (query r of the KV head), channel c at
+// r * kQRow + (c / 32) * 40 + c % 32.  The padding spreads the 16-byte reads
+// of one warp (8 rows x 4 channel blocks, the KIVI-style key path) over all
+// banks: row strides are an odd number of 16-byte units and block strides
+// two units more than a multiple of eight.
+constexpr int kQRow = 164;
+__device__ __forceinline__ int qidx(int r, int c) { return r * kQRow + (c >> 5) * 40 + (c & 31); }
+
 template <int NT>
 struct SmemLayout {
-  static constexpr int q = kStageOff + kBufBytes;  // float q[NT * 8][128]
-  static constexpr int bar = q + NT * 8 * kD * 4;  // mbarrier per stage (4), abort flag
+  static constexpr int q = kStageOff + kBufBytes;  // float q[NT * 8][kQRow] (qidx)
+  static constexpr int bar = q + NT * 8 * kQRow * 4;  // mbarrier per stage (4), abort flag
   static constexpr int bytes = bar + 64 + 1024;    // + alignment slack
 };
 constexpr int kMaxStages = 4;
@@ -297,11 +305,12 @@ template <int NT>
 __device__ __forceinline__ void qfrag_natural(uint32_t (&qb)[NT][8][2], const float* q_s, int g, int tq) {
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
-    const float* qr = q_s + (nt * 8 + g) * kD;
+    const int r = nt * 8 + g;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      qb[nt][j][0] = pack_bf16x2(qr[16 * j + 2 * tq], qr[16 * j + 2 * tq + 1]);
-      qb[nt][j][1] = pack_bf16x2(qr[16 * j + 2 * tq + 8], qr[16 * j + 2 * tq + 9]);
+      const int c = 16 * j + 2 * tq;
+      qb[nt][j][0] = pack_bf16x2(q_s[qidx(r, c)], q_s[qidx(r, c + 1)]);
+      qb[nt][j][1] = pack_bf16x2(q_s[qidx(r, c + 8)], q_s[qidx(r, c + 9)]);
     }
   }
 }
@@ -336,7 +345,7 @@ __device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (
                                             const float* q_s, int g, int tq) {
 #pragma unroll
   for (int nt = 0; nt < NT; ++nt) {
-    const float* qr = q_s + (nt * 8 + g) * kD;
+    const int r = nt * 8 + g;
     float a1 = 0.f, a0 = 0.f;
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
@@ -345,7 +354,7 @@ __device__ __forceinline__ void qfrag_token(uint32_t (&qb)[NT][8][2], uint32_t (
       const float f = (BITS != 4) ? 1.0f / (float)(1 << pos3(j)) : 1.0f;  // exact
 #pragma unroll
       for (int hh = 0; hh < 2; ++hh) {
-        const float x0 = qr[c[2 * hh]] * f, x1 = qr[c[2 * hh + 1]] * f;
+        const float x0 = q_s[qidx(r, c[2 * hh])] * f, x1 = q_s[qidx(r, c[2 * hh + 1])] * f;
         uint32_t hi, lo = 0u;
         if (ROT) {
           split_pair(x0, x1, hi, lo);
@@ -600,7 +609,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       uint32_t qh[NT][8][2], qlo[NT][8][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
-        const float* qr = q_s + (nt * 8 + g) * kD;
+        const float* qr = q_s + (nt * 8 + g) * kQRow;
         float zpart = 0.f;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
@@ -608,7 +617,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           const int c0 = 32 * tq + 4 * j;
           float2 m[4];
           meta_quad<MB>(kmp, gm + c0, m);
-          const float4 qv = *reinterpret_cast<const float4*>(qr + c0);
+          const float4 qv = *reinterpret_cast<const float4*>(qr + tq * 40 + 4 * j);  // channels c0..c0+3
           split_pair(qv.x * m[0].x, qv.y * m[1].x, qh[nt][j][0], qlo[nt][j][0]);
           split_pair(qv.z * m[2].x, qv.w * m[3].x, qh[nt][j][1], qlo[nt][j][1]);
           zpart = fmaf(qv.x, m[0].y, zpart);
@@ -1042,7 +1051,8 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   for (int k = 0; k < QV; ++k) {
     const int i = tid + k * kThreads;
     if (i < NT * 8 * 16) {
-      float4* dst = reinterpret_cast<float4*>(q_s + i * 8);
+      // piece i: row i / 16, channels 8 (i % 16) .. + 7
+      float4* dst = reinterpret_cast<float4*>(q_s + qidx(i >> 4, 8 * (i & 15)));
       float f[8];
       bf16x2_to_f32(qv[k].x, f[0], f[1]);
       bf16x2_to_f32(qv[k].y, f[2], f[3]);
@@ -1057,10 +1067,10 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
     for (int j = warp; j < G; j += kWarps) {
       float x[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) x[i] = q_s[j * kD + lane * 4 + i];
+      for (int i = 0; i < 4; ++i) x[i] = q_s[qidx(j, lane * 4 + i)];
       fwht128_warp(x, lane);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) q_s[j * kD + lane * 4 + i] = x[i];
+      for (int i = 0; i < 4; ++i) q_s[qidx(j, lane * 4 + i)] = x[i];
     }
     __syncthreads();
   }
