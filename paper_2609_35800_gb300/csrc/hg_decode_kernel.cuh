@@ -58,13 +58,12 @@ constexpr int kPartialStride = kD + 4;  // m, l, 2 pad, o[128]: rows of 528 byte
 // Shared memory, from a 1024-byte aligned base (swizzled TMA boxes need it).
 constexpr int kStageOff = 0;                    // pipeline buffer
 // Four CTAs per SM for up to 8 queries per KV head (NT = 1), two above.
-// Staged queries: row r (query r of the KV head), channel c at
-// r * kQRow + (c / 32) * 40 + c % 32.  The padding spreads the 16-byte reads
-// of one warp (8 rows x 4 channel blocks, the KIVI-style key path) over all
-// banks: row strides are an odd number of 16-byte units and block strides
-// two units more than a multiple of eight.
-constexpr int kQRow = 164;
-__device__ __forceinline__ int qidx(int r, int c) { return r * kQRow + (c >> 5) * 40 + (c & 31); }
+// Staged queries: row r (query r of the KV head), channel c at r * kQRow + c.
+// The row stride of 36 16-byte units (4 mod 8) spreads the 16-byte reads of
+// one warp in the KIVI-style key path (8 rows x 4 consecutive channel
+// quads) over all banks.
+constexpr int kQRow = 144;
+__device__ __forceinline__ int qidx(int r, int c) { return r * kQRow + c; }
 
 template <int NT>
 struct SmemLayout {
@@ -613,11 +612,12 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         float zpart = 0.f;
 #pragma unroll
         for (int j = 0; j < 8; ++j) {
-          // k-slots 2tq, 2tq+1, 2tq+8, 2tq+9 of k-step j <-> channels 32tq + 4j + 0..3
-          const int c0 = 32 * tq + 4 * j;
+          // k-slots 2tq, 2tq+1, 2tq+8, 2tq+9 of k-step j <-> channels 16j + 4tq + 0..3
+          // (the four tq lanes read four different banks of codes and metadata)
+          const int c0 = 16 * j + 4 * tq;
           float2 m[4];
           meta_quad<MB>(kmp, gm + c0, m);
-          const float4 qv = *reinterpret_cast<const float4*>(qr + tq * 40 + 4 * j);  // channels c0..c0+3
+          const float4 qv = *reinterpret_cast<const float4*>(qr + c0);
           split_pair(qv.x * m[0].x, qv.y * m[1].x, qh[nt][j][0], qlo[nt][j][0]);
           split_pair(qv.z * m[2].x, qv.w * m[3].x, qh[nt][j][1], qlo[nt][j][1]);
           zpart = fmaf(qv.x, m[0].y, zpart);
@@ -636,7 +636,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       const uint32_t sel4 = (uint32_t)(g >> 1) | ((uint32_t)(4 + (g >> 1)) << 8);
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
-        const int c0 = 32 * tq + 4 * j;
+        const int c0 = 16 * j + 4 * tq;
         uint32_t w[4][4];
 #pragma unroll
         for (int cc = 0; cc < 4; ++cc) {
