@@ -509,6 +509,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 #pragma unroll
         for (int i = 0; i < 4; ++i) acc[s][nt][i] = 0.f;
     float zk[NT][2];  // KIVI-style: sum_c q_c z_c of the group, per query column
+    uint32_t qh[NT][8][2], qlo[NT][8][2];  // KIVI-style: the group's scaled queries (hi + lo)
 #pragma unroll
     for (int nt = 0; nt < NT; ++nt) zk[nt][0] = zk[nt][1] = 0.f;
 
@@ -605,7 +606,6 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         for (int i = 0; i < 4; ++i) acc[0][nt][i] += acc2[nt][i];
     } else {  // K_KIVI: group u of the tile; channel c has (scale, zero) = meta[u][c]
       const int gm = u * kD;  // first metadata pair of the group
-      uint32_t qh[NT][8][2], qlo[NT][8][2];
 #pragma unroll
       for (int nt = 0; nt < NT; ++nt) {
         const float* qr = q_s + (nt * 8 + g) * kQRow;
@@ -631,52 +631,60 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
         zk[nt][0] = __shfl_sync(kFull, zpart, (2 * tq) << 2);
         zk[nt][1] = __shfl_sync(kFull, zpart, (2 * tq + 1) << 2);
       }
-      const uint32_t* gc = kc32 + u * kD * BITS;  // [128 channels][BITS words], token order
-      // byte selector: byte (g/2) of a -> byte 0, byte (g/2) of b -> byte 2
-      const uint32_t sel4 = (uint32_t)(g >> 1) | ((uint32_t)(4 + (g >> 1)) << 8);
+    }
+
+    // ---------------- per slice: (KIVI-style keys: scores), softmax, then P.V ----------------
+    // The loop stays rolled: for KIVI-style keys (two slices per unit) an
+    // unrolled copy doubles the longest code path of the kernel.
+#pragma unroll 1
+    for (int s = 0; s < SPU; ++s) {
+      const int tok0 = (u * SPU + s) * 16;
+      if (tok0 >= nvalid) break;
+      float ks[NT][4];  // KIVI-style: this slice's scores against the scaled queries
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int c0 = 16 * j + 4 * tq;
-        uint32_t w[4][4];
+      for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-        for (int cc = 0; cc < 4; ++cc) {
-          if (BITS == 2) {
-            const uint2 t2 = *reinterpret_cast<const uint2*>(gc + (c0 + cc) * 2);
-            w[cc][0] = t2.x;
-            w[cc][1] = t2.y;
-            w[cc][2] = w[cc][3] = 0u;
-          } else if (BITS == 3) {  // two 2-bit words, then the bit-2 plane of the 32 tokens
-            w[cc][0] = gc[(c0 + cc) * 3];
-            w[cc][1] = gc[(c0 + cc) * 3 + 1];
-            w[cc][2] = gc[(c0 + cc) * 3 + 2];
-            w[cc][3] = 0u;
-          } else {
-            const uint4 t4 = *reinterpret_cast<const uint4*>(gc + (c0 + cc) * 4);
-            w[cc][0] = t4.x;
-            w[cc][1] = t4.y;
-            w[cc][2] = t4.z;
-            w[cc][3] = t4.w;
+        for (int i = 0; i < 4; ++i) ks[nt][i] = 0.f;
+      if (KM == K_KIVI) {
+        const uint32_t* gc = kc32 + u * kD * BITS;  // [128 channels][BITS words], token order
+        // byte selector: byte (g/2) of a -> byte 0, byte (g/2) of b -> byte 2
+        const uint32_t sel4 = (uint32_t)(g >> 1) | ((uint32_t)(4 + (g >> 1)) << 8);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          const int c0 = 16 * j + 4 * tq;
+          // per channel: the word(s) of tokens 16s..16s+15 (3 bits: and the bit-2 plane)
+          uint32_t w[4][2];
+#pragma unroll
+          for (int cc = 0; cc < 4; ++cc) {
+            if (BITS == 2) {
+              w[cc][0] = gc[(c0 + cc) * 2 + s];
+              w[cc][1] = 0u;
+            } else if (BITS == 3) {
+              w[cc][0] = gc[(c0 + cc) * 3 + s];
+              w[cc][1] = gc[(c0 + cc) * 3 + 2];
+            } else {
+              const uint2 t2 = *reinterpret_cast<const uint2*>(gc + (c0 + cc) * 4 + 2 * s);
+              w[cc][0] = t2.x;
+              w[cc][1] = t2.y;
+            }
           }
-        }
-#pragma unroll
-        for (int s = 0; s < 2; ++s) {
           uint32_t a[4];
           if (BITS == 2) {
-            // word s of a channel: tokens 16s..16s+15; its low half holds the first 8
-            a[0] = pair2<2>(prmt(w[0][s], w[1][s], 0x5410) >> (2 * g));
-            a[1] = pair2<2>(prmt(w[0][s], w[1][s], 0x7632) >> (2 * g));
-            a[2] = pair2<2>(prmt(w[2][s], w[3][s], 0x5410) >> (2 * g));
-            a[3] = pair2<2>(prmt(w[2][s], w[3][s], 0x7632) >> (2 * g));
+            // the word's low half holds tokens 16s..16s+7, its high half the next 8
+            a[0] = pair2<2>(prmt(w[0][0], w[1][0], 0x5410) >> (2 * g));
+            a[1] = pair2<2>(prmt(w[0][0], w[1][0], 0x7632) >> (2 * g));
+            a[2] = pair2<2>(prmt(w[2][0], w[3][0], 0x5410) >> (2 * g));
+            a[3] = pair2<2>(prmt(w[2][0], w[3][0], 0x7632) >> (2 * g));
           } else if (BITS == 3) {
             // bit 2 of token 16s + i: plane byte s (i < 8) or 2 + s (i >= 8), bit i % 8
-            const uint32_t lo0 = prmt(w[0][s], w[1][s], 0x5410) >> (2 * g);
-            const uint32_t lo1 = prmt(w[0][s], w[1][s], 0x7632) >> (2 * g);
-            const uint32_t lo2 = prmt(w[2][s], w[3][s], 0x5410) >> (2 * g);
-            const uint32_t lo3 = prmt(w[2][s], w[3][s], 0x7632) >> (2 * g);
-            const uint32_t h0 = prmt(w[0][2], w[1][2], plane_sel(s)) >> g;
-            const uint32_t h1 = prmt(w[0][2], w[1][2], plane_sel(2 + s)) >> g;
-            const uint32_t h2 = prmt(w[2][2], w[3][2], plane_sel(s)) >> g;
-            const uint32_t h3 = prmt(w[2][2], w[3][2], plane_sel(2 + s)) >> g;
+            const uint32_t lo0 = prmt(w[0][0], w[1][0], 0x5410) >> (2 * g);
+            const uint32_t lo1 = prmt(w[0][0], w[1][0], 0x7632) >> (2 * g);
+            const uint32_t lo2 = prmt(w[2][0], w[3][0], 0x5410) >> (2 * g);
+            const uint32_t lo3 = prmt(w[2][0], w[3][0], 0x7632) >> (2 * g);
+            const uint32_t h0 = prmt(w[0][1], w[1][1], plane_sel(s)) >> g;
+            const uint32_t h1 = prmt(w[0][1], w[1][1], plane_sel(2 + s)) >> g;
+            const uint32_t h2 = prmt(w[2][1], w[3][1], plane_sel(s)) >> g;
+            const uint32_t h3 = prmt(w[2][1], w[3][1], plane_sel(2 + s)) >> g;
             a[0] = pair2<3>((lo0 & 0x00030003u) | ((h0 & 0x00010001u) << 2));
             a[1] = pair2<3>((lo1 & 0x00030003u) | ((h1 & 0x00010001u) << 2));
             a[2] = pair2<3>((lo2 & 0x00030003u) | ((h2 & 0x00010001u) << 2));
@@ -684,25 +692,18 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
           } else {
             // words 2s, 2s+1 of a channel: tokens 16s..16s+7 and 16s+8..16s+15
             const int sh = 4 * (g & 1);
-            a[0] = pair2<4>(prmt(w[0][2 * s], w[1][2 * s], sel4) >> sh);
-            a[1] = pair2<4>(prmt(w[0][2 * s + 1], w[1][2 * s + 1], sel4) >> sh);
-            a[2] = pair2<4>(prmt(w[2][2 * s], w[3][2 * s], sel4) >> sh);
-            a[3] = pair2<4>(prmt(w[2][2 * s + 1], w[3][2 * s + 1], sel4) >> sh);
+            a[0] = pair2<4>(prmt(w[0][0], w[1][0], sel4) >> sh);
+            a[1] = pair2<4>(prmt(w[0][1], w[1][1], sel4) >> sh);
+            a[2] = pair2<4>(prmt(w[2][0], w[3][0], sel4) >> sh);
+            a[3] = pair2<4>(prmt(w[2][1], w[3][1], sel4) >> sh);
           }
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            mma_bf16(acc[s][nt], a, qh[nt][j][0], qh[nt][j][1]);
-            mma_bf16(acc[s][nt], a, qlo[nt][j][0], qlo[nt][j][1]);
+            mma_bf16(ks[nt], a, qh[nt][j][0], qh[nt][j][1]);
+            mma_bf16(ks[nt], a, qlo[nt][j][0], qlo[nt][j][1]);
           }
         }
       }
-    }
-
-    // ---------------- per slice: softmax, then P.V ----------------
-#pragma unroll
-    for (int s = 0; s < SPU; ++s) {
-      const int tok0 = (u * SPU + s) * 16;
-      if (tok0 >= nvalid) break;
       float sc[NT][4];
       if (KM == K_TOKEN) {
         // acc = sum_d (128 + f c_d) (q_d / f) = 128 s1 + q.c, so
@@ -721,7 +722,7 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
 #pragma unroll
-          for (int i = 0; i < 4; ++i) sc[nt][i] = (acc[s][nt][i] + zk[nt][i & 1]) * scale_log2;
+          for (int i = 0; i < 4; ++i) sc[nt][i] = (ks[nt][i] + zk[nt][i & 1]) * scale_log2;
       } else {
 #pragma unroll
         for (int nt = 0; nt < NT; ++nt)
