@@ -51,6 +51,8 @@ def parse_args_from(argv):
                     help="metadata per group: fp32 pair (64) or binary16 pair (32, Sec. 5.4)")
     ap.add_argument("--bits", type=int, default=0, choices=[0, 2, 3, 4],
                     help="code width override (0: the workload's own)")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="layer-count override (0: the workload's own), e.g. for a small profile")
     ap.add_argument("--salient-permille", type=int, default=0,
                     help="AKVQ-style salient tokens kept BF16 per head (Sec. 4; 20 = 2%%)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -308,6 +310,8 @@ def _workload(args):
     w = wl.WORKLOADS[args.workload]
     if args.meta_bits != w.meta_bits:
         w = dataclasses.replace(w, meta_bits=args.meta_bits, name=w.name + "_meta%d" % args.meta_bits)
+    if args.layers and args.layers != w.layers:
+        w = dataclasses.replace(w, layers=args.layers, name=w.name + "_%dlayers" % args.layers)
     if args.bits and args.bits != w.bits:
         w = dataclasses.replace(w, bits=args.bits, name=w.name + "_%dbit" % args.bits)
     if args.salient_permille != w.salient_permille:
