@@ -513,40 +513,46 @@ def run_gpu(args):
 
 
 def run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream):
-    """Same step driven from pinned host buffers through the C ABI."""
+    """Same step driven from pinned host buffers through the C ABI.  The
+    prefill K (and V) of all layers sit in one pinned buffer each, and every
+    decode step's query, new keys and new values in one pinned buffer, so a
+    step is two prefill copies, then per decode step one copy in and one out."""
     import torch
 
     import paper_2609_35800_gb300 as hg
     L, S = w.layers, w.decode_steps
-    hk = [k.cpu().pin_memory() for k, _ in prefill]
-    hv = [v.cpu().pin_memory() for _, v in prefill]
-    hq = [q.cpu().pin_memory() for q in qs]
-    hkn = [kn.cpu().pin_memory() for kn, _ in news]
-    hvn = [vn.cpu().pin_memory() for _, vn in news]
+    hk = torch.stack([k for k, _ in prefill]).cpu().pin_memory()
+    hv = torch.stack([v for _, v in prefill]).cpu().pin_memory()
+    nq, nk = qs[0].numel(), news[0][0].numel()
+    hin = torch.empty((S, nq + 2 * nk), dtype=qs[0].dtype).pin_memory()
+    for st in range(S):
+        hin[st, :nq].copy_(qs[st].reshape(-1).cpu())
+        hin[st, nq:nq + nk].copy_(news[st][0].reshape(-1).cpu())
+        hin[st, nq + nk:].copy_(news[st][1].reshape(-1).cpu())
     hout = torch.empty((S,) + tuple(qs[0].shape), dtype=qs[0].dtype).pin_memory()
-    dk = [torch.empty_like(k) for k, _ in prefill]
-    dv = [torch.empty_like(v) for _, v in prefill]
-    dq = torch.empty_like(qs[0])
-    dkn = torch.empty_like(news[0][0])
-    dvn = torch.empty_like(news[0][1])
+    dk = torch.empty_like(hk, device=dev)
+    dv = torch.empty_like(hv, device=dev)
+    din = torch.empty(nq + 2 * nk, dtype=qs[0].dtype, device=dev)
+    dq = din[:nq].view(qs[0].shape)
+    dkn = din[nq:nq + nk].view(news[0][0].shape)
+    dvn = din[nq + nk:].view(news[0][1].shape)
     dout = torch.empty_like(qs[0])
-    h2d = sum(t.numel() * 2 for t in hk + hv + hq + hkn + hvn)
+    dks = [dk[l] for l in range(L)]
+    dvs = [dv[l] for l in range(L)]
+    h2d = (hk.numel() + hv.numel() + hin.numel()) * 2
     d2h = hout.numel() * 2
 
     def step():
-        for l in range(L):
-            dk[l].copy_(hk[l], non_blocking=True)
-            dv[l].copy_(hv[l], non_blocking=True)
+        dk.copy_(hk, non_blocking=True)
+        dv.copy_(hv, non_blocking=True)
         for l0 in range(0, L, 64):
             n = min(64, L - l0)
-            hg.hg_quantize_kv(runner.cache, l0, dk[l0:l0 + n], dv[l0:l0 + n], stream)
-        for s in range(S):
-            dq.copy_(hq[s], non_blocking=True)
-            dkn.copy_(hkn[s], non_blocking=True)
-            dvn.copy_(hvn[s], non_blocking=True)
+            hg.hg_quantize_kv(runner.cache, l0, dks[l0:l0 + n], dvs[l0:l0 + n], stream)
+        for st in range(S):
+            din.copy_(hin[st], non_blocking=True)
             hg.hg_decode_step(runner.cache, 0, L, dq, dkn, dvn, dout, 0.0, runner.ws, runner.ws_bytes,
                               stream)
-            hout[s].copy_(dout, non_blocking=True)
+            hout[st].copy_(dout, non_blocking=True)
 
     for _ in range(max(1, args.warmup)):
         step()
