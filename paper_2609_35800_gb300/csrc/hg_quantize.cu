@@ -17,6 +17,7 @@
 
 #include "hg_common.cuh"
 #include "hg_internal.h"
+#include "hg_mma.cuh"
 
 namespace hg {
 
@@ -155,6 +156,8 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
   // The warp's tokens t0 + warp + 4i, one at a time, the next token's K and V
   // loaded while this one is processed.  The loop stays rolled: the token
   // body is long, and eight unrolled copies of it thrash the instruction cache.
+  // (Staging the whole tile in shared memory with asynchronous copies first
+  // measured slower for this kernel.)
   uint2 kn = make_uint2(0u, 0u), vn = make_uint2(0u, 0u);
   if (t0 + warp < t1) {
     kn = ldg8(K + (size_t)(t0 + warp) * kD + lane * 4);
@@ -441,12 +444,16 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
   const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
 
   __shared__ __align__(16) char rows[2][kQTok][kQPitch];
-  // coalesced staging: chunk c = 16 bytes of one row
+  // coalesced staging, chunk c = 16 bytes of one row, as asynchronous copies
+  // (all of a thread's chunks in flight at once rather than one load-store
+  // round trip after another)
   for (int c = tid; c < 2 * n * 16; c += kThreads) {
     const int kv = c / (n * 16), rem = c - kv * (n * 16);
     const int r = rem >> 4, col = rem & 15;
-    *reinterpret_cast<uint4*>(&rows[kv][r][col * 16]) = ldg16((kv ? src_v : src_k) + (size_t)r * 256 + col * 16);
+    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
   }
+  cp_async_commit();
+  cp_async_wait<0>();
   __syncthreads();
 
   const int kv = tid >> 6, r = tid & (kQTok - 1);
