@@ -919,6 +919,21 @@ __device__ __forceinline__ void compute_tile(WarpState<NT, NZOf<VM>::value>& ws,
       }
     }
   }
+  if (VM == V_TOKEN) {
+    // Fold the tile's 1024 offsets into the accumulators.  Both grow with the
+    // segment while their difference (the value sum) stays small; left to the
+    // end of a long segment (thousands of tokens in one CTA), the fp32
+    // accumulation error of the large common part would show in the result.
+#pragma unroll
+    for (int nt = 0; nt < NT; ++nt) {
+#pragma unroll
+      for (int mt = 0; mt < 8; ++mt)
+#pragma unroll
+        for (int i = 0; i < 4; ++i) ws.o[nt][mt][i] -= ws.corr[nt][i];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) ws.corr[nt][i] = 0.f;
+    }
+  }
 }
 
 // ---------------------------------------------------------------------------

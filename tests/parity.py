@@ -51,34 +51,47 @@ def _meta_words(meta, meta16):
     return meta.view(np.uint32)
 
 
-def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, rows=None):
-    """Bit-exact comparison of every region of one layer (or the given heads / rows)."""
+def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, rows=None,
+                      local=False):
+    """Bit-exact comparison of every region of one layer (or the given heads / rows).
+
+    local: k_bits, v_bits and the oracle output o hold only the given rows and
+    heads (index [i][j] for rows[i], heads[j]), and the arena is read region
+    by region from the device (caches too large to copy whole)."""
     w = runner.w
     m16 = w.meta_bits == 32
-    if arena is None:
-        arena = runner.arena.cpu().numpy()
+    if local:
+        def rd(off, nbytes, dtype):
+            return runner.arena[off: off + nbytes].cpu().numpy().view(dtype)
+    else:
+        if arena is None:
+            arena = runner.arena.cpu().numpy()
+
+        def rd(off, nbytes, dtype):
+            return _slice(arena, off, nbytes, dtype)
     B, H, T = w.batch, w.kv_heads, w.seq_len
     s, nq = w.img_start, o["nq"]
     W = 128 * w.bits // 32
     heads = range(H) if heads is None else heads
     rows = range(B) if rows is None else rows
     ns = o["n_salient"]
-    for h in heads:
+    for hi, h in enumerate(heads):
         r = hg.hg_cache_head_regions(runner.cache, layer, h)
         assert r.nq == nq
         cls = r.head_class
         assert r.n_salient == (ns if cls == hg.HG_HEAD_QUANTIZED else 0)
         nc = 0 if cls == hg.HG_HEAD_PROTECTED else nq - r.n_salient
         assert r.n_coded == nc
-        for b in rows:
+        for bi, b in enumerate(rows):
+            ob, oh = (bi, hi) if local else (b, h)  # oracle / input index of (b, h)
             if cls == hg.HG_HEAD_PROTECTED:
                 toks = np.arange(T)
             elif r.n_salient:
                 # leading text, salient image tokens in order, trailing text
-                sal = o["salient"][b, h]
+                sal = o["salient"][ob, oh]
                 toks = np.concatenate([np.arange(0, s), s + sal, np.arange(s + nq, T)])
                 nblk = (nq + 31) // 32
-                words = _slice(arena, r.sal + b * r.sal_bstride, nblk * 8, np.uint32)
+                words = rd(r.sal + b * r.sal_bstride, nblk * 8, np.uint32)
                 want = np.zeros(nblk, np.uint32)
                 for i in sal:
                     want[i >> 5] |= np.uint32(1 << (i & 31))
@@ -88,27 +101,27 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
             else:
                 toks = np.concatenate([np.arange(0, s), np.arange(s + nq, T)])
             assert r.bf16_prefill == toks.size
-            kb = _slice(arena, r.kb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
-            vb = _slice(arena, r.vb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
-            assert np.array_equal(kb, k_bits[b, h, toks]), (layer, h, b, "kb")
-            assert np.array_equal(vb, v_bits[b, h, toks]), (layer, h, b, "vb")
-            kmeta_n = o["k_meta"][b, h].size if w.base == 1 else 2 * nc
-            vmeta_n = o["v_meta"][b, h].size * nc // max(nq, 1)
+            kb = rd(r.kb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
+            vb = rd(r.vb + b * r.kb_bstride, toks.size * 256, np.uint16).reshape(-1, 128)
+            assert np.array_equal(kb, k_bits[ob, oh, toks]), (layer, h, b, "kb")
+            assert np.array_equal(vb, v_bits[ob, oh, toks]), (layer, h, b, "vb")
+            kmeta_n = o["k_meta"][ob, oh].size if w.base == 1 else 2 * nc
+            vmeta_n = o["v_meta"][ob, oh].size * nc // max(nq, 1)
             if cls == hg.HG_HEAD_QUANTIZED and nc:
-                kw = _slice(arena, r.kq + b * r.kq_bstride, nc * W * 4, np.uint32)
-                ek = _meta_words(o["k_meta"][b, h][:kmeta_n], m16)
-                km = _slice(arena, r.kqm + b * r.kqm_bstride, ek.nbytes, np.uint32)
-                assert np.array_equal(kw, o["k_words"][b, h][:nc * W]), (layer, h, b, "kq")
+                kw = rd(r.kq + b * r.kq_bstride, nc * W * 4, np.uint32)
+                ek = _meta_words(o["k_meta"][ob, oh][:kmeta_n], m16)
+                km = rd(r.kqm + b * r.kqm_bstride, ek.nbytes, np.uint32)
+                assert np.array_equal(kw, o["k_words"][ob, oh][:nc * W]), (layer, h, b, "kq")
                 assert np.array_equal(km, ek), (layer, h, b, "kqm")
             if cls != hg.HG_HEAD_PROTECTED and nc:
-                vw = _slice(arena, r.vq + b * r.vq_bstride, nc * W * 4, np.uint32)
-                ev = _meta_words(o["v_meta"][b, h][:vmeta_n], m16)
-                vm = _slice(arena, r.vqm + b * r.vqm_bstride, ev.nbytes, np.uint32)
-                assert np.array_equal(vw, o["v_words"][b, h][:nc * W]), (layer, h, b, "vq")
+                vw = rd(r.vq + b * r.vq_bstride, nc * W * 4, np.uint32)
+                ev = _meta_words(o["v_meta"][ob, oh][:vmeta_n], m16)
+                vm = rd(r.vqm + b * r.vqm_bstride, ev.nbytes, np.uint32)
+                assert np.array_equal(vw, o["v_words"][ob, oh][:nc * W]), (layer, h, b, "vq")
                 assert np.array_equal(vm, ev), (layer, h, b, "vqm")
             if cls == hg.HG_HEAD_KEYS_ONLY and nq:
-                ki = _slice(arena, r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)
-                assert np.array_equal(ki, k_bits[b, h, s:s + nq]), (layer, h, b, "kimg")
+                ki = rd(r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)
+                assert np.array_equal(ki, k_bits[ob, oh, s:s + nq]), (layer, h, b, "kimg")
 
 
 def attention_reference(runner, o, q_bits, appended_k, appended_v, sigma):
