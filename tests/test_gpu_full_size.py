@@ -4,6 +4,8 @@ bench.py times: one quantize call over all layers, then fused decode steps
 sampled (layer, batch row, KV head) triples one by one: the head's arena
 regions bit for bit, and its G query heads' attention outputs after every
 step within the tolerance of the parity tests."""
+import dataclasses
+
 import numpy as np
 import pytest
 import torch
@@ -40,9 +42,16 @@ def _samples(w, mask, seed):
     return picks
 
 
-@pytest.mark.parametrize("name", ["qwen25vl7b", "llavanext7b", "internvl25_8b", "qwen25vl72b"])
-def test_full_size_sampled_parity(name):
-    w = wl.WORKLOADS[name]
+# the four benchmark shapes, then options of the next rows at full size
+VARIANTS = [("qwen25vl7b", {}), ("llavanext7b", {}), ("internvl25_8b", {}), ("qwen25vl72b", {}),
+            ("internvl25_8b", {"salient_permille": 20}), ("qwen25vl7b", {"bits": 3}),
+            ("llavanext7b", {"bits": 3}), ("qwen25vl72b", {"meta_bits": 32})]
+
+
+@pytest.mark.parametrize("name,opts", VARIANTS,
+                         ids=[n + "".join("-%s%s" % kv for kv in o.items()) for n, o in VARIANTS])
+def test_full_size_sampled_parity(name, opts):
+    w = dataclasses.replace(wl.WORKLOADS[name], **opts)
     runner = CacheRunner(w)
     runner.quantize_all()
     G = w.q_heads // w.kv_heads
