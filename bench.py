@@ -461,6 +461,8 @@ def run_gpu(args):
     achieved = dec_bytes_mean / (dec_ms * 1e-3) / 1e9
     traffic = profiled_traffic(w.name)
 
+    extra = decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream)
+
     e2e = None
     if not args.no_e2e:
         e2e = run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream)
@@ -495,6 +497,7 @@ def run_gpu(args):
                      "peak_source": peak_src + " hbm_gbs (burst copy)"},
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
+        "decode_variants": extra,
     }
     if e2e is not None:
         line["e2e"] = e2e
@@ -510,6 +513,71 @@ def run_gpu(args):
     if dist is not None:
         dist.destroy_process_group()
     return 0
+
+
+def decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream):
+    """Two other ways to launch the same decode steps, reported beside the
+    headline (which they do not change): one launch per layer (append and
+    attention of a single layer each), L2 flushed before every step; and the
+    whole decode loop captured in one CUDA graph and replayed (launch costs
+    gone; the cache stays in L2 between steps, as it would when nothing else
+    runs between decode steps)."""
+    import torch
+
+    import paper_2609_35800_gb300 as hg
+    L, S = w.layers, w.decode_steps
+    out = torch.empty_like(qs[0])
+    dec_bytes_mean = (sum(dec_b) + S * app_b) / S
+    res = {}
+    # one launch per layer
+    hg.hg_cache_reset_appended(runner.cache)
+    n_steps = min(S, 8)
+    times = []
+    for st in range(n_steps):
+        cushion()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for l in range(L):
+            hg.hg_decode_step(runner.cache, l, 1, qs[st][l], news[st][0][l], news[st][1][l], out[l],
+                              0.0, runner.ws, runner.ws_bytes, stream)
+        a1.record(stream)
+        times.append((a0, a1))
+    torch.cuda.synchronize()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in times)
+    res["per_layer_launches"] = {"ms_per_decode_step": round(ms, 4), "launches_per_step": L,
+                                 "GBps": round(dec_bytes_mean / (ms * 1e-3) / 1e9, 1),
+                                 "steps_timed": n_steps, "l2": "flushed before every step"}
+    # the decode loop as one CUDA graph (layer-batched launches)
+    hg.hg_cache_reset_appended(runner.cache)
+    graph = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        with torch.cuda.graph(graph, stream=side):
+            cap = torch.cuda.current_stream()
+            for st in range(S):
+                hg.hg_decode_step(runner.cache, 0, L, qs[st], news[st][0], news[st][1], out, 0.0,
+                                  runner.ws, runner.ws_bytes, cap)
+    torch.cuda.current_stream().wait_stream(side)
+    graph.replay()
+    torch.cuda.synchronize()
+    reps = []
+    for _ in range(5):
+        cushion()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        graph.replay()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        reps.append(a0.elapsed_time(a1) / S)
+    best, med = min(reps), statistics.median(reps)
+    res["graph_replay"] = {"ms_per_decode_step_best": round(best, 4),
+                           "ms_per_decode_step_median": round(med, 4),
+                           "GBps_best": round(dec_bytes_mean / (best * 1e-3) / 1e9, 1),
+                           "decode_tokens_per_s_best": round(w.batch / (best * 1e-3), 1),
+                           "l2": "flushed before each replay of the %d-step loop only" % S}
+    hg.hg_cache_reset_appended(runner.cache)
+    return res
 
 
 def run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream):
