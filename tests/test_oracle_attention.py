@@ -116,3 +116,49 @@ def test_storage_k_only_saving_about_22_percent(oracle):
     kv = oracle.image_bits_per_elem(2, 32, 0.125, 0)
     ko = oracle.image_bits_per_elem(2, 32, 0.125, 1)
     assert round(100 * (kv - ko) / kv) == 22
+
+
+def _brute_attention(q, K, V, sigma):
+    """Scalar double-precision decode attention written out term by term for tiny
+    shapes: softmax over every token of sigma * <q, k_t>, then the weighted sum of
+    the values; query head qh reads KV head qh // G."""
+    B, Hq, D = len(q), len(q[0]), len(q[0][0])
+    H, T = len(K[0]), len(K[0][0])
+    G = Hq // H
+    out = [[[0.0] * D for _ in range(Hq)] for _ in range(B)]
+    for b in range(B):
+        for qh in range(Hq):
+            h = qh // G
+            scores = []
+            for t in range(T):
+                acc = 0.0
+                for d in range(D):
+                    acc += q[b][qh][d] * K[b][h][t][d]
+                scores.append(sigma * acc)
+            top = max(scores)
+            w = [math.exp(x - top) for x in scores]
+            z = math.fsum(w)
+            for d in range(D):
+                out[b][qh][d] = math.fsum(w[t] * V[b][h][t][d] for t in range(T)) / z
+    return out
+
+
+@pytest.mark.parametrize("B,Hq,H,T,sigma,scale", [
+    (1, 1, 1, 1, 0.0883883476, 1.0),    # one token: the output is its value
+    (2, 4, 2, 3, 0.0883883476, 1.0),
+    (1, 6, 2, 8, 0.2, 3.0),             # G = 3, sharp softmax
+    (2, 2, 2, 5, 1.0, 0.5),             # MHA
+    (1, 8, 1, 7, 0.05, 40.0),           # scores far beyond exp's range without the shift
+])
+def test_matches_brute_force_on_tiny_shapes(oracle, B, Hq, H, T, sigma, scale):
+    rng = np.random.default_rng(100 + T * 7 + Hq)
+    qb = _bits(rng.standard_normal((B, Hq, 128)) * scale)
+    K = rng.standard_normal((B, H, T, 128)) * scale
+    V = rng.standard_normal((B, H, T, 128))
+    got = oracle.attention_layer(qb, K, V, sigma)
+    want = np.array(_brute_attention(_f32(qb).astype(np.float64).tolist(), K.tolist(),
+                                      V.tolist(), sigma))
+    assert np.allclose(got, want, rtol=1e-12, atol=1e-13)
+    if T == 1:
+        for qh in range(Hq):
+            assert np.allclose(got[:, qh], V[:, qh * H // Hq, 0], atol=1e-15)
