@@ -109,30 +109,64 @@ CLOCK_FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.a
 
 
 class ClockSampler:
-    def __init__(self, device_index):
+    """nvidia-smi sampling of SM clocks and throttle reasons around a timed
+    region: entering waits (up to `start_timeout` s) for the first sample so
+    the sampler is live when the region starts; `summary` keeps the samples
+    that arrived inside the region (plus the first one after it, which covers
+    its tail), or every sample when none did."""
+
+    def __init__(self, device_index, period_ms=100, start_timeout=5.0, cmd=None):
         self.proc = None
         self.idx = device_index
+        self.period_ms = period_ms
+        self.start_timeout = start_timeout
+        self.cmd = cmd or ["nvidia-smi"]
+        self.stamped = []
+        self.lines = []
+        self.t0 = self.t1 = None
+        self._reader = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            if line.strip():
+                self.stamped.append((time.perf_counter(), line))
 
     def __enter__(self):
+        import threading
         try:
             self.proc = subprocess.Popen(
-                ["nvidia-smi", "--query-gpu=" + CLOCK_FIELDS, "--format=csv,noheader,nounits",
-                 "-i", str(self.idx), "-lms", "200"],
+                self.cmd + ["--query-gpu=" + CLOCK_FIELDS, "--format=csv,noheader,nounits",
+                            "-i", str(self.idx), "-lms", str(self.period_ms)],
                 stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
         except OSError:
             self.proc = None
+        if self.proc is not None:
+            self._reader = threading.Thread(target=self._read, daemon=True)
+            self._reader.start()
+            deadline = time.perf_counter() + self.start_timeout
+            while not self.stamped and self.proc.poll() is None and time.perf_counter() < deadline:
+                time.sleep(0.01)
+        self.t0 = time.perf_counter()
         return self
 
     def __exit__(self, *exc):
-        self.lines = []
+        self.t1 = time.perf_counter()
         if self.proc is not None:
+            # let the sample in progress at the region's end arrive
+            deadline = self.t1 + 2.5 * self.period_ms * 1e-3
+            while (self.proc.poll() is None and time.perf_counter() < deadline
+                   and not any(t >= self.t1 for t, _ in self.stamped)):
+                time.sleep(0.01)
             self.proc.terminate()
             try:
-                out, _ = self.proc.communicate(timeout=5)
+                self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
-                out, _ = self.proc.communicate()
-            self.lines = [l for l in out.splitlines() if l.strip()]
+                self.proc.wait()
+            self._reader.join(timeout=5)
+        inside = [l for t, l in self.stamped if self.t0 <= t < self.t1]
+        after = [l for t, l in self.stamped if t >= self.t1][:1]
+        self.lines = (inside + after) or [l for _, l in self.stamped]
 
     def summary(self):
         sm, mx, reasons = [], [], set()
