@@ -43,7 +43,7 @@ def parse_args():
 def parse_args_from(argv):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="headguard", choices=["headguard", "reference"])
     ap.add_argument("--workload", default="qwen25vl7b")
@@ -115,7 +115,7 @@ class ClockSampler:
     that arrived inside the region (plus the first one after it, which covers
     its tail), or every sample when none did."""
 
-    def __init__(self, device_index, period_ms=100, start_timeout=5.0, cmd=None):
+    def __init__(self, device_index, period_ms=50, start_timeout=5.0, cmd=None):
         self.proc = None
         self.idx = device_index
         self.period_ms = period_ms
