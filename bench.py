@@ -57,6 +57,8 @@ def parse_args_from(argv):
                     help="AKVQ-style salient tokens kept BF16 per head (Sec. 4; 20 = 2%%)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-variants", action="store_true",
+                    help="skip the per-layer-launch and graph-replay decode variants")
     return ap.parse_args(argv)
 
 
@@ -427,7 +429,9 @@ def run_gpu(args):
     sigma = 0.0
     quant_b, dec_b, app_b = geometry_bytes(runner)
     step_bytes = quant_b + sum(dec_b) + S * app_b
-    launches_per_step = (L + 63) // 64 + S * ((L + 63) // 64)
+    # quantize: one launch per 64 layers, preceded by the salient-token selection when on
+    q_launches = (L + 63) // 64 * (2 if (w.salient_permille > 0 and w.image > 0) else 1)
+    launches_per_step = q_launches + S * ((L + 63) // 64)
 
     def cushion():
         flush.zero_()            # evict L2 (write a buffer larger than L2) ...
@@ -495,7 +499,9 @@ def run_gpu(args):
     achieved = dec_bytes_mean / (dec_ms * 1e-3) / 1e9
     traffic = profiled_traffic(w.name)
 
-    extra = decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream)
+    extra = None
+    if not args.no_variants:
+        extra = decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream)
 
     e2e = None
     if not args.no_e2e:
@@ -531,8 +537,9 @@ def run_gpu(args):
                      "peak_source": peak_src + " hbm_gbs (burst copy)"},
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
-        "decode_variants": extra,
     }
+    if extra is not None:
+        line["decode_variants"] = extra
     if e2e is not None:
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
