@@ -3,7 +3,9 @@
 Thin ctypes marshalling over ``libheadguard.so`` (declared in
 ``include/headguard.h``): every function here has the C entry point's name,
 converts its arguments (torch tensors -> device pointers, streams -> handles)
-and raises :class:`HGError` on a non-zero status.  All computation happens in
+and raises :class:`HGError` on a non-zero status (and ValueError, before the
+call, when a tensor argument is not a dense CUDA tensor holding the bytes the
+call reads or writes through it).  All computation happens in
 the library's CUDA kernels; there is no Python or CPU fallback, and importing
 the compute functions without the built library raises.
 """
@@ -123,13 +125,34 @@ def _check(status, where):
         raise HGError(status, where)
 
 
-def _ptr(x):
-    """Device/host address of a tensor (data_ptr), an int, or None."""
-    if x is None:
-        return None
-    if isinstance(x, int):
-        return x
-    return x.data_ptr()
+def _devs(where, *specs):
+    """Addresses of device buffer arguments, each given as (x, nbytes, name).
+    A torch tensor must be dense and hold at least `nbytes` bytes (the extent
+    the library reads or writes through it) -- checked for every argument
+    first -- and live on a CUDA device; an int is taken as a raw device
+    address whose extent the caller vouches for, None as a null pointer
+    (which the library rejects)."""
+    for x, nbytes, name in specs:
+        if x is None or isinstance(x, int):
+            continue
+        if not x.is_contiguous():
+            raise ValueError("%s: %s must be contiguous" % (where, name))
+        have = x.numel() * x.element_size()
+        if have < nbytes:
+            raise ValueError("%s: %s holds %d bytes, the call touches %d"
+                             % (where, name, have, nbytes))
+    for x, _, name in specs:
+        if x is not None and not isinstance(x, int) and not x.is_cuda:
+            raise ValueError("%s: %s must be a CUDA tensor" % (where, name))
+    return [x if (x is None or isinstance(x, int)) else x.data_ptr() for x, _, _ in specs]
+
+
+def _extent(cache, *dims, elem=2):
+    """Bytes of a dense [dims...][head_dim] array of `elem`-byte entries."""
+    n = elem * cache.shape.head_dim
+    for d in dims:
+        n *= max(int(d), 0)
+    return n
 
 
 def _stream(stream):
@@ -182,7 +205,8 @@ def hg_cache_create(shape, config, head_mask, arena, arena_bytes=None):
     if arena_bytes is None:
         arena_bytes = arena.numel() * arena.element_size()
     h = ctypes.c_void_p()
-    _check(library().hg_cache_create(ctypes.byref(shape), ctypes.byref(config), mp, _ptr(arena),
+    ap, = _devs("hg_cache_create", (arena, arena_bytes, "arena"))
+    _check(library().hg_cache_create(ctypes.byref(shape), ctypes.byref(config), mp, ap,
                                      arena_bytes, ctypes.byref(h)), "hg_cache_create")
     return Cache(h, arena, shape, config, m.copy())
 
@@ -210,21 +234,33 @@ def hg_cache_reset_appended(cache):
 
 def hg_quantize_kv(cache, layer_begin, k_list, v_list, stream=None):
     n = len(k_list)
-    assert len(v_list) == n
-    karr = (ctypes.c_void_p * n)(*[_ptr(k) for k in k_list])
-    varr = (ctypes.c_void_p * n)(*[_ptr(v) for v in v_list])
+    if len(v_list) != n:
+        raise ValueError("hg_quantize_kv: %d key and %d value tensors" % (n, len(v_list)))
+    sh = cache.shape
+    need = _extent(cache, sh.batch, sh.num_kv_heads, sh.seq_len)
+    ptrs = _devs("hg_quantize_kv", *([(k, need, "k[%d]" % i) for i, k in enumerate(k_list)] +
+                                     [(v, need, "v[%d]" % i) for i, v in enumerate(v_list)]))
+    karr = (ctypes.c_void_p * n)(*ptrs[:n])
+    varr = (ctypes.c_void_p * n)(*ptrs[n:])
     _check(library().hg_quantize_kv(cache.handle, layer_begin, n, karr, varr, _stream(stream)),
            "hg_quantize_kv")
 
 
 def hg_dequantize_kv(cache, layer, k_out, v_out, out_fp32, stream=None):
-    _check(library().hg_dequantize_kv(cache.handle, layer, _ptr(k_out), _ptr(v_out),
-                                      1 if out_fp32 else 0, _stream(stream)), "hg_dequantize_kv")
+    sh = cache.shape
+    t = sh.seq_len + max(hg_cache_appended(cache, layer), 0)
+    need = _extent(cache, sh.batch, sh.num_kv_heads, t, elem=4 if out_fp32 else 2)
+    kp, vp = _devs("hg_dequantize_kv", (k_out, need, "k_out"), (v_out, need, "v_out"))
+    _check(library().hg_dequantize_kv(cache.handle, layer, kp, vp, 1 if out_fp32 else 0,
+                                      _stream(stream)), "hg_dequantize_kv")
 
 
 def hg_append_kv(cache, layer_begin, layer_count, k_new, v_new, stream=None):
-    _check(library().hg_append_kv(cache.handle, layer_begin, layer_count, _ptr(k_new),
-                                  _ptr(v_new), _stream(stream)), "hg_append_kv")
+    sh = cache.shape
+    need = _extent(cache, layer_count, sh.batch, sh.num_kv_heads)
+    kp, vp = _devs("hg_append_kv", (k_new, need, "k_new"), (v_new, need, "v_new"))
+    _check(library().hg_append_kv(cache.handle, layer_begin, layer_count, kp, vp,
+                                  _stream(stream)), "hg_append_kv")
 
 
 def hg_decode_workspace_size(cache, layer_count):
@@ -237,21 +273,23 @@ def hg_decode_workspace_size(cache, layer_count):
 def hg_workspace_clear(workspace, nbytes=None, stream=None):
     if nbytes is None:
         nbytes = workspace.numel() * workspace.element_size()
-    _check(library().hg_workspace_clear(_ptr(workspace), nbytes, _stream(stream)),
-           "hg_workspace_clear")
+    wp, = _devs("hg_workspace_clear", (workspace, nbytes, "workspace"))
+    _check(library().hg_workspace_clear(wp, nbytes, _stream(stream)), "hg_workspace_clear")
 
 
 def hg_workspace_status(workspace, stream=None):
     """Status word of a decode workspace (waits for the stream); 0 = healthy."""
     out = ctypes.c_uint32(0)
-    _check(library().hg_workspace_status(_ptr(workspace), ctypes.byref(out), _stream(stream)),
+    wp, = _devs("hg_workspace_status", (workspace, 4, "workspace"))
+    _check(library().hg_workspace_status(wp, ctypes.byref(out), _stream(stream)),
            "hg_workspace_status")
     return out.value
 
 
 def hg_check_bounded_wait(word, rounds, stream=None):
     """Run the bounded-wait self-check into the device word `word` (see the header)."""
-    _check(library().hg_check_bounded_wait(_ptr(word), int(rounds), _stream(stream)),
+    wp, = _devs("hg_check_bounded_wait", (word, 4, "word"))
+    _check(library().hg_check_bounded_wait(wp, int(rounds), _stream(stream)),
            "hg_check_bounded_wait")
 
 
@@ -272,10 +310,13 @@ def hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, 
                         workspace_bytes=None, stream=None):
     if workspace_bytes is None:
         workspace_bytes = workspace.numel() * workspace.element_size()
-    _check(library().hg_decode_attention(cache.handle, layer_begin, layer_count, _ptr(q),
-                                         _ptr(out), float(softmax_scale), _ptr(workspace),
-                                         workspace_bytes, _stream(stream)),
-           "hg_decode_attention")
+    sh = cache.shape
+    need = _extent(cache, layer_count, sh.batch, sh.num_q_heads)
+    qp, op, wp = _devs("hg_decode_attention", (q, need, "q"), (out, need, "out"),
+                       (workspace, workspace_bytes, "workspace"))
+    _check(library().hg_decode_attention(cache.handle, layer_begin, layer_count, qp, op,
+                                         float(softmax_scale), wp, workspace_bytes,
+                                         _stream(stream)), "hg_decode_attention")
 
 
 def hg_decode_step(cache, layer_begin, layer_count, q, k_new, v_new, out, softmax_scale, workspace,
@@ -283,16 +324,25 @@ def hg_decode_step(cache, layer_begin, layer_count, q, k_new, v_new, out, softma
     """Append the step's K/V and run decode attention including it, in one launch."""
     if workspace_bytes is None:
         workspace_bytes = workspace.numel() * workspace.element_size()
-    _check(library().hg_decode_step(cache.handle, layer_begin, layer_count, _ptr(q), _ptr(k_new),
-                                    _ptr(v_new), _ptr(out), float(softmax_scale), _ptr(workspace),
-                                    workspace_bytes, _stream(stream)), "hg_decode_step")
+    sh = cache.shape
+    nq = _extent(cache, layer_count, sh.batch, sh.num_q_heads)
+    nkv = _extent(cache, layer_count, sh.batch, sh.num_kv_heads)
+    qp, kp, vp, op, wp = _devs("hg_decode_step", (q, nq, "q"), (k_new, nkv, "k_new"),
+                               (v_new, nkv, "v_new"), (out, nq, "out"),
+                               (workspace, workspace_bytes, "workspace"))
+    _check(library().hg_decode_step(cache.handle, layer_begin, layer_count, qp, kp, vp, op,
+                                    float(softmax_scale), wp, workspace_bytes, _stream(stream)),
+           "hg_decode_step")
 
 
 def hg_decode_attention_noalloc(cache, layer_begin, layer_count, q, out, softmax_scale,
                                 stream=None):
     """Decode attention with the library's static 32 MiB scratch as workspace (no allocation)."""
-    _check(library().hg_decode_attention_noalloc(cache.handle, layer_begin, layer_count, _ptr(q),
-                                                 _ptr(out), float(softmax_scale), _stream(stream)),
+    sh = cache.shape
+    need = _extent(cache, layer_count, sh.batch, sh.num_q_heads)
+    qp, op = _devs("hg_decode_attention_noalloc", (q, need, "q"), (out, need, "out"))
+    _check(library().hg_decode_attention_noalloc(cache.handle, layer_begin, layer_count, qp, op,
+                                                 float(softmax_scale), _stream(stream)),
            "hg_decode_attention_noalloc")
 
 
