@@ -89,3 +89,33 @@ def test_raw_addresses_reach_the_library(cache):
     with pytest.raises(hg.HGError) as e:
         hg.hg_quantize_kv(cache, 0, [(1 << 40) + 8], [1 << 40], stream=0)
     assert e.value.status == 2
+
+
+@pytest.mark.parametrize("name", ["tiny", "qwen25vl7b"])
+def test_generated_inputs_pass_the_extent_checks(name):
+    """The inputs the runner, the tests and the bench hand to the binding (the
+    workload generators' shapes, whole or one layer at a time) pass every
+    extent check: on CPU the only complaint left is the device."""
+    build.build()
+    w = wl.WORKLOADS[name]
+    mask = wl.protection_mask(w).numpy()
+    sh, cf = shape_of(w), config_of(w)
+    c = hg.hg_cache_create(sh, cf, mask, 1 << 40, hg.hg_cache_layout(sh, cf, mask))
+    k, v = wl.layer_kv(w, 0, "cpu")
+    q = wl.step_query(w, 0, "cpu")
+    kn, vn = wl.step_new_kv(w, 0, "cpu")
+    out = torch.empty_like(q)
+    ws = torch.zeros(hg.hg_decode_workspace_size(c, w.layers), dtype=torch.uint8)
+    k32 = torch.empty(w.batch, w.kv_heads, w.seq_len, 128, dtype=torch.float32)
+    cuda = "must be a CUDA tensor"
+    _raises(lambda: hg.hg_quantize_kv(c, 0, [k] * w.layers, [v] * w.layers), cuda)
+    _raises(lambda: hg.hg_append_kv(c, 0, w.layers, kn, vn), cuda)
+    _raises(lambda: hg.hg_decode_attention(c, 0, w.layers, q, out, 0.0, ws), cuda)
+    _raises(lambda: hg.hg_decode_step(c, 0, w.layers, q, kn, vn, out, 0.0, ws), cuda)
+    _raises(lambda: hg.hg_decode_attention_noalloc(c, 0, w.layers, q, out, 0.0), cuda)
+    last = w.layers - 1
+    _raises(lambda: hg.hg_decode_step(c, last, 1, q[last], kn[last], vn[last], out[last], 0.0, ws),
+            cuda)
+    _raises(lambda: hg.hg_dequantize_kv(c, 0, k32, k32, True), cuda)
+    _raises(lambda: hg.hg_dequantize_kv(c, 0, k, v, False), cuda)
+    _raises(lambda: hg.hg_workspace_clear(ws), cuda)
