@@ -12,7 +12,7 @@
  *     "Applying protection");
  *   - reconstruct the cache as floating point (Sec. 4, simulated quantization:
  *     values rounded to the quantizer's levels and reconstructed as floats);
- *   - grouped-query decode attention that reads packed 2/4-bit codes and BF16
+ *   - grouped-query decode attention that reads packed 2/3/4-bit codes and BF16
  *     entries in one pass.
  *
  * Conventions shared by every entry point
@@ -32,7 +32,10 @@
  *              launched; a call that returns an error has enqueued nothing and
  *              changed no state.  HG_ERR_CUDA reports a launch error returned
  *              by the CUDA runtime (cudaGetLastError after the launch).
- *              Device code performs no waits of any kind.
+ *              The only polling waits in device code are decode CTAs waiting
+ *              on mbarriers for their own tile copies, each bounded: one that runs out
+ *              sets the workspace status word (hg_workspace_status) instead
+ *              of hanging.
  *   Threads    A hg_cache may be used from one host thread at a time.
  */
 #ifndef HEADGUARD_H
