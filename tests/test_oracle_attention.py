@@ -162,3 +162,50 @@ def test_matches_brute_force_on_tiny_shapes(oracle, B, Hq, H, T, sigma, scale):
     if T == 1:
         for qh in range(Hq):
             assert np.allclose(got[:, qh], V[:, qh * H // Hq, 0], atol=1e-15)
+
+
+def test_common_key_shift_leaves_the_output(oracle):
+    # adding one vector u to every key of a head adds sigma * <q, u> to every
+    # score of that head, which the softmax cancels
+    rng = np.random.default_rng(11)
+    K = rng.standard_normal((2, 2, 23, 128))
+    V = rng.standard_normal((2, 2, 23, 128))
+    q = _bits(rng.standard_normal((2, 6, 128)))
+    u = rng.standard_normal((2, 2, 1, 128)) * 5
+    a = oracle.attention_layer(q, K, V, 0.09)
+    b = oracle.attention_layer(q, K + u, V, 0.09)
+    assert np.allclose(a, b, atol=1e-12)
+
+
+def test_affine_in_the_values(oracle):
+    rng = np.random.default_rng(12)
+    K = rng.standard_normal((1, 2, 19, 128))
+    V = rng.standard_normal((1, 2, 19, 128))
+    q = _bits(rng.standard_normal((1, 4, 128)))
+    a = oracle.attention_layer(q, K, V, 0.1)
+    b = oracle.attention_layer(q, K, 2.5 * V - 0.75, 0.1)
+    assert np.allclose(b, 2.5 * a - 0.75, atol=1e-12)
+
+
+def test_query_scale_equals_softmax_scale(oracle):
+    # doubling q (exact in BF16) is the same as doubling sigma
+    rng = np.random.default_rng(13)
+    K = rng.standard_normal((1, 1, 31, 128))
+    V = rng.standard_normal((1, 1, 31, 128))
+    q = rng.standard_normal((1, 3, 128))
+    a = oracle.attention_layer(_bits(2 * _f32(_bits(q))), K, V, 0.07)
+    b = oracle.attention_layer(_bits(q), K, V, 0.14)
+    assert np.allclose(a, b, atol=1e-13)
+
+
+def test_replicated_heads_equal_grouped_heads(oracle):
+    # G = 1 with each KV head copied to the query heads of its group equals the
+    # grouped-query layout
+    rng = np.random.default_rng(14)
+    B, H, G, T = 2, 3, 4, 11
+    K = rng.standard_normal((B, H, T, 128))
+    V = rng.standard_normal((B, H, T, 128))
+    q = _bits(rng.standard_normal((B, H * G, 128)))
+    gqa = oracle.attention_layer(q, K, V, 0.09)
+    mha = oracle.attention_layer(q, np.repeat(K, G, axis=1), np.repeat(V, G, axis=1), 0.09)
+    assert np.array_equal(gqa, mha)
