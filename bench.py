@@ -356,6 +356,20 @@ def _workload(args):
     return w
 
 
+def workload_config(w):
+    """The line's `config` (the same for both arms): the workload by name and shape."""
+    from paper_2609_35800_gb300 import workloads as wl
+    return {"workload": w.name, "layers": w.layers, "batch": w.batch,
+            "q_heads": w.q_heads, "kv_heads": w.kv_heads,
+            "tokens": "%d text + %d image + %d text" % (w.text_prefix, w.image, w.text_suffix),
+            "base": ["minmax", "kivi", "akvq"][w.base], "bits": w.bits,
+            "keys_only": w.keys_only, "protected_heads": int(wl.protection_mask(w).sum()),
+            "decode_steps": w.decode_steps,
+            "l2": "flushed (512 MiB write + read) before every timed launch group",
+            "launch": "quantize: all layers per launch; each decode step: one launch appending the "
+                      "new K/V and attending over all layers"}
+
+
 def run_reference(args):
     from paper_2609_35800_gb300 import workloads as wl
     rank = int(os.environ.get("RANK", "0"))
@@ -378,7 +392,7 @@ def run_reference(args):
         "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
         "ms_per_step": round(1000 * tot_s / max(1, args.steps), 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "fp32/fp64", "data": "synthetic",
-        "config": {"workload": w.name, "sample": sample},
+        "config": workload_config(w),
         "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
                          "kind": "oracle", "sample": sample},
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
@@ -512,15 +526,7 @@ def run_gpu(args):
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
         "dtype": "fp32", "data": "synthetic",
-        "config": {"workload": w.name, "layers": L, "batch": w.batch,
-                   "q_heads": w.q_heads, "kv_heads": w.kv_heads,
-                   "tokens": "%d text + %d image + %d text" % (w.text_prefix, w.image,
-                                                               w.text_suffix),
-                   "base": ["minmax", "kivi", "akvq"][w.base], "bits": w.bits,
-                   "keys_only": w.keys_only, "protected_heads": int(runner.mask.sum()),
-                   "decode_steps": S, "l2": "flushed (512 MiB write + read) before every timed launch group",
-                   "launch": "quantize: all layers per launch; each decode step: one launch appending the "
-                             "new K/V and attending over all layers"},
+        "config": workload_config(w),
         "pct_of_8TBps": round(100 * value / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_hbm": round(100 * value / peak, 2),
         "decode_tokens_per_s": round(tok_s, 1),
