@@ -521,6 +521,11 @@ def run_gpu(args):
     if not args.no_e2e:
         e2e = run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream)
 
+    try:
+        deq = time_dequantize(runner, w, dec_b, dev, cushion, stream)
+    except Exception as exc:  # a side measurement never costs the line
+        deq = {"error": "%s: %s" % (type(exc).__name__, exc)}
+
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
@@ -534,6 +539,7 @@ def run_gpu(args):
             "quantize": {"ms": round(quant_ms, 4), "GBps": round(quant_b / quant_ms / 1e6, 1)},
             "decode_step (append + attention, one launch)": {"ms": round(dec_ms, 4),
                                                                "GBps": round(achieved, 1)},
+            "dequantize (all layers, not part of the step)": deq,
         },
         "step_bytes": step_bytes,
         "wall_s_timed_region": round(t_wall, 4),
@@ -625,6 +631,38 @@ def decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream):
                            "l2": "flushed before each replay of the %d-step loop only" % S}
     hg.hg_cache_reset_appended(runner.cache)
     return res
+
+
+def time_dequantize(runner, w, dec_b, dev, cushion, stream, reps=3):
+    """Reconstruction of every layer as BF16 (Sec. 4: code * scale + zero, the
+    AKVQ-style keys rotated back; text, protected and appended entries copied),
+    one launch per layer, L2 flushed before each group of L launches.  Bytes:
+    the cache entries a decode step reads (codes, metadata, BF16 rows) plus the
+    two BF16 outputs [B][H_kv][T + appended][128]."""
+    import torch
+
+    import paper_2609_35800_gb300 as hg
+    L, B, H, Hq = w.layers, w.batch, w.kv_heads, w.q_heads
+    app = hg.hg_cache_appended(runner.cache, 0)
+    q_rows = L * B * Hq * 256
+    dec_static = dec_b[0] - L * H * B * 512 - 2 * q_rows  # cache bytes without appended rows
+    tt = w.seq_len + app
+    nbytes = dec_static + L * H * B * app * 512 + L * 2 * B * H * tt * 256
+    k16 = torch.empty((B, H, tt, 128), dtype=torch.bfloat16, device=dev)
+    v16 = torch.empty_like(k16)
+    times = []
+    for _ in range(reps):
+        cushion()
+        a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for l in range(L):
+            hg.hg_dequantize_kv(runner.cache, l, k16, v16, False, stream)
+        a1.record(stream)
+        times.append((a0, a1))
+    torch.cuda.synchronize()
+    ms = statistics.mean(a.elapsed_time(b) for a, b in times)
+    return {"ms": round(ms, 4), "GBps": round(nbytes / (ms * 1e-3) / 1e9, 1), "launches": L,
+            "appended": app, "bytes": nbytes, "l2": "flushed before each group of launches"}
 
 
 def run_e2e(args, runner, w, prefill, qs, news, step_bytes, dev, stream):

@@ -25,3 +25,43 @@ def test_overrides_rename_the_workload():
     c = bench.workload_config(bench._workload(args))
     assert c["workload"] == "internvl25_8b_meta32_4layers_salient20"
     assert c["layers"] == 4 and c["base"] == "akvq" and c["bits"] == 4
+
+
+def test_dequantize_bytes_on_the_one_layer_cache(monkeypatch):
+    """The dequantize side measurement counts the cache entries a decode step
+    reads plus the two BF16 outputs; driven here on CPU with the library calls
+    and CUDA events stubbed out."""
+    import types
+
+    import torch
+
+    import bench
+    import paper_2609_35800_gb300 as hg
+    from paper_2609_35800_gb300 import build, workloads as wl
+    from paper_2609_35800_gb300.runner import config_of, shape_of
+    build.build()
+    w = wl.WORKLOADS["tiny"]
+    mask = wl.protection_mask(w).numpy()
+    sh, cf = shape_of(w), config_of(w)
+    cache = hg.hg_cache_create(sh, cf, mask, 1 << 40, hg.hg_cache_layout(sh, cf, mask))
+    runner = types.SimpleNamespace(w=w, cache=cache)
+    _, dec_b, _ = bench.geometry_bytes(runner)
+
+    calls = []
+
+    class Ev:
+        def record(self, stream):
+            pass
+
+        def elapsed_time(self, other):
+            return 0.5
+
+    monkeypatch.setattr(torch.cuda, "Event", lambda enable_timing=True: Ev())
+    monkeypatch.setattr(torch.cuda, "synchronize", lambda: None)
+    monkeypatch.setattr(hg, "hg_dequantize_kv", lambda c, l, k, v, f, s: calls.append((l, k.shape)))
+    r = bench.time_dequantize(runner, w, dec_b, "cpu", lambda: None, None)
+    # 3 quantized heads: 64 text rows + 256 coded tokens (2 x 32 code bytes,
+    # 2 x 8 metadata bytes); protected head 1: 320 BF16 rows; outputs K and V
+    want = 3 * (64 * 512 + 256 * 2 * (32 + 8)) + 320 * 512 + 2 * 4 * 320 * 256
+    assert r["bytes"] == want and r["appended"] == 0 and r["launches"] == 1
+    assert r["ms"] == 0.5 and calls == [(0, (1, 4, 320, 128))] * 3
