@@ -73,6 +73,14 @@ def _status(f, *a):
     ({}, dict(base=0, salient_permille=20), 3),
     ({}, dict(base=1, salient_permille=20), 3),
     ({}, dict(base=2, keys_only=1, salient_permille=20), 3),
+    (dict(max_new_tokens=-1), {}, 1),
+    (dict(img_start=-1), {}, 1),
+    (dict(num_layers=0), {}, 1),
+    (dict(img_len=-1), {}, 1),
+    (dict(seq_len=1 << 28, img_start=0), {}, 3),          # token index range
+    (dict(batch=20000), {}, 3),                            # batch x KV heads > grid.y
+    ({}, dict(base=1, kivi_group_channels=16), 3),
+    (dict(seq_len=60100, img_start=50, img_len=60000), dict(base=2, salient_permille=20), 3),
 ])
 def test_layout_validation(lib, shape_kw, cfg_kw, status):
     mask = np.zeros((3, max(4, shape_kw.get("num_kv_heads", 4))), np.uint8)
@@ -275,3 +283,12 @@ def test_workspace_size_grows_with_layers(lib):
 def test_status_strings(lib):
     for s in range(8):
         assert isinstance(hg.hg_status_string(s), str) and hg.hg_status_string(s)
+
+
+def test_salient_selection_size_limit(lib):
+    # one score per image token in the selection kernel's shared memory: 40000
+    # image tokens fit, 60000 do not (the case above)
+    mask = np.zeros((3, 4), np.uint8)
+    n = hg.hg_cache_layout(_shape(seq_len=40100, img_start=50, img_len=40000),
+                           _cfg(base=2, salient_permille=20), mask)
+    assert n > 0
