@@ -174,7 +174,8 @@ hg_status hg_cache_layout(const hg_shape *shape, const hg_quant_config *config,
 
 /* Create the descriptor of a cache stored in `arena` (device, 256-byte aligned,
  * at least hg_cache_layout bytes; its contents need no initialisation).  The
- * descriptor copies shape, config and mask.  Host only; no CUDA call.
+ * descriptor copies shape, config and mask (the fixed head set chosen offline,
+ * Sec. 3).  Host only; no CUDA call.
  * The arena must outlive the descriptor's use; hg_cache_destroy frees only the
  * descriptor. */
 hg_status hg_cache_create(const hg_shape *shape, const hg_quant_config *config,
@@ -182,14 +183,18 @@ hg_status hg_cache_create(const hg_shape *shape, const hg_quant_config *config,
                           hg_cache **out);
 void hg_cache_destroy(hg_cache *cache);
 
-/* Region map of one (layer, head).  Host only. */
+/* Region map of one (layer, head): where its BF16 rows, codes and metadata sit
+ * in the arena.  The packed layout is this library's (the paper stores no
+ * packed cache, Sec. 4).  Host only. */
 hg_status hg_cache_head_regions(const hg_cache *cache, int32_t layer, int32_t head,
                                 hg_head_regions *out);
 
-/* Number of decode tokens appended so far to `layer` (host state). */
+/* Number of decode tokens appended so far to `layer` (host state; generated
+ * tokens are text and stay BF16, Sec. 3). */
 int32_t hg_cache_appended(const hg_cache *cache, int32_t layer);
 
-/* Forget appended tokens (all layers); device memory is not touched. */
+/* Forget appended tokens (all layers); device memory is not touched.  (Cache
+ * bookkeeping; the paper has no counterpart.) */
 hg_status hg_cache_reset_appended(hg_cache *cache);
 
 /* Quantize-pack layers [layer_begin, layer_begin + layer_count) from their BF16
@@ -218,12 +223,15 @@ hg_status hg_append_kv(hg_cache *cache, int32_t layer_begin, int32_t layer_count
                        const void *k_new, const void *v_new, hg_stream_t stream);
 
 /* Workspace bytes hg_decode_attention needs for a launch over layer_count
- * layers (any appended count up to max_new_tokens). */
+ * layers (any appended count up to max_new_tokens).  The workspace holds the
+ * split-K partials of the decode kernel (a GPU work decomposition; the paper
+ * has no counterpart). */
 hg_status hg_decode_workspace_size(const hg_cache *cache, int32_t layer_count, size_t *bytes);
 
-/* Zero a workspace (cudaMemsetAsync).  Required once before its first use;
- * decode attention leaves it zeroed again on completion.  Layout: a 512-byte
- * header holding a status word at byte 0, split counters, split partials. */
+/* Zero a workspace (cudaMemsetAsync; no counterpart in the paper).  Required
+ * once before its first use; decode attention leaves it zeroed again on
+ * completion.  Layout: a 512-byte header holding a status word at byte 0,
+ * split counters, split partials. */
 hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
 
 /* Health of the decode launches that used a workspace: waits for `stream`,
@@ -250,7 +258,10 @@ hg_status hg_check_bounded_wait(void *word, uint32_t rounds, hg_stream_t stream)
 
 /* Grouped-query decode attention of one step over layers
  * [layer_begin, +layer_count), reading packed codes and BF16 entries in one
- * pass.  q: device BF16 [layer_count][batch][num_q_heads][128]; out: device
+ * pass: attention over the mixed-precision cache of Sec. 3 (protected and text
+ * entries BF16, the other image entries the base quantizer's reconstruction,
+ * which Sec. 4 feeds to attention as floating point; here the codes enter the
+ * contraction directly).  q: device BF16 [layer_count][batch][num_q_heads][128]; out: device
  * BF16, same shape.  Query head qh attends with KV head qh / G over every
  * token of that head (prefill text, image, appended), with
  * score = softmax_scale * <q, k>; softmax_scale <= 0 selects 1/sqrt(128).
@@ -260,9 +271,9 @@ hg_status hg_decode_attention(const hg_cache *cache, int32_t layer_begin, int32_
                               const void *q, void *out, float softmax_scale,
                               void *workspace, size_t workspace_bytes, hg_stream_t stream);
 
-/* One decode step in one launch: append the step's K/V (as hg_append_kv) and
- * run grouped-query decode attention over every token including the new one
- * (as hg_decode_attention).  k_new / v_new: device BF16
+/* One decode step in one launch: append the step's K/V (as hg_append_kv; text,
+ * BF16, Sec. 3) and run grouped-query decode attention over every token
+ * including the new one (as hg_decode_attention, Sec. 3 / Sec. 4).  k_new / v_new: device BF16
  * [layer_count][batch][num_kv_heads][128]; the other arguments as for
  * hg_decode_attention.  The work item that holds the new position reads it
  * from k_new / v_new and also stores it into the cache.  Returns
@@ -316,7 +327,7 @@ hg_status hg_cache_image_bits_per_elem(const hg_cache *cache, double *bits);
 hg_status hg_select_heads(const float *g_scores, const float *o_scores, int32_t num_layers,
                           int32_t num_q_heads, int32_t num_kv_heads, int32_t k, uint8_t *mask_out);
 
-/* Static description of a status code. */
+/* Static description of a status code (no counterpart in the paper). */
 const char *hg_status_string(hg_status status);
 
 #ifdef __cplusplus
