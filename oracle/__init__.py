@@ -8,7 +8,7 @@ import this package; the product library never does.
 
 Every function cites the paper passage it follows (section numbers of
 "HeadGuard: Selective Head Protection for Low-Bit VLM KV-Cache
-Quantization"); the readings R1-R12 are stated in ``hg_oracle.c``.
+Quantization"); the readings R1-R16 are stated in ``hg_oracle.c``.
 """
 import ctypes
 import os

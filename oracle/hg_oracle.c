@@ -41,6 +41,7 @@
  *      zero are stored as binary16 (round to nearest even, magnitudes above
  *      65504 saturate to 65504), and the codes are computed against the
  *      stored values, so reconstruction uses exactly what is stored.
+ *   R14 one contiguous image span [s, s + n), the same for every batch row.
  *   R15 AKVQ-style salient tokens (Sec. 4, optional): in each (batch row, KV
  *      head) whose image keys are quantized, the keys and values of the ns
  *      image tokens with the largest squared key norm stay BF16, ties to the
