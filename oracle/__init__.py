@@ -204,9 +204,10 @@ def quantize_layer(k_bits, v_bits, s, n, base, bits, head_mask, keys_only,
     Returns a dict with per-(b,h) arrays:
       nq, kq, vq [B,H,T], k_words [B,H,...], k_meta, v_words, v_meta (shapes as
       documented in hg_oracle.c), k_deq, v_deq [B,H,T,128] fp32, k_att fp64.
-    n_salient > 0 (R15): heads with quantized keys keep that many image tokens
-    BF16 (indices in salient [B,H,n_salient]); their codes and metadata fill
-    the first nq - n_salient token slots.
+    n_salient > 0 (R15): every head that is not protected K+V keeps that many
+    image tokens' keys and values BF16 (indices in salient [B,H,n_salient]; a
+    K-only protected head's image keys are BF16 anyway); their codes and
+    metadata fill the first nq - n_salient token slots.
     """
     k_bits = _c(k_bits, np.uint16)
     v_bits = _c(v_bits, np.uint16)

@@ -43,14 +43,19 @@
  *      stored values, so reconstruction uses exactly what is stored.
  *   R14 one contiguous image span [s, s + n), the same for every batch row.
  *   R15 AKVQ-style salient tokens (Sec. 4, optional): in each (batch row, KV
- *      head) whose image keys are quantized, the keys and values of the ns
- *      image tokens with the largest squared key norm stay BF16, ties to the
- *      lower token index; ns = ceil(n * permille / 1000) ("a nominal 2%" is
- *      permille 20).  The norm is taken on the unrotated BF16 key in binary32
- *      in the fixed order of hgo_key_norm2, so that both implementations rank
- *      the same values.  The remaining image tokens are quantized in order and
- *      stored compacted.  Built for the AKVQ-style base without K-only
- *      protection.
+ *      head) that is not protected K+V, the keys and values of the ns image
+ *      tokens with the largest squared key norm stay BF16, ties to the lower
+ *      token index; ns = ceil(n * permille / 1000) ("a nominal 2%" is
+ *      permille 20).  Sec. 4 keeps salient tokens whether or not a head is
+ *      protected, so under K-only protection a protected head (whose image keys are BF16
+ *      already) keeps its salient tokens' values BF16 and codes the rest of
+ *      its image values.  The norm is taken on the unrotated BF16 key in
+ *      binary32 in the fixed order of hgo_key_norm2, so that both
+ *      implementations rank the same values.  The remaining image tokens are
+ *      quantized in order and stored compacted.  Built for the per-token
+ *      bases (the paper's salient tokens belong to the AKVQ-style base; the
+ *      KIVI-style key groups of 32 consecutive tokens leave no room for
+ *      them).
  *   R16 3-bit codes (the paper's 3-bit setting, Sec. 4 / Tab. 1): a group of
  *      n codes (n a multiple of 32) is stored as n/16 words holding bits 0-1
  *      of every code in the 2-bit packing, then n/32 words holding bit 2 of
@@ -326,11 +331,13 @@ float hgo_key_norm2(const uint16_t *krow);
 void hgo_select_salient(const float *score, int n, int ns, int32_t *idx);
 
 /*
- * n_salient > 0 (R15; per-token bases without K-only protection): for a head
- * whose image keys are quantized, the n_salient image tokens of largest key
+ * n_salient > 0 (R15; per-token bases): for a head that is not protected K+V
+ * (its image values are quantized), the n_salient image tokens of largest key
  * norm keep BF16 keys and values, their image-relative indices go to
  * `salient` (ascending), and the other image tokens are quantized in order
- * into the first nq - n_salient slots of the code and metadata arrays.
+ * into the first nq - n_salient slots of the code and metadata arrays.  A
+ * K-only protected head keeps every image key BF16, so only its values are
+ * affected.
  */
 int hgo_quantize_head_s(const uint16_t *k, const uint16_t *v, int T, int s, int n,
                         int base, int bits, int meta16, int protect, int keys_only,
@@ -351,7 +358,7 @@ int hgo_quantize_head_s(const uint16_t *k, const uint16_t *v, int T, int s, int 
 
     /* R15: which image tokens stay BF16 (sal[i] for image token s + i) */
     uint8_t *sal = (uint8_t *)calloc((size_t)(nq > 0 ? nq : 1), 1);
-    if (n_salient > 0 && quant_k && !keys_only && base != HGO_BASE_KIVI && nq > 0) {
+    if (n_salient > 0 && quant_v && base != HGO_BASE_KIVI && nq > 0) {
         float *score = (float *)malloc(sizeof(float) * (size_t)nq);
         for (int i = 0; i < nq; ++i) score[i] = hgo_key_norm2(k + (long)(s + i) * D);
         hgo_select_salient(score, nq, n_salient, salient);
@@ -539,7 +546,7 @@ int hgo_quantize_layer_s(const uint16_t *k, const uint16_t *v, int B, int H, int
     const int D = HGO_D;
     const int nq = hgo_quantized_count(T, s, n, base, group_tokens, residual);
     if (n_salient < 0 || n_salient > nq) return -1;
-    if (n_salient > 0 && (keys_only || base == HGO_BASE_KIVI)) return -1; /* R15 */
+    if (n_salient > 0 && base == HGO_BASE_KIVI) return -1; /* R15: per-token bases only */
     const long kw = (long)nq * D * bits / 32;
     const long km = (base == HGO_BASE_KIVI) ? (long)(nq / group_tokens) * D * 2 : (long)nq * 2;
     const long vm = (base == HGO_BASE_KIVI) ? (long)nq * (D / group_channels) * 2 : (long)nq * 2;

@@ -168,8 +168,101 @@ def test_unsupported_combinations_are_rejected(oracle):
     rng = np.random.default_rng(1)
     k = _bf16_bits(rng, (1, 2, 80, 128))
     v = _bf16_bits(rng, (1, 2, 80, 128))
-    with pytest.raises(ValueError):  # K-only protection
-        oracle.quantize_layer(k, v, 4, 64, 2, 2, np.array([0, 1], np.uint8), 1, n_salient=2)
     with pytest.raises(ValueError):  # KIVI-style groups
         oracle.quantize_layer(k, v, 4, 64, 1, 2, np.array([0, 1], np.uint8), 0, residual=0,
                               n_salient=2)
+
+
+# --------------------------------------------------------------------------
+# K-only protection (Sec. 4 keeps salient tokens whether or not a head is
+# protected; a K-only protected head keeps its image keys BF16, so only its
+# salient tokens' values are kept BF16 -- reading R15)
+# --------------------------------------------------------------------------
+
+def test_keys_only_hand_example(oracle):
+    """One K-only protected head, 8 text + 64 image + 8 text tokens, 4 salient
+    tokens (permille 50: ceil(3.2)).  Image keys are zero except tokens 3, 17,
+    40, 41 (image-relative), whose channel 5 holds 6, 9, 7, 8: those four are
+    the salient ones.  Their values stay BF16; image token 4 is the fourth
+    coded value (slot 3), token 18 slot 16, token 42 slot 38."""
+    T, s, n = 80, 8, 64
+    k = np.zeros((1, 1, T, 128), np.int64)
+    for i, x in ((3, 6), (17, 9), (40, 7), (41, 8)):
+        k[0, 0, s + i, 5] = x
+    k[0, 0, :s, :] = 50  # text keys are not ranked: only image tokens are candidates
+    kb = _bf16_of_int(k)
+    rng = np.random.default_rng(12)
+    v = _bf16_bits(rng, (1, 1, T, 128))
+    ns = oracle.salient_count(n, 50)
+    assert ns == 4
+    o = oracle.quantize_layer(kb, v, s, n, 2, 4, np.array([1], np.uint8), 1, n_salient=ns)
+    assert list(o["salient"][0, 0]) == [3, 17, 40, 41]
+    assert not o["kq"].any()                                   # every key BF16
+    assert np.array_equal(o["k_deq"][0, 0], _f32(kb[0, 0]))
+    for i in (3, 17, 40, 41):
+        assert o["vq"][0, 0, s + i] == 0
+        assert np.array_equal(o["v_deq"][0, 0, s + i], _f32(v[0, 0, s + i]))
+    W = 16  # 4-bit words per 128-channel token
+    for i, slot in ((0, 0), (4, 3), (18, 16), (42, 38), (63, 59)):
+        assert o["vq"][0, 0, s + i] == 1
+        codes, sc, z = oracle.quantize_group(_f32(v[0, 0, s + i]), 4)
+        assert np.array_equal(o["v_words"][0, 0][slot * W:(slot + 1) * W], oracle.pack(codes, 4))
+        assert o["v_meta"][0, 0][2 * slot] == sc and o["v_meta"][0, 0][2 * slot + 1] == z
+
+
+@pytest.mark.parametrize("base,bits", [(2, 4), (2, 2), (0, 2), (2, 3)])
+def test_keys_only_selection_and_compacted_values(oracle, base, bits):
+    """Every head with coded values (quantized heads and K-only protected heads)
+    ranks its image tokens by exact integer key norms; the salient tokens keep
+    BF16 keys and values and the rest is the base on the compacted sequence
+    (for a K-only protected head: values only, every key BF16)."""
+    mask = np.array([0, 1, 0, 1], np.uint8)
+    B, H, T, s, n = 2, 4, 150, 11, 128
+    rng = np.random.default_rng(20 + bits)
+    k = _bf16_of_int(rng.integers(-7, 8, (B, H, T, 128)))
+    v = _bf16_bits(rng, (B, H, T, 128))
+    ns = oracle.salient_count(n, 40)
+    assert ns == 6
+    o = oracle.quantize_layer(k, v, s, n, base, bits, mask, 1, n_salient=ns)
+    W = 128 * bits // 32
+    nc = n - ns
+    for b in range(B):
+        for h in range(H):
+            norms = (_f32(k[b, h, s:s + n]).astype(np.int64) ** 2).sum(axis=1)
+            order = sorted(range(n), key=lambda i: (-norms[i], i))
+            sal = o["salient"][b, h]
+            assert list(sal) == sorted(order[:ns])
+            keep = np.setdiff1d(np.arange(n), sal)
+            for i in sal:
+                assert o["vq"][b, h, s + i] == 0 and o["kq"][b, h, s + i] == 0
+                assert np.array_equal(o["v_deq"][b, h, s + i], _f32(v[b, h, s + i]))
+                assert np.array_equal(o["k_deq"][b, h, s + i], _f32(k[b, h, s + i]))
+            toks = np.concatenate([np.arange(s), s + keep, np.arange(s + n, T)])
+            r = oracle.quantize_layer(k[b:b + 1, h:h + 1][:, :, toks], v[b:b + 1, h:h + 1][:, :, toks],
+                                      s, nc, base, bits, mask[h:h + 1], 1)
+            assert np.array_equal(o["v_words"][b, h][:nc * W], r["v_words"][0, 0][:nc * W])
+            assert np.array_equal(o["v_meta"][b, h][:nc * 2], r["v_meta"][0, 0][:nc * 2])
+            assert np.array_equal(o["v_deq"][b, h][toks], r["v_deq"][0, 0])
+            assert np.array_equal(o["k_deq"][b, h][toks], r["k_deq"][0, 0])
+            if mask[h]:
+                assert not o["kq"][b, h].any()
+                assert np.array_equal(o["k_deq"][b, h], _f32(k[b, h]))
+            else:
+                assert np.array_equal(o["k_words"][b, h][:nc * W], r["k_words"][0, 0][:nc * W])
+                assert np.array_equal(o["k_meta"][b, h][:nc * 2], r["k_meta"][0, 0][:nc * 2])
+                assert np.all(o["kq"][b, h, s + keep] == 1)
+
+
+def test_keys_only_all_protected_matches_k_plus_v_values(oracle):
+    """With every head K-only protected, the values (and their salient tokens)
+    are exactly those of the quantized heads of a K+V-free mask: the selection
+    depends on the keys only, never on the protection of the keys."""
+    rng = np.random.default_rng(31)
+    B, H, T, s, n = 1, 3, 90, 5, 70
+    k = _bf16_bits(rng, (B, H, T, 128))
+    v = _bf16_bits(rng, (B, H, T, 128))
+    ns = oracle.salient_count(n, 20)
+    a = oracle.quantize_layer(k, v, s, n, 2, 4, np.ones(H, np.uint8), 1, n_salient=ns)
+    q = oracle.quantize_layer(k, v, s, n, 2, 4, np.zeros(H, np.uint8), 0, n_salient=ns)
+    for key in ("salient", "v_words", "v_meta", "v_deq", "vq"):
+        assert np.array_equal(a[key], q[key]), key
