@@ -98,12 +98,13 @@ typedef struct hg_shape {
  * pair; 32 = a binary16 pair, the Sec. 5.4 storage model (2.25 bits per element
  * at 2 bits): scale and zero are rounded to nearest-even binary16 (magnitudes
  * >= 65504 saturate) and the codes are computed against the stored values.
- * salient_permille (0 = off; AKVQ-style base without keys_only, else
- * HG_ERR_UNSUPPORTED): Sec. 4's salient tokens.  In every (batch row, KV head)
- * whose image keys are quantized, ceil(nq * salient_permille / 1000) image
- * tokens (20: the paper's nominal 2%) with the largest squared norm of the
- * unrotated BF16 key keep BF16 keys and values; ties go to the lower token
- * index.  The squared norm is summed in binary32 in a fixed order: 32 partial
+ * salient_permille (0 = off; AKVQ-style base only, else HG_ERR_UNSUPPORTED):
+ * Sec. 4's salient tokens, kept whether or not a head is protected.  In every
+ * (batch row, KV head) that is not protected K+V, ceil(nq * salient_permille /
+ * 1000) image tokens (20: the paper's nominal 2%) with the largest squared
+ * norm of the unrotated BF16 key keep BF16 keys and values (a keys-only
+ * protected head keeps every image key BF16 anyway, so there only its salient
+ * values change); ties go to the lower token index.  The squared norm is summed in binary32 in a fixed order: 32 partial
  * sums of channels 4l..4l+3, ((x0^2 + x1^2) + x2^2) + x3^2, then five rounds
  * in which partial l adds partial (l xor m), m = 16, 8, 4, 2, 1.  The other
  * image tokens are coded in order, compacted. */
@@ -145,8 +146,10 @@ typedef enum hg_head_class {
  *   vq / vqm  value codes [batch][nq][4*bits] (channel order), metadata
  *             [batch][nq][groups], groups = 1 (per token) or 4 (KIVI-style,
  *             channels 32j..32j+31).
- *   kimg      BF16 [batch][nq][128] image keys of a keys-only protected head.
- *   sal       salient-token map of a quantized head (salient tokens only):
+ *   kimg      BF16 [batch][n_coded][128] image keys of a keys-only protected
+ *             head (with salient tokens: those of the coded tokens, compacted;
+ *             the salient tokens' keys sit in kb).
+ *   sal       salient-token map of a head with coded values (salient tokens only):
  *             per batch row uint32 [ceil(nq/32)] (bit j of word w: image
  *             token 32w + j is salient), then int32 [ceil(nq/32)] (salient
  *             tokens before block w), row stride sal_bstride.
@@ -154,7 +157,7 @@ typedef enum hg_head_class {
  * except for KIVI-style, where only whole 32-token groups inside
  * [img_start, min(img_start + img_len, seq_len - kivi_residual)) are coded.
  * The code and metadata arrays hold n_coded tokens (nq less the n_salient
- * salient tokens of a quantized head), in token order. */
+ * salient tokens of a head with coded values), in token order. */
 typedef struct hg_head_regions {
     int32_t head_class;
     int32_t nq;
@@ -207,13 +210,15 @@ hg_status hg_cache_reset_appended(hg_cache *cache);
 hg_status hg_quantize_kv(hg_cache *cache, int32_t layer_begin, int32_t layer_count,
                          const void *const *k, const void *const *v, hg_stream_t stream);
 
-/* Reconstruct one layer as floating point (Sec. 4: code * scale + zero, the
- * AKVQ-style keys rotated back).  k_out / v_out: device
- * [batch][num_kv_heads][seq_len + appended][128], fp32 when out_fp32 != 0, else
- * BF16 (round to nearest even), tokens in original order followed by the
- * appended ones.  BF16 entries are copied exactly. */
-hg_status hg_dequantize_kv(const hg_cache *cache, int32_t layer, void *k_out, void *v_out,
-                           int32_t out_fp32, hg_stream_t stream);
+/* Reconstruct layers [layer_begin, layer_begin + layer_count) as floating
+ * point (Sec. 4: code * scale + zero, the AKVQ-style keys rotated back).
+ * k_out / v_out: device [layer_count][batch][num_kv_heads][seq_len + appended][128],
+ * fp32 when out_fp32 != 0, else BF16 (round to nearest even), tokens in
+ * original order followed by the appended ones.  BF16 entries are copied
+ * exactly.  Every layer of the range must hold the same number of appended
+ * tokens (HG_ERR_INVALID_ARG otherwise); one launch per 64 layers. */
+hg_status hg_dequantize_kv(const hg_cache *cache, int32_t layer_begin, int32_t layer_count,
+                           void *k_out, void *v_out, int32_t out_fp32, hg_stream_t stream);
 
 /* Append one decode token's K/V to layers [layer_begin, +layer_count) (text
  * tokens stay BF16, Sec. 3).  k_new / v_new: device BF16
@@ -231,7 +236,9 @@ hg_status hg_decode_workspace_size(const hg_cache *cache, int32_t layer_count, s
 /* Zero a workspace (cudaMemsetAsync; no counterpart in the paper).  Required
  * once before its first use; decode attention leaves it zeroed again on
  * completion.  Layout: a 512-byte header holding a status word at byte 0,
- * split counters, split partials. */
+ * split counters, split partials.  workspace NULL: clear the status word of
+ * the scratch array hg_decode_attention_noalloc uses on the current device
+ * (`bytes` is ignored). */
 hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
 
 /* Health of the decode launches that used a workspace: waits for `stream`,
@@ -241,8 +248,11 @@ hg_status hg_workspace_clear(void *workspace, size_t bytes, hg_stream_t stream);
  * let the copies it had issued land before exiting.  Decode CTAs wait with a
  * bound instead of hanging; after a non-zero status the outputs of the
  * launches since the last clear are undefined and the workspace must be
- * cleared (hg_workspace_clear) before it is used again.  (Failure detection
- * of the kernels; the paper has no counterpart.) */
+ * cleared (hg_workspace_clear) before it is used again.  workspace NULL: the
+ * status word of the scratch array hg_decode_attention_noalloc uses on the
+ * current device, which collects the failures of every allocation-free call
+ * since it was last cleared with hg_workspace_clear(NULL, 0, stream).
+ * (Failure detection of the kernels; the paper has no counterpart.) */
 hg_status hg_workspace_status(const void *workspace, uint32_t *status, hg_stream_t stream);
 
 /* Self-check of the bounded wait that guards every decode tile (failure
@@ -298,9 +308,15 @@ hg_status hg_decode_step(hg_cache *cache, int32_t layer_begin, int32_t layer_cou
  *   Set-up    the first call on a device (with that device current) looks up
  *             the array's device address with cudaGetSymbolAddress; make that
  *             first call before any stream capture.
- *   Sharing   every call uses the same array and clears the part it needs
+ *   Sharing   every call uses the same array and clears its split counters
  *             (cudaMemsetAsync) before launching; calls that overlap on the
  *             GPU (different streams, or threads on the same device) race.
+ *   Errors    the argument checks and the size limit run before anything is
+ *             enqueued.  A bounded wait that runs out (see Errors above) sets
+ *             the array's status word, which later calls leave set: read it
+ *             with hg_workspace_status(NULL, &status, stream) and reset it
+ *             with hg_workspace_clear(NULL, 0, stream); a non-zero word means
+ *             the outputs of the calls since the last reset are undefined.
  * No cudaMalloc, cudaFree or other allocating routine is called. */
 hg_status hg_decode_attention_noalloc(const hg_cache *cache, int32_t layer_begin,
                                       int32_t layer_count, const void *q, void *out,

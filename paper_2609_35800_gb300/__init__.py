@@ -99,7 +99,7 @@ def library():
         "hg_cache_appended": ([P, i32], i32),
         "hg_cache_reset_appended": ([P], st),
         "hg_quantize_kv": ([P, i32, i32, P, P, P], st),
-        "hg_dequantize_kv": ([P, i32, P, P, i32, P], st),
+        "hg_dequantize_kv": ([P, i32, i32, P, P, i32, P], st),
         "hg_append_kv": ([P, i32, i32, P, P, P], st),
         "hg_decode_workspace_size": ([P, i32, ctypes.POINTER(sz)], st),
         "hg_workspace_clear": ([P, sz, P], st),
@@ -246,13 +246,15 @@ def hg_quantize_kv(cache, layer_begin, k_list, v_list, stream=None):
            "hg_quantize_kv")
 
 
-def hg_dequantize_kv(cache, layer, k_out, v_out, out_fp32, stream=None):
+def hg_dequantize_kv(cache, layer_begin, layer_count, k_out, v_out, out_fp32, stream=None):
+    """Reconstruct layers [layer_begin, +layer_count) into k_out / v_out
+    [layer_count][B][H_kv][T + appended][128] (fp32 or BF16)."""
     sh = cache.shape
-    t = sh.seq_len + max(hg_cache_appended(cache, layer), 0)
-    need = _extent(cache, sh.batch, sh.num_kv_heads, t, elem=4 if out_fp32 else 2)
+    t = sh.seq_len + max(hg_cache_appended(cache, layer_begin), 0)
+    need = _extent(cache, layer_count, sh.batch, sh.num_kv_heads, t, elem=4 if out_fp32 else 2)
     kp, vp = _devs("hg_dequantize_kv", (k_out, need, "k_out"), (v_out, need, "v_out"))
-    _check(library().hg_dequantize_kv(cache.handle, layer, kp, vp, 1 if out_fp32 else 0,
-                                      _stream(stream)), "hg_dequantize_kv")
+    _check(library().hg_dequantize_kv(cache.handle, layer_begin, layer_count, kp, vp,
+                                      1 if out_fp32 else 0, _stream(stream)), "hg_dequantize_kv")
 
 
 def hg_append_kv(cache, layer_begin, layer_count, k_new, v_new, stream=None):
@@ -271,14 +273,20 @@ def hg_decode_workspace_size(cache, layer_count):
 
 
 def hg_workspace_clear(workspace, nbytes=None, stream=None):
-    if nbytes is None:
+    """Zero a decode workspace; workspace None clears the status word of the
+    allocation-free entry point's scratch on the current device."""
+    if workspace is None:
+        nbytes = 0
+    elif nbytes is None:
         nbytes = workspace.numel() * workspace.element_size()
     wp, = _devs("hg_workspace_clear", (workspace, nbytes, "workspace"))
     _check(library().hg_workspace_clear(wp, nbytes, _stream(stream)), "hg_workspace_clear")
 
 
 def hg_workspace_status(workspace, stream=None):
-    """Status word of a decode workspace (waits for the stream); 0 = healthy."""
+    """Status word of a decode workspace (waits for the stream); 0 = healthy.
+    workspace None: the status word of the allocation-free entry point's scratch
+    on the current device."""
     out = ctypes.c_uint32(0)
     wp, = _devs("hg_workspace_status", (workspace, 4, "workspace"))
     _check(library().hg_workspace_status(wp, ctypes.byref(out), _stream(stream)),

@@ -56,10 +56,9 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   if (c->keys_only != 0 && c->keys_only != 1) return HG_ERR_INVALID_ARG;
   if (c->meta_bits != 0 && c->meta_bits != 32 && c->meta_bits != 64) return HG_ERR_INVALID_ARG;
   if (c->salient_permille < 0 || c->salient_permille > 1000) return HG_ERR_INVALID_ARG;
-  // salient tokens (Sec. 4) belong to the AKVQ-style base; K-only protection
-  // would keep salient values of protected heads BF16 too, which is not built
-  if (c->salient_permille > 0 && (c->base != HG_BASE_AKVQ_HADAMARD || c->keys_only))
-    return HG_ERR_UNSUPPORTED;
+  // salient tokens (Sec. 4) belong to the AKVQ-style base (with K+V or K-only
+  // protection)
+  if (c->salient_permille > 0 && c->base != HG_BASE_AKVQ_HADAMARD) return HG_ERR_UNSUPPORTED;
   if (c->base == HG_BASE_KIVI) {
     if (c->kivi_group_tokens != kKiviGroup || c->kivi_group_channels != kKiviGroup)
       return HG_ERR_UNSUPPORTED;
@@ -198,7 +197,7 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
       if (cls == kProtected) {
         total += d.T * sb.bf16;
       } else {
-        const int nc = cls == kKeysOnly ? d.nq : ncoded(d);
+        const int nc = ncoded(d);
         total += (d.T - nc) * sb.bf16 + nc * (cls == kKeysOnly ? sb.coded_k : sb.coded_u);
       }
     }
@@ -213,13 +212,14 @@ DecodePlan plan_decode(const hg_cache* c, int begin, int count) {
   for (int iter = 0; iter < 64; ++iter, item *= 1.05) {
     p.cbU = chunk_tokens(d.T - ncoded(d) + d.S_new, sb.bf16, item, 64);
     p.cqU = chunk_tokens(ncoded(d), sb.coded_u, item, 64);
-    p.cqK = chunk_tokens(d.nq, sb.coded_k, item, 64);
+    p.cqK = chunk_tokens(ncoded(d), sb.coded_k, item, 64);
     p.cbP = chunk_tokens(d.T + d.S_new, sb.bf16, item, 64);
     long long items = 0;
     for (int l = begin; l < begin + count; ++l)
       items += (long long)d.B * row_chunks(d, c->layer_mask[l], counts_of(d, d.S_new, p));
     if (items <= wave) break;
-    if (p.cbU >= d.T - ncoded(d) + d.S_new && p.cqU >= ncoded(d) && p.cqK >= d.nq && p.cbP >= d.T + d.S_new)
+    if (p.cbU >= d.T - ncoded(d) + d.S_new && p.cqU >= ncoded(d) && p.cqK >= ncoded(d) &&
+        p.cbP >= d.T + d.S_new)
       break;
   }
   // The merging CTA stages every split's partial of a head in its stage buffer.
@@ -381,8 +381,8 @@ hg_status hg_cache_head_regions(const hg_cache* c, int32_t layer, int32_t head, 
   out->kimg_bstride = hd.kimg_bs;
   out->sal = abs(hd.sal);
   out->sal_bstride = hd.sal_bs;
-  out->n_coded = hd.cls == kProtected ? 0 : (hd.cls == kKeysOnly ? c->d.nq : ncoded(c->d));
-  out->n_salient = hd.cls == kQuantized ? c->d.ns : 0;
+  out->n_coded = hd.cls == kProtected ? 0 : ncoded(c->d);
+  out->n_salient = hd.cls == kProtected ? 0 : c->d.ns;
   return HG_OK;
 }
 
@@ -430,21 +430,31 @@ hg_status hg_quantize_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count,
   return HG_OK;
 }
 
-hg_status hg_dequantize_kv(const hg_cache* c, int32_t layer, void* k_out, void* v_out,
-                           int32_t out_fp32, hg_stream_t stream) {
-  if (!range_ok(c, layer, 1) || !k_out || !v_out) return HG_ERR_INVALID_ARG;
+hg_status hg_dequantize_kv(const hg_cache* c, int32_t layer_begin, int32_t layer_count, void* k_out,
+                           void* v_out, int32_t out_fp32, hg_stream_t stream) {
+  if (!range_ok(c, layer_begin, layer_count) || !k_out || !v_out) return HG_ERR_INVALID_ARG;
   if (!aligned16(k_out) || !aligned16(v_out)) return HG_ERR_ALIGNMENT;
-  DequantParams p;
-  std::memset(&p, 0, sizeof p);
-  p.d = c->d;
-  p.arena = c->arena;
-  p.layer_base = c->layer_base[layer];
-  p.mask = c->layer_mask[layer];
-  p.appended = c->appended[layer];
-  p.out_fp32 = out_fp32 ? 1 : 0;
-  p.k_out = k_out;
-  p.v_out = v_out;
-  return cuda_status(launch_dequantize(p, reinterpret_cast<cudaStream_t>(stream)));
+  const int appended = c->appended[layer_begin];
+  for (int i = 1; i < layer_count; ++i)
+    if (c->appended[layer_begin + i] != appended) return HG_ERR_INVALID_ARG;
+  const Dims& d = c->d;
+  const size_t layer_bytes = (size_t)d.B * d.H * (size_t)(d.T + appended) * kD * (out_fp32 ? 4 : 2);
+  for (int done = 0; done < layer_count; done += kMaxLayersPerLaunch) {
+    const int n = std::min(kMaxLayersPerLaunch, layer_count - done);
+    DequantParams p;
+    std::memset(&p, 0, sizeof p);
+    p.d = d;
+    p.arena = c->arena;
+    p.n_layers = n;
+    fill_table(c, layer_begin + done, n, &p.lt);
+    p.appended = appended;
+    p.out_fp32 = out_fp32 ? 1 : 0;
+    p.k_out = static_cast<char*>(k_out) + (size_t)done * layer_bytes;
+    p.v_out = static_cast<char*>(v_out) + (size_t)done * layer_bytes;
+    const hg_status st = cuda_status(launch_dequantize(p, reinterpret_cast<cudaStream_t>(stream)));
+    if (st != HG_OK) return st;
+  }
+  return HG_OK;
 }
 
 hg_status hg_append_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count, const void* k_new,
@@ -487,7 +497,14 @@ hg_status hg_decode_workspace_size(const hg_cache* c, int32_t layer_count, size_
 }
 
 hg_status hg_workspace_clear(void* ws, size_t bytes, hg_stream_t stream) {
-  if (!ws) return HG_ERR_INVALID_ARG;
+  if (!ws) {
+    // the allocation-free entry point's scratch: its header (status word);
+    // its split counters are cleared by every call
+    void* scratch = nullptr;
+    const hg_status st = noalloc_scratch_address(&scratch);
+    if (st != HG_OK) return st;
+    return cuda_status(cudaMemsetAsync(scratch, 0, kWsHeaderBytes, reinterpret_cast<cudaStream_t>(stream)));
+  }
   return cuda_status(cudaMemsetAsync(ws, 0, bytes, reinterpret_cast<cudaStream_t>(stream)));
 }
 
@@ -501,7 +518,13 @@ hg_status hg_check_bounded_wait(void* word, uint32_t rounds, hg_stream_t stream)
 }
 
 hg_status hg_workspace_status(const void* ws, uint32_t* status, hg_stream_t stream) {
-  if (!ws || !status) return HG_ERR_INVALID_ARG;
+  if (!status) return HG_ERR_INVALID_ARG;
+  if (!ws) {  // the allocation-free entry point's scratch on the current device
+    void* scratch = nullptr;
+    const hg_status st = noalloc_scratch_address(&scratch);
+    if (st != HG_OK) return st;
+    ws = scratch;
+  }
   if (!aligned16(ws)) return HG_ERR_ALIGNMENT;
   const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   uint32_t v = 0;
@@ -542,7 +565,7 @@ int order_items(const hg_cache* c, int begin, int count, const DecodeParams& p, 
         int nb;
         const int ni = head_chunks(cls, cc, &nb);
         const int blen = (cls == kProtected ? d.T : d.T - d.nq + d.ns) + L.appended;
-        const int clen = cls == kKeysOnly ? d.nq : ncoded(d);
+        const int clen = ncoded(d);
         const int bc = (cls == kProtected) ? p.plan.cbP : p.plan.cbU;
         const int qc = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
         const double qb = (cls == kKeysOnly) ? sb.coded_k : sb.coded_u;
@@ -667,6 +690,31 @@ hg_status hg_decode_step(hg_cache* c, int32_t layer_begin, int32_t layer_count, 
   return st;
 }
 
+}  // extern "C"
+
+namespace hg {
+
+hg_status decode_attention_on_scratch(const hg_cache* c, int32_t layer_begin, int32_t layer_count,
+                                      const void* q, void* out, float softmax_scale, void* scratch,
+                                      size_t scratch_bytes, hg_stream_t stream) {
+  hg_status st = decode_checks(c, layer_begin, layer_count, q, out, softmax_scale, scratch, scratch_bytes);
+  if (st != HG_OK) return st;
+  st = arena_tensor_map(c);
+  if (st != HG_OK) return st;
+  // launches over more than kMaxLayersPerLaunch layers reuse the counters of
+  // the first group, and every launch leaves them at zero again
+  const size_t counters = ws_counter_bytes(c->d, std::min<int>(layer_count, kMaxLayersPerLaunch));
+  if (cudaMemsetAsync(static_cast<char*>(scratch) + kWsHeaderBytes, 0, counters,
+                      reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return HG_ERR_CUDA;
+  return decode_launch(c, layer_begin, layer_count, q, nullptr, nullptr, out, softmax_scale, scratch,
+                       scratch_bytes, stream);
+}
+
+}  // namespace hg
+
+extern "C" {
+
 hg_status hg_select_heads(const float* g_scores, const float* o_scores, int32_t num_layers, int32_t num_q_heads,
                           int32_t num_kv_heads, int32_t k, uint8_t* mask_out) {
   if (!g_scores || !o_scores || !mask_out || num_layers <= 0 || num_q_heads <= 0 || num_kv_heads <= 0)
@@ -720,9 +768,9 @@ hg_status hg_cache_image_bits_per_elem(const hg_cache* c, double* bits) {
   for (int l = 0; l < d.L; ++l) {
     for (int h = 0; h < d.H; ++h) {
       const int cls = head_class(d, c->layer_mask[l], h);
-      // salient image tokens (quantized heads only) are BF16 like the
+      // salient image tokens (heads with coded values) are BF16 like the
       // image tokens outside the eligible span
-      const double coded = cls == kKeysOnly ? d.nq : ncoded(d), bf16 = d.n - coded;
+      const double coded = ncoded(d), bf16 = d.n - coded;
       double kb = 0, vb = 0;
       if (cls == kQuantized) {
         kb = coded * (code_bits + kmeta_tok) + bf16 * 16.0 * kD;

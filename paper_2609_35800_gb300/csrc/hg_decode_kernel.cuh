@@ -41,6 +41,8 @@
 #pragma once
 #include <cuda_runtime.h>
 
+#include <atomic>
+
 #include "hg_common.cuh"
 #include "hg_internal.h"
 #include "hg_mma.cuh"
@@ -1256,7 +1258,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   } else {
     const int c = (cls == kKeysOnly) ? p.plan.cqK : p.plan.cqU;
     tb = (r - nb) * c;
-    te = min(tb + c, cls == kKeysOnly ? d.nq : ncoded(d));
+    te = min(tb + c, ncoded(d));
   }
   const int tid = threadIdx.x;
   const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
@@ -1371,11 +1373,13 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
 
 template <int BITS, int NT, int BASE, int MB>
 cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
-  static bool configured[64] = {};
+  // set once per device; host threads that race here both set the same
+  // attributes, and the flags themselves are atomic
+  static std::atomic<bool> configured[64];
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
   if (e != cudaSuccess) return e;
-  if (dev < 64 && !configured[dev]) {
+  if (dev < 0 || dev >= 64 || !configured[dev].load(std::memory_order_acquire)) {
     e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE, MB>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              SmemLayout<NT>::bytes);
     if (e != cudaSuccess) return e;
@@ -1383,7 +1387,7 @@ cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
     e = cudaFuncSetAttribute(decode_kernel<BITS, NT, BASE, MB>, cudaFuncAttributePreferredSharedMemoryCarveout,
                              cudaSharedmemCarveoutMaxShared);
     if (e != cudaSuccess) return e;
-    configured[dev] = true;
+    if (dev >= 0 && dev < 64) configured[dev].store(true, std::memory_order_release);
   }
   (void)grid_x;
   decode_kernel<BITS, NT, BASE, MB><<<p.total_items, kThreads, SmemLayout<NT>::bytes, s>>>(p);

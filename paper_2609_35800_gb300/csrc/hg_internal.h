@@ -5,6 +5,7 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include "../../include/headguard.h"
 #include "hg_layout.cuh"
 
 namespace hg {
@@ -30,11 +31,11 @@ struct QuantizeParams {
 struct DequantParams {
   Dims d;
   const char* arena;
-  uint64_t layer_base;
-  uint64_t mask;
-  int appended;
+  int n_layers;
+  LayerTable lt;
+  int appended;  // appended tokens, the same in every layer of the launch
   int out_fp32;
-  void* k_out;
+  void* k_out;   // [n_layers][B][H][T + appended][128]
   void* v_out;
 };
 
@@ -125,5 +126,17 @@ cudaError_t launch_wait_probe(uint32_t* result, uint32_t rounds, cudaStream_t s)
 cudaError_t launch_decode_m16(const DecodeParams& p, int grid_x, cudaStream_t s);
 // Most splits of one head the decode kernel's merge can take.
 int decode_max_splits(int G);
+
+// Decode attention with a scratch array as its workspace (the allocation-free
+// entry point): the argument checks of hg_decode_attention and the arena's
+// tensor map first, then a clear of the split counters only (the status word
+// is left as the previous calls left it), then the launch.
+hg_status decode_attention_on_scratch(const hg_cache* cache, int32_t layer_begin, int32_t layer_count,
+                                      const void* q, void* out, float softmax_scale, void* scratch,
+                                      size_t scratch_bytes, hg_stream_t stream);
+// Device address of the allocation-free entry point's scratch array on the
+// current device (its first 512 bytes are a workspace header with the status
+// word at byte 0).
+hg_status noalloc_scratch_address(void** out);
 
 }  // namespace hg

@@ -54,11 +54,11 @@ HG_HD int quantized_count(int T, int s, int n, int base, int residual) {
   return (span / kKiviGroup) * kKiviGroup;
 }
 
-// Image tokens stored coded per head with coded values: the eligible span less
-// the salient tokens (heads whose keys are quantized; no salient tokens exist
-// together with keys-only heads).
+// Image tokens stored coded per head with coded values (quantized heads and
+// keys-only heads): the eligible span less the salient tokens.  A keys-only
+// head keeps the coded tokens' keys as BF16 rows, compacted the same way.
 HG_HD int ncoded(const Dims& d) { return d.nq - d.ns; }
-// Salient-token map of one (batch row, quantized head): a bit per image token
+// Salient-token map of one (batch row, head with coded values): a bit per image token
 // in 32-token blocks (uint32 [nblk]), then the number of salient tokens before
 // each block (int32 [nblk]); rows padded to 16 bytes.
 HG_HD int sal_blocks(const Dims& d) { return (d.nq + 31) / 32; }
@@ -100,7 +100,7 @@ HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
   g.n_PK = d.keys_only ? g.n_prot : 0;
   g.n_PKV = d.keys_only ? 0 : g.n_prot;
   g.n_VQ = g.n_U + g.n_PK;
-  const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
+  const uint64_t B = (uint64_t)d.B;
   const uint64_t nc = (uint64_t)ncoded(d);
   const uint64_t tok_bf16 = (uint64_t)d.H * cap_unprot(d) + (uint64_t)g.n_PKV * nc;
   g.bf16_bytes = align_up(B * tok_bf16 * kD * 2);
@@ -111,8 +111,8 @@ HG_HD LayerGeom layer_geom(const Dims& d, uint64_t mask) {
   g.kqm = off; off += align_up((uint64_t)g.n_U * B * kmeta_stride(d));
   g.vq = off; off += align_up((uint64_t)g.n_VQ * B * nc * code_bytes_per_token(d));
   g.vqm = off; off += align_up((uint64_t)g.n_VQ * B * vmeta_stride(d));
-  g.kimg = off; off += align_up((uint64_t)g.n_PK * B * nq * kD * 2);
-  g.sal = off; off += align_up((uint64_t)g.n_U * B * sal_stride(d));
+  g.kimg = off; off += align_up((uint64_t)g.n_PK * B * nc * kD * 2);
+  g.sal = off; off += align_up((uint64_t)g.n_VQ * B * sal_stride(d));
   g.size = off;
   return g;
 }
@@ -136,7 +136,7 @@ HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
   HeadGeom r;
   const uint64_t below = (h == 0) ? 0ull : (g.mask & ((h >= 64) ? ~0ull : ((1ull << h) - 1ull)));
   const int prot_below = popc64(below);
-  const uint64_t B = (uint64_t)d.B, nq = (uint64_t)d.nq;
+  const uint64_t B = (uint64_t)d.B;
   r.cls = head_class(d, g.mask, h);
   r.bf16_prefill = (r.cls == kProtected) ? d.T : d.T - d.nq + d.ns;
   r.cap = r.bf16_prefill + d.S_new;
@@ -151,19 +151,19 @@ HG_HD HeadGeom head_geom(const Dims& d, const LayerGeom& g, int h) {
   r.kqm_bs = kmeta_stride(d);
   r.vq_bs = nc * code_bytes_per_token(d);
   r.vqm_bs = vmeta_stride(d);
-  r.kimg_bs = nq * kD * 2;
+  r.kimg_bs = nc * kD * 2;
   r.sal_bs = sal_stride(d);
   r.kq = r.kqm = r.vq = r.vqm = r.kimg = r.sal = kNone;
   if (r.cls == kQuantized) {
     const uint64_t u = (uint64_t)(h - prot_below);
     r.kq = g.kq + u * B * r.kq_bs;
     r.kqm = g.kqm + u * B * r.kqm_bs;
-    if (d.ns > 0) r.sal = g.sal + u * B * r.sal_bs;
   }
   if (r.cls != kProtected) {
     const uint64_t vr = d.keys_only ? (uint64_t)h : (uint64_t)(h - prot_below);
     r.vq = g.vq + vr * B * r.vq_bs;
     r.vqm = g.vqm + vr * B * r.vqm_bs;
+    if (d.ns > 0) r.sal = g.sal + vr * B * r.sal_bs;
   }
   if (r.cls == kKeysOnly) {
     r.kimg = g.kimg + (uint64_t)prot_below * B * r.kimg_bs;
@@ -201,7 +201,7 @@ HG_HD ChunkCounts chunk_counts(const Dims& d, int appended, int cbU, int cqU, in
   ChunkCounts c;
   c.nbU = cdiv(d.T - d.nq + d.ns + appended, cbU);
   c.nqU = cdiv(ncoded(d), cqU);
-  c.nqK = cdiv(d.nq, cqK);
+  c.nqK = cdiv(ncoded(d), cqK);
   c.nbP = cdiv(d.T + appended, cbP);
   return c;
 }

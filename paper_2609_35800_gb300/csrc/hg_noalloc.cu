@@ -9,29 +9,42 @@
 // device array of kScratchBytes (32 MiB) that every GPU loading this library
 // keeps until the process exits.  Nothing here calls cudaMalloc, cudaFree or
 // any other allocating routine.
+//
+// The array is laid out as a decode workspace: a 512-byte header whose first
+// word is the status word, the split counters, the split partials.  Every call
+// clears the counters it uses; the status word is sticky (a wait that ran out
+// in any call stays visible) until the caller clears it, and both are reached
+// through hg_workspace_status / hg_workspace_clear with a null workspace.
 #include <cuda_runtime.h>
 
 #include <cstdint>
 #include <mutex>
 
 #include "../../include/headguard.h"
+#include "hg_internal.h"
 
 namespace {
 
 constexpr size_t kScratchBytes = size_t(32) << 20;
 constexpr int kMaxDevices = 64;
 
-// The shared scratch.  In host code this name is only a stand-in for the
-// device array, never a usable address; the address comes from
-// cudaGetSymbolAddress below.
+// The shared scratch (zero when the library's module is loaded).  In host code
+// this name is only a stand-in for the device array, never a usable address;
+// the address comes from cudaGetSymbolAddress below.
 __device__ __align__(256) unsigned char g_scratch[kScratchBytes];
 
 std::mutex g_mutex;
 void* g_scratch_ptr[kMaxDevices] = {};
 
+bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+}  // namespace
+
+namespace hg {
+
 // Device address of the scratch on the current device; looked up (and the
 // library's module loaded) on the first call for that device.
-hg_status scratch_address(void** out) {
+hg_status noalloc_scratch_address(void** out) {
   int dev = -1;
   if (cudaGetDevice(&dev) != cudaSuccess) return HG_ERR_CUDA;
   if (dev < 0 || dev >= kMaxDevices) return HG_ERR_UNSUPPORTED;
@@ -45,14 +58,13 @@ hg_status scratch_address(void** out) {
   return HG_OK;
 }
 
-bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
-
-}  // namespace
+}  // namespace hg
 
 extern "C" hg_status hg_decode_attention_noalloc(const hg_cache* cache, int32_t layer_begin,
                                                  int32_t layer_count, const void* q, void* out,
                                                  float softmax_scale, hg_stream_t stream) {
-  // Same argument checks as hg_decode_attention, done before anything is enqueued.
+  // The host-side checks of hg_decode_attention that need no workspace, and
+  // the size limit, before anything else.
   if (!cache || layer_begin < 0 || layer_count < 1 || !q || !out) return HG_ERR_INVALID_ARG;
   if (hg_cache_appended(cache, layer_begin) < 0 ||
       hg_cache_appended(cache, layer_begin + layer_count - 1) < 0)
@@ -64,12 +76,10 @@ extern "C" hg_status hg_decode_attention_noalloc(const hg_cache* cache, int32_t 
   if (st != HG_OK) return st;
   if (need > kScratchBytes) return HG_ERR_WORKSPACE_TOO_SMALL;
   void* scratch = nullptr;
-  st = scratch_address(&scratch);
+  st = hg::noalloc_scratch_address(&scratch);
   if (st != HG_OK) return st;
-  // The array keeps whatever the previous call left; the status word and the
-  // split counters must start at zero.
-  if (cudaMemsetAsync(scratch, 0, need, reinterpret_cast<cudaStream_t>(stream)) != cudaSuccess)
-    return HG_ERR_CUDA;
-  return hg_decode_attention(cache, layer_begin, layer_count, q, out, softmax_scale, scratch,
-                             kScratchBytes, stream);
+  // The remaining checks, then a clear of the split counters (the array keeps
+  // whatever the previous call left), then the launch.
+  return hg::decode_attention_on_scratch(cache, layer_begin, layer_count, q, out, softmax_scale, scratch,
+                                         kScratchBytes, stream);
 }

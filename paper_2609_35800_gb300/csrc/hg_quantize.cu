@@ -60,25 +60,6 @@ __device__ __forceinline__ void store_token_codes(uint32_t* row, const uint32_t 
   }
 }
 
-// Codes of channels 4l..4l+3 of one token from its packed row.
-__device__ __forceinline__ void load_token_codes(const uint32_t* row, int bits, int lane,
-                                                 uint32_t (&c)[4]) {
-  if (bits == 2 || bits == 3) {
-    const uint32_t byte = (__ldg(row + (lane >> 2)) >> (8 * (lane & 3))) & 0xffu;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) c[i] = (byte >> (2 * i)) & 3u;
-    if (bits == 3) {
-      const uint32_t hp = __ldg(row + 8 + (lane >> 3)) >> plane_base(lane);
-#pragma unroll
-      for (int i = 0; i < 4; ++i) c[i] |= ((hp >> i) & 1u) << 2;
-    }
-  } else {
-    const uint32_t half = (__ldg(row + (lane >> 1)) >> (16 * (lane & 1))) & 0xffffu;
-#pragma unroll
-    for (int i = 0; i < 4; ++i) c[i] = (half >> (4 * i)) & 15u;
-  }
-}
-
 __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
   bf16x2_to_f32(w.x, x[0], x[1]);
   bf16x2_to_f32(w.y, x[2], x[3]);
@@ -138,14 +119,15 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
 
   __shared__ __align__(16) uint16_t ktile[kTile][kD];
 
-  // AKVQ-style salient tokens (Sec. 4): the map of this tile's image tokens.
-  // Image tiles start on the image's 32-token blocks, so one map word covers
-  // the tile: a salient token goes to BF16 position qs + (its rank among the
-  // salient tokens), every other image token to coded slot ti - (the salient
-  // tokens before it).
+  // AKVQ-style salient tokens (Sec. 4): the map of this tile's image tokens,
+  // in every head whose image values are coded (quantized and keys-only
+  // heads).  Image tiles start on the image's 32-token blocks, so one map
+  // word covers the tile: a salient token goes to BF16 position qs + (its
+  // rank among the salient tokens), every other image token to coded slot
+  // ti - (the salient tokens before it).
   uint32_t sbits = 0u;
   int srank = 0;
-  const bool sal_tile = d.ns > 0 && hd.cls == kQuantized && t0 >= qs && t0 < qe;
+  const bool sal_tile = d.ns > 0 && hd.cls != kProtected && t0 >= qs && t0 < qe;
   if (sal_tile) {
     const char* sm = Lb + hd.sal + b * hd.sal_bs;
     const int w = (t0 - qs) >> 5;
@@ -197,8 +179,8 @@ quantize_kernel(const __grid_constant__ QuantizeParams p) {
         store_token_codes(crow, c, d.bits, lane);
         if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, sc, z, m16);
       }
-    } else if (coded && hd.cls == kKeysOnly) {
-      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2) = kri;
+    } else if (coded && hd.cls == kKeysOnly && !sal) {
+      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ci * kD + lane * 4) * 2) = kri;
     } else {
       const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
       *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) = kri;
@@ -489,7 +471,7 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
 
 // ---------------------------------------------------------------------------
 // AKVQ-style salient tokens (Sec. 4): one CTA per (batch row, KV head, layer);
-// heads whose image keys are not quantized return.  Squared key norms of the
+// protected K+V heads (no coded image entries) return.  Squared key norms of the
 // image tokens in the fixed binary32 order (a warp per token: lane l sums
 // channels 4l..4l+3, then five butterfly rounds of pairwise sums), ns rounds
 // of a CTA-wide arg-max (largest score, ties to the lower index), then the
@@ -503,7 +485,7 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
   const int b = bh / d.H, h = bh % d.H;
   const LayerGeom g = layer_geom(d, p.lt.mask[li]);
   const HeadGeom hd = head_geom(d, g, h);
-  if (hd.cls != kQuantized || d.ns <= 0) return;
+  if (hd.cls == kProtected || d.ns <= 0) return;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
   const int nq = d.nq, nblk = sal_blocks(d);
   extern __shared__ __align__(16) float sal_smem[];
@@ -580,95 +562,180 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
   }
 }
 
-// Reconstruct one layer as floats in original token order (then appended).
-__global__ void __launch_bounds__(kThreads)
+// ---------------------------------------------------------------------------
+// Reconstruction (Sec. 4: codes to floats, code * scale + zero; AKVQ-style keys
+// rotated back; BF16 entries copied), every layer of the launch in original
+// token order followed by the appended tokens.  One CTA per (32-token tile,
+// batch row, KV head, layer); a half-warp owns one token row of K or of V,
+// lane j of it channels 8j..8j+7, so every output row is one 256-byte (BF16)
+// or 512-byte (fp32) store of 16 lanes and each lane issues its code,
+// metadata and row loads independently.  The AKVQ-style inverse rotation runs
+// its first three butterfly stages inside a lane and the last four across the
+// half-warp, in the same order as the forward transform.
+// ---------------------------------------------------------------------------
+constexpr int kDqThreads = 256;
+constexpr int kDqTile = 32;
+
+__device__ __forceinline__ void bf16x8_to_f32(const uint4& w, float (&x)[8]) {
+  bf16x2_to_f32(w.x, x[0], x[1]);
+  bf16x2_to_f32(w.y, x[2], x[3]);
+  bf16x2_to_f32(w.z, x[4], x[5]);
+  bf16x2_to_f32(w.w, x[6], x[7]);
+}
+
+// Codes of channels 8c..8c+7 of a per-token packed row (channel order; 3 bits:
+// the 2-bit half-word, then the plane byte of channels 8c..8c+7, which holds
+// them in order at byte ((c >> 1) & 1) | ((c & 1) << 1) of plane word c / 4).
+__device__ __forceinline__ void row_codes8(const uint32_t* row, int bits, int c, uint32_t (&code)[8]) {
+  if (bits == 4) {
+    const uint32_t w = __ldg(row + c);
+#pragma unroll
+    for (int i = 0; i < 8; ++i) code[i] = (w >> (4 * i)) & 15u;
+    return;
+  }
+  const uint32_t half = (__ldg(row + (c >> 1)) >> (16 * (c & 1))) & 0xffffu;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) code[i] = (half >> (2 * i)) & 3u;
+  if (bits == 3) {
+    const uint32_t pl = __ldg(row + 8 + (c >> 2)) >> (8 * (((c >> 1) & 1) | ((c & 1) << 1)));
+#pragma unroll
+    for (int i = 0; i < 8; ++i) code[i] |= ((pl >> i) & 1u) << 2;
+  }
+}
+
+// Code of token e (0..31) of one KIVI-style key group row (one channel, token order).
+__device__ __forceinline__ uint32_t kivi_code(const uint32_t* row, int bits, int e) {
+  if (bits == 3) {
+    const uint32_t lo = (__ldg(row + e / 16) >> (2 * (e % 16))) & 3u;
+    const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
+    return lo | (((__ldg(row + 2) >> pp) & 1u) << 2);
+  }
+  const int per = 32 / bits;
+  return (__ldg(row + e / per) >> (bits * (e % per))) & ((1u << bits) - 1u);
+}
+
+// Normalised Hadamard-128 of a vector spread over a half-warp, lane j holding
+// channels 8j..8j+7: stages h = 1, 2, 4 in the lane, h = 8..64 with lane
+// j ^ (h / 8); butterflies (a, b) -> (a + b, a - b), one multiply at the end.
+__device__ __forceinline__ void fwht128_half(float (&x)[8], int j) {
+#pragma unroll
+  for (int h = 1; h < 8; h <<= 1) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      if (i & h) continue;
+      const float a = x[i], b = x[i + h];
+      x[i] = __fadd_rn(a, b);
+      x[i + h] = __fsub_rn(a, b);
+    }
+  }
+#pragma unroll
+  for (int m = 1; m < 16; m <<= 1) {
+    const bool upper = (j & m) != 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const float p = __shfl_xor_sync(kFull, x[i], m);
+      x[i] = upper ? __fsub_rn(p, x[i]) : __fadd_rn(x[i], p);
+    }
+  }
+  const float c = hadamard_c();
+#pragma unroll
+  for (int i = 0; i < 8; ++i) x[i] = __fmul_rn(x[i], c);
+}
+
+__global__ void __launch_bounds__(kDqThreads)
 dequantize_kernel(const __grid_constant__ DequantParams p) {
   const Dims& d = p.d;
-  const int bh = blockIdx.y;
+  const int li = blockIdx.z, bh = blockIdx.y;
   const int b = bh / d.H, h = bh % d.H;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int Tt = d.T + p.appended;
-  const LayerGeom g = layer_geom(d, p.mask);
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
   const HeadGeom hd = head_geom(d, g, h);
-  const char* Lb = p.arena + p.layer_base;
+  const char* Lb = p.arena + p.lt.base[li];
   const int qs = d.s, qe = d.s + d.nq;
   const int W = kD * d.bits / 32;
   const bool m16 = d.meta16 != 0;
+  const int j = threadIdx.x & 15;  // channels 8j..8j+7
+  const size_t out_row0 = (((size_t)li * d.B + b) * d.H + h) * (size_t)Tt;
 
-  for (int t = blockIdx.x * kTile + warp; t < min(Tt, (int)(blockIdx.x + 1) * kTile); t += 4) {
+  // unit u: K (u < 512) or V, token (u >> 4) & 31 of the tile; unrolled so
+  // that the loads of a thread's four units are in flight together
+#pragma unroll
+  for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
+    const bool is_k = u < kDqTile * 16;
+    const int t = blockIdx.x * kDqTile + ((u >> 4) & (kDqTile - 1));
+    if (t >= Tt) continue;  // uniform over the half-warp
     const bool coded = (t >= qs) && (t < qe);
     const int ti = t - qs;
     int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token (Sec. 4)
     bool sal = false;
-    if (coded && d.ns > 0 && hd.cls == kQuantized) {
+    if (coded && d.ns > 0 && hd.cls != kProtected) {
       const char* sm = Lb + hd.sal + b * hd.sal_bs;
-      const int w = ti >> 5, j = ti & 31;
+      const int w = ti >> 5, e = ti & 31;
       const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
       const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
-                       __popc(sb & ((1u << j) - 1u));
-      sal = (sb >> j) & 1u;
+                       __popc(sb & ((1u << e) - 1u));
+      sal = (sb >> e) & 1u;
       ci = ti - rank;
       spos = qs + rank;
     }
     const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
-    float xk[4], xv[4];
-    if (coded && hd.cls == kQuantized && !sal) {
-      uint32_t c[4];
-      if (d.base == kKivi) {
-        const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
-        const int per = 32 / d.bits;
-        const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs);
-        const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
+    float x[8];
+    if (is_k) {
+      if (coded && hd.cls == kQuantized && !sal) {
+        uint32_t code[8];
+        float2 m[8];
+        if (d.base == kKivi) {
+          const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
+          const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) +
+                                  ((size_t)grp * kD + 8 * j) * d.bits;
+          const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
 #pragma unroll
-        for (int i = 0; i < 4; ++i) {
-          const size_t row = (size_t)grp * kD + lane * 4 + i;
-          uint32_t code;
-          if (d.bits == 3) {
-            const uint32_t lo = (__ldg(codes + row * 3 + e / 16) >> (2 * (e % 16))) & 3u;
-            const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
-            code = lo | (((__ldg(codes + row * 3 + 2) >> pp) & 1u) << 2);
-          } else {
-            const uint32_t w = __ldg(codes + row * d.bits + e / per);
-            code = (w >> (d.bits * (e % per))) & ((1u << d.bits) - 1u);
+          for (int i = 0; i < 8; ++i) {
+            code[i] = kivi_code(codes + i * d.bits, d.bits, e);
+            m[i] = load_meta(meta, (size_t)grp * kD + 8 * j + i, m16);
           }
-          const float2 m = load_meta(meta, row, m16);
-          xk[i] = dequant1(code, m.x, m.y);
+        } else {
+          row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W, d.bits, j,
+                     code);
+          const float2 m0 = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, m16);
+#pragma unroll
+          for (int i = 0; i < 8; ++i) m[i] = m0;
         }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) x[i] = dequant1(code[i], m[i].x, m[i].y);
+        if (d.base == kAkvq) fwht128_half(x, j);  // inverse rotation (H is self-inverse)
       } else {
-        load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W,
-                         d.bits, lane, c);
-        const float2 m = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, m16);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) xk[i] = dequant1(c[i], m.x, m.y);
-        if (d.base == kAkvq) fwht128_warp(xk, lane);  // inverse rotation (H is self-inverse)
+        const char* src = (coded && hd.cls == kKeysOnly && !sal)
+                              ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
+                              : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
+        bf16x8_to_f32(ldg16(src + j * 16), x);
       }
-    } else if (coded && hd.cls == kKeysOnly) {
-      bf16x4_to_f32(ldg8(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ti * kD + lane * 4) * 2), xk);
     } else {
-      bf16x4_to_f32(ldg8(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2), xk);
-    }
-    if (coded && hd.cls != kProtected && !sal) {
-      uint32_t c[4];
-      load_token_codes(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
-                       d.bits, lane, c);
-      const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
-                                 (size_t)ci * vgroups(d) + (d.base == kKivi ? (lane >> 3) : 0), m16);
+      if (coded && hd.cls != kProtected && !sal) {
+        uint32_t code[8];
+        row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W, d.bits, j,
+                   code);
+        // KIVI-style: 32-channel groups, channels 8j.. in group j / 4
+        const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
+                                   (size_t)ci * vgroups(d) + (d.base == kKivi ? (j >> 2) : 0), m16);
 #pragma unroll
-      for (int i = 0; i < 4; ++i) xv[i] = dequant1(c[i], m.x, m.y);
-    } else {
-      bf16x4_to_f32(ldg8(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2), xv);
+        for (int i = 0; i < 8; ++i) x[i] = dequant1(code[i], m.x, m.y);
+      } else {
+        bf16x8_to_f32(ldg16(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256 + j * 16), x);
+      }
     }
-    const size_t o = (((size_t)b * d.H + h) * Tt + t) * kD + lane * 4;
+    const size_t o = (out_row0 + t) * kD + 8 * j;
+    void* dst = is_k ? p.k_out : p.v_out;
     if (p.out_fp32) {
-      reinterpret_cast<float4*>(p.k_out)[o / 4] = make_float4(xk[0], xk[1], xk[2], xk[3]);
-      reinterpret_cast<float4*>(p.v_out)[o / 4] = make_float4(xv[0], xv[1], xv[2], xv[3]);
+      float4* f = reinterpret_cast<float4*>(static_cast<float*>(dst) + o);
+      f[0] = make_float4(x[0], x[1], x[2], x[3]);
+      f[1] = make_float4(x[4], x[5], x[6], x[7]);
     } else {
-      reinterpret_cast<uint2*>(p.k_out)[o / 4] =
-          make_uint2(f32_to_bf16_rn(xk[0]) | (f32_to_bf16_rn(xk[1]) << 16),
-                     f32_to_bf16_rn(xk[2]) | (f32_to_bf16_rn(xk[3]) << 16));
-      reinterpret_cast<uint2*>(p.v_out)[o / 4] =
-          make_uint2(f32_to_bf16_rn(xv[0]) | (f32_to_bf16_rn(xv[1]) << 16),
-                     f32_to_bf16_rn(xv[2]) | (f32_to_bf16_rn(xv[3]) << 16));
+      *reinterpret_cast<uint4*>(static_cast<uint16_t*>(dst) + o) =
+          make_uint4(f32_to_bf16_rn(x[0]) | (f32_to_bf16_rn(x[1]) << 16),
+                     f32_to_bf16_rn(x[2]) | (f32_to_bf16_rn(x[3]) << 16),
+                     f32_to_bf16_rn(x[4]) | (f32_to_bf16_rn(x[5]) << 16),
+                     f32_to_bf16_rn(x[6]) | (f32_to_bf16_rn(x[7]) << 16));
     }
   }
 }
@@ -731,8 +798,8 @@ cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s) {
 
 cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s) {
   const int Tt = p.d.T + p.appended;
-  dim3 grid((Tt + kTile - 1) / kTile, p.d.B * p.d.H, 1);
-  dequantize_kernel<<<grid, kThreads, 0, s>>>(p);
+  dim3 grid((Tt + kDqTile - 1) / kDqTile, p.d.B * p.d.H, p.n_layers);
+  dequantize_kernel<<<grid, kDqThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -79,7 +79,7 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
         r = hg.hg_cache_head_regions(runner.cache, layer, h)
         assert r.nq == nq
         cls = r.head_class
-        assert r.n_salient == (ns if cls == hg.HG_HEAD_QUANTIZED else 0)
+        assert r.n_salient == (0 if cls == hg.HG_HEAD_PROTECTED else ns)
         nc = 0 if cls == hg.HG_HEAD_PROTECTED else nq - r.n_salient
         assert r.n_coded == nc
         for bi, b in enumerate(rows):
@@ -119,9 +119,11 @@ def check_arena_layer(runner, layer, k_bits, v_bits, o, arena=None, heads=None, 
                 vm = rd(r.vqm + b * r.vqm_bstride, ev.nbytes, np.uint32)
                 assert np.array_equal(vw, o["v_words"][ob, oh][:nc * W]), (layer, h, b, "vq")
                 assert np.array_equal(vm, ev), (layer, h, b, "vqm")
-            if cls == hg.HG_HEAD_KEYS_ONLY and nq:
-                ki = rd(r.kimg + b * r.kimg_bstride, nq * 256, np.uint16).reshape(-1, 128)
-                assert np.array_equal(ki, k_bits[ob, oh, s:s + nq]), (layer, h, b, "kimg")
+            if cls == hg.HG_HEAD_KEYS_ONLY and nc:
+                # image keys of the coded tokens (the salient ones are in kb), compacted
+                coded = np.setdiff1d(np.arange(nq), o["salient"][ob, oh]) if r.n_salient else np.arange(nq)
+                ki = rd(r.kimg + b * r.kimg_bstride, nc * 256, np.uint16).reshape(-1, 128)
+                assert np.array_equal(ki, k_bits[ob, oh, s + coded]), (layer, h, b, "kimg")
 
 
 def attention_reference(runner, o, q_bits, appended_k, appended_v, sigma):
@@ -148,3 +150,63 @@ def assert_close(got_bf16_bits, ref, where=""):
                              "(max abs err %.3g)" % (where, bad.sum(), bad.size, tuple(i),
                                                      g[tuple(i)], ref[tuple(i)], err.max()))
     return float(err.max())
+
+
+def layer_block(runner, layer):
+    """Host copy of one layer's block of the arena: (numpy bytes, base offset)."""
+    w = runner.w
+    lo, hi = None, 0
+    for h in range(w.kv_heads):
+        r = hg.hg_cache_head_regions(runner.cache, layer, h)
+        for off, stride in ((r.kb, r.kb_bstride), (r.vb, r.kb_bstride), (r.kq, r.kq_bstride),
+                            (r.kqm, r.kqm_bstride), (r.vq, r.vq_bstride), (r.vqm, r.vqm_bstride),
+                            (r.kimg, r.kimg_bstride), (r.sal, r.sal_bstride)):
+            if off == hg.NONE_OFFSET:
+                continue
+            lo = off if lo is None else min(lo, off)
+            hi = max(hi, off + w.batch * stride)
+    return runner.arena[lo:hi].cpu().numpy(), lo
+
+
+def check_arena_layer_blocks(runner, layer, k_bits, v_bits, o, block=None):
+    """Bit-exact comparison of every region of one layer, all batch rows of a
+    head at once (caches without salient tokens).  k_bits, v_bits: uint16
+    [B][H][T][128]; o: the oracle's quantize_layer output for the same layer."""
+    w = runner.w
+    assert not o["n_salient"]
+    m16 = w.meta_bits == 32
+    arena, base = block if block is not None else layer_block(runner, layer)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    s, nq = w.img_start, o["nq"]
+    W = 128 * w.bits // 32
+
+    def rows(off, stride, n, dtype):
+        a = arena[off - base: off - base + B * stride].reshape(B, stride)
+        return a[:, :n * np.dtype(dtype).itemsize].view(dtype)
+
+    for h in range(H):
+        r = hg.hg_cache_head_regions(runner.cache, layer, h)
+        cls = r.head_class
+        assert r.nq == nq and r.n_salient == 0
+        toks = np.arange(T) if cls == hg.HG_HEAD_PROTECTED else np.concatenate([np.arange(s), np.arange(s + nq, T)])
+        assert r.bf16_prefill == toks.size
+        kb = rows(r.kb, r.kb_bstride, toks.size * 128, np.uint16)
+        vb = rows(r.vb, r.kb_bstride, toks.size * 128, np.uint16)
+        assert np.array_equal(kb, k_bits[:, h][:, toks].reshape(B, -1)), (layer, h, "kb")
+        assert np.array_equal(vb, v_bits[:, h][:, toks].reshape(B, -1)), (layer, h, "vb")
+        if cls == hg.HG_HEAD_PROTECTED or not nq:
+            continue
+        if cls == hg.HG_HEAD_QUANTIZED:
+            kw = rows(r.kq, r.kq_bstride, nq * W, np.uint32)
+            assert np.array_equal(kw, o["k_words"][:, h, :nq * W]), (layer, h, "kq")
+            ek = _meta_words(o["k_meta"][:, h], m16)
+            km = rows(r.kqm, r.kqm_bstride, ek.shape[1], np.uint32)
+            assert np.array_equal(km, ek), (layer, h, "kqm")
+        else:
+            ki = rows(r.kimg, r.kimg_bstride, nq * 128, np.uint16)
+            assert np.array_equal(ki, k_bits[:, h, s:s + nq].reshape(B, -1)), (layer, h, "kimg")
+        vw = rows(r.vq, r.vq_bstride, nq * W, np.uint32)
+        assert np.array_equal(vw, o["v_words"][:, h, :nq * W]), (layer, h, "vq")
+        ev = _meta_words(o["v_meta"][:, h], m16)
+        vm = rows(r.vqm, r.vqm_bstride, ev.shape[1], np.uint32)
+        assert np.array_equal(vm, ev), (layer, h, "vqm")

@@ -72,7 +72,6 @@ def _status(f, *a):
     ({}, dict(base=2, salient_permille=1001), 1),
     ({}, dict(base=0, salient_permille=20), 3),
     ({}, dict(base=1, salient_permille=20), 3),
-    ({}, dict(base=2, keys_only=1, salient_permille=20), 3),
     (dict(max_new_tokens=-1), {}, 1),
     (dict(img_start=-1), {}, 1),
     (dict(num_layers=0), {}, 1),
@@ -121,7 +120,11 @@ ODD = {"odd_nq_minmax": wl.custom("odd", 3, 3, 16, 4, 64, 333, 17, wl.BASE_MINMA
        "salient_akvq": wl.custom("sal", 3, 2, 16, 4, 9, 333, 17, wl.BASE_AKVQ, 4, 0,
                                  salient_permille=20),
        "salient_all": wl.custom("sal2", 2, 3, 8, 8, 5, 70, 9, wl.BASE_AKVQ, 2, 0,
-                                salient_permille=1000)}
+                                salient_permille=1000),
+       "salient_akvq_konly": wl.custom("salk", 3, 2, 16, 4, 9, 333, 17, wl.BASE_AKVQ, 4, 1,
+                                       salient_permille=20),
+       "salient_akvq3_konly": wl.custom("salk3", 2, 3, 8, 8, 5, 131, 40, wl.BASE_AKVQ, 3, 1,
+                                        salient_permille=40)}
 
 
 @pytest.mark.parametrize("name", list(wl.WORKLOADS) + list(ODD))
@@ -266,7 +269,7 @@ def test_calls_validate_before_any_launch(lib):
         hg.hg_decode_attention(cache, 0, 2, base, base, float("nan"), base, need, stream=0)
     assert e.value.status == 1
     with pytest.raises(hg.HGError) as e:
-        hg.hg_dequantize_kv(cache, 2, base, base, 1, stream=0)
+        hg.hg_dequantize_kv(cache, 2, 1, base, base, 1, stream=0)
     assert e.value.status == 1
     assert hg.hg_cache_appended(cache, 0) == 0
     assert hg.hg_cache_appended(cache, 5) == -1

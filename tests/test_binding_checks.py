@@ -64,11 +64,11 @@ def test_decode_inputs(cache):
 
 def test_dequantize_outputs(cache):
     # fp32 output needs 4 bytes per entry; nothing appended yet: T tokens
-    _raises(lambda: hg.hg_dequantize_kv(cache, 0, _bf16(B, H, T, 128), _bf16(B, H, T, 128), True),
+    _raises(lambda: hg.hg_dequantize_kv(cache, 0, 1, _bf16(B, H, T, 128), _bf16(B, H, T, 128), True),
             "k_out holds")
     k32 = torch.zeros((B, H, T, 128), dtype=torch.float32)
-    _raises(lambda: hg.hg_dequantize_kv(cache, 0, k32, k32, True), "must be a CUDA tensor")
-    _raises(lambda: hg.hg_dequantize_kv(cache, 0, _bf16(B, H, T, 128), _bf16(B, H, T, 128), False),
+    _raises(lambda: hg.hg_dequantize_kv(cache, 0, 1, k32, k32, True), "must be a CUDA tensor")
+    _raises(lambda: hg.hg_dequantize_kv(cache, 0, 1, _bf16(B, H, T, 128), _bf16(B, H, T, 128), False),
             "must be a CUDA tensor")
 
 
@@ -116,6 +116,6 @@ def test_generated_inputs_pass_the_extent_checks(name):
     last = w.layers - 1
     _raises(lambda: hg.hg_decode_step(c, last, 1, q[last], kn[last], vn[last], out[last], 0.0, ws),
             cuda)
-    _raises(lambda: hg.hg_dequantize_kv(c, 0, k32, k32, True), cuda)
-    _raises(lambda: hg.hg_dequantize_kv(c, 0, k, v, False), cuda)
+    _raises(lambda: hg.hg_dequantize_kv(c, 0, 1, k32, k32, True), cuda)
+    _raises(lambda: hg.hg_dequantize_kv(c, 0, 1, k, v, False), cuda)
     _raises(lambda: hg.hg_workspace_clear(ws), cuda)

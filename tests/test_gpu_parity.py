@@ -121,16 +121,17 @@ def test_fused_decode_step(case):
     runner, kept, outs = _run_and_check(w, fused=True)
     assert hg.hg_cache_appended(runner.cache, 0) == w.decode_steps
     Tt = w.seq_len + w.decode_steps
-    k32 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
+    # every layer in one reconstruction launch
+    k32 = torch.empty(w.layers, w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
     v32 = torch.empty_like(k32)
+    hg.hg_dequantize_kv(runner.cache, 0, w.layers, k32, v32, True)
+    torch.cuda.synchronize()
     for l in range(w.layers):
-        hg.hg_dequantize_kv(runner.cache, l, k32, v32, True)
-        torch.cuda.synchronize()
         for step in range(w.decode_steps):
             k_new, v_new = wl.step_new_kv(w, step, "cuda")
-            assert np.array_equal(k32[:, :, w.seq_len + step].cpu().numpy(),
+            assert np.array_equal(k32[l, :, :, w.seq_len + step].cpu().numpy(),
                                   k_new[l].float().cpu().numpy())
-            assert np.array_equal(v32[:, :, w.seq_len + step].cpu().numpy(),
+            assert np.array_equal(v32[l, :, :, w.seq_len + step].cpu().numpy(),
                                   v_new[l].float().cpu().numpy())
 
 
@@ -207,6 +208,11 @@ SALIENT = [
     (("akvq4_sal_all", 1, 2, 8, 2, 5, 70, 9, A, 4, 0, 2, [], 32), 1000),
     (("akvq2_sal_g16", 1, 1, 32, 2, 16, 200, 16, A, 2, 0, 2, [(0, 1)], 32), 20),
     (("akvq2_sal_long", 1, 1, 28, 4, 50, 3000, 50, A, 2, 0, 2, [(0, 0)], 32), 20),
+    # K-only protection: a protected head keeps its salient tokens' values BF16
+    (("akvq4_konly_sal", 2, 2, 16, 4, 64, 333, 17, A, 4, 1, 3, [(0, 3), (1, 0), (1, 2)], 32), 20),
+    (("akvq2_konly_sal_unaligned", 1, 3, 8, 4, 13, 250, 30, A, 2, 1, 2, [(0, 1)], 32), 40),
+    (("akvq3_konly_sal", 1, 2, 8, 4, 20, 150, 30, A, 3, 1, 2, [(0, 0), (0, 2)], 32), 100),
+    (("akvq4_konly_sal_all_protected", 1, 1, 8, 2, 5, 300, 9, A, 4, 1, 2, [(0, 0), (0, 1)], 32), 20),
 ]
 
 
@@ -243,8 +249,10 @@ def test_dequantize_bit_exact(case, meta_bits):
     _dequantize_bit_exact(_workload(case, meta_bits))
 
 
-@pytest.mark.parametrize("case,permille", [SALIENT[0], SALIENT[1], SALIENT[3]],
-                         ids=["akvq4", "akvq2_unaligned", "all"])
+@pytest.mark.parametrize("case,permille", [SALIENT[0], SALIENT[1], SALIENT[3], SALIENT[6], SALIENT[7],
+                                          SALIENT[9]],
+                         ids=["akvq4", "akvq2_unaligned", "all", "konly4", "konly2_unaligned",
+                              "konly_all_protected"])
 def test_salient_dequantize_bit_exact(case, permille):
     _dequantize_bit_exact(_workload(case, salient_permille=permille))
 
@@ -256,15 +264,21 @@ def _dequantize_bit_exact(w):
     k_new, v_new = wl.step_new_kv(w, 0, "cuda")
     hg.hg_append_kv(runner.cache, 0, w.layers, k_new, v_new)
     Tt = w.seq_len + 1
+    # all layers in one launch (fp32 and BF16 outputs), and each layer alone (fp32)
+    K32 = torch.empty(w.layers, w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
+    V32 = torch.empty_like(K32)
+    hg.hg_dequantize_kv(runner.cache, 0, w.layers, K32, V32, True)
+    K16 = torch.empty(w.layers, w.batch, w.kv_heads, Tt, 128, dtype=torch.bfloat16, device="cuda")
+    V16 = torch.empty_like(K16)
+    hg.hg_dequantize_kv(runner.cache, 0, w.layers, K16, V16, False)
     for l, (k, v) in enumerate(kept):
         o = oracle_layer(runner, l, bits16(k), bits16(v))
         k32 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.float32, device="cuda")
         v32 = torch.empty_like(k32)
-        hg.hg_dequantize_kv(runner.cache, l, k32, v32, True)
-        k16 = torch.empty(w.batch, w.kv_heads, Tt, 128, dtype=torch.bfloat16, device="cuda")
-        v16 = torch.empty_like(k16)
-        hg.hg_dequantize_kv(runner.cache, l, k16, v16, False)
+        hg.hg_dequantize_kv(runner.cache, l, 1, k32, v32, True)
         torch.cuda.synchronize()
+        assert torch.equal(k32, K32[l]) and torch.equal(v32, V32[l])
+        k16, v16 = K16[l], V16[l]
         kd = np.concatenate([o["k_deq"], (bits16(k_new[l]).astype(np.uint32) << 16)
                              .view(np.float32)[:, :, None]], axis=2)
         vd = np.concatenate([o["v_deq"], (bits16(v_new[l]).astype(np.uint32) << 16)
@@ -368,7 +382,7 @@ def test_meta16_extreme_ranges(base, bits):
     hg.hg_quantize_kv(runner.cache, 0, [k], [v])
     k32 = torch.empty(B, H, T, 128, dtype=torch.float32, device="cuda")
     v32 = torch.empty_like(k32)
-    hg.hg_dequantize_kv(runner.cache, 0, k32, v32, True)
+    hg.hg_dequantize_kv(runner.cache, 0, 1, k32, v32, True)
     torch.cuda.synchronize()
     kb, vb = bits16(k), bits16(v)
     o = oracle_layer(runner, 0, kb, vb)
