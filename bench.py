@@ -88,6 +88,7 @@ def geometry_bytes(runner):
                 per_b_write += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
                 per_b_read_dec += nq * code_tok + r.kqm_bstride + nq * code_tok + r.vqm_bstride
             elif r.head_class == hg.HG_HEAD_KEYS_ONLY:
+                per_b_write += r.sal_bstride
                 per_b_write += nq * 256 + nq * code_tok + r.vqm_bstride
                 per_b_read_dec += nq * 256 + nq * code_tok + r.vqm_bstride
             quant += B * (T * 512 + per_b_write)
@@ -250,9 +251,30 @@ def profiled_traffic(workload):
 # CPU oracle timing (cpu_baseline and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_sample(w, n_layers, n_steps):
+def cpu_model():
+    """Host CPU model string (lscpu, else /proc/cpuinfo, else the machine type)."""
+    import platform
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        for line in open("/proc/cpuinfo"):
+            if line.lower().startswith("model name"):
+                return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
+def oracle_sample(w, n_layers, n_steps, parts=None):
     """Time the oracle on the first n_layers layers: quantize, then n_steps decode
-    steps of attention over those layers.  Returns (bytes, seconds, threads)."""
+    steps of attention over those layers.  Returns (bytes, seconds, threads);
+    with `parts` (a dict) also fills in the quantize and decode shares:
+    quant_bytes, quant_s, dec_bytes, dec_s."""
     import numpy as np
     import torch
 
@@ -270,6 +292,7 @@ def oracle_sample(w, n_layers, n_steps):
     secs = 0.0
     nbytes = 0
     outs = []
+    q_secs = 0.0
     for l in range(n_layers):
         k, v = wl.layer_kv(w, l, "cpu")
         kb, vb = bits(k), bits(v)
@@ -278,6 +301,7 @@ def oracle_sample(w, n_layers, n_steps):
                                   int(w.keys_only), w.kivi_group_tokens, w.kivi_group_channels,
                                   w.kivi_residual, meta16=w.meta_bits == 32, n_salient=ns)
         secs += time.perf_counter() - t0
+        q_secs += time.perf_counter() - t0
         nq = o["nq"] - ns  # coded tokens per quantized head
         code_tok = 128 * w.bits // 8
         n_prot = int(mask[l].sum())
@@ -292,6 +316,7 @@ def oracle_sample(w, n_layers, n_steps):
                        + coded_heads_v * (nq * code_tok + meta_v))
         nbytes += B * H * T * 512 + written
         outs.append(o)
+    q_bytes = nbytes
     app_k = [[] for _ in range(n_layers)]
     app_v = [[] for _ in range(n_layers)]
     for s in range(n_steps):
@@ -311,7 +336,22 @@ def oracle_sample(w, n_layers, n_steps):
             # same per-token bytes as the packed cache the GPU reads
             nbytes += _decode_bytes_layer(w, mask[l], outs[l]["nq"], Tt - T, ns) + 2 * B * w.q_heads * 256
     threads = int(os.environ.get("OMP_NUM_THREADS", os.cpu_count() or 1))
+    if parts is not None:
+        parts.update(quant_bytes=q_bytes, quant_s=q_secs, dec_bytes=nbytes - q_bytes,
+                     dec_s=secs - q_secs)
     return nbytes, secs, threads
+
+
+def cpu_baseline_fields(w, n_layers, n_steps, parts):
+    """The oracle's quantize GB/s and decode tokens/s from one timed sample
+    (decode tokens/s scaled to all layers when the sample holds fewer)."""
+    dec_tok = w.batch * n_steps / parts["dec_s"] * (n_layers / w.layers) if parts["dec_s"] > 0 else None
+    return {"quantize_GBps": round(parts["quant_bytes"] / parts["quant_s"] / 1e9, 4),
+            "decode_GBps": round(parts["dec_bytes"] / parts["dec_s"] / 1e9, 4),
+            "decode_tokens_per_s": round(dec_tok, 3) if dec_tok else None,
+            "decode_tokens_per_s_basis": ("timed over all %d layers" % w.layers if n_layers == w.layers
+                                          else "extrapolated from %d of %d layers" % (n_layers, w.layers)),
+            "nproc": os.cpu_count(), "cpu_model": cpu_model()}
 
 
 def _decode_bytes_layer(w, mask_row, nq, appended, ns=0):
@@ -326,7 +366,7 @@ def _decode_bytes_layer(w, mask_row, nq, appended, ns=0):
         if prot and not w.keys_only:
             tot += (T + appended) * 512
         elif prot:
-            tot += (T - nq + appended) * 512 + nq * (256 + code_tok + vmeta)
+            tot += (T - nq + ns + appended) * 512 + (nq - ns) * (256 + code_tok + vmeta)
         else:
             tot += (T - nq + ns + appended) * 512 + (nq - ns) * (2 * code_tok + kmeta + vmeta)
     return B * tot
@@ -379,8 +419,9 @@ def run_reference(args):
     n_layers, n_steps = cpu_sample_plan(w)
     vals = []
     tot_s = 0.0
+    parts = {}
     for i in range(args.warmup + args.steps):
-        nb, secs, threads = oracle_sample(w, n_layers, n_steps)
+        nb, secs, threads = oracle_sample(w, n_layers, n_steps, parts)
         if i >= args.warmup:
             vals.append(nb / secs / 1e9)
             tot_s += secs
@@ -393,8 +434,9 @@ def run_reference(args):
         "ms_per_step": round(1000 * tot_s / max(1, args.steps), 3), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "fp32/fp64", "data": "synthetic",
         "config": workload_config(w),
-        "cpu_baseline": {"value": round(value, 4), "unit": "GB/s", "cores": threads,
-                         "kind": "oracle", "sample": sample},
+        "cpu_baseline": dict({"value": round(value, 4), "unit": "GB/s", "cores": threads,
+                              "kind": "oracle", "sample": sample},
+                             **cpu_baseline_fields(w, n_layers, n_steps, parts)),
         "e2e": {"value": round(value, 4), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -530,7 +572,7 @@ def run_gpu(args):
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms_step, 4),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "fp32", "data": "synthetic",
+        "dtype": "bf16/fp16 MMA operands, fp32 accumulate; fp32 quantizer", "data": "synthetic",
         "config": workload_config(w),
         "pct_of_8TBps": round(100 * value / NOMINAL_HBM_GBS, 2),
         "pct_of_measured_hbm": round(100 * value / peak, 2),
@@ -556,11 +598,13 @@ def run_gpu(args):
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_layers, n_steps = cpu_sample_plan(w)
-        nb, secs, threads = oracle_sample(w, n_layers, n_steps)
-        line["cpu_baseline"] = {
+        parts = {}
+        nb, secs, threads = oracle_sample(w, n_layers, n_steps, parts)
+        line["cpu_baseline"] = dict({
             "value": round(nb / secs / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
             "sample": "%s: oracle quantize of %d layer(s) then %d decode step(s) of fp64 attention "
-                      "over them; timed oracle calls only" % (w.name, n_layers, n_steps)}
+                      "over them; timed oracle calls only" % (w.name, n_layers, n_steps)},
+            **cpu_baseline_fields(w, n_layers, n_steps, parts))
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
@@ -633,12 +677,13 @@ def decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream):
     return res
 
 
-def time_dequantize(runner, w, dec_b, dev, cushion, stream, reps=3):
+def time_dequantize(runner, w, dec_b, dev, cushion, stream, reps=3, budget_bytes=4 << 30):
     """Reconstruction of every layer as BF16 (Sec. 4: code * scale + zero, the
-    AKVQ-style keys rotated back; text, protected and appended entries copied),
-    one launch per layer, L2 flushed before each group of L launches.  Bytes:
-    the cache entries a decode step reads (codes, metadata, BF16 rows) plus the
-    two BF16 outputs [B][H_kv][T + appended][128]."""
+    AKVQ-style keys rotated back; text, protected and appended entries copied):
+    one launch over as many layers as fit `budget_bytes` of output per tensor
+    (all of them on the smaller caches), L2 flushed before each group of
+    launches.  Bytes: the cache entries a decode step reads (codes, metadata,
+    BF16 rows) plus the two BF16 outputs [layers][B][H_kv][T + appended][128]."""
     import torch
 
     import paper_2609_35800_gb300 as hg
@@ -648,20 +693,24 @@ def time_dequantize(runner, w, dec_b, dev, cushion, stream, reps=3):
     dec_static = dec_b[0] - L * H * B * 512 - 2 * q_rows  # cache bytes without appended rows
     tt = w.seq_len + app
     nbytes = dec_static + L * H * B * app * 512 + L * 2 * B * H * tt * 256
-    k16 = torch.empty((B, H, tt, 128), dtype=torch.bfloat16, device=dev)
+    per_layer = B * H * tt * 256
+    chunk = max(1, min(L, budget_bytes // per_layer))
+    k16 = torch.empty((chunk, B, H, tt, 128), dtype=torch.bfloat16, device=dev)
     v16 = torch.empty_like(k16)
     times = []
     for _ in range(reps):
         cushion()
         a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a0.record(stream)
-        for l in range(L):
-            hg.hg_dequantize_kv(runner.cache, l, k16, v16, False, stream)
+        for l0 in range(0, L, chunk):
+            n = min(chunk, L - l0)
+            hg.hg_dequantize_kv(runner.cache, l0, n, k16, v16, False, stream)
         a1.record(stream)
         times.append((a0, a1))
     torch.cuda.synchronize()
     ms = statistics.mean(a.elapsed_time(b) for a, b in times)
-    return {"ms": round(ms, 4), "GBps": round(nbytes / (ms * 1e-3) / 1e9, 1), "launches": L,
+    return {"ms": round(ms, 4), "GBps": round(nbytes / (ms * 1e-3) / 1e9, 1),
+            "launches": (L + chunk - 1) // chunk, "layers_per_launch": chunk,
             "appended": app, "bytes": nbytes, "l2": "flushed before each group of launches"}
 
 

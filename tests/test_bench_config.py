@@ -58,10 +58,11 @@ def test_dequantize_bytes_on_the_one_layer_cache(monkeypatch):
 
     monkeypatch.setattr(torch.cuda, "Event", lambda enable_timing=True: Ev())
     monkeypatch.setattr(torch.cuda, "synchronize", lambda: None)
-    monkeypatch.setattr(hg, "hg_dequantize_kv", lambda c, l, k, v, f, s: calls.append((l, k.shape)))
+    monkeypatch.setattr(hg, "hg_dequantize_kv",
+                        lambda c, l, n, k, v, f, s: calls.append((l, n, k.shape)))
     r = bench.time_dequantize(runner, w, dec_b, "cpu", lambda: None, None)
     # 3 quantized heads: 64 text rows + 256 coded tokens (2 x 32 code bytes,
     # 2 x 8 metadata bytes); protected head 1: 320 BF16 rows; outputs K and V
     want = 3 * (64 * 512 + 256 * 2 * (32 + 8)) + 320 * 512 + 2 * 4 * 320 * 256
     assert r["bytes"] == want and r["appended"] == 0 and r["launches"] == 1
-    assert r["ms"] == 0.5 and calls == [(0, (1, 4, 320, 128))] * 3
+    assert r["ms"] == 0.5 and calls == [(0, 1, (1, 1, 4, 320, 128))] * 3
