@@ -644,6 +644,27 @@ def decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream):
     res["per_layer_launches"] = {"ms_per_decode_step": round(ms, 4), "launches_per_step": L,
                                  "GBps": round(dec_bytes_mean / (ms * 1e-3) / 1e9, 1),
                                  "steps_timed": n_steps, "l2": "flushed before every step"}
+    # append and attention as two launches per step (hg_append_kv, then
+    # hg_decode_attention), both over all layers
+    hg.hg_cache_reset_appended(runner.cache)
+    times = []
+    for st in range(n_steps):
+        cushion()
+        a0, a1, a2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+        a0.record(stream)
+        hg.hg_append_kv(runner.cache, 0, L, news[st][0], news[st][1], stream)
+        a1.record(stream)
+        hg.hg_decode_attention(runner.cache, 0, L, qs[st], out, 0.0, runner.ws, runner.ws_bytes, stream)
+        a2.record(stream)
+        times.append((a0, a1, a2))
+    torch.cuda.synchronize()
+    app_ms = statistics.mean(a.elapsed_time(b) for a, b, _ in times)
+    att_ms = statistics.mean(b.elapsed_time(c) for _, b, c in times)
+    res["append_then_attention"] = {
+        "append_ms": round(app_ms, 4), "append_GBps": round(app_b / (app_ms * 1e-3) / 1e9, 1),
+        "attention_ms": round(att_ms, 4),
+        "attention_GBps": round((dec_bytes_mean - app_b) / (att_ms * 1e-3) / 1e9, 1),
+        "steps_timed": n_steps, "l2": "flushed before every step"}
     # the decode loop as one CUDA graph (layer-batched launches)
     hg.hg_cache_reset_appended(runner.cache)
     graph = torch.cuda.CUDAGraph()

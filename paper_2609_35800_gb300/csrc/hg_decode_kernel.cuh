@@ -1027,9 +1027,16 @@ __device__ __noinline__ void combine_pass(const float* src, int n, int sstride, 
 // One work item with a given key / value mode: pipeline, then per-warp results
 // into shared memory (m, l, o[q][channel]).
 // ---------------------------------------------------------------------------
+// 16-byte pieces of the staged queries per thread (piece i: query row i / 16,
+// channels 8 (i % 16) .. + 7).
+template <int NT>
+struct QPieces {
+  static constexpr int n = (NT * 8 * 16 + kThreads - 1) / kThreads;
+};
+
 template <int BITS, int NT, int KM, int VM, bool ROT, int MB>
 __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int te, const DecodeParams& p,
-                                         const uint16_t* qg, int G, float* parts) {
+                                         const uint4 (&qv)[QPieces<NT>::n], int G, float* parts) {
   using TL = Tile<BITS, KM, VM, MB>;
   constexpr int NZ = NZOf<VM>::value;
   const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
@@ -1046,15 +1053,7 @@ __device__ __forceinline__ void run_item(char* smem, const Seg& sg, int tb, int 
   const uint32_t st0 = smem_u32(stages);
   const uint32_t bars = smem_u32(smem + SmemLayout<NT>::bar);
   volatile int* abort = reinterpret_cast<volatile int*>(smem + SmemLayout<NT>::bar + 8 * kMaxStages);
-  // The queries are requested first: they gate every warp's first tile and
-  // would otherwise queue behind the CTAs' tile traffic.
-  constexpr int QV = (NT * 8 * 16 + kThreads - 1) / kThreads;  // 16-byte query pieces per thread
-  uint4 qv[QV];
-#pragma unroll
-  for (int k = 0; k < QV; ++k) {
-    const int i = tid + k * kThreads;
-    qv[k] = (i < G * 16) ? ldg16(qg + i * 8) : make_uint4(0u, 0u, 0u, 0u);
-  }
+  constexpr int QV = QPieces<NT>::n;
   // Only the first tile goes in flight now: with every CTA of the launch
   // starting at once, first tiles alone make a burst the memory system serves
   // quickly, so compute starts early; the other stages are filled once the
@@ -1239,6 +1238,17 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
       r -= n0;
     }
   }
+  // The queries are requested before anything else that depends on the
+  // record: they gate every warp's first tile, and their latency now overlaps
+  // the geometry below and the first tile's copy.
+  const int G = d.G;
+  const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
+  uint4 qv[QPieces<NT>::n];
+#pragma unroll
+  for (int k = 0; k < QPieces<NT>::n; ++k) {
+    const int i = threadIdx.x + k * kThreads;
+    qv[k] = (i < G * 16) ? ldg16(qg + i * 8) : make_uint4(0u, 0u, 0u, 0u);
+  }
   const DecodeLayer& L = p.layer[li];
   const uint64_t mask = p.lt.mask[li];
   const ChunkCounts cc = {L.nbU, L.nqU, L.nqK, L.nbP};
@@ -1248,7 +1258,6 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   const LayerGeom lg = layer_geom(d, mask);
   const HeadGeom hd = head_geom(d, lg, h);
   const char* Lb = p.arena + p.lt.base[li];
-  const int G = d.G;
   const bool coded = r >= nb;
   int tb, te;
   if (!coded) {
@@ -1261,7 +1270,6 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     te = min(tb + c, ncoded(d));
   }
   const int tid = threadIdx.x;
-  const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
 
   // the warps' (m, l, o) partials [warp][16][132], in the stage buffer once the
   // tiles are consumed (the same row layout as the split partials)
@@ -1293,7 +1301,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
       }
     }
     __syncthreads();  // barriers initialised, new row stored
-    run_item<BITS, NT, K_BF16, V_BF16, false, MB>(smem, sg, tb, te, p, qg, G, parts);
+    run_item<BITS, NT, K_BF16, V_BF16, false, MB>(smem, sg, tb, te, p, qv, G, parts);
   } else if (hd.cls == kKeysOnly) {
     __syncthreads();  // barriers initialised
     sg.k = Lb + hd.kimg + b * hd.kimg_bs;
@@ -1301,9 +1309,9 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_BF16, V_KIVI, false, MB>(smem, sg, tb, te, p, qg, G, parts);
+      run_item<BITS, NT, K_BF16, V_KIVI, false, MB>(smem, sg, tb, te, p, qv, G, parts);
     else
-      run_item<BITS, NT, K_BF16, V_TOKEN, false, MB>(smem, sg, tb, te, p, qg, G, parts);
+      run_item<BITS, NT, K_BF16, V_TOKEN, false, MB>(smem, sg, tb, te, p, qv, G, parts);
   } else {
     __syncthreads();  // barriers initialised
     sg.kc = Lb + hd.kq + b * hd.kq_bs;
@@ -1311,11 +1319,11 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
     sg.vc = Lb + hd.vq + b * hd.vq_bs;
     sg.vm = Lb + hd.vqm + b * hd.vqm_bs;
     if (BASE == kKivi)
-      run_item<BITS, NT, K_KIVI, V_KIVI, false, MB>(smem, sg, tb, te, p, qg, G, parts);
+      run_item<BITS, NT, K_KIVI, V_KIVI, false, MB>(smem, sg, tb, te, p, qv, G, parts);
     else if (BASE == kAkvq)
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, true, MB>(smem, sg, tb, te, p, qg, G, parts);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, true, MB>(smem, sg, tb, te, p, qv, G, parts);
     else
-      run_item<BITS, NT, K_TOKEN, V_TOKEN, false, MB>(smem, sg, tb, te, p, qg, G, parts);
+      run_item<BITS, NT, K_TOKEN, V_TOKEN, false, MB>(smem, sg, tb, te, p, qv, G, parts);
   }
   __syncthreads();
 

@@ -370,6 +370,20 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   }
   if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
     const float r = __frcp_rn(scale);
+    // Two channels per paired operation: d = fl(x - min), then
+    // T' = RN(d r + C) with C = 192.5 + 4 * 2^-16.  In [128, 256) the grid is
+    // 2^-16, so T' is T = RN(d r + 192) moved by 0x8004 units (one unit more
+    // or less when d r + 192 falls exactly between two grid points, where the
+    // shift by an even count flips the tie-break).  Bits 16.. of T' are then
+    // floor(d r + 0.5) away from ties, and the error of T' against the exact
+    // quotient is below two units (0.5 FMA rounding, 1/16 for r, 1/16 for
+    // the reference division, 1 for the tie-break), so every element within
+    // two units of the half-integer boundary -- T' low bits in [2, 6] -- is
+    // among those with low bits in [0, 7], which take the exact rule.
+    const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
+    const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
+    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
+    const uint64_t c2 = f32x2(cbits, cbits);
     // chunks of 8 channels (one uint4 of the row): 16 code bits (2-bit) or 32
     // (4-bit); the loop stays rolled (by two) so the code is small and stays
     // in the instruction cache
@@ -378,15 +392,27 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
     for (int k = 0; k < 16; ++k) {
       const uint4 v = r4[k];
       const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint32_t a[8];
+      uint32_t low = 0xffffffffu;  // per 16-bit half: the smallest masked low bits seen
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint64_t x2 = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 8k + 2i, 8k + 2i + 1
+        const uint64_t t2 = f32x2_fma(f32x2_sub(x2, mn2), r2, c2);
+        a[2 * i] = (uint32_t)t2;
+        a[2 * i + 1] = (uint32_t)(t2 >> 32);
+        low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
+      }
       uint32_t c8[8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const uint32_t hw = w[i >> 1];
-        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
-        const uint32_t a = __float_as_uint(__fmaf_rn(d, r, 192.0f)) + 0x8001u;
-        // BF16 data puts many quotients exactly on half-integers: those (and
-        // anything within a unit of one) take the exact rule
-        c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : ((a >> 16) & L);
+      for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
+      if (__vcmpeq2(low, 0u)) {  // a near-tie in this chunk (about one chunk in 500): the exact rule
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (a[i] & 0xfff8u) continue;
+          const uint32_t hw = w[i >> 1];
+          const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
+          c8[i] = exact_code(d, scale, levels);
+        }
       }
       emit_chunk<BITS>(k, c8, codes, prev, plane);
     }
@@ -569,12 +595,19 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
 // batch row, KV head, layer); a half-warp owns one token row of K or of V,
 // lane j of it channels 8j..8j+7, so every output row is one 256-byte (BF16)
 // or 512-byte (fp32) store of 16 lanes and each lane issues its code,
-// metadata and row loads independently.  The AKVQ-style inverse rotation runs
+// metadata and row loads independently (all four units of a thread at once).
+// A BF16 entry written as BF16 is copied as it is.  The AKVQ-style inverse rotation runs
 // its first three butterfly stages inside a lane and the last four across the
 // half-warp, in the same order as the forward transform.
 // ---------------------------------------------------------------------------
 constexpr int kDqThreads = 256;
 constexpr int kDqTile = 32;
+
+// Two floats to BF16 bits (round to nearest even, low half first): one cvt.
+__device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
+  const __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<const uint32_t*>(&h);
+}
 
 __device__ __forceinline__ void bf16x8_to_f32(const uint4& w, float (&x)[8]) {
   bf16x2_to_f32(w.x, x[0], x[1]);
@@ -642,7 +675,7 @@ __device__ __forceinline__ void fwht128_half(float (&x)[8], int j) {
   for (int i = 0; i < 8; ++i) x[i] = __fmul_rn(x[i], c);
 }
 
-__global__ void __launch_bounds__(kDqThreads)
+__global__ void __launch_bounds__(kDqThreads, 5)
 dequantize_kernel(const __grid_constant__ DequantParams p) {
   const Dims& d = p.d;
   const int li = blockIdx.z, bh = blockIdx.y;
@@ -657,8 +690,8 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
   const int j = threadIdx.x & 15;  // channels 8j..8j+7
   const size_t out_row0 = (((size_t)li * d.B + b) * d.H + h) * (size_t)Tt;
 
-  // unit u: K (u < 512) or V, token (u >> 4) & 31 of the tile; unrolled so
-  // that the loads of a thread's four units are in flight together
+  // unit u: K (u < 16 * kDqTile) or V, token (u >> 4) % kDqTile of the tile;
+  // unrolled so that the loads of a thread's four units are in flight together
 #pragma unroll
   for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
     const bool is_k = u < kDqTile * 16;
@@ -679,7 +712,11 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
       spos = qs + rank;
     }
     const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
+    const size_t o = (out_row0 + t) * kD + 8 * j;
+    void* dst = is_k ? p.k_out : p.v_out;
     float x[8];
+    bool raw = false;  // a BF16 entry: `w` holds its 16 bytes
+    uint4 w = make_uint4(0u, 0u, 0u, 0u);
     if (is_k) {
       if (coded && hd.cls == kQuantized && !sal) {
         uint32_t code[8];
@@ -708,7 +745,8 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
         const char* src = (coded && hd.cls == kKeysOnly && !sal)
                               ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
                               : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
-        bf16x8_to_f32(ldg16(src + j * 16), x);
+        w = ldg16(src + j * 16);
+        raw = true;
       }
     } else {
       if (coded && hd.cls != kProtected && !sal) {
@@ -721,21 +759,20 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
 #pragma unroll
         for (int i = 0; i < 8; ++i) x[i] = dequant1(code[i], m.x, m.y);
       } else {
-        bf16x8_to_f32(ldg16(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256 + j * 16), x);
+        w = ldg16(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256 + j * 16);
+        raw = true;
       }
     }
-    const size_t o = (out_row0 + t) * kD + 8 * j;
-    void* dst = is_k ? p.k_out : p.v_out;
     if (p.out_fp32) {
+      if (raw) bf16x8_to_f32(w, x);
       float4* f = reinterpret_cast<float4*>(static_cast<float*>(dst) + o);
       f[0] = make_float4(x[0], x[1], x[2], x[3]);
       f[1] = make_float4(x[4], x[5], x[6], x[7]);
     } else {
-      *reinterpret_cast<uint4*>(static_cast<uint16_t*>(dst) + o) =
-          make_uint4(f32_to_bf16_rn(x[0]) | (f32_to_bf16_rn(x[1]) << 16),
-                     f32_to_bf16_rn(x[2]) | (f32_to_bf16_rn(x[3]) << 16),
-                     f32_to_bf16_rn(x[4]) | (f32_to_bf16_rn(x[5]) << 16),
-                     f32_to_bf16_rn(x[6]) | (f32_to_bf16_rn(x[7]) << 16));
+      if (!raw)
+        w = make_uint4(pack_bf16x2_rn(x[0], x[1]), pack_bf16x2_rn(x[2], x[3]), pack_bf16x2_rn(x[4], x[5]),
+                       pack_bf16x2_rn(x[6], x[7]));
+      *reinterpret_cast<uint4*>(static_cast<uint16_t*>(dst) + o) = w;
     }
   }
 }
