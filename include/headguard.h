@@ -24,7 +24,10 @@
  *              allocation is the hg_cache descriptor itself.
  *   Tensors    Device tensors are dense row-major BF16 (uint16 bit patterns)
  *              unless stated otherwise, head_dim = 128, and must be 16-byte
- *              aligned.
+ *              aligned.  The per-step decode inputs and outputs (q, k_new,
+ *              v_new, out) may instead be pinned host memory, which the
+ *              kernels read and write directly over the host link (no copy
+ *              engine round trip for a step's few hundred kilobytes).
  *   Streams    Every device operation is enqueued on the given stream
  *              (hg_stream_t is cudaStream_t; NULL means the legacy default
  *              stream) and returns before the GPU work completes.

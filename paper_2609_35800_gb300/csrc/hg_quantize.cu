@@ -434,9 +434,146 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   }
 }
 
+// ---------------------------------------------------------------------------
+// AKVQ-style keys (Sec. 4), one thread per vector: the BF16 row is widened
+// into 64 packed fp32 pairs (channels 2m, 2m + 1), rotated by the normalised
+// Hadamard-128 in registers -- stage h = 1 inside each pair, stages h = 2..64
+// on whole pairs (both halves of a pair meet the same partner offset), the
+// 1/sqrt(128) factor once at the end, the same butterflies in the same order
+// as the warp-wide transform -- and quantized per token like the min-max
+// rows above, with the same exact code rule.
+// ---------------------------------------------------------------------------
+__device__ __forceinline__ float pair_lo(uint64_t x) { return __uint_as_float((uint32_t)x); }
+__device__ __forceinline__ float pair_hi(uint64_t x) { return __uint_as_float((uint32_t)(x >> 32)); }
+
 template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
+  const uint32_t* r32 = reinterpret_cast<const uint32_t*>(row_s);
+  uint64_t xp[64];
+#pragma unroll
+  for (int m = 0; m < 64; ++m) {
+    const uint32_t w = r32[m];
+    const float a = __uint_as_float(w << 16), b = __uint_as_float(w & 0xffff0000u);
+    xp[m] = f32x2(__float_as_uint(__fadd_rn(a, b)), __float_as_uint(__fsub_rn(a, b)));  // stage h = 1
+  }
+#pragma unroll
+  for (int hp = 1; hp < 64; hp <<= 1) {  // stage h = 2 hp
+#pragma unroll
+    for (int m = 0; m < 64; ++m) {
+      if (m & hp) continue;
+      const uint64_t a = xp[m], b = xp[m + hp];
+      xp[m] = f32x2_add(a, b);
+      xp[m + hp] = f32x2_sub(a, b);
+    }
+  }
+  {
+    const uint32_t cb = __float_as_uint(hadamard_c());
+    const uint64_t c2 = f32x2(cb, cb);
+#pragma unroll
+    for (int m = 0; m < 64; ++m) xp[m] = f32x2_mul(xp[m], c2);
+  }
+  // min / max of the rotated vector (exact; signed zeros folded to +0)
+  float mn = fminf(pair_lo(xp[0]), pair_hi(xp[0])), mx = fmaxf(pair_lo(xp[0]), pair_hi(xp[0]));
+  {
+    float mn1 = fminf(pair_lo(xp[1]), pair_hi(xp[1])), mx1 = fmaxf(pair_lo(xp[1]), pair_hi(xp[1]));
+#pragma unroll
+    for (int m = 2; m < 64; m += 2) {
+      mn = fminf(mn, fminf(pair_lo(xp[m]), pair_hi(xp[m])));
+      mx = fmaxf(mx, fmaxf(pair_lo(xp[m]), pair_hi(xp[m])));
+      mn1 = fminf(mn1, fminf(pair_lo(xp[m + 1]), pair_hi(xp[m + 1])));
+      mx1 = fmaxf(mx1, fmaxf(pair_lo(xp[m + 1]), pair_hi(xp[m + 1])));
+    }
+    mn = fminf(mn, mn1);
+    mx = fmaxf(mx, mx1);
+  }
+  mn = __fadd_rn(mn, 0.0f);
+  mx = __fadd_rn(mx, 0.0f);
+  constexpr uint32_t L = (1u << BITS) - 1u;
+  const float levels = (float)L;
+  float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  if (M16) {
+    scale = half_sat(scale);
+    mn = half_sat(mn);
+  }
+  store_meta(meta, mi, scale, mn, M16);
+  constexpr int W = 4 * BITS;
+  if (scale == 0.0f) {
+#pragma unroll
+    for (int i = 0; i < W; ++i) codes[i] = 0u;
+    return;
+  }
+  uint32_t prev = 0u, plane = 0u;
+  if (M16) {  // as the min-max rows: the quotient clamped, then the same near-tie rule
+    const float r = __frcp_rn(scale);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      uint32_t c8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const uint64_t x2 = xp[4 * k + (i >> 1)];
+        const float d = __fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn);
+        const float q = fminf(fmaxf(__fmul_rn(d, r), -1.0f), levels + 1.0f);
+        const uint32_t a = __float_as_uint(__fadd_rn(q, 192.0f)) + 0x8001u;
+        const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
+        c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
+      }
+      emit_chunk<BITS>(k, c8, codes, prev, plane);
+    }
+    return;
+  }
+  if (scale >= 2.3509887e-38f) {  // the fast rule of the min-max rows (see there)
+    const float r = __frcp_rn(scale);
+    const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
+    const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
+    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
+    const uint64_t c2 = f32x2(cbits, cbits);
+#pragma unroll
+    for (int k = 0; k < 16; ++k) {
+      uint32_t a[8];
+      uint32_t low = 0xffffffffu;
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const uint64_t t2 = f32x2_fma(f32x2_sub(xp[4 * k + i], mn2), r2, c2);
+        a[2 * i] = (uint32_t)t2;
+        a[2 * i + 1] = (uint32_t)(t2 >> 32);
+        low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
+      }
+      uint32_t c8[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
+      if (__vcmpeq2(low, 0u)) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          if (a[i] & 0xfff8u) continue;
+          const uint64_t x2 = xp[4 * k + (i >> 1)];
+          c8[i] = exact_code(__fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn), scale, levels);
+        }
+      }
+      emit_chunk<BITS>(k, c8, codes, prev, plane);
+    }
+    return;
+  }
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {  // tiny scale: the exact rule throughout
+    uint32_t c8[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint64_t x2 = xp[4 * k + (i >> 1)];
+      c8[i] = exact_code(__fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn), scale, levels);
+    }
+    emit_chunk<BITS>(k, c8, codes, prev, plane);
+  }
+}
+
+// The per-token bases, one thread per vector: min-max rows (Sec. 1) and
+// AKVQ-style rows (Sec. 4: keys rotated first; values per token, unrotated).
+// With salient tokens (AKVQ-style, Sec. 4) a thread finds its token in the
+// head's map: a salient token's K and V rows go to the BF16 region at
+// position s + (its rank), every other image token to coded slot ti - (the
+// salient tokens before it).
+template <int BITS, bool M16, int BASE>
 __global__ void __launch_bounds__(kThreads)
-quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
+quantize_token_kernel(const __grid_constant__ QuantizeParams p) {
   const Dims& d = p.d;
   const int li = blockIdx.z, bh = blockIdx.y;
   const int b = bh / d.H, h = bh % d.H;
@@ -469,30 +606,40 @@ quantize_minmax_kernel(const __grid_constant__ QuantizeParams p) {
   const int t = t0 + r;
   const bool coded = t >= d.s && t < d.s + d.nq;
   const int ti = t - d.s;
+  int ci = ti, pos = bf16_pos(d, hd.cls, t);
+  bool sal = false;
+  if (BASE == kAkvq && coded && d.ns > 0 && hd.cls != kProtected) {
+    const char* sm = Lb + hd.sal + b * hd.sal_bs;
+    const int w = ti >> 5, e = ti & 31;
+    const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
+    const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
+                     __popc(sb & ((1u << e) - 1u));
+    sal = (sb >> e) & 1u;
+    ci = ti - rank;
+    if (sal) pos = d.s + rank;
+  }
   const char* row_s = rows[kv][r];
   constexpr int W = 4 * BITS;
+  char* dst;
   if (kv == 0) {
-    if (coded && hd.cls == kQuantized) {
-      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ti * W,
-                                    Lb + hd.kqm + b * hd.kqm_bs, ti);
+    if (coded && hd.cls == kQuantized && !sal) {
+      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
+      if (BASE == kAkvq) quantize_row_rotated<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
+      else quantize_row_token<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
       return;
     }
-    char* dst = (coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
-                                               : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+    dst = (coded && hd.cls == kKeysOnly && !sal) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
+                                                 : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
   } else {
-    if (coded && hd.cls != kProtected) {
-      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
-                                    Lb + hd.vqm + b * hd.vqm_bs, ti);
+    if (coded && hd.cls != kProtected && !sal) {
+      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
+                                    Lb + hd.vqm + b * hd.vqm_bs, ci);
       return;
     }
-    char* dst = Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
-#pragma unroll
-    for (int k = 0; k < 16; ++k)
-      reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+    dst = Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256;
   }
+#pragma unroll
+  for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
 }
 
 // ---------------------------------------------------------------------------
@@ -681,8 +828,12 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
   const int li = blockIdx.z, bh = blockIdx.y;
   const int b = bh / d.H, h = bh % d.H;
   const int Tt = d.T + p.appended;
-  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-  const HeadGeom hd = head_geom(d, g, h);
+  // the head's region map, computed once for the CTA (64-bit arithmetic that
+  // would otherwise cost every warp more instructions than its four units)
+  __shared__ HeadGeom s_hd;
+  if (threadIdx.x == 0) s_hd = head_geom(d, layer_geom(d, p.lt.mask[li]), h);
+  __syncthreads();
+  const HeadGeom& hd = s_hd;
   const char* Lb = p.arena + p.lt.base[li];
   const int qs = d.s, qe = d.s + d.nq;
   const int W = kD * d.bits / 32;
@@ -799,25 +950,28 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 
 }  // namespace
 
-cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
-  if (p.d.base == kMinMax) {  // one thread per vector
-    dim3 grid((p.d.T + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
-    const bool m16 = p.d.meta16 != 0;
-    if (p.d.bits == 2) {
-      if (m16) quantize_minmax_kernel<2, true><<<grid, kThreads, 0, s>>>(p);
-      else quantize_minmax_kernel<2, false><<<grid, kThreads, 0, s>>>(p);
-    } else if (p.d.bits == 3) {
-      if (m16) quantize_minmax_kernel<3, true><<<grid, kThreads, 0, s>>>(p);
-      else quantize_minmax_kernel<3, false><<<grid, kThreads, 0, s>>>(p);
-    } else {
-      if (m16) quantize_minmax_kernel<4, true><<<grid, kThreads, 0, s>>>(p);
-      else quantize_minmax_kernel<4, false><<<grid, kThreads, 0, s>>>(p);
-    }
-    return cudaGetLastError();
+template <int BASE>
+cudaError_t launch_token(const QuantizeParams& p, cudaStream_t s) {
+  dim3 grid((p.d.T + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
+  const bool m16 = p.d.meta16 != 0;
+  if (p.d.bits == 2) {
+    if (m16) quantize_token_kernel<2, true, BASE><<<grid, kThreads, 0, s>>>(p);
+    else quantize_token_kernel<2, false, BASE><<<grid, kThreads, 0, s>>>(p);
+  } else if (p.d.bits == 3) {
+    if (m16) quantize_token_kernel<3, true, BASE><<<grid, kThreads, 0, s>>>(p);
+    else quantize_token_kernel<3, false, BASE><<<grid, kThreads, 0, s>>>(p);
+  } else {
+    if (m16) quantize_token_kernel<4, true, BASE><<<grid, kThreads, 0, s>>>(p);
+    else quantize_token_kernel<4, false, BASE><<<grid, kThreads, 0, s>>>(p);
   }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
+  if (p.d.base == kMinMax) return launch_token<kMinMax>(p, s);  // one thread per vector
+  if (p.d.base == kAkvq) return launch_token<kAkvq>(p, s);
   dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
-  if (p.d.base == kKivi) quantize_kernel<kKivi><<<grid, kThreads, 0, s>>>(p);
-  else quantize_kernel<kAkvq><<<grid, kThreads, 0, s>>>(p);
+  quantize_kernel<kKivi><<<grid, kThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 

@@ -404,3 +404,24 @@ def test_bounded_wait_gives_up_and_flags():
     assert int(word[0].item()) == 3
     # the device still works: an ordinary decode afterwards is correct
     _run_and_check(_workload(CASES[1]))
+
+
+def test_decode_step_reads_and_writes_pinned_host_memory():
+    """The decode step's query, new K/V and output may live in pinned host
+    memory (addressable from the device): the result is bit-identical to the
+    same step on device buffers, and the new tokens land in the cache."""
+    w = _workload(CASES[0])
+    ra, rb = CacheRunner(w), CacheRunner(w)
+    ra.quantize_all()
+    rb.quantize_all()
+    for step in range(w.decode_steps):
+        k_new, v_new = wl.step_new_kv(w, step, "cuda")
+        q = wl.step_query(w, step, "cuda")
+        out = torch.empty_like(q)
+        hg.hg_decode_step(ra.cache, 0, w.layers, q, k_new, v_new, out, SIGMA, ra.ws, ra.ws_bytes)
+        hq, hk, hv = q.cpu().pin_memory(), k_new.cpu().pin_memory(), v_new.cpu().pin_memory()
+        hout = torch.full(q.shape, float("nan"), dtype=q.dtype).pin_memory()
+        hg.hg_decode_step(rb.cache, 0, w.layers, hq.data_ptr(), hk.data_ptr(), hv.data_ptr(),
+                          hout.data_ptr(), SIGMA, rb.ws, rb.ws_bytes)
+        torch.cuda.synchronize()
+        assert torch.equal(hout.view(torch.int16), out.cpu().view(torch.int16)), "step %d" % step
