@@ -1206,6 +1206,11 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   // swizzled TMA boxes need 1024-byte aligned shared addresses
   char* smem = smem_raw + ((1024u - (smem_u32(smem_raw) & 1023u)) & 1023u);
   const Dims& d = p.d;
+  // Programmatic dependent launch: the next launch on the stream (the next
+  // layer's or step's decode) may be scheduled as soon as every CTA of this
+  // one runs; it builds its prologue from its parameters and waits (below)
+  // before it touches memory that earlier kernels write.
+  grid_launch_dependents();
   if ((int)blockIdx.x >= p.total_items) return;
   if (threadIdx.x == 0) {
     const uint32_t bars = smem_u32(smem + SmemLayout<NT>::bar);
@@ -1238,17 +1243,7 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
       r -= n0;
     }
   }
-  // The queries are requested before anything else that depends on the
-  // record: they gate every warp's first tile, and their latency now overlaps
-  // the geometry below and the first tile's copy.
   const int G = d.G;
-  const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
-  uint4 qv[QPieces<NT>::n];
-#pragma unroll
-  for (int k = 0; k < QPieces<NT>::n; ++k) {
-    const int i = threadIdx.x + k * kThreads;
-    qv[k] = (i < G * 16) ? ldg16(qg + i * 8) : make_uint4(0u, 0u, 0u, 0u);
-  }
   const DecodeLayer& L = p.layer[li];
   const uint64_t mask = p.lt.mask[li];
   const ChunkCounts cc = {L.nbU, L.nqU, L.nqK, L.nbP};
@@ -1258,6 +1253,19 @@ decode_kernel(const __grid_constant__ DecodeParams p) {
   const LayerGeom lg = layer_geom(d, mask);
   const HeadGeom hd = head_geom(d, lg, h);
   const char* Lb = p.arena + p.lt.base[li];
+  // Everything above comes from the launch parameters.  From here on the CTA
+  // reads the queries, the new K/V, the arena and the workspace, which the
+  // kernels before this one on the stream write.
+  grid_dependency_wait();
+  // The queries are requested first: they gate every warp's first tile, and
+  // their latency overlaps the first tile's copy.
+  const uint16_t* qg = p.q + (((size_t)li * d.B + b) * d.Hq + (size_t)h * G) * kD;
+  uint4 qv[QPieces<NT>::n];
+#pragma unroll
+  for (int k = 0; k < QPieces<NT>::n; ++k) {
+    const int i = threadIdx.x + k * kThreads;
+    qv[k] = (i < G * 16) ? ldg16(qg + i * 8) : make_uint4(0u, 0u, 0u, 0u);
+  }
   const bool coded = r >= nb;
   int tb, te;
   if (!coded) {
@@ -1398,7 +1406,18 @@ cudaError_t launch_t(const DecodeParams& p, int grid_x, cudaStream_t s) {
     if (dev >= 0 && dev < 64) configured[dev].store(true, std::memory_order_release);
   }
   (void)grid_x;
-  decode_kernel<BITS, NT, BASE, MB><<<p.total_items, kThreads, SmemLayout<NT>::bytes, s>>>(p);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((unsigned)p.total_items, 1, 1);
+  cfg.blockDim = dim3(kThreads, 1, 1);
+  cfg.dynamicSmemBytes = SmemLayout<NT>::bytes;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  e = cudaLaunchKernelEx(&cfg, decode_kernel<BITS, NT, BASE, MB>, p);
+  if (e != cudaSuccess) return e;
   return cudaGetLastError();
 }
 

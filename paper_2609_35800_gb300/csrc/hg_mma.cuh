@@ -58,6 +58,16 @@ __device__ __forceinline__ uint64_t f32x2_fma(uint64_t a, uint64_t b, uint64_t c
   return r;
 }
 
+// Programmatic dependent launch (PTX griddepcontrol): let the next grid on the
+// stream be scheduled once every CTA of this one has issued this (or exited),
+// and wait until the grids this one depends on have completed and their
+// memory operations are visible.  Both are no-ops for a launch without a
+// programmatic dependency.
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;\n" ::: "memory");
+}
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;\n" ::: "memory"); }
+
 // Transpose of an 8x8 16-bit matrix held one row-pair per lane.
 __device__ __forceinline__ uint32_t movtrans(uint32_t x) {
   uint32_t y;
