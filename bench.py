@@ -567,6 +567,10 @@ def run_gpu(args):
         deq = time_dequantize(runner, w, dec_b, dev, cushion, stream)
     except Exception as exc:  # a side measurement never costs the line
         deq = {"error": "%s: %s" % (type(exc).__name__, exc)}
+    try:
+        floors = measure_floors(int(dec_bytes_mean), cushion, stream, dev)
+    except Exception as exc:
+        floors = {"error": "%s: %s" % (type(exc).__name__, exc)}
 
     line = {
         "metric": METRIC, "value": round(value, 2), "unit": "GB/s", "n_gpus": world,
@@ -589,6 +593,7 @@ def run_gpu(args):
                      "frac": round(achieved / peak, 4), "traffic": traffic,
                      "kernel": "decode_kernel (hg_decode_step)",
                      "peak_source": peak_src + " hbm_gbs (burst copy)"},
+        "floors": floors,
         "clocks": clk.summary(),
         "gpu_launches": launches_per_step * args.steps,
     }
@@ -696,6 +701,36 @@ def decode_variants(args, runner, w, qs, news, dec_b, app_b, cushion, stream):
                            "l2": "flushed before each replay of the %d-step loop only" % S}
     hg.hg_cache_reset_appended(runner.cache)
     return res
+
+
+def measure_floors(nbytes, cushion, stream, dev, reps=10):
+    """Fixed costs of an event-timed launch on this device, for reading the
+    decode fraction: two events with nothing between them, one near-empty
+    kernel, and a plain read of the decode step's byte count by torch's own
+    reduction (the same L2 flush before each).  Medians in microseconds."""
+    import torch
+    buf = torch.ones(max(1, nbytes // 4), dtype=torch.int32, device=dev)
+
+    def timed(fn):
+        ts = []
+        for _ in range(reps):
+            cushion()
+            a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a0.record(stream)
+            fn()
+            a1.record(stream)
+            ts.append((a0, a1))
+        torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) * 1000.0 for a, b in ts)
+
+    events = timed(lambda: None)
+    empty = timed(lambda: torch.cuda._sleep(0))
+    read = timed(lambda: buf.max())
+    return {"events_only_us": round(events, 2), "empty_kernel_us": round(empty, 2),
+            "read_same_bytes_us": round(read, 2), "read_bytes": buf.numel() * 4,
+            "read_GBps": round(buf.numel() * 4 / (read * 1e-6) / 1e9, 1),
+            "how": "CUDA events on the launching stream after the same L2 flush; the read is "
+                   "torch.max over an int32 buffer of the decode step's byte count"}
 
 
 def time_dequantize(runner, w, dec_b, dev, cushion, stream, reps=3, budget_bytes=4 << 30):

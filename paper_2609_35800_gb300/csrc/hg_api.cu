@@ -413,7 +413,6 @@ hg_status hg_quantize_kv(hg_cache* c, int32_t layer_begin, int32_t layer_count,
     p.arena = c->arena;
     p.n_layers = n;
     p.tile_origin = d.s % 32;
-    p.n_tiles = (d.T - p.tile_origin + 32 + 31) / 32;
     fill_table(c, layer_begin + done, n, &p.lt);
     for (int i = 0; i < n; ++i) {
       p.k[i] = static_cast<const uint16_t*>(k[done + i]);

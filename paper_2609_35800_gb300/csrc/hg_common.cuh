@@ -120,38 +120,6 @@ __device__ __forceinline__ uint32_t code_of(float d, float scale, float r, float
   return (uint32_t)rq;
 }
 
-// Group quantizer over a group spread across GL consecutive lanes (aligned),
-// 4 values per lane.  min / max by butterflies (exact), signed zeros folded to
-// +0, scale = (max - min) / (2^bits - 1), code = round-half-even((x - min) /
-// scale) clamped to the levels, codes 0 when scale == 0, zero = min.  With
-// m16 the scale and zero are first rounded to binary16 and the codes taken
-// against the rounded pair.
-template <int GL>
-__device__ __forceinline__ void quantize_group4(const float (&x)[4], int bits, bool m16, uint32_t (&code)[4],
-                                                float& scale, float& zero) {
-  float mn = fminf(fminf(x[0], x[1]), fminf(x[2], x[3]));
-  float mx = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-#pragma unroll
-  for (int o = 1; o < GL; o <<= 1) {
-    mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
-    mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-  }
-  mn = __fadd_rn(mn, 0.0f);
-  mx = __fadd_rn(mx, 0.0f);
-  const float levels = (float)((1 << bits) - 1);
-  scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
-  zero = mn;
-  if (m16) {
-    scale = half_sat(scale);
-    zero = half_sat(zero);
-  }
-  const bool fast = scale >= 2.3509887e-38f;  // 2^-125
-  const float r = __frcp_rn(fast ? scale : 1.0f);
-#pragma unroll
-  for (int i = 0; i < 4; ++i)
-    code[i] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[i], zero), scale, r, levels, fast);
-}
-
 // Reconstruction fl32(fl32(code * scale) + zero).
 __device__ __forceinline__ float dequant1(uint32_t code, float scale, float zero) {
   return __fadd_rn(__fmul_rn((float)code, scale), zero);

@@ -21,8 +21,7 @@ struct QuantizeParams {
   Dims d;
   char* arena;
   int n_layers;
-  int n_tiles;      // 32-token tiles per (row, head)
-  int tile_origin;  // tile i covers [tile_origin - 32 + 32 i, +32) clipped to [0, T)
+  int tile_origin;  // s mod 32: KIVI-style tile i covers [tile_origin - 32 + 64 i, +64) clipped to [0, T)
   LayerTable lt;
   const uint16_t* k[kMaxLayersPerLaunch];
   const uint16_t* v[kMaxLayersPerLaunch];

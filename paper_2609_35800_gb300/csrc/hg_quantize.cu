@@ -1,15 +1,15 @@
 // Quantize-pack, dequantize and append kernels of the HeadGuard KV cache.
 //
 // Quantize (Sec. 3 "Applying protection" over the Sec. 1 / Sec. 4 bases).
-// Per-token min-max base: quantize_minmax_kernel below, one thread per
-// vector.  KIVI- and AKVQ-style bases: quantize_kernel,
-// one CTA per (32-token tile, batch row, KV head, layer).  The head's class
-// and the image span are resolved once per CTA, so protected heads and text
-// tokens take a uniform BF16 copy path.  A warp owns one token at a time,
-// each lane four consecutive channels; per-token groups reduce their min /
-// max with warp butterflies, KIVI-style value groups (32 channels) with
-// 8-lane butterflies, and KIVI-style key groups (32 tokens of one channel) are
-// quantized by one thread per channel from a shared-memory copy of the tile.
+// Every base stages a 64-token tile of one (layer, batch row, KV head) in
+// shared memory with coalesced asynchronous copies and then works one thread
+// per vector: per-token min-max rows (Sec. 1), AKVQ-style rows (Sec. 4: keys
+// rotated by the Hadamard-128 in registers first), KIVI-style value rows
+// (four 32-channel groups) and KIVI-style key groups (one thread per channel
+// over 32 consecutive image tokens).  The head's class and the image span are
+// resolved once per CTA, so protected heads and text tokens take a uniform
+// BF16 copy path.  Codes, scales and zeros follow the group quantizer exactly
+// (round half to even of the IEEE quotient, no contraction).
 #include <climits>
 
 #include <cuda_bf16.h>
@@ -24,41 +24,7 @@ namespace hg {
 namespace {
 
 constexpr int kThreads = 128;
-constexpr int kTile = 32;
 constexpr unsigned kFull = 0xffffffffu;
-
-// 3-bit codes (the 2-bit low part, then the bit-2 plane): bit position, in
-// plane word l / 8, of the bit 2 of channel 4l (channels 4l..4l+3 follow it).
-// Channel e sits at e mod 32 with index bits 3 and 4 exchanged.
-__device__ __forceinline__ int plane_base(int lane) {
-  return 4 * (lane & 1) + 8 * ((lane >> 2) & 1) + 16 * ((lane >> 1) & 1);
-}
-
-// Pack one token's 128 codes (lane l holds channels 4l..4l+3) in channel order,
-// LSB-first, and store its 4*bits words (3 bits: 8 words of bits 0-1, then 4
-// plane words of bit 2).
-__device__ __forceinline__ void store_token_codes(uint32_t* row, const uint32_t (&c)[4], int bits,
-                                                  int lane) {
-  if (bits == 2 || bits == 3) {
-    uint32_t x = ((c[0] & 3u) | ((c[1] & 3u) << 2) | ((c[2] & 3u) << 4) | ((c[3] & 3u) << 6)) << (8 * (lane & 3));
-    x |= __shfl_xor_sync(kFull, x, 1);
-    x |= __shfl_xor_sync(kFull, x, 2);
-    if ((lane & 3) == 0) row[lane >> 2] = x;
-    if (bits == 3) {
-      uint32_t hp = (((c[0] >> 2) & 1u) | (((c[1] >> 2) & 1u) << 1) | (((c[2] >> 2) & 1u) << 2) |
-                     (((c[3] >> 2) & 1u) << 3))
-                    << plane_base(lane);
-      hp |= __shfl_xor_sync(kFull, hp, 1);
-      hp |= __shfl_xor_sync(kFull, hp, 2);
-      hp |= __shfl_xor_sync(kFull, hp, 4);
-      if ((lane & 7) == 0) row[8 + (lane >> 3)] = hp;
-    }
-  } else {
-    uint32_t x = (c[0] | (c[1] << 4) | (c[2] << 8) | (c[3] << 12)) << (16 * (lane & 1));
-    x |= __shfl_xor_sync(kFull, x, 1);
-    if ((lane & 1) == 0) row[lane >> 1] = x;
-  }
-}
 
 __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
   bf16x2_to_f32(w.x, x[0], x[1]);
@@ -89,160 +55,6 @@ __device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGrou
 #pragma unroll
   for (int e = 0; e < kKiviGroup; ++e)
     code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], zero), scale, r, levels, fast);
-}
-
-template <int BASE>
-__global__ void __launch_bounds__(kThreads)
-quantize_kernel(const __grid_constant__ QuantizeParams p) {
-  const Dims& d = p.d;
-  const int tile = blockIdx.x, bh = blockIdx.y, li = blockIdx.z;
-  const int b = bh / d.H, h = bh % d.H;
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-
-  int t0 = p.tile_origin - kTile + kTile * tile;
-  int t1 = t0 + kTile;
-  if (t0 < 0) t0 = 0;
-  if (t1 > d.T) t1 = d.T;
-  if (t0 >= t1) return;
-
-  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-  const HeadGeom hd = head_geom(d, g, h);
-  char* Lb = p.arena + p.lt.base[li];
-  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T;
-  const uint16_t* K = p.k[li] + row0 * kD;
-  const uint16_t* V = p.v[li] + row0 * kD;
-  const int qs = d.s, qe = d.s + d.nq;
-  const int W = kD * d.bits / 32;  // code words per token
-  const bool m16 = d.meta16 != 0;
-  // A whole KIVI-style key group of a quantized head: tokens [t0, t0 + 32).
-  const bool kivi_k_tile = (BASE == kKivi) && (hd.cls == kQuantized) && t0 >= qs && t1 <= qe;
-
-  __shared__ __align__(16) uint16_t ktile[kTile][kD];
-
-  // AKVQ-style salient tokens (Sec. 4): the map of this tile's image tokens,
-  // in every head whose image values are coded (quantized and keys-only
-  // heads).  Image tiles start on the image's 32-token blocks, so one map
-  // word covers the tile: a salient token goes to BF16 position qs + (its
-  // rank among the salient tokens), every other image token to coded slot
-  // ti - (the salient tokens before it).
-  uint32_t sbits = 0u;
-  int srank = 0;
-  const bool sal_tile = d.ns > 0 && hd.cls != kProtected && t0 >= qs && t0 < qe;
-  if (sal_tile) {
-    const char* sm = Lb + hd.sal + b * hd.sal_bs;
-    const int w = (t0 - qs) >> 5;
-    sbits = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
-    srank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w);
-  }
-
-  // The warp's tokens t0 + warp + 4i, one at a time, the next token's K and V
-  // loaded while this one is processed.  The loop stays rolled: the token
-  // body is long, and eight unrolled copies of it thrash the instruction cache.
-  // (Staging the whole tile in shared memory with asynchronous copies first
-  // measured slower for this kernel.)
-  uint2 kn = make_uint2(0u, 0u), vn = make_uint2(0u, 0u);
-  if (t0 + warp < t1) {
-    kn = ldg8(K + (size_t)(t0 + warp) * kD + lane * 4);
-    vn = ldg8(V + (size_t)(t0 + warp) * kD + lane * 4);
-  }
-#pragma unroll 1
-  for (int t = t0 + warp; t < t1; t += 4) {
-    const uint2 kri = kn, vri = vn;
-    if (t + 4 < t1) {
-      kn = ldg8(K + (size_t)(t + 4) * kD + lane * 4);
-      vn = ldg8(V + (size_t)(t + 4) * kD + lane * 4);
-    }
-    const bool coded = (t >= qs) && (t < qe);
-    const int ti = t - qs;
-    int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token
-    bool sal = false;
-    if (sal_tile && coded) {
-      const int j = t - t0;
-      const int rank = srank + __popc(sbits & ((1u << j) - 1u));
-      sal = (sbits >> j) & 1u;
-      ci = ti - rank;
-      spos = qs + rank;
-    }
-
-    // ---- key ----
-    if (coded && hd.cls == kQuantized && !sal) {
-      if (BASE == kKivi) {
-        *reinterpret_cast<uint2*>(&ktile[t - t0][lane * 4]) = kri;
-      } else {
-        float x[4];
-        bf16x4_to_f32(kri, x);
-        if (BASE == kAkvq) fwht128_warp(x, lane);  // rotate, then per-token RTN
-        uint32_t c[4];
-        float sc, z;
-        quantize_group4<32>(x, d.bits, m16, c, sc, z);
-        uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
-        store_token_codes(crow, c, d.bits, lane);
-        if (lane == 0) store_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, sc, z, m16);
-      }
-    } else if (coded && hd.cls == kKeysOnly && !sal) {
-      *reinterpret_cast<uint2*>(Lb + hd.kimg + b * hd.kimg_bs + ((size_t)ci * kD + lane * 4) * 2) = kri;
-    } else {
-      const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
-      *reinterpret_cast<uint2*>(Lb + hd.kb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) = kri;
-    }
-
-    // ---- value (never rotated) ----
-    if (coded && hd.cls != kProtected && !sal) {
-      float x[4];
-      bf16x4_to_f32(vri, x);
-      uint32_t c[4];
-      float sc, z;
-      char* meta = Lb + hd.vqm + b * hd.vqm_bs;
-      const size_t mi = (size_t)ci * vgroups(d);
-      if (BASE == kKivi) {
-        quantize_group4<8>(x, d.bits, m16, c, sc, z);  // 32-channel groups: lanes 8j..8j+7
-        if ((lane & 7) == 0) store_meta(meta, mi + (lane >> 3), sc, z, m16);
-      } else {
-        quantize_group4<32>(x, d.bits, m16, c, sc, z);
-        if (lane == 0) store_meta(meta, mi, sc, z, m16);
-      }
-      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W;
-      store_token_codes(crow, c, d.bits, lane);
-    } else {
-      const int pos = sal ? spos : bf16_pos(d, hd.cls, t);
-      *reinterpret_cast<uint2*>(Lb + hd.vb + b * hd.kb_bs + ((size_t)pos * kD + lane * 4) * 2) = vri;
-    }
-  }
-
-  if (!kivi_k_tile) return;  // uniform over the CTA
-  __syncthreads();
-  // KIVI-style keys: thread c quantizes channel c over the 32-token group.
-  const int c = threadIdx.x;
-  float x[kKiviGroup];
-#pragma unroll
-  for (int e = 0; e < kKiviGroup; ++e) x[e] = bf16_to_f32(ktile[e][c]);
-  uint32_t code[kKiviGroup];
-  float sc, z;
-  quantize_group_serial(x, d.bits, m16, code, sc, z);
-  const int grp = (t0 - qs) / kKiviGroup;
-  uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * d.bits;
-  if (d.bits == 3) {  // two words of bits 0-1 (16 tokens each), then the bit-2 plane
-    uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
-#pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      lo0 |= (code[e] & 3u) << (2 * e);
-      lo1 |= (code[16 + e] & 3u) << (2 * e);
-    }
-#pragma unroll
-    for (int e = 0; e < 32; ++e)
-      hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
-    dst[0] = lo0;
-    dst[1] = lo1;
-    dst[2] = hp;
-  } else {
-    const int per = 32 / d.bits;
-    for (int w = 0; w < d.bits; ++w) {
-      uint32_t word = 0;
-      for (int e = 0; e < per; ++e) word |= code[w * per + e] << (d.bits * e);
-      dst[w] = word;
-    }
-  }
-  store_meta(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + c, sc, z, m16);
 }
 
 // ---------------------------------------------------------------------------
@@ -303,16 +115,98 @@ __device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32
   }
 }
 
+// Codes of the 8 channels of one chunk (four BF16 pairs w[0..3]) in a group
+// with minimum mn and step scale > 0, r = RN(1 / scale):
+//   M16 (binary16 metadata, always a normal r): a binary16 scale is at least
+//     2^-24, so r is finite.  The rounded zero and scale can put a quotient
+//     outside [0, levels]: q = d r is clamped to [-1, levels + 1] (which
+//     decides no code differently), then T = RN(q + 192) lies in
+//     [191, 193 + levels] and bits 16.. of T + 0x8001, less 0x4340, are the
+//     unclamped code.  The two roundings (q, then T) keep T within 2^-16 of
+//     fl(d / scale) + 192 for quotients that can decide a code, so an element
+//     whose low bits are not within one unit of 0x8000 rounds as the exact
+//     rule does; the others take it.
+//   fast (scale >= 2^-125, 1 / scale finite): two channels per paired
+//     operation, d = fl(x - min), then T' = RN(d r + C) with
+//     C = 192.5 + 4 * 2^-16.  In [128, 256) the grid is 2^-16, so T' is
+//     T = RN(d r + 192) moved by 0x8004 units (one unit more or less when
+//     d r + 192 falls exactly between two grid points, where the shift by an
+//     even count flips the tie-break).  Bits 16.. of T' are then
+//     floor(d r + 0.5) away from ties, and the error of T' against the exact
+//     quotient is below two units (0.5 FMA rounding, 1/16 for r, 1/16 for the
+//     reference division, 1 for the tie-break), so every element within two
+//     units of the half-integer boundary -- T' low bits in [2, 6] -- is among
+//     those with low bits in [0, 7], which take the exact rule.
+//   otherwise (tiny scale): the exact rule for every element.
 template <int BITS, bool M16>
-__device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
-  const uint4* r4 = reinterpret_cast<const uint4*>(row_s);
-  __nv_bfloat162 mn2, mx2;
-  {
-    const uint4 v = r4[0];
-    mn2 = mx2 = *reinterpret_cast<const __nv_bfloat162*>(&v.x);
+__device__ __forceinline__ void chunk_codes(const uint32_t (&w)[4], float mn, float scale, float r, bool fast,
+                                            uint32_t (&c8)[8]) {
+  constexpr uint32_t L = (1u << BITS) - 1u;
+  const float levels = (float)L;
+  if (M16) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t hw = w[i >> 1];
+      const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
+      const float q = fminf(fmaxf(__fmul_rn(d, r), -1.0f), levels + 1.0f);
+      const uint32_t a = __float_as_uint(__fadd_rn(q, 192.0f)) + 0x8001u;
+      const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
+      c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
+    }
+    return;
+  }
+  if (fast) {
+    const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
+    const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
+    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
+    const uint64_t c2 = f32x2(cbits, cbits);
+    uint32_t a[8];
+    uint32_t low = 0xffffffffu;  // per 16-bit half: the smallest masked low bits seen
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const uint64_t x2 = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1 of the chunk
+      const uint64_t t2 = f32x2_fma(f32x2_sub(x2, mn2), r2, c2);
+      a[2 * i] = (uint32_t)t2;
+      a[2 * i + 1] = (uint32_t)(t2 >> 32);
+      low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
+    }
+#pragma unroll
+    for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
+    if (__vcmpeq2(low, 0u)) {  // a near-tie in this chunk (about one chunk in 500): the exact rule
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (a[i] & 0xfff8u) continue;
+        const uint32_t hw = w[i >> 1];
+        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
+        c8[i] = exact_code(d, scale, levels);
+      }
+    }
+    return;
   }
 #pragma unroll
-  for (int k = 0; k < 16; ++k) {
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t hw = w[i >> 1];
+    const float x = __uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16));
+    c8[i] = exact_code(__fsub_rn(x, mn), scale, levels);
+  }
+}
+
+// One group of a BF16 row: chunks [k0, k0 + nk) (8 channels each) with their
+// min / max over bf16x2 pairs (exact), signed zeros folded to +0,
+// scale = fl((max - min) / levels), metadata stored at index mi (binary16
+// pair with M16: codes against the rounded pair), codes 0 when scale == 0,
+// each chunk's codes emitted into the packed row.  The chunk loop stays rolled
+// (by two) so that the code is small and stays in the instruction cache.
+template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int nk, uint32_t* codes, char* meta,
+                                                   size_t mi, uint32_t& prev, uint32_t& plane) {
+  __nv_bfloat162 mn2, mx2;
+  {
+    const uint4 v = r4[k0];
+    mn2 = mx2 = *reinterpret_cast<const __nv_bfloat162*>(&v.x);
+  }
+#pragma unroll 4
+  for (int k = k0; k < k0 + nk; ++k) {
     const uint4 v = r4[k];
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
@@ -326,112 +220,46 @@ __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* 
   float mx = fmaxf(__low2float(mx2), __high2float(mx2));
   mn = __fadd_rn(mn, 0.0f);  // -0 -> +0
   mx = __fadd_rn(mx, 0.0f);
-  constexpr uint32_t L = (1u << BITS) - 1u;
-  const float levels = (float)L;
+  const float levels = (float)((1u << BITS) - 1u);
   float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
   if (M16) {  // binary16 metadata: codes against the stored pair
     scale = half_sat(scale);
     mn = half_sat(mn);
   }
   store_meta(meta, mi, scale, mn, M16);
-  constexpr int W = 4 * BITS;  // code words per token
-  if (scale == 0.0f) {  // constant vector (or a step below binary16 range): every code 0
-#pragma unroll
-    for (int i = 0; i < W; ++i) codes[i] = 0u;
-    return;
-  }
-  if (M16) {
-    // A binary16 scale is at least 2^-24, so r is finite.  The rounded zero
-    // and scale can put a quotient outside [0, levels]: q = d r is clamped to
-    // [-1, levels + 1] (which decides no code differently), then T =
-    // RN(q + 192) lies in [191, 193 + levels] and bits 16.. of T + 0x8001,
-    // less 0x4340, are the unclamped code.  The two roundings (q, then T) keep
-    // T within 2^-16 of fl(d / scale) + 192 for quotients that can decide a
-    // code, so the near-tie test is the same as below.
-    const float r = __frcp_rn(scale);
-    uint32_t prev = 0u, plane = 0u;
+  const bool fast = scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
+  const float r = (M16 || fast) ? __frcp_rn(scale) : 1.0f;
 #pragma unroll 2
-    for (int k = 0; k < 16; ++k) {
-      const uint4 v = r4[k];
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint32_t c8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const uint32_t hw = w[i >> 1];
-        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
-        const float q = fminf(fmaxf(__fmul_rn(d, r), -1.0f), levels + 1.0f);
-        const uint32_t a = __float_as_uint(__fadd_rn(q, 192.0f)) + 0x8001u;
-        const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
-        c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
-      }
-      emit_chunk<BITS>(k, c8, codes, prev, plane);
-    }
-    return;
-  }
-  if (scale >= 2.3509887e-38f) {  // 2^-125: 1 / scale is finite
-    const float r = __frcp_rn(scale);
-    // Two channels per paired operation: d = fl(x - min), then
-    // T' = RN(d r + C) with C = 192.5 + 4 * 2^-16.  In [128, 256) the grid is
-    // 2^-16, so T' is T = RN(d r + 192) moved by 0x8004 units (one unit more
-    // or less when d r + 192 falls exactly between two grid points, where the
-    // shift by an even count flips the tie-break).  Bits 16.. of T' are then
-    // floor(d r + 0.5) away from ties, and the error of T' against the exact
-    // quotient is below two units (0.5 FMA rounding, 1/16 for r, 1/16 for
-    // the reference division, 1 for the tie-break), so every element within
-    // two units of the half-integer boundary -- T' low bits in [2, 6] -- is
-    // among those with low bits in [0, 7], which take the exact rule.
-    const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
-    const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
-    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
-    const uint64_t c2 = f32x2(cbits, cbits);
-    // chunks of 8 channels (one uint4 of the row): 16 code bits (2-bit) or 32
-    // (4-bit); the loop stays rolled (by two) so the code is small and stays
-    // in the instruction cache
-    uint32_t prev = 0u, plane = 0u;
-#pragma unroll 2
-    for (int k = 0; k < 16; ++k) {
-      const uint4 v = r4[k];
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint32_t a[8];
-      uint32_t low = 0xffffffffu;  // per 16-bit half: the smallest masked low bits seen
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint64_t x2 = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 8k + 2i, 8k + 2i + 1
-        const uint64_t t2 = f32x2_fma(f32x2_sub(x2, mn2), r2, c2);
-        a[2 * i] = (uint32_t)t2;
-        a[2 * i + 1] = (uint32_t)(t2 >> 32);
-        low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
-      }
-      uint32_t c8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
-      if (__vcmpeq2(low, 0u)) {  // a near-tie in this chunk (about one chunk in 500): the exact rule
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          if (a[i] & 0xfff8u) continue;
-          const uint32_t hw = w[i >> 1];
-          const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
-          c8[i] = exact_code(d, scale, levels);
-        }
-      }
-      emit_chunk<BITS>(k, c8, codes, prev, plane);
-    }
-    return;
-  }
-  // tiny scale: the exact rule throughout
-  uint32_t prev = 0u, plane = 0u;
-#pragma unroll 1
-  for (int k = 0; k < 16; ++k) {
+  for (int k = k0; k < k0 + nk; ++k) {
+    const uint4 v = r4[k];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
     uint32_t c8[8];
+    if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int e = 8 * k + i;
-      const uint32_t hw = reinterpret_cast<const uint32_t*>(row_s)[e >> 1];
-      const float x = __uint_as_float((e & 1) ? (hw & 0xffff0000u) : (hw << 16));
-      c8[i] = exact_code(__fsub_rn(x, mn), scale, levels);
+      for (int i = 0; i < 8; ++i) c8[i] = 0u;
+    } else {
+      chunk_codes<BITS, M16>(w, mn, scale, r, fast, c8);
     }
     emit_chunk<BITS>(k, c8, codes, prev, plane);
   }
+}
+
+// Per-token min-max over the whole 128-channel row (Sec. 1), one group.
+template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
+  uint32_t prev = 0u, plane = 0u;
+  quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 0, 16, codes, meta, mi, prev, plane);
+}
+
+// KIVI-style values (Sec. 4): four groups of 32 channels per token
+// (metadata mi .. mi + 3); the packing is the per-token one (channel order).
+template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_row_kivi_v(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
+  uint32_t prev = 0u, plane = 0u;
+#pragma unroll 1
+  for (int j = 0; j < 4; ++j)
+    quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 4 * j, 4, codes, meta, mi + j, prev,
+                                  plane);
 }
 
 // ---------------------------------------------------------------------------
@@ -640,6 +468,115 @@ quantize_token_kernel(const __grid_constant__ QuantizeParams p) {
   }
 #pragma unroll
   for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+}
+
+// ---------------------------------------------------------------------------
+// KIVI-style base (Sec. 4), on staged rows as above: one CTA per (64-token
+// tile, batch row, KV head, layer), tiles aligned so that the image's 32-token
+// key groups (anchored at the image start) never straddle two tiles.  Values
+// of every head whose image values are coded: one thread per token row, four
+// 32-channel groups.  Keys of a quantized head: once the rows are staged,
+// thread c quantizes channel c over each whole key group of the tile (32
+// consecutive image tokens, packed in token order).  Every other row (text,
+// the BF16 residual window and a trailing partial group, protected heads,
+// keys of keys-only heads) is copied.
+// ---------------------------------------------------------------------------
+template <int BITS, bool M16>
+__global__ void __launch_bounds__(kThreads)
+quantize_kivi_kernel(const __grid_constant__ QuantizeParams p) {
+  const Dims& d = p.d;
+  const int li = blockIdx.z, bh = blockIdx.y;
+  const int b = bh / d.H, h = bh % d.H;
+  // tile i: [origin - 32 + 64 i, + 64) clipped to [0, T), origin = s mod 32
+  const int tlo = p.tile_origin - kKiviGroup + kQTok * (int)blockIdx.x;
+  const int t0 = max(tlo, 0), t1 = min(tlo + kQTok, d.T);
+  const int n = t1 - t0;
+  if (n <= 0) return;
+  const int tid = threadIdx.x;
+  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+  const HeadGeom hd = head_geom(d, g, h);
+  char* Lb = p.arena + p.lt.base[li];
+  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + t0;
+  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
+  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
+
+  __shared__ __align__(16) char rows[2][kQTok][kQPitch];
+  for (int c = tid; c < 2 * n * 16; c += kThreads) {
+    const int kv = c / (n * 16), rem = c - kv * (n * 16);
+    const int r = rem >> 4, col = rem & 15;
+    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
+  }
+  cp_async_commit();
+  cp_async_wait<0>();
+  __syncthreads();
+
+  const int qs = d.s, qe = d.s + d.nq;
+  constexpr int W = 4 * BITS;
+  const int kv = tid >> 6, r = tid & (kQTok - 1);
+  if (r < n) {
+    const int t = t0 + r;
+    const bool coded = t >= qs && t < qe;
+    const int ti = t - qs;
+    const char* row_s = rows[kv][r];
+    char* dst = nullptr;
+    if (kv == 0) {
+      if (!(coded && hd.cls == kQuantized))  // quantized keys: by channel below
+        dst = (coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
+                                             : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
+    } else if (coded && hd.cls != kProtected) {
+      quantize_row_kivi_v<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+                                     Lb + hd.vqm + b * hd.vqm_bs, (size_t)ti * 4);
+    } else {
+      dst = Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
+    }
+    if (dst) {
+#pragma unroll
+      for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+    }
+  }
+  if (hd.cls != kQuantized) return;  // uniform over the CTA
+
+  // KIVI-style keys: thread c quantizes channel c over each whole group of the
+  // tile (the staged rows are only read, so no further barrier is needed)
+  const bool m16 = M16;
+  const int c = tid;
+#pragma unroll 1
+  for (int g0 = tlo; g0 < tlo + kQTok; g0 += kKiviGroup) {
+    if (g0 < qs || g0 + kKiviGroup > qe || g0 < t0 || g0 + kKiviGroup > t1) continue;
+    float x[kKiviGroup];
+#pragma unroll
+    for (int e = 0; e < kKiviGroup; ++e)
+      x[e] = bf16_to_f32(*reinterpret_cast<const uint16_t*>(&rows[0][g0 - t0 + e][2 * c]));
+    uint32_t code[kKiviGroup];
+    float sc, z;
+    quantize_group_serial(x, BITS, m16, code, sc, z);
+    const int grp = (g0 - qs) / kKiviGroup;
+    uint32_t* dstc = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * BITS;
+    if (BITS == 3) {  // two words of bits 0-1 (16 tokens each), then the bit-2 plane
+      uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
+#pragma unroll
+      for (int e = 0; e < 16; ++e) {
+        lo0 |= (code[e] & 3u) << (2 * e);
+        lo1 |= (code[16 + e] & 3u) << (2 * e);
+      }
+#pragma unroll
+      for (int e = 0; e < 32; ++e)
+        hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
+      dstc[0] = lo0;
+      dstc[1] = lo1;
+      dstc[2] = hp;
+    } else {
+      constexpr int per = 32 / (BITS == 3 ? 2 : BITS);
+#pragma unroll
+      for (int w = 0; w < BITS; ++w) {
+        uint32_t word = 0;
+#pragma unroll
+        for (int e = 0; e < per; ++e) word |= code[w * per + e] << (BITS * e);
+        dstc[w] = word;
+      }
+    }
+    store_meta(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + c, sc, z, m16);
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -967,12 +904,28 @@ cudaError_t launch_token(const QuantizeParams& p, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
-  if (p.d.base == kMinMax) return launch_token<kMinMax>(p, s);  // one thread per vector
-  if (p.d.base == kAkvq) return launch_token<kAkvq>(p, s);
-  dim3 grid(p.n_tiles, p.d.B * p.d.H, p.n_layers);
-  quantize_kernel<kKivi><<<grid, kThreads, 0, s>>>(p);
+cudaError_t launch_kivi(const QuantizeParams& p, cudaStream_t s) {
+  // 64-token tiles from s mod 32 - 32 (image groups never straddle a tile)
+  dim3 grid((p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
+  const bool m16 = p.d.meta16 != 0;
+  if (p.d.bits == 2) {
+    if (m16) quantize_kivi_kernel<2, true><<<grid, kThreads, 0, s>>>(p);
+    else quantize_kivi_kernel<2, false><<<grid, kThreads, 0, s>>>(p);
+  } else if (p.d.bits == 3) {
+    if (m16) quantize_kivi_kernel<3, true><<<grid, kThreads, 0, s>>>(p);
+    else quantize_kivi_kernel<3, false><<<grid, kThreads, 0, s>>>(p);
+  } else {
+    if (m16) quantize_kivi_kernel<4, true><<<grid, kThreads, 0, s>>>(p);
+    else quantize_kivi_kernel<4, false><<<grid, kThreads, 0, s>>>(p);
+  }
   return cudaGetLastError();
+}
+
+cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
+  // one thread per vector for every base (the KIVI-style keys: per channel)
+  if (p.d.base == kMinMax) return launch_token<kMinMax>(p, s);
+  if (p.d.base == kAkvq) return launch_token<kAkvq>(p, s);
+  return launch_kivi(p, s);
 }
 
 cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s) {
