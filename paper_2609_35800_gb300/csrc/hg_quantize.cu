@@ -31,32 +31,6 @@ __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
   bf16x2_to_f32(w.y, x[2], x[3]);
 }
 
-// One 32-value group held by a single thread (KIVI-style key channel group).
-__device__ __forceinline__ void quantize_group_serial(const float (&x)[kKiviGroup], int bits, bool m16,
-                                                      uint32_t (&code)[kKiviGroup], float& scale,
-                                                      float& zero) {
-  float mn = x[0], mx = x[0];
-#pragma unroll
-  for (int e = 1; e < kKiviGroup; ++e) {
-    mn = fminf(mn, x[e]);
-    mx = fmaxf(mx, x[e]);
-  }
-  mn = __fadd_rn(mn, 0.0f);
-  mx = __fadd_rn(mx, 0.0f);
-  const float levels = (float)((1 << bits) - 1);
-  scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
-  zero = mn;
-  if (m16) {
-    scale = half_sat(scale);
-    zero = half_sat(zero);
-  }
-  const bool fast = scale >= 2.3509887e-38f;  // 2^-125
-  const float r = __frcp_rn(fast ? scale : 1.0f);
-#pragma unroll
-  for (int e = 0; e < kKiviGroup; ++e)
-    code[e] = (scale == 0.0f) ? 0u : code_of(__fsub_rn(x[e], zero), scale, r, levels, fast);
-}
-
 // ---------------------------------------------------------------------------
 // Per-token min-max base: one thread per (token, K or V) vector.
 //
@@ -87,32 +61,173 @@ __device__ __noinline__ uint32_t exact_code(float d, float scale, float levels) 
 // Eight codes of channels 8k..8k+7 into the packed row: 4 bits -> word k;
 // 2 bits -> half of word k/2; 3 bits -> the same 2-bit half plus one byte of
 // plane word 8 + k/4 (byte ((k >> 1) & 1) | ((k & 1) << 1): channel index bits
-// 3 and 4 exchanged), each word stored once complete.
+// 3 and 4 exchanged), each word stored once complete.  `lo` holds the chunk's
+// 32 (4-bit) or 16 (2- and 3-bit) code bits, `hb` the 8 bit-2 bits (3-bit).
 template <int BITS>
-__device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32_t* codes, uint32_t& prev,
-                                           uint32_t& plane) {
+__device__ __forceinline__ void store_chunk(int k, uint32_t lo, uint32_t hb, uint32_t* codes, uint32_t& prev,
+                                            uint32_t& plane) {
   if (BITS == 4) {
-    uint32_t w = 0u;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) w |= c[i] << (4 * i);
-    codes[k] = w;
+    codes[k] = lo;
     return;
   }
-  uint32_t lo = 0u;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) lo |= (c[i] & 3u) << (2 * i);
   if (k & 1) codes[k >> 1] = prev | (lo << 16);
   else prev = lo;
   if (BITS == 3) {
-    uint32_t hb = 0u;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) hb |= ((c[i] >> 2) & 1u) << i;
     plane |= hb << (8 * (((k >> 1) & 1) | ((k & 1) << 1)));
     if ((k & 3) == 3) {
       codes[8 + (k >> 2)] = plane;
       plane = 0u;
     }
   }
+}
+
+template <int BITS>
+__device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32_t* codes, uint32_t& prev,
+                                           uint32_t& plane) {
+  uint32_t lo = 0u, hb = 0u;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    lo |= (BITS == 4) ? (c[i] << (4 * i)) : ((c[i] & 3u) << (2 * i));
+    if (BITS == 3) hb |= ((c[i] >> 2) & 1u) << i;
+  }
+  store_chunk<BITS>(k, lo, hb, codes, prev, plane);
+}
+
+// The same from the eight T' words of the fast rule (code in bits 16..): each
+// code is shifted straight into its packed position (one shift and one
+// and-or per element instead of extracting it first).
+template <int BITS>
+__device__ __forceinline__ void emit_from_T(int k, const uint32_t (&a)[8], uint32_t* codes, uint32_t& prev,
+                                            uint32_t& plane) {
+  uint32_t lo = 0u, hb = 0u;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    if (BITS == 4) {
+      const uint32_t x = (4 * i >= 16) ? (a[i] << (4 * i - 16)) : (a[i] >> (16 - 4 * i));
+      lo |= x & (15u << (4 * i));
+    } else {
+      lo |= (a[i] >> (16 - 2 * i)) & (3u << (2 * i));
+      if (BITS == 3) hb |= (a[i] >> (18 - i)) & (1u << i);
+    }
+  }
+  store_chunk<BITS>(k, lo, hb, codes, prev, plane);
+}
+
+// T' = RN(fl(x - min) r + C) for the four channel pairs of a chunk (the fast
+// rule of chunk_codes), element 2i + j from half j of pair i.  Returns true
+// when no element has T' low bits in [0, 7] (then every code is bits 16.. of
+// T'); false when some element is near a tie and must take the exact rule.
+__device__ __forceinline__ bool chunk_T(const uint64_t (&x2)[4], uint64_t mn2, uint64_t r2, uint64_t c2,
+                                        uint32_t (&a)[8]) {
+  uint32_t low = 0xffffffffu;  // per 16-bit half: the smallest low bits seen
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    const uint64_t t2 = f32x2_fma(f32x2_sub(x2[i], mn2), r2, c2);
+    a[2 * i] = (uint32_t)t2;
+    a[2 * i + 1] = (uint32_t)(t2 >> 32);
+    low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410));
+  }
+  return __vcmpleu2(low, 0x00070007u) == 0u;
+}
+
+// Pack and store the 32 codes of one KIVI-style key group row (one channel,
+// token order): 2 / 4 bits as `bits` words, 3 bits as two words of bits 0-1
+// (16 tokens each) and the bit-2 plane.
+template <int BITS>
+__device__ __forceinline__ void store_key_group(uint32_t* dst, const uint32_t (&code)[kKiviGroup]) {
+  if (BITS == 3) {
+    uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      lo0 |= (code[e] & 3u) << (2 * e);
+      lo1 |= (code[16 + e] & 3u) << (2 * e);
+    }
+#pragma unroll
+    for (int e = 0; e < 32; ++e)
+      hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
+    dst[0] = lo0;
+    dst[1] = lo1;
+    dst[2] = hp;
+  } else {
+    constexpr int per = 32 / (BITS == 3 ? 2 : BITS);
+#pragma unroll
+    for (int w = 0; w < BITS; ++w) {
+      uint32_t word = 0;
+#pragma unroll
+      for (int e = 0; e < per; ++e) word |= code[w * per + e] << (BITS * e);
+      dst[w] = word;
+    }
+  }
+}
+
+// Two adjacent channels (2c, 2c + 1) of one KIVI-style key group: the 32
+// bf16x2 words of the group's tokens at `col` (the group's first staged row,
+// then a row pitch apart).  min / max of both channels at once over bf16x2
+// pairs (exact); with fp32 metadata and both steps at least 2^-125, the codes
+// of both channels come from the paired rule of the token rows (per-lane
+// minimum and reciprocal), otherwise each channel takes the scalar group
+// quantizer.  Codes and metadata as for one channel.
+template <int BITS, bool M16>
+__device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst0, uint32_t* dst1, char* meta,
+                                                  size_t mi) {
+  uint32_t w[kKiviGroup];
+#pragma unroll
+  for (int e = 0; e < kKiviGroup; ++e) w[e] = *reinterpret_cast<const uint32_t*>(col + (size_t)e * kQPitch);
+  __nv_bfloat162 mn2 = *reinterpret_cast<const __nv_bfloat162*>(&w[0]), mx2 = mn2;
+#pragma unroll
+  for (int e = 1; e < kKiviGroup; ++e) {
+    const __nv_bfloat162 h = *reinterpret_cast<const __nv_bfloat162*>(&w[e]);
+    mn2 = __hmin2(mn2, h);
+    mx2 = __hmax2(mx2, h);
+  }
+  constexpr uint32_t L = (1u << BITS) - 1u;
+  const float levels = (float)L;
+  float mn[2] = {__fadd_rn(__low2float(mn2), 0.0f), __fadd_rn(__high2float(mn2), 0.0f)};
+  const float mx[2] = {__fadd_rn(__low2float(mx2), 0.0f), __fadd_rn(__high2float(mx2), 0.0f)};
+  float sc[2];
+#pragma unroll
+  for (int j = 0; j < 2; ++j) {
+    sc[j] = __fdiv_rn(__fsub_rn(mx[j], mn[j]), levels);
+    if (M16) {
+      sc[j] = half_sat(sc[j]);
+      mn[j] = half_sat(mn[j]);
+    }
+    store_meta(meta, mi + j, sc[j], mn[j], M16);
+  }
+  uint32_t c0[kKiviGroup], c1[kKiviGroup];
+  if (!M16 && sc[0] >= 2.3509887e-38f && sc[1] >= 2.3509887e-38f) {
+    const float r0 = __frcp_rn(sc[0]), r1 = __frcp_rn(sc[1]);
+    const uint64_t mn2p = f32x2(__float_as_uint(mn[0]), __float_as_uint(mn[1]));
+    const uint64_t r2 = f32x2(__float_as_uint(r0), __float_as_uint(r1));
+    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16 (see chunk_codes)
+    const uint64_t c2 = f32x2(cbits, cbits);
+#pragma unroll
+    for (int e = 0; e < kKiviGroup; ++e) {
+      const uint64_t t2 = f32x2_fma(f32x2_sub(f32x2(w[e] << 16, w[e] & 0xffff0000u), mn2p), r2, c2);
+      const uint32_t a0 = (uint32_t)t2, a1 = (uint32_t)(t2 >> 32);
+      c0[e] = (a0 >> 16) & L;
+      c1[e] = (a1 >> 16) & L;
+      if (!(a0 & 0xfff8u))
+        c0[e] = exact_code(__fsub_rn(__uint_as_float(w[e] << 16), mn[0]), sc[0], levels);
+      if (!(a1 & 0xfff8u))
+        c1[e] = exact_code(__fsub_rn(__uint_as_float(w[e] & 0xffff0000u), mn[1]), sc[1], levels);
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const bool fast = sc[j] >= 2.3509887e-38f;  // 2^-125
+      const float r = __frcp_rn(fast ? sc[j] : 1.0f);
+#pragma unroll
+      for (int e = 0; e < kKiviGroup; ++e) {
+        const float x = __uint_as_float(j ? (w[e] & 0xffff0000u) : (w[e] << 16));
+        const uint32_t c = (sc[j] == 0.0f) ? 0u : code_of(__fsub_rn(x, mn[j]), sc[j], r, levels, fast);
+        if (j) c1[e] = c;
+        else c0[e] = c;
+      }
+    }
+  }
+  store_key_group<BITS>(dst0, c0);
+  store_key_group<BITS>(dst1, c1);
 }
 
 // Codes of the 8 channels of one chunk (four BF16 pairs w[0..3]) in a group
@@ -136,14 +251,15 @@ __device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32
 //     quotient is below two units (0.5 FMA rounding, 1/16 for r, 1/16 for the
 //     reference division, 1 for the tie-break), so every element within two
 //     units of the half-integer boundary -- T' low bits in [2, 6] -- is among
-//     those with low bits in [0, 7], which take the exact rule.
+//     those with low bits in [0, 7], which take the exact rule (chunk_T,
+//     emit_from_T; a chunk with such an element goes through chunk_near_tie).
 //   otherwise (tiny scale): the exact rule for every element.
 template <int BITS, bool M16>
-__device__ __forceinline__ void chunk_codes(const uint32_t (&w)[4], float mn, float scale, float r, bool fast,
+__device__ __forceinline__ void chunk_codes(const uint32_t (&w)[4], float mn, float scale, float r,
                                             uint32_t (&c8)[8]) {
   constexpr uint32_t L = (1u << BITS) - 1u;
   const float levels = (float)L;
-  if (M16) {
+  if constexpr (M16) {
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const uint32_t hw = w[i >> 1];
@@ -153,42 +269,26 @@ __device__ __forceinline__ void chunk_codes(const uint32_t (&w)[4], float mn, fl
       const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
       c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
     }
-    return;
-  }
-  if (fast) {
-    const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
-    const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
-    const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
-    const uint64_t c2 = f32x2(cbits, cbits);
-    uint32_t a[8];
-    uint32_t low = 0xffffffffu;  // per 16-bit half: the smallest masked low bits seen
+  } else {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const uint64_t x2 = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1 of the chunk
-      const uint64_t t2 = f32x2_fma(f32x2_sub(x2, mn2), r2, c2);
-      a[2 * i] = (uint32_t)t2;
-      a[2 * i + 1] = (uint32_t)(t2 >> 32);
-      low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t hw = w[i >> 1];
+      const float x = __uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16));
+      c8[i] = exact_code(__fsub_rn(x, mn), scale, levels);
     }
-#pragma unroll
-    for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
-    if (__vcmpeq2(low, 0u)) {  // a near-tie in this chunk (about one chunk in 500): the exact rule
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        if (a[i] & 0xfff8u) continue;
-        const uint32_t hw = w[i >> 1];
-        const float d = __fsub_rn(__uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16)), mn);
-        c8[i] = exact_code(d, scale, levels);
-      }
-    }
-    return;
   }
+}
+
+// Codes of a chunk that has an element near a tie: bits 16.. of T' for the
+// others, the exact rule for the elements with T' low bits in [0, 7].
+// x(i) gives element i's value.
+template <int BITS, class X>
+__device__ __forceinline__ void chunk_near_tie(const uint32_t (&a)[8], X x, float mn, float scale,
+                                               uint32_t (&c8)[8]) {
+  constexpr uint32_t L = (1u << BITS) - 1u;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t hw = w[i >> 1];
-    const float x = __uint_as_float((i & 1) ? (hw & 0xffff0000u) : (hw << 16));
-    c8[i] = exact_code(__fsub_rn(x, mn), scale, levels);
-  }
+  for (int i = 0; i < 8; ++i)
+    c8[i] = (a[i] & 0xfff8u) ? ((a[i] >> 16) & L) : exact_code(__fsub_rn(x(i), mn), scale, (float)L);
 }
 
 // One group of a BF16 row: chunks [k0, k0 + nk) (8 channels each) with their
@@ -227,18 +327,34 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
     mn = half_sat(mn);
   }
   store_meta(meta, mi, scale, mn, M16);
-  const bool fast = scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
+  const bool fast = !M16 && scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
   const float r = (M16 || fast) ? __frcp_rn(scale) : 1.0f;
+  const uint64_t mnp = f32x2(__float_as_uint(mn), __float_as_uint(mn));
+  const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
+  const uint32_t cbits = __float_as_uint(192.50006103515625f);  // C = 192.5 + 4 * 2^-16
+  const uint64_t c2 = f32x2(cbits, cbits);
 #pragma unroll 2
   for (int k = k0; k < k0 + nk; ++k) {
     const uint4 v = r4[k];
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
     uint32_t c8[8];
-    if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
+    if (fast) {
+      uint64_t x2[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1
+      uint32_t a[8];
+      if (chunk_T(x2, mnp, r2, c2, a)) {
+        emit_from_T<BITS>(k, a, codes, prev, plane);
+        continue;
+      }
+      // a near-tie in this chunk (about one chunk in 500): the exact rule for it
+      chunk_near_tie<BITS>(a, [&](int i) { return __uint_as_float((i & 1) ? (w[i >> 1] & 0xffff0000u) : (w[i >> 1] << 16)); },
+                           mn, scale, c8);
+    } else if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
 #pragma unroll
       for (int i = 0; i < 8; ++i) c8[i] = 0u;
     } else {
-      chunk_codes<BITS, M16>(w, mn, scale, r, fast, c8);
+      chunk_codes<BITS, M16>(w, mn, scale, r, c8);
     }
     emit_chunk<BITS>(k, c8, codes, prev, plane);
   }
@@ -349,7 +465,7 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
     }
     return;
   }
-  if (scale >= 2.3509887e-38f) {  // the fast rule of the min-max rows (see there)
+  if (scale >= 2.3509887e-38f) {  // the fast rule of the min-max rows (chunk_T)
     const float r = __frcp_rn(scale);
     const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
     const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
@@ -357,27 +473,16 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
     const uint64_t c2 = f32x2(cbits, cbits);
 #pragma unroll
     for (int k = 0; k < 16; ++k) {
+      const uint64_t x2[4] = {xp[4 * k], xp[4 * k + 1], xp[4 * k + 2], xp[4 * k + 3]};
       uint32_t a[8];
-      uint32_t low = 0xffffffffu;
-#pragma unroll
-      for (int i = 0; i < 4; ++i) {
-        const uint64_t t2 = f32x2_fma(f32x2_sub(xp[4 * k + i], mn2), r2, c2);
-        a[2 * i] = (uint32_t)t2;
-        a[2 * i + 1] = (uint32_t)(t2 >> 32);
-        low = __vminu2(low, __byte_perm(a[2 * i], a[2 * i + 1], 0x5410) & 0xfff8fff8u);
+      if (chunk_T(x2, mn2, r2, c2, a)) {
+        emit_from_T<BITS>(k, a, codes, prev, plane);
+      } else {
+        uint32_t c8[8];
+        chunk_near_tie<BITS>(a, [&](int i) { return (i & 1) ? pair_hi(x2[i >> 1]) : pair_lo(x2[i >> 1]); }, mn,
+                             scale, c8);
+        emit_chunk<BITS>(k, c8, codes, prev, plane);
       }
-      uint32_t c8[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) c8[i] = (a[i] >> 16) & L;
-      if (__vcmpeq2(low, 0u)) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          if (a[i] & 0xfff8u) continue;
-          const uint64_t x2 = xp[4 * k + (i >> 1)];
-          c8[i] = exact_code(__fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn), scale, levels);
-        }
-      }
-      emit_chunk<BITS>(k, c8, codes, prev, plane);
     }
     return;
   }
@@ -393,82 +498,96 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
   }
 }
 
-// The per-token bases, one thread per vector: min-max rows (Sec. 1) and
-// AKVQ-style rows (Sec. 4: keys rotated first; values per token, unrotated).
-// With salient tokens (AKVQ-style, Sec. 4) a thread finds its token in the
-// head's map: a salient token's K and V rows go to the BF16 region at
-// position s + (its rank), every other image token to coded slot ti - (the
-// salient tokens before it).
-template <int BITS, bool M16, int BASE>
-__global__ void __launch_bounds__(kThreads)
-quantize_token_kernel(const __grid_constant__ QuantizeParams p) {
-  const Dims& d = p.d;
-  const int li = blockIdx.z, bh = blockIdx.y;
-  const int b = bh / d.H, h = bh % d.H;
-  const int t0 = blockIdx.x * kQTok;
-  const int n = min(kQTok, d.T - t0);
-  if (n <= 0) return;
-  const int tid = threadIdx.x;
-  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-  const HeadGeom hd = head_geom(d, g, h);
-  char* Lb = p.arena + p.lt.base[li];
-  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + t0;
-  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
-  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
-
-  __shared__ __align__(16) char rows[2][kQTok][kQPitch];
-  // coalesced staging, chunk c = 16 bytes of one row, as asynchronous copies
-  // (all of a thread's chunks in flight at once rather than one load-store
-  // round trip after another)
-  for (int c = tid; c < 2 * n * 16; c += kThreads) {
-    const int kv = c / (n * 16), rem = c - kv * (n * 16);
-    const int r = rem >> 4, col = rem & 15;
-    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
-  }
-  cp_async_commit();
-  cp_async_wait<0>();
-  __syncthreads();
-
-  const int kv = tid >> 6, r = tid & (kQTok - 1);
-  if (r >= n) return;
-  const int t = t0 + r;
-  const bool coded = t >= d.s && t < d.s + d.nq;
-  const int ti = t - d.s;
-  int ci = ti, pos = bf16_pos(d, hd.cls, t);
-  bool sal = false;
-  if (BASE == kAkvq && coded && d.ns > 0 && hd.cls != kProtected) {
-    const char* sm = Lb + hd.sal + b * hd.sal_bs;
-    const int w = ti >> 5, e = ti & 31;
-    const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
-    const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
-                     __popc(sb & ((1u << e) - 1u));
-    sal = (sb >> e) & 1u;
-    ci = ti - rank;
-    if (sal) pos = d.s + rank;
-  }
-  const char* row_s = rows[kv][r];
-  constexpr int W = 4 * BITS;
-  char* dst;
-  if (kv == 0) {
-    if (coded && hd.cls == kQuantized && !sal) {
-      uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
-      if (BASE == kAkvq) quantize_row_rotated<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
-      else quantize_row_token<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
-      return;
-    }
-    dst = (coded && hd.cls == kKeysOnly && !sal) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
-                                                 : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
-  } else {
-    if (coded && hd.cls != kProtected && !sal) {
-      quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
-                                    Lb + hd.vqm + b * hd.vqm_bs, ci);
-      return;
-    }
-    dst = Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256;
-  }
+__device__ __forceinline__ void copy_row(char* dst, const char* row_s) {
 #pragma unroll
   for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
 }
+
+// Staged rows of one tile: K rows [0][r], V rows [1][r], r < n, 272-byte pitch.
+typedef char StagedRows[2][kQTok][kQPitch];
+
+// Token span of a tile: rows r < n hold tokens t0 + r.
+struct TileSpan {
+  int t0, n, tlo;  // tlo: the unclipped tile start (KIVI-style tiles)
+};
+
+// Coalesced staging of a tile's K and V rows, 16 bytes of one row per
+// asynchronous copy (every chunk of a thread in flight at once); the caller
+// commits the group.
+__device__ __forceinline__ void stage_rows(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
+                                           StagedRows& rows) {
+  const Dims& d = p.d;
+  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + sp.t0;
+  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
+  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
+  for (int c = threadIdx.x; c < 2 * sp.n * 16; c += kThreads) {
+    const int kv = c / (sp.n * 16), rem = c - kv * (sp.n * 16);
+    const int r = rem >> 4, col = rem & 15;
+    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
+  }
+}
+
+// The per-token bases, one thread per vector: min-max rows (Sec. 1) and
+// AKVQ-style rows (Sec. 4: keys rotated first; values per token, unrotated).
+// Tiles of 64 tokens from token 0.  With salient tokens (AKVQ-style, Sec. 4)
+// a thread finds its token in the head's map: a salient token's K and V rows
+// go to the BF16 region at position s + (its rank), every other image token
+// to coded slot ti - (the salient tokens before it).
+template <int BITS, bool M16, int BASE>
+struct TokenTiles {
+  static __device__ __forceinline__ int count(const QuantizeParams& p) { return (p.d.T + kQTok - 1) / kQTok; }
+  static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
+    TileSpan sp;
+    sp.t0 = sp.tlo = tx * kQTok;
+    sp.n = min(kQTok, p.d.T - sp.t0);
+    return sp;
+  }
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
+                                                 const StagedRows& rows) {
+    const Dims& d = p.d;
+    const int tid = threadIdx.x;
+    const int kv = tid >> 6, r = tid & (kQTok - 1);
+    if (r >= sp.n) return;
+    const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+    const HeadGeom hd = head_geom(d, g, h);
+    char* Lb = p.arena + p.lt.base[li];
+    const int t = sp.t0 + r;
+    const bool coded = t >= d.s && t < d.s + d.nq;
+    const int ti = t - d.s;
+    int ci = ti, pos = bf16_pos(d, hd.cls, t);
+    bool sal = false;
+    if (BASE == kAkvq && coded && d.ns > 0 && hd.cls != kProtected) {
+      const char* sm = Lb + hd.sal + b * hd.sal_bs;
+      const int w = ti >> 5, e = ti & 31;
+      const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
+      const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
+                       __popc(sb & ((1u << e) - 1u));
+      sal = (sb >> e) & 1u;
+      ci = ti - rank;
+      if (sal) pos = d.s + rank;
+    }
+    const char* row_s = rows[kv][r];
+    constexpr int W = 4 * BITS;
+    if (kv == 0) {
+      if (coded && hd.cls == kQuantized && !sal) {
+        uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
+        if (BASE == kAkvq) quantize_row_rotated<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
+        else quantize_row_token<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
+        return;
+      }
+      char* dst = (coded && hd.cls == kKeysOnly && !sal) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
+                                                         : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
+      copy_row(dst, row_s);
+    } else {
+      if (coded && hd.cls != kProtected && !sal) {
+        quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
+                                      Lb + hd.vqm + b * hd.vqm_bs, ci);
+        return;
+      }
+      copy_row(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256, row_s);
+    }
+  }
+};
 
 // ---------------------------------------------------------------------------
 // KIVI-style base (Sec. 4), on staged rows as above: one CTA per (64-token
@@ -482,101 +601,83 @@ quantize_token_kernel(const __grid_constant__ QuantizeParams p) {
 // keys of keys-only heads) is copied.
 // ---------------------------------------------------------------------------
 template <int BITS, bool M16>
-__global__ void __launch_bounds__(kThreads)
-quantize_kivi_kernel(const __grid_constant__ QuantizeParams p) {
-  const Dims& d = p.d;
-  const int li = blockIdx.z, bh = blockIdx.y;
-  const int b = bh / d.H, h = bh % d.H;
-  // tile i: [origin - 32 + 64 i, + 64) clipped to [0, T), origin = s mod 32
-  const int tlo = p.tile_origin - kKiviGroup + kQTok * (int)blockIdx.x;
-  const int t0 = max(tlo, 0), t1 = min(tlo + kQTok, d.T);
-  const int n = t1 - t0;
-  if (n <= 0) return;
-  const int tid = threadIdx.x;
-  const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-  const HeadGeom hd = head_geom(d, g, h);
-  char* Lb = p.arena + p.lt.base[li];
-  const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + t0;
-  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
-  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
-
-  __shared__ __align__(16) char rows[2][kQTok][kQPitch];
-  for (int c = tid; c < 2 * n * 16; c += kThreads) {
-    const int kv = c / (n * 16), rem = c - kv * (n * 16);
-    const int r = rem >> 4, col = rem & 15;
-    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
+struct KiviTiles {
+  // tile x: [origin - 32 + 64 x, + 64) clipped to [0, T), origin = s mod 32
+  static __device__ __forceinline__ int count(const QuantizeParams& p) {
+    return (p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
   }
+  static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
+    TileSpan sp;
+    sp.tlo = p.tile_origin - kKiviGroup + kQTok * tx;
+    sp.t0 = max(sp.tlo, 0);
+    sp.n = min(sp.tlo + kQTok, p.d.T) - sp.t0;
+    return sp;
+  }
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
+                                                 const StagedRows& rows) {
+    const Dims& d = p.d;
+    const int tid = threadIdx.x;
+    const LayerGeom g = layer_geom(d, p.lt.mask[li]);
+    const HeadGeom hd = head_geom(d, g, h);
+    char* Lb = p.arena + p.lt.base[li];
+    const int qs = d.s, qe = d.s + d.nq;
+    const int t0 = sp.t0, t1 = sp.t0 + sp.n, tlo = sp.tlo;
+    constexpr int W = 4 * BITS;
+    const int kv = tid >> 6, r = tid & (kQTok - 1);
+    if (r < sp.n) {
+      const int t = t0 + r;
+      const bool coded = t >= qs && t < qe;
+      const int ti = t - qs;
+      const char* row_s = rows[kv][r];
+      if (kv == 0) {
+        if (!(coded && hd.cls == kQuantized))  // quantized keys: by channel below
+          copy_row((coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
+                                                  : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256,
+                   row_s);
+      } else if (coded && hd.cls != kProtected) {
+        quantize_row_kivi_v<BITS, M16>(row_s,
+                                       reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+                                       Lb + hd.vqm + b * hd.vqm_bs, (size_t)ti * 4);
+      } else {
+        copy_row(Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256, row_s);
+      }
+    }
+    if (hd.cls != kQuantized) return;  // uniform over the CTA
+
+    // KIVI-style keys: both whole groups of the tile at once, thread c taking
+    // channels 2 (c % 64) and 2 (c % 64) + 1 of group c / 64 (the staged rows
+    // are only read)
+    const int g0 = tlo + kKiviGroup * (tid >> 6), c2 = tid & 63;
+    if (g0 >= qs && g0 + kKiviGroup <= qe && g0 >= t0 && g0 + kKiviGroup <= t1) {
+      const int grp = (g0 - qs) / kKiviGroup;
+      uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + 2 * c2) * BITS;
+      quantize_key_pair<BITS, M16>(&rows[0][g0 - t0][4 * c2], dst, dst + BITS, Lb + hd.kqm + b * hd.kqm_bs,
+                                   (size_t)grp * kD + 2 * c2);
+    }
+  }
+};
+
+// The quantizer kernel: one CTA per tile, tiles numbered (tile, batch row x
+// KV head, layer) with the tile index fastest.  A CTA stages its tile, waits
+// for the copies and codes it; the copies of other resident CTAs overlap its
+// work.  (Persistent CTAs that stage the next tile into a second buffer while
+// coding the current one measured 5-45% slower: the second buffer halves the
+// resident CTAs.)
+template <class TP>
+__global__ void __launch_bounds__(kThreads) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
+  __shared__ __align__(16) StagedRows rows;
+  const int nx = TP::count(p), nbh = p.d.B * p.d.H;
+  const int i = blockIdx.x;
+  const int tx = i % nx, rest = i / nx, bh = rest % nbh, li = rest / nbh;
+  if (li >= p.n_layers) return;
+  const int b = bh / p.d.H, h = bh % p.d.H;
+  const TileSpan sp = TP::span(p, tx);
+  if (sp.n <= 0) return;
+  stage_rows(p, li, b, h, sp, rows);
   cp_async_commit();
   cp_async_wait<0>();
   __syncthreads();
-
-  const int qs = d.s, qe = d.s + d.nq;
-  constexpr int W = 4 * BITS;
-  const int kv = tid >> 6, r = tid & (kQTok - 1);
-  if (r < n) {
-    const int t = t0 + r;
-    const bool coded = t >= qs && t < qe;
-    const int ti = t - qs;
-    const char* row_s = rows[kv][r];
-    char* dst = nullptr;
-    if (kv == 0) {
-      if (!(coded && hd.cls == kQuantized))  // quantized keys: by channel below
-        dst = (coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
-                                             : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
-    } else if (coded && hd.cls != kProtected) {
-      quantize_row_kivi_v<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
-                                     Lb + hd.vqm + b * hd.vqm_bs, (size_t)ti * 4);
-    } else {
-      dst = Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256;
-    }
-    if (dst) {
-#pragma unroll
-      for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
-    }
-  }
-  if (hd.cls != kQuantized) return;  // uniform over the CTA
-
-  // KIVI-style keys: thread c quantizes channel c over each whole group of the
-  // tile (the staged rows are only read, so no further barrier is needed)
-  const bool m16 = M16;
-  const int c = tid;
-#pragma unroll 1
-  for (int g0 = tlo; g0 < tlo + kQTok; g0 += kKiviGroup) {
-    if (g0 < qs || g0 + kKiviGroup > qe || g0 < t0 || g0 + kKiviGroup > t1) continue;
-    float x[kKiviGroup];
-#pragma unroll
-    for (int e = 0; e < kKiviGroup; ++e)
-      x[e] = bf16_to_f32(*reinterpret_cast<const uint16_t*>(&rows[0][g0 - t0 + e][2 * c]));
-    uint32_t code[kKiviGroup];
-    float sc, z;
-    quantize_group_serial(x, BITS, m16, code, sc, z);
-    const int grp = (g0 - qs) / kKiviGroup;
-    uint32_t* dstc = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + c) * BITS;
-    if (BITS == 3) {  // two words of bits 0-1 (16 tokens each), then the bit-2 plane
-      uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
-#pragma unroll
-      for (int e = 0; e < 16; ++e) {
-        lo0 |= (code[e] & 3u) << (2 * e);
-        lo1 |= (code[16 + e] & 3u) << (2 * e);
-      }
-#pragma unroll
-      for (int e = 0; e < 32; ++e)
-        hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
-      dstc[0] = lo0;
-      dstc[1] = lo1;
-      dstc[2] = hp;
-    } else {
-      constexpr int per = 32 / (BITS == 3 ? 2 : BITS);
-#pragma unroll
-      for (int w = 0; w < BITS; ++w) {
-        uint32_t word = 0;
-#pragma unroll
-        for (int e = 0; e < per; ++e) word |= code[w * per + e] << (BITS * e);
-        dstc[w] = word;
-      }
-    }
-    store_meta(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + c, sc, z, m16);
-  }
+  TP::process(p, li, b, h, sp, rows);
 }
 
 // ---------------------------------------------------------------------------
@@ -887,45 +988,31 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 
 }  // namespace
 
-template <int BASE>
-cudaError_t launch_token(const QuantizeParams& p, cudaStream_t s) {
-  dim3 grid((p.d.T + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
-  const bool m16 = p.d.meta16 != 0;
-  if (p.d.bits == 2) {
-    if (m16) quantize_token_kernel<2, true, BASE><<<grid, kThreads, 0, s>>>(p);
-    else quantize_token_kernel<2, false, BASE><<<grid, kThreads, 0, s>>>(p);
-  } else if (p.d.bits == 3) {
-    if (m16) quantize_token_kernel<3, true, BASE><<<grid, kThreads, 0, s>>>(p);
-    else quantize_token_kernel<3, false, BASE><<<grid, kThreads, 0, s>>>(p);
-  } else {
-    if (m16) quantize_token_kernel<4, true, BASE><<<grid, kThreads, 0, s>>>(p);
-    else quantize_token_kernel<4, false, BASE><<<grid, kThreads, 0, s>>>(p);
-  }
+// Launch of the quantizer kernel over every tile of the launch's layers.
+template <class TP>
+cudaError_t launch_tiles(const QuantizeParams& p, int tiles_x, cudaStream_t s) {
+  const long long total = (long long)tiles_x * p.d.B * p.d.H * p.n_layers;
+  quantize_tiles_kernel<TP><<<(unsigned)total, kThreads, 0, s>>>(p);
   return cudaGetLastError();
 }
 
-cudaError_t launch_kivi(const QuantizeParams& p, cudaStream_t s) {
-  // 64-token tiles from s mod 32 - 32 (image groups never straddle a tile)
-  dim3 grid((p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok, p.d.B * p.d.H, p.n_layers);
-  const bool m16 = p.d.meta16 != 0;
-  if (p.d.bits == 2) {
-    if (m16) quantize_kivi_kernel<2, true><<<grid, kThreads, 0, s>>>(p);
-    else quantize_kivi_kernel<2, false><<<grid, kThreads, 0, s>>>(p);
-  } else if (p.d.bits == 3) {
-    if (m16) quantize_kivi_kernel<3, true><<<grid, kThreads, 0, s>>>(p);
-    else quantize_kivi_kernel<3, false><<<grid, kThreads, 0, s>>>(p);
-  } else {
-    if (m16) quantize_kivi_kernel<4, true><<<grid, kThreads, 0, s>>>(p);
-    else quantize_kivi_kernel<4, false><<<grid, kThreads, 0, s>>>(p);
+template <int BITS, bool M16>
+cudaError_t launch_quantize_bits(const QuantizeParams& p, cudaStream_t s) {
+  const Dims& d = p.d;
+  if (d.base == kKivi) {
+    const int tx = (d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
+    return launch_tiles<KiviTiles<BITS, M16>>(p, tx, s);
   }
-  return cudaGetLastError();
+  const int tx = (d.T + kQTok - 1) / kQTok;
+  if (d.base == kAkvq) return launch_tiles<TokenTiles<BITS, M16, kAkvq>>(p, tx, s);
+  return launch_tiles<TokenTiles<BITS, M16, kMinMax>>(p, tx, s);
 }
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
-  // one thread per vector for every base (the KIVI-style keys: per channel)
-  if (p.d.base == kMinMax) return launch_token<kMinMax>(p, s);
-  if (p.d.base == kAkvq) return launch_token<kAkvq>(p, s);
-  return launch_kivi(p, s);
+  const bool m16 = p.d.meta16 != 0;
+  if (p.d.bits == 2) return m16 ? launch_quantize_bits<2, true>(p, s) : launch_quantize_bits<2, false>(p, s);
+  if (p.d.bits == 3) return m16 ? launch_quantize_bits<3, true>(p, s) : launch_quantize_bits<3, false>(p, s);
+  return m16 ? launch_quantize_bits<4, true>(p, s) : launch_quantize_bits<4, false>(p, s);
 }
 
 cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s) {
