@@ -66,3 +66,47 @@ def test_dequantize_bytes_on_the_one_layer_cache(monkeypatch):
     want = 3 * (64 * 512 + 256 * 2 * (32 + 8)) + 320 * 512 + 2 * 4 * 320 * 256
     assert r["bytes"] == want and r["appended"] == 0 and r["launches"] == 1
     assert r["ms"] == 0.5 and calls == [(0, 1, (1, 1, 4, 320, 128))] * 3
+
+
+def test_cpu_baseline_fields_split_quantize_and_decode():
+    """The oracle's quantize GB/s and decode tokens/s from one timed sample;
+    decode tokens/s scaled to all layers when the sample holds fewer."""
+    import bench
+    from paper_2609_35800_gb300 import workloads as wl
+    w = wl.WORKLOADS["qwen25vl7b"]
+    parts = {"quant_bytes": 2e9, "quant_s": 4.0, "dec_bytes": 3e9, "dec_s": 2.0}
+    f = bench.cpu_baseline_fields(w, 28, 8, parts)
+    assert f["quantize_GBps"] == 0.5 and f["decode_GBps"] == 1.5
+    assert f["decode_tokens_per_s"] == 1 * 8 / 2.0  # batch 1, 8 steps over all 28 layers in 2 s
+    assert "all 28 layers" in f["decode_tokens_per_s_basis"]
+    assert f["nproc"] == os.cpu_count() and f["cpu_model"]
+    g = bench.cpu_baseline_fields(w, 7, 8, parts)  # a quarter of the layers: a quarter of the time per token
+    assert g["decode_tokens_per_s"] == 1 * 8 / 2.0 * 7 / 28
+    assert "extrapolated from 7 of 28" in g["decode_tokens_per_s_basis"]
+
+
+def test_floors_on_stubbed_events(monkeypatch):
+    """measure_floors times three things with the same L2 flush before each
+    repetition and reports medians; driven here with stub events on CPU."""
+    import types
+
+    import torch
+
+    import bench
+    ticks = iter(range(1000))
+    flushes = []
+
+    class Ev:
+        def record(self, stream):
+            self.t = next(ticks)
+
+        def elapsed_time(self, other):
+            return (other.t - self.t) * 1e-3  # ms: one tick = 1 us
+
+    monkeypatch.setattr(torch.cuda, "Event", lambda enable_timing=True: Ev())
+    monkeypatch.setattr(torch.cuda, "synchronize", lambda: None)
+    monkeypatch.setattr(torch.cuda, "_sleep", lambda n: None)
+    f = bench.measure_floors(4096, lambda: flushes.append(1), None, "cpu", reps=3)
+    assert len(flushes) == 9
+    assert f["events_only_us"] == 1.0 and f["empty_kernel_us"] == 1.0 and f["read_same_bytes_us"] == 1.0
+    assert f["read_bytes"] == 4096 and f["read_GBps"] > 0
