@@ -23,7 +23,6 @@ namespace hg {
 
 namespace {
 
-constexpr int kThreads = 128;
 constexpr unsigned kFull = 0xffffffffu;
 
 __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
@@ -503,38 +502,47 @@ __device__ __forceinline__ void copy_row(char* dst, const char* row_s) {
   for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
 }
 
-// Staged rows of one tile: K rows [0][r], V rows [1][r], r < n, 272-byte pitch.
-typedef char StagedRows[2][kQTok][kQPitch];
+// Staged rows of one tile: part pi (K rows, V rows, or both: K then V) at
+// [pi][r], r < n, 272-byte pitch.
+template <int NP>
+using StagedRows = char[NP][kQTok][kQPitch];
 
 // Token span of a tile: rows r < n hold tokens t0 + r.
 struct TileSpan {
   int t0, n, tlo;  // tlo: the unclipped tile start (KIVI-style tiles)
 };
 
-// Coalesced staging of a tile's K and V rows, 16 bytes of one row per
-// asynchronous copy (every chunk of a thread in flight at once); the caller
-// commits the group.
+// Coalesced staging of a tile's rows (PARTS: 1 = K, 2 = V, 3 = K then V), 16
+// bytes of one row per asynchronous copy (every chunk of a thread in flight at
+// once); the caller commits the group.
+template <int PARTS>
 __device__ __forceinline__ void stage_rows(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                           StagedRows& rows) {
+                                           StagedRows<PARTS == 3 ? 2 : 1>& rows) {
+  constexpr int NP = PARTS == 3 ? 2 : 1;
   const Dims& d = p.d;
   const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + sp.t0;
   const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
   const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
-  for (int c = threadIdx.x; c < 2 * sp.n * 16; c += kThreads) {
-    const int kv = c / (sp.n * 16), rem = c - kv * (sp.n * 16);
+  for (int c = threadIdx.x; c < NP * sp.n * 16; c += blockDim.x) {
+    const int pi = c / (sp.n * 16), rem = c - pi * (sp.n * 16);
     const int r = rem >> 4, col = rem & 15;
-    cp_async16(smem_u32(&rows[kv][r][col * 16]), (kv ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
+    const bool v = PARTS == 2 || (PARTS == 3 && pi == 1);
+    cp_async16(smem_u32(&rows[pi][r][col * 16]), (v ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
   }
 }
 
 // The per-token bases, one thread per vector: min-max rows (Sec. 1) and
 // AKVQ-style rows (Sec. 4: keys rotated first; values per token, unrotated).
-// Tiles of 64 tokens from token 0.  With salient tokens (AKVQ-style, Sec. 4)
-// a thread finds its token in the head's map: a salient token's K and V rows
-// go to the BF16 region at position s + (its rank), every other image token
-// to coded slot ti - (the salient tokens before it).
-template <int BITS, bool M16, int BASE>
+// Tiles of 64 tokens from token 0; a CTA takes the K rows, the V rows or both
+// (PARTS 1, 2, 3).  With salient tokens (AKVQ-style, Sec. 4) a thread finds its
+// token in the head's map: a salient token's K and V rows go to the BF16
+// region at position s + (its rank), every other image token to coded slot
+// ti - (the salient tokens before it).
+template <int BITS, bool M16, int BASE, int PARTS>
 struct TokenTiles {
+  static constexpr int kParts = PARTS;
+  static constexpr int kNP = PARTS == 3 ? 2 : 1;
+  static constexpr int kBlock = kQTok * kNP;
   static __device__ __forceinline__ int count(const QuantizeParams& p) { return (p.d.T + kQTok - 1) / kQTok; }
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
@@ -543,10 +551,11 @@ struct TokenTiles {
     return sp;
   }
   static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                                 const StagedRows& rows) {
+                                                 const StagedRows<kNP>& rows) {
     const Dims& d = p.d;
     const int tid = threadIdx.x;
-    const int kv = tid >> 6, r = tid & (kQTok - 1);
+    const int pi = tid >> 6, r = tid & (kQTok - 1);
+    const int kv = PARTS == 3 ? pi : (PARTS == 1 ? 0 : 1);
     if (r >= sp.n) return;
     const LayerGeom g = layer_geom(d, p.lt.mask[li]);
     const HeadGeom hd = head_geom(d, g, h);
@@ -566,7 +575,7 @@ struct TokenTiles {
       ci = ti - rank;
       if (sal) pos = d.s + rank;
     }
-    const char* row_s = rows[kv][r];
+    const char* row_s = rows[pi][r];
     constexpr int W = 4 * BITS;
     if (kv == 0) {
       if (coded && hd.cls == kQuantized && !sal) {
@@ -602,6 +611,9 @@ struct TokenTiles {
 // ---------------------------------------------------------------------------
 template <int BITS, bool M16>
 struct KiviTiles {
+  static constexpr int kParts = 3;
+  static constexpr int kNP = 2;
+  static constexpr int kBlock = 2 * kQTok;
   // tile x: [origin - 32 + 64 x, + 64) clipped to [0, T), origin = s mod 32
   static __device__ __forceinline__ int count(const QuantizeParams& p) {
     return (p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
@@ -614,7 +626,7 @@ struct KiviTiles {
     return sp;
   }
   static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                                 const StagedRows& rows) {
+                                                 const StagedRows<kNP>& rows) {
     const Dims& d = p.d;
     const int tid = threadIdx.x;
     const LayerGeom g = layer_geom(d, p.lt.mask[li]);
@@ -664,8 +676,8 @@ struct KiviTiles {
 // coding the current one measured 5-45% slower: the second buffer halves the
 // resident CTAs.)
 template <class TP>
-__global__ void __launch_bounds__(kThreads) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
-  __shared__ __align__(16) StagedRows rows;
+__global__ void __launch_bounds__(TP::kBlock) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
+  __shared__ __align__(16) StagedRows<TP::kNP> rows;
   const int nx = TP::count(p), nbh = p.d.B * p.d.H;
   const int i = blockIdx.x;
   const int tx = i % nx, rest = i / nx, bh = rest % nbh, li = rest / nbh;
@@ -673,7 +685,7 @@ __global__ void __launch_bounds__(kThreads) quantize_tiles_kernel(const __grid_c
   const int b = bh / p.d.H, h = bh % p.d.H;
   const TileSpan sp = TP::span(p, tx);
   if (sp.n <= 0) return;
-  stage_rows(p, li, b, h, sp, rows);
+  stage_rows<TP::kParts>(p, li, b, h, sp, rows);
   cp_async_commit();
   cp_async_wait<0>();
   __syncthreads();
@@ -860,7 +872,7 @@ __device__ __forceinline__ void fwht128_half(float (&x)[8], int j) {
   for (int i = 0; i < 8; ++i) x[i] = __fmul_rn(x[i], c);
 }
 
-__global__ void __launch_bounds__(kDqThreads, 5)
+__global__ void __launch_bounds__(kDqThreads, 6)
 dequantize_kernel(const __grid_constant__ DequantParams p) {
   const Dims& d = p.d;
   const int li = blockIdx.z, bh = blockIdx.y;
@@ -992,7 +1004,7 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 template <class TP>
 cudaError_t launch_tiles(const QuantizeParams& p, int tiles_x, cudaStream_t s) {
   const long long total = (long long)tiles_x * p.d.B * p.d.H * p.n_layers;
-  quantize_tiles_kernel<TP><<<(unsigned)total, kThreads, 0, s>>>(p);
+  quantize_tiles_kernel<TP><<<(unsigned)total, TP::kBlock, 0, s>>>(p);
   return cudaGetLastError();
 }
 
@@ -1004,8 +1016,15 @@ cudaError_t launch_quantize_bits(const QuantizeParams& p, cudaStream_t s) {
     return launch_tiles<KiviTiles<BITS, M16>>(p, tx, s);
   }
   const int tx = (d.T + kQTok - 1) / kQTok;
-  if (d.base == kAkvq) return launch_tiles<TokenTiles<BITS, M16, kAkvq>>(p, tx, s);
-  return launch_tiles<TokenTiles<BITS, M16, kMinMax>>(p, tx, s);
+  if (d.base == kAkvq) {
+    // keys and values in CTAs of their own: a rotated key row holds 64 fp32
+    // pairs in registers, a value row far fewer, and a kernel's threads all
+    // get the larger count -- split, twice as many key rows are resident
+    const cudaError_t e = launch_tiles<TokenTiles<BITS, M16, kAkvq, 1>>(p, tx, s);
+    if (e != cudaSuccess) return e;
+    return launch_tiles<TokenTiles<BITS, M16, kAkvq, 2>>(p, tx, s);
+  }
+  return launch_tiles<TokenTiles<BITS, M16, kMinMax, 3>>(p, tx, s);
 }
 
 cudaError_t launch_quantize(const QuantizeParams& p, cudaStream_t s) {
