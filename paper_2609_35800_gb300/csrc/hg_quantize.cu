@@ -129,33 +129,19 @@ __device__ __forceinline__ bool chunk_T(const uint64_t (&x2)[4], uint64_t mn2, u
   return __vcmpleu2(low, 0x00070007u) == 0u;
 }
 
-// Pack and store the 32 codes of one KIVI-style key group row (one channel,
-// token order): 2 / 4 bits as `bits` words, 3 bits as two words of bits 0-1
-// (16 tokens each) and the bit-2 plane.
+// Code e (0..31, token order) of one KIVI-style key group row into its packed
+// words: 2 / 4 bits at word e / (32 / bits), bit bits * (e mod 32 / bits); 3
+// bits: bits 0-1 at word e / 16, bit 2 e mod 16, and bit 2 into plane word 2 at
+// bit e with index bits 3 and 4 exchanged.  e is a compile-time constant after
+// unrolling, so each is one shift and one or.
 template <int BITS>
-__device__ __forceinline__ void store_key_group(uint32_t* dst, const uint32_t (&code)[kKiviGroup]) {
+__device__ __forceinline__ void add_key_code(uint32_t (&wd)[BITS], int e, uint32_t c) {
   if (BITS == 3) {
-    uint32_t lo0 = 0u, lo1 = 0u, hp = 0u;
-#pragma unroll
-    for (int e = 0; e < 16; ++e) {
-      lo0 |= (code[e] & 3u) << (2 * e);
-      lo1 |= (code[16 + e] & 3u) << (2 * e);
-    }
-#pragma unroll
-    for (int e = 0; e < 32; ++e)
-      hp |= ((code[e] >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
-    dst[0] = lo0;
-    dst[1] = lo1;
-    dst[2] = hp;
+    wd[e / 16] |= (c & 3u) << (2 * (e % 16));
+    wd[2] |= ((c >> 2) & 1u) << ((e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4));
   } else {
     constexpr int per = 32 / (BITS == 3 ? 2 : BITS);
-#pragma unroll
-    for (int w = 0; w < BITS; ++w) {
-      uint32_t word = 0;
-#pragma unroll
-      for (int e = 0; e < per; ++e) word |= code[w * per + e] << (BITS * e);
-      dst[w] = word;
-    }
+    wd[e / per] |= c << (BITS * (e % per));
   }
 }
 
@@ -193,7 +179,9 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
     }
     store_meta(meta, mi + j, sc[j], mn[j], M16);
   }
-  uint32_t c0[kKiviGroup], c1[kKiviGroup];
+  uint32_t wd0[BITS], wd1[BITS];  // the two channels' packed words, filled code by code
+#pragma unroll
+  for (int i = 0; i < BITS; ++i) wd0[i] = wd1[i] = 0u;
   if (!M16 && sc[0] >= 2.3509887e-38f && sc[1] >= 2.3509887e-38f) {
     const float r0 = __frcp_rn(sc[0]), r1 = __frcp_rn(sc[1]);
     const uint64_t mn2p = f32x2(__float_as_uint(mn[0]), __float_as_uint(mn[1]));
@@ -204,12 +192,11 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
     for (int e = 0; e < kKiviGroup; ++e) {
       const uint64_t t2 = f32x2_fma(f32x2_sub(f32x2(w[e] << 16, w[e] & 0xffff0000u), mn2p), r2, c2);
       const uint32_t a0 = (uint32_t)t2, a1 = (uint32_t)(t2 >> 32);
-      c0[e] = (a0 >> 16) & L;
-      c1[e] = (a1 >> 16) & L;
-      if (!(a0 & 0xfff8u))
-        c0[e] = exact_code(__fsub_rn(__uint_as_float(w[e] << 16), mn[0]), sc[0], levels);
-      if (!(a1 & 0xfff8u))
-        c1[e] = exact_code(__fsub_rn(__uint_as_float(w[e] & 0xffff0000u), mn[1]), sc[1], levels);
+      uint32_t k0 = (a0 >> 16) & L, k1 = (a1 >> 16) & L;
+      if (!(a0 & 0xfff8u)) k0 = exact_code(__fsub_rn(__uint_as_float(w[e] << 16), mn[0]), sc[0], levels);
+      if (!(a1 & 0xfff8u)) k1 = exact_code(__fsub_rn(__uint_as_float(w[e] & 0xffff0000u), mn[1]), sc[1], levels);
+      add_key_code<BITS>(wd0, e, k0);
+      add_key_code<BITS>(wd1, e, k1);
     }
   } else {
 #pragma unroll
@@ -220,13 +207,16 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
       for (int e = 0; e < kKiviGroup; ++e) {
         const float x = __uint_as_float(j ? (w[e] & 0xffff0000u) : (w[e] << 16));
         const uint32_t c = (sc[j] == 0.0f) ? 0u : code_of(__fsub_rn(x, mn[j]), sc[j], r, levels, fast);
-        if (j) c1[e] = c;
-        else c0[e] = c;
+        if (j) add_key_code<BITS>(wd1, e, c);
+        else add_key_code<BITS>(wd0, e, c);
       }
     }
   }
-  store_key_group<BITS>(dst0, c0);
-  store_key_group<BITS>(dst1, c1);
+#pragma unroll
+  for (int i = 0; i < BITS; ++i) {
+    dst0[i] = wd0[i];
+    dst1[i] = wd1[i];
+  }
 }
 
 // Codes of the 8 channels of one chunk (four BF16 pairs w[0..3]) in a group
