@@ -454,7 +454,7 @@ hg_status hg_dequantize_kv(const hg_cache* c, int32_t layer_begin, int32_t layer
     p.out_fp32 = out_fp32 ? 1 : 0;
     p.k_out = static_cast<char*>(k_out) + (size_t)done * layer_bytes;
     p.v_out = static_cast<char*>(v_out) + (size_t)done * layer_bytes;
-    const hg_status st = cuda_status(launch_dequantize(p, reinterpret_cast<cudaStream_t>(stream)));
+    const hg_status st = cuda_status(launch_dequantize(p, sm_count(), reinterpret_cast<cudaStream_t>(stream)));
     if (st != HG_OK) return st;
   }
   return HG_OK;

@@ -117,7 +117,8 @@ cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s);
 // bit per image token.
 inline size_t salient_smem_bytes(const Dims& d) { return (size_t)d.nq * 4 + (size_t)sal_blocks(d) * 4; }
 constexpr size_t kMaxSalientSmem = 200 * 1024;
-cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s);
+// Reconstruction of the launch's layers; sm_count sizes the tile spans.
+cudaError_t launch_dequantize(const DequantParams& p, int sm_count, cudaStream_t s);
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s);
 cudaError_t launch_decode(const DecodeParams& p, int grid_x, cudaStream_t s);
 cudaError_t launch_wait_probe(uint32_t* result, uint32_t rounds, cudaStream_t s);

@@ -10,6 +10,7 @@
 // resolved once per CTA, so protected heads and text tokens take a uniform
 // BF16 copy path.  Codes, scales and zeros follow the group quantizer exactly
 // (round half to even of the IEEE quotient, no contraction).
+#include <algorithm>
 #include <climits>
 
 #include <cuda_bf16.h>
@@ -540,15 +541,13 @@ struct TokenTiles {
     sp.n = min(kQTok, p.d.T - sp.t0);
     return sp;
   }
-  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                                 const StagedRows<kNP>& rows) {
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, const TileSpan& sp,
+                                                 const StagedRows<kNP>& rows, const HeadGeom& hd) {
     const Dims& d = p.d;
     const int tid = threadIdx.x;
     const int pi = tid >> 6, r = tid & (kQTok - 1);
     const int kv = PARTS == 3 ? pi : (PARTS == 1 ? 0 : 1);
     if (r >= sp.n) return;
-    const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-    const HeadGeom hd = head_geom(d, g, h);
     char* Lb = p.arena + p.lt.base[li];
     const int t = sp.t0 + r;
     const bool coded = t >= d.s && t < d.s + d.nq;
@@ -615,12 +614,10 @@ struct KiviTiles {
     sp.n = min(sp.tlo + kQTok, p.d.T) - sp.t0;
     return sp;
   }
-  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                                 const StagedRows<kNP>& rows) {
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, const TileSpan& sp,
+                                                 const StagedRows<kNP>& rows, const HeadGeom& hd) {
     const Dims& d = p.d;
     const int tid = threadIdx.x;
-    const LayerGeom g = layer_geom(d, p.lt.mask[li]);
-    const HeadGeom hd = head_geom(d, g, h);
     char* Lb = p.arena + p.lt.base[li];
     const int qs = d.s, qe = d.s + d.nq;
     const int t0 = sp.t0, t1 = sp.t0 + sp.n, tlo = sp.tlo;
@@ -668,6 +665,7 @@ struct KiviTiles {
 template <class TP>
 __global__ void __launch_bounds__(TP::kBlock) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
   __shared__ __align__(16) StagedRows<TP::kNP> rows;
+  __shared__ HeadGeom s_hd;
   const int nx = TP::count(p), nbh = p.d.B * p.d.H;
   const int i = blockIdx.x;
   const int tx = i % nx, rest = i / nx, bh = rest % nbh, li = rest / nbh;
@@ -677,9 +675,12 @@ __global__ void __launch_bounds__(TP::kBlock) quantize_tiles_kernel(const __grid
   if (sp.n <= 0) return;
   stage_rows<TP::kParts>(p, li, b, h, sp, rows);
   cp_async_commit();
+  // the head's region map, once for the CTA while its copies are in flight
+  // (64-bit arithmetic that would otherwise run in every thread)
+  if (threadIdx.x == 0) s_hd = head_geom(p.d, layer_geom(p.d, p.lt.mask[li]), h);
   cp_async_wait<0>();
   __syncthreads();
-  TP::process(p, li, b, h, sp, rows);
+  TP::process(p, li, b, sp, rows, s_hd);
 }
 
 // ---------------------------------------------------------------------------
@@ -862,8 +863,12 @@ __device__ __forceinline__ void fwht128_half(float (&x)[8], int j) {
   for (int i = 0; i < 8; ++i) x[i] = __fmul_rn(x[i], c);
 }
 
-__global__ void __launch_bounds__(kDqThreads, 6)
-dequantize_kernel(const __grid_constant__ DequantParams p) {
+// BITS, BASE and M16 are compile-time, so each (code width, base, metadata
+// width) runs code of its own; a CTA takes a span of consecutive tiles of one
+// (row, head, layer), so the head's region map and its barrier are paid once
+// per span.
+template <int BITS, int BASE, bool M16>
+__global__ void __launch_bounds__(kDqThreads, 6) dequantize_kernel(const __grid_constant__ DequantParams p) {
   const Dims& d = p.d;
   const int li = blockIdx.z, bh = blockIdx.y;
   const int b = bh / d.H, h = bh % d.H;
@@ -876,94 +881,100 @@ dequantize_kernel(const __grid_constant__ DequantParams p) {
   const HeadGeom& hd = s_hd;
   const char* Lb = p.arena + p.lt.base[li];
   const int qs = d.s, qe = d.s + d.nq;
-  const int W = kD * d.bits / 32;
-  const bool m16 = d.meta16 != 0;
+  constexpr int W = kD * BITS / 32;
   const int j = threadIdx.x & 15;  // channels 8j..8j+7
   const size_t out_row0 = (((size_t)li * d.B + b) * d.H + h) * (size_t)Tt;
+  const int ntiles = (Tt + kDqTile - 1) / kDqTile;
+  const int span = (ntiles + (int)gridDim.x - 1) / (int)gridDim.x;
+  const int x1 = min(((int)blockIdx.x + 1) * span, ntiles);
 
-  // unit u: K (u < 16 * kDqTile) or V, token (u >> 4) % kDqTile of the tile;
-  // unrolled so that the loads of a thread's four units are in flight together
+#pragma unroll 1
+  for (int x = blockIdx.x * span; x < x1; ++x) {
+    // unit u: K (u < 16 * kDqTile) or V, token (u >> 4) % kDqTile of the
+    // tile; unrolled so that the loads of a thread's four units are in flight
+    // together
 #pragma unroll
-  for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
-    const bool is_k = u < kDqTile * 16;
-    const int t = blockIdx.x * kDqTile + ((u >> 4) & (kDqTile - 1));
-    if (t >= Tt) continue;  // uniform over the half-warp
-    const bool coded = (t >= qs) && (t < qe);
-    const int ti = t - qs;
-    int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token (Sec. 4)
-    bool sal = false;
-    if (coded && d.ns > 0 && hd.cls != kProtected) {
-      const char* sm = Lb + hd.sal + b * hd.sal_bs;
-      const int w = ti >> 5, e = ti & 31;
-      const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
-      const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
-                       __popc(sb & ((1u << e) - 1u));
-      sal = (sb >> e) & 1u;
-      ci = ti - rank;
-      spos = qs + rank;
-    }
-    const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
-    const size_t o = (out_row0 + t) * kD + 8 * j;
-    void* dst = is_k ? p.k_out : p.v_out;
-    float x[8];
-    bool raw = false;  // a BF16 entry: `w` holds its 16 bytes
-    uint4 w = make_uint4(0u, 0u, 0u, 0u);
-    if (is_k) {
-      if (coded && hd.cls == kQuantized && !sal) {
-        uint32_t code[8];
-        float2 m[8];
-        if (d.base == kKivi) {
-          const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
-          const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) +
-                                  ((size_t)grp * kD + 8 * j) * d.bits;
-          const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
+    for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
+      const bool is_k = u < kDqTile * 16;
+      const int t = x * kDqTile + ((u >> 4) & (kDqTile - 1));
+      if (t >= Tt) continue;  // uniform over the half-warp
+      const bool coded = (t >= qs) && (t < qe);
+      const int ti = t - qs;
+      int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token (Sec. 4)
+      bool sal = false;
+      if (BASE == kAkvq && coded && d.ns > 0 && hd.cls != kProtected) {
+        const char* sm = Lb + hd.sal + b * hd.sal_bs;
+        const int w = ti >> 5, e = ti & 31;
+        const uint32_t sb = __ldg(reinterpret_cast<const uint32_t*>(sm) + w);
+        const int rank = __ldg(reinterpret_cast<const int*>(sm + (size_t)sal_blocks(d) * 4) + w) +
+                         __popc(sb & ((1u << e) - 1u));
+        sal = (sb >> e) & 1u;
+        ci = ti - rank;
+        spos = qs + rank;
+      }
+      const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
+      const size_t o = (out_row0 + t) * kD + 8 * j;
+      void* dst = is_k ? p.k_out : p.v_out;
+      float x8[8];
+      bool raw = false;  // a BF16 entry: `w` holds its 16 bytes
+      uint4 w = make_uint4(0u, 0u, 0u, 0u);
+      if (is_k) {
+        if (coded && hd.cls == kQuantized && !sal) {
+          uint32_t code[8];
+          float2 m[8];
+          if (BASE == kKivi) {
+            const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
+            const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) +
+                                    ((size_t)grp * kD + 8 * j) * BITS;
+            const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            code[i] = kivi_code(codes + i * d.bits, d.bits, e);
-            m[i] = load_meta(meta, (size_t)grp * kD + 8 * j + i, m16);
+            for (int i = 0; i < 8; ++i) {
+              code[i] = kivi_code(codes + i * BITS, BITS, e);
+              m[i] = load_meta(meta, (size_t)grp * kD + 8 * j + i, M16);
+            }
+          } else {
+            row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W, BITS, j,
+                       code);
+            const float2 m0 = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, M16);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) m[i] = m0;
           }
+#pragma unroll
+          for (int i = 0; i < 8; ++i) x8[i] = dequant1(code[i], m[i].x, m[i].y);
+          if (BASE == kAkvq) fwht128_half(x8, j);  // inverse rotation (H is self-inverse)
         } else {
-          row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W, d.bits, j,
-                     code);
-          const float2 m0 = load_meta(Lb + hd.kqm + b * hd.kqm_bs, ci, m16);
-#pragma unroll
-          for (int i = 0; i < 8; ++i) m[i] = m0;
+          const char* src = (coded && hd.cls == kKeysOnly && !sal)
+                                ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
+                                : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
+          w = ldg16(src + j * 16);
+          raw = true;
         }
-#pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] = dequant1(code[i], m[i].x, m[i].y);
-        if (d.base == kAkvq) fwht128_half(x, j);  // inverse rotation (H is self-inverse)
       } else {
-        const char* src = (coded && hd.cls == kKeysOnly && !sal)
-                              ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
-                              : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
-        w = ldg16(src + j * 16);
-        raw = true;
-      }
-    } else {
-      if (coded && hd.cls != kProtected && !sal) {
-        uint32_t code[8];
-        row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W, d.bits, j,
-                   code);
-        // KIVI-style: 32-channel groups, channels 8j.. in group j / 4
-        const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
-                                   (size_t)ci * vgroups(d) + (d.base == kKivi ? (j >> 2) : 0), m16);
+        if (coded && hd.cls != kProtected && !sal) {
+          uint32_t code[8];
+          row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W, BITS, j,
+                     code);
+          // KIVI-style: 32-channel groups, channels 8j.. in group j / 4
+          const float2 m = load_meta(Lb + hd.vqm + b * hd.vqm_bs,
+                                     (size_t)ci * vgroups(d) + (BASE == kKivi ? (j >> 2) : 0), M16);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) x[i] = dequant1(code[i], m.x, m.y);
-      } else {
-        w = ldg16(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256 + j * 16);
-        raw = true;
+          for (int i = 0; i < 8; ++i) x8[i] = dequant1(code[i], m.x, m.y);
+        } else {
+          w = ldg16(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256 + j * 16);
+          raw = true;
+        }
       }
-    }
-    if (p.out_fp32) {
-      if (raw) bf16x8_to_f32(w, x);
-      float4* f = reinterpret_cast<float4*>(static_cast<float*>(dst) + o);
-      f[0] = make_float4(x[0], x[1], x[2], x[3]);
-      f[1] = make_float4(x[4], x[5], x[6], x[7]);
-    } else {
-      if (!raw)
-        w = make_uint4(pack_bf16x2_rn(x[0], x[1]), pack_bf16x2_rn(x[2], x[3]), pack_bf16x2_rn(x[4], x[5]),
-                       pack_bf16x2_rn(x[6], x[7]));
-      *reinterpret_cast<uint4*>(static_cast<uint16_t*>(dst) + o) = w;
+      if (p.out_fp32) {
+        if (raw) bf16x8_to_f32(w, x8);
+        float4* f = reinterpret_cast<float4*>(static_cast<float*>(dst) + o);
+        f[0] = make_float4(x8[0], x8[1], x8[2], x8[3]);
+        f[1] = make_float4(x8[4], x8[5], x8[6], x8[7]);
+      } else {
+        if (!raw)
+          w = make_uint4(pack_bf16x2_rn(x8[0], x8[1]), pack_bf16x2_rn(x8[2], x8[3]),
+                         pack_bf16x2_rn(x8[4], x8[5]), pack_bf16x2_rn(x8[6], x8[7]));
+        *reinterpret_cast<uint4*>(static_cast<uint16_t*>(dst) + o) = w;
+      }
     }
   }
 }
@@ -1036,11 +1047,35 @@ cudaError_t launch_salient(const QuantizeParams& p, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_dequantize(const DequantParams& p, cudaStream_t s) {
-  const int Tt = p.d.T + p.appended;
-  dim3 grid((Tt + kDqTile - 1) / kDqTile, p.d.B * p.d.H, p.n_layers);
-  dequantize_kernel<<<grid, kDqThreads, 0, s>>>(p);
+template <int BITS, int BASE, bool M16>
+cudaError_t launch_dequantize_t(const DequantParams& p, dim3 grid, cudaStream_t s) {
+  dequantize_kernel<BITS, BASE, M16><<<grid, kDqThreads, 0, s>>>(p);
   return cudaGetLastError();
+}
+
+template <int BITS>
+cudaError_t launch_dequantize_bits(const DequantParams& p, dim3 grid, cudaStream_t s) {
+  const bool m16 = p.d.meta16 != 0;
+  if (p.d.base == kKivi)
+    return m16 ? launch_dequantize_t<BITS, kKivi, true>(p, grid, s) : launch_dequantize_t<BITS, kKivi, false>(p, grid, s);
+  if (p.d.base == kAkvq)
+    return m16 ? launch_dequantize_t<BITS, kAkvq, true>(p, grid, s) : launch_dequantize_t<BITS, kAkvq, false>(p, grid, s);
+  return m16 ? launch_dequantize_t<BITS, kMinMax, true>(p, grid, s)
+             : launch_dequantize_t<BITS, kMinMax, false>(p, grid, s);
+}
+
+cudaError_t launch_dequantize(const DequantParams& p, int sm_count, cudaStream_t s) {
+  const int Tt = p.d.T + p.appended;
+  const int ntiles = (Tt + kDqTile - 1) / kDqTile;
+  // spans of several tiles once the grid holds more than 16 waves of 6 CTAs
+  // per SM (at most 8 tiles a CTA)
+  const long long groups = (long long)p.d.B * p.d.H * p.n_layers;
+  const long long waves16 = 16LL * 6 * (sm_count > 0 ? sm_count : 1);
+  const int span = (int)std::max(1LL, std::min(8LL, groups * ntiles / waves16));
+  dim3 grid((ntiles + span - 1) / span, p.d.B * p.d.H, p.n_layers);
+  if (p.d.bits == 2) return launch_dequantize_bits<2>(p, grid, s);
+  if (p.d.bits == 3) return launch_dequantize_bits<3>(p, grid, s);
+  return launch_dequantize_bits<4>(p, grid, s);
 }
 
 cudaError_t launch_append(const AppendParams& p, cudaStream_t s) {
