@@ -50,7 +50,7 @@ __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
 // within one unit of 0x8000 rounds the same way as the reference.
 // Uncoded vectors (text, protected heads, keys of keys-only heads) are copied.
 // ---------------------------------------------------------------------------
-constexpr int kQTok = 64;
+constexpr int kQTok = 32;
 constexpr int kQPitch = 272;
 
 // Round-half-even of fl(d / scale), clamped to the levels (IEEE division).
@@ -281,12 +281,24 @@ __device__ __forceinline__ void chunk_near_tie(const uint32_t (&a)[8], X x, floa
     c8[i] = (a[i] & 0xfff8u) ? ((a[i] >> 16) & L) : exact_code(__fsub_rn(x(i), mn), scale, (float)L);
 }
 
+// Chunks per store unit of the packed row: the chunks whose codes share the
+// words that a chunk's codes go into (4 bits: one word per chunk; 2 bits: two
+// chunks per word; 3 bits: four chunks per plane word).
+template <int BITS>
+constexpr int kChunksPerUnit = BITS == 4 ? 1 : (BITS == 2 ? 2 : 4);
+
 // One group of a BF16 row: chunks [k0, k0 + nk) (8 channels each) with their
 // min / max over bf16x2 pairs (exact), signed zeros folded to +0,
 // scale = fl((max - min) / levels), metadata stored at index mi (binary16
 // pair with M16: codes against the rounded pair), codes 0 when scale == 0,
 // each chunk's codes emitted into the packed row.  The chunk loop stays rolled
 // (by two) so that the code is small and stays in the instruction cache.
+// A chunk with an element near a tie (fast rule) is emitted with its fast
+// codes and flagged; after the loop each thread codes the store units of its
+// flagged chunks again, the flagged elements by the exact rule, and stores
+// them over the first ones.  The threads of a warp do this side by side, so a
+// warp pays for the largest number of flagged units of one thread instead of
+// running every thread's near ties one after another inside the loop.
 template <int BITS, bool M16>
 __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int nk, uint32_t* codes, char* meta,
                                                    size_t mi, uint32_t& prev, uint32_t& plane) {
@@ -323,6 +335,7 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
   const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
   const uint32_t cbits = __float_as_uint(192.50006103515625f);  // C = 192.5 + 4 * 2^-16
   const uint64_t c2 = f32x2(cbits, cbits);
+  uint32_t ties = 0u;  // bit k - k0: chunk k has an element near a tie
 #pragma unroll 2
   for (int k = k0; k < k0 + nk; ++k) {
     const uint4 v = r4[k];
@@ -333,13 +346,9 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
 #pragma unroll
       for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1
       uint32_t a[8];
-      if (chunk_T(x2, mnp, r2, c2, a)) {
-        emit_from_T<BITS>(k, a, codes, prev, plane);
-        continue;
-      }
-      // a near-tie in this chunk (about one chunk in 500): the exact rule for it
-      chunk_near_tie<BITS>(a, [&](int i) { return __uint_as_float((i & 1) ? (w[i >> 1] & 0xffff0000u) : (w[i >> 1] << 16)); },
-                           mn, scale, c8);
+      if (!chunk_T(x2, mnp, r2, c2, a)) ties |= 1u << (k - k0);  // about one chunk in 100
+      emit_from_T<BITS>(k, a, codes, prev, plane);
+      continue;
     } else if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
 #pragma unroll
       for (int i = 0; i < 8; ++i) c8[i] = 0u;
@@ -347,6 +356,25 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
       chunk_codes<BITS, M16>(w, mn, scale, r, c8);
     }
     emit_chunk<BITS>(k, c8, codes, prev, plane);
+  }
+  constexpr int U = kChunksPerUnit<BITS>;
+  while (ties) {
+    const int u0 = k0 + (((__ffs(ties) - 1) / U) * U);  // first chunk of the unit
+    ties &= ~(((1u << U) - 1u) << (u0 - k0));
+    uint32_t up = 0u, upl = 0u;
+#pragma unroll 1
+    for (int k = u0; k < u0 + U; ++k) {
+      const uint4 v = r4[k];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      uint64_t x2[4];
+#pragma unroll
+      for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);
+      uint32_t a[8], c8[8];
+      chunk_T(x2, mnp, r2, c2, a);
+      chunk_near_tie<BITS>(a, [&](int i) { return __uint_as_float((i & 1) ? (w[i >> 1] & 0xffff0000u) : (w[i >> 1] << 16)); },
+                           mn, scale, c8);
+      emit_chunk<BITS>(k, c8, codes, up, upl);
+    }
   }
 }
 
@@ -493,60 +521,51 @@ __device__ __forceinline__ void copy_row(char* dst, const char* row_s) {
   for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
 }
 
-// Staged rows of one tile: part pi (K rows, V rows, or both: K then V) at
-// [pi][r], r < n, 272-byte pitch.
-template <int NP>
-using StagedRows = char[NP][kQTok][kQPitch];
+// Staged rows of one warp tile: row r < n holds token t0 + r, 272-byte pitch.
+using StagedRows = char[kQTok][kQPitch];
 
 // Token span of a tile: rows r < n hold tokens t0 + r.
 struct TileSpan {
   int t0, n, tlo;  // tlo: the unclipped tile start (KIVI-style tiles)
 };
 
-// Coalesced staging of a tile's rows (PARTS: 1 = K, 2 = V, 3 = K then V), 16
-// bytes of one row per asynchronous copy (every chunk of a thread in flight at
-// once); the caller commits the group.
-template <int PARTS>
-__device__ __forceinline__ void stage_rows(const QuantizeParams& p, int li, int b, int h, const TileSpan& sp,
-                                           StagedRows<PARTS == 3 ? 2 : 1>& rows) {
-  constexpr int NP = PARTS == 3 ? 2 : 1;
+// Coalesced staging of one part (K or V rows) of a tile by the CTA's warp:
+// lane l copies 16-byte chunks l, l + 32, ... of the tile's contiguous rows
+// (every chunk in flight at once); the caller commits the group.
+__device__ __forceinline__ void stage_rows(const QuantizeParams& p, int li, int b, int h, int kv, const TileSpan& sp,
+                                           StagedRows& rows) {
   const Dims& d = p.d;
   const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + sp.t0;
-  const char* src_k = reinterpret_cast<const char*>(p.k[li] + row0 * kD);
-  const char* src_v = reinterpret_cast<const char*>(p.v[li] + row0 * kD);
-  for (int c = threadIdx.x; c < NP * sp.n * 16; c += blockDim.x) {
-    const int pi = c / (sp.n * 16), rem = c - pi * (sp.n * 16);
-    const int r = rem >> 4, col = rem & 15;
-    const bool v = PARTS == 2 || (PARTS == 3 && pi == 1);
-    cp_async16(smem_u32(&rows[pi][r][col * 16]), (v ? src_v : src_k) + (size_t)r * 256 + col * 16, 16);
+  const char* src = reinterpret_cast<const char*>((kv ? p.v[li] : p.k[li]) + row0 * kD);
+  for (int c = threadIdx.x; c < sp.n * 16; c += 32) {
+    const int r = c >> 4, col = c & 15;
+    cp_async16(smem_u32(&rows[r][col * 16]), src + (size_t)r * 256 + col * 16, 16);
   }
 }
 
 // The per-token bases, one thread per vector: min-max rows (Sec. 1) and
 // AKVQ-style rows (Sec. 4: keys rotated first; values per token, unrotated).
-// Tiles of 64 tokens from token 0; a CTA takes the K rows, the V rows or both
-// (PARTS 1, 2, 3).  With salient tokens (AKVQ-style, Sec. 4) a thread finds its
-// token in the head's map: a salient token's K and V rows go to the BF16
-// region at position s + (its rank), every other image token to coded slot
-// ti - (the salient tokens before it).
+// Tiles of 32 tokens from token 0; a CTA (one warp) takes the K rows or the V
+// rows of a tile (PARTS 1: K only, 2: V only, 3: both, as two CTAs).  With
+// salient tokens (AKVQ-style, Sec. 4) a thread finds its token in the head's
+// map: a salient token's K and V rows go to the BF16 region at position
+// s + (its rank), every other image token to coded slot ti - (the salient
+// tokens before it).
 template <int BITS, bool M16, int BASE, int PARTS>
 struct TokenTiles {
-  static constexpr int kParts = PARTS;
-  static constexpr int kNP = PARTS == 3 ? 2 : 1;
-  static constexpr int kBlock = kQTok * kNP;
+  static constexpr int kNParts = PARTS == 3 ? 2 : 1;
   static __device__ __forceinline__ int count(const QuantizeParams& p) { return (p.d.T + kQTok - 1) / kQTok; }
+  static __device__ __forceinline__ int part(int i) { return PARTS == 3 ? i : (PARTS == 1 ? 0 : 1); }
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
     sp.t0 = sp.tlo = tx * kQTok;
     sp.n = min(kQTok, p.d.T - sp.t0);
     return sp;
   }
-  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, const TileSpan& sp,
-                                                 const StagedRows<kNP>& rows, const HeadGeom& hd) {
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int kv, const TileSpan& sp,
+                                                 const StagedRows& rows, const HeadGeom& hd) {
     const Dims& d = p.d;
-    const int tid = threadIdx.x;
-    const int pi = tid >> 6, r = tid & (kQTok - 1);
-    const int kv = PARTS == 3 ? pi : (PARTS == 1 ? 0 : 1);
+    const int r = threadIdx.x;
     if (r >= sp.n) return;
     char* Lb = p.arena + p.lt.base[li];
     const int t = sp.t0 + r;
@@ -564,7 +583,7 @@ struct TokenTiles {
       ci = ti - rank;
       if (sal) pos = d.s + rank;
     }
-    const char* row_s = rows[pi][r];
+    const char* row_s = rows[r];
     constexpr int W = 4 * BITS;
     if (kv == 0) {
       if (coded && hd.cls == kQuantized && !sal) {
@@ -588,25 +607,24 @@ struct TokenTiles {
 };
 
 // ---------------------------------------------------------------------------
-// KIVI-style base (Sec. 4), on staged rows as above: one CTA per (64-token
-// tile, batch row, KV head, layer), tiles aligned so that the image's 32-token
-// key groups (anchored at the image start) never straddle two tiles.  Values
-// of every head whose image values are coded: one thread per token row, four
-// 32-channel groups.  Keys of a quantized head: once the rows are staged,
-// thread c quantizes channel c over each whole key group of the tile (32
+// KIVI-style base (Sec. 4), on staged rows as above: one CTA (one warp) per
+// (32-token tile, K or V rows, batch row, KV head, layer), tiles aligned so
+// that each of the image's 32-token key groups (anchored at the image start)
+// is one whole tile.  Values of every head whose image values are coded: one
+// thread per token row, four 32-channel groups.  Keys of a quantized head:
+// lane c quantizes channel pairs c and c + 32 over the tile's key group (32
 // consecutive image tokens, packed in token order).  Every other row (text,
 // the BF16 residual window and a trailing partial group, protected heads,
 // keys of keys-only heads) is copied.
 // ---------------------------------------------------------------------------
 template <int BITS, bool M16>
 struct KiviTiles {
-  static constexpr int kParts = 3;
-  static constexpr int kNP = 2;
-  static constexpr int kBlock = 2 * kQTok;
-  // tile x: [origin - 32 + 64 x, + 64) clipped to [0, T), origin = s mod 32
+  static constexpr int kNParts = 2;
+  // tile x: [origin - 32 + 32 x, + 32) clipped to [0, T), origin = s mod 32
   static __device__ __forceinline__ int count(const QuantizeParams& p) {
     return (p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
   }
+  static __device__ __forceinline__ int part(int i) { return i; }
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
     sp.tlo = p.tile_origin - kKiviGroup + kQTok * tx;
@@ -614,73 +632,74 @@ struct KiviTiles {
     sp.n = min(sp.tlo + kQTok, p.d.T) - sp.t0;
     return sp;
   }
-  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, const TileSpan& sp,
-                                                 const StagedRows<kNP>& rows, const HeadGeom& hd) {
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int kv, const TileSpan& sp,
+                                                 const StagedRows& rows, const HeadGeom& hd) {
     const Dims& d = p.d;
-    const int tid = threadIdx.x;
+    const int lane = threadIdx.x;
     char* Lb = p.arena + p.lt.base[li];
     const int qs = d.s, qe = d.s + d.nq;
-    const int t0 = sp.t0, t1 = sp.t0 + sp.n, tlo = sp.tlo;
+    const int t0 = sp.t0, tlo = sp.tlo;
     constexpr int W = 4 * BITS;
-    const int kv = tid >> 6, r = tid & (kQTok - 1);
-    if (r < sp.n) {
-      const int t = t0 + r;
+    if (kv == 1) {
+      if (lane >= sp.n) return;
+      const int t = t0 + lane;
       const bool coded = t >= qs && t < qe;
       const int ti = t - qs;
-      const char* row_s = rows[kv][r];
-      if (kv == 0) {
-        if (!(coded && hd.cls == kQuantized))  // quantized keys: by channel below
-          copy_row((coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ti * 256
-                                                  : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256,
-                   row_s);
-      } else if (coded && hd.cls != kProtected) {
-        quantize_row_kivi_v<BITS, M16>(row_s,
-                                       reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
+      if (coded && hd.cls != kProtected)
+        quantize_row_kivi_v<BITS, M16>(rows[lane], reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ti * W,
                                        Lb + hd.vqm + b * hd.vqm_bs, (size_t)ti * 4);
-      } else {
-        copy_row(Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256, row_s);
+      else
+        copy_row(Lb + hd.vb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256, rows[lane]);
+      return;
+    }
+    // keys: a whole image key group of a quantized head, by channel pairs
+    // (uniform over the warp), else the rows are copied
+    if (hd.cls == kQuantized && tlo >= qs && tlo + kKiviGroup <= qe && tlo == t0 && sp.n == kKiviGroup) {
+      const int grp = (tlo - qs) / kKiviGroup;
+#pragma unroll 1
+      for (int c2 = lane; c2 < 64; c2 += 32) {
+        uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + 2 * c2) * BITS;
+        quantize_key_pair<BITS, M16>(&rows[0][4 * c2], dst, dst + BITS, Lb + hd.kqm + b * hd.kqm_bs,
+                                     (size_t)grp * kD + 2 * c2);
       }
+      return;
     }
-    if (hd.cls != kQuantized) return;  // uniform over the CTA
-
-    // KIVI-style keys: both whole groups of the tile at once, thread c taking
-    // channels 2 (c % 64) and 2 (c % 64) + 1 of group c / 64 (the staged rows
-    // are only read)
-    const int g0 = tlo + kKiviGroup * (tid >> 6), c2 = tid & 63;
-    if (g0 >= qs && g0 + kKiviGroup <= qe && g0 >= t0 && g0 + kKiviGroup <= t1) {
-      const int grp = (g0 - qs) / kKiviGroup;
-      uint32_t* dst = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + ((size_t)grp * kD + 2 * c2) * BITS;
-      quantize_key_pair<BITS, M16>(&rows[0][g0 - t0][4 * c2], dst, dst + BITS, Lb + hd.kqm + b * hd.kqm_bs,
-                                   (size_t)grp * kD + 2 * c2);
-    }
+    if (lane >= sp.n) return;
+    const int t = t0 + lane;
+    const bool coded = t >= qs && t < qe;
+    if (coded && hd.cls == kQuantized) return;  // unreachable: coded key groups are whole tiles
+    copy_row((coded && hd.cls == kKeysOnly) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)(t - qs) * 256
+                                            : Lb + hd.kb + b * hd.kb_bs + (size_t)bf16_pos(d, hd.cls, t) * 256,
+             rows[lane]);
   }
 };
 
-// The quantizer kernel: one CTA per tile, tiles numbered (tile, batch row x
-// KV head, layer) with the tile index fastest.  A CTA stages its tile, waits
-// for the copies and codes it; the copies of other resident CTAs overlap its
-// work.  (Persistent CTAs that stage the next tile into a second buffer while
-// coding the current one measured 5-45% slower: the second buffer halves the
-// resident CTAs.)
+// The quantizer kernel: one CTA of one warp per (tile, part), numbered
+// (part, tile, batch row x KV head, layer) with the part fastest.  A warp
+// stages its 32 rows, waits for its own copies and codes them; no CTA-wide
+// barrier, so the warps of an SM (23 resident) run out of step and one
+// warp's loads overlap another's coding.
 template <class TP>
-__global__ void __launch_bounds__(TP::kBlock) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
-  __shared__ __align__(16) StagedRows<TP::kNP> rows;
+__global__ void __launch_bounds__(32) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
+  __shared__ __align__(16) StagedRows rows;
   __shared__ HeadGeom s_hd;
   const int nx = TP::count(p), nbh = p.d.B * p.d.H;
   const int i = blockIdx.x;
-  const int tx = i % nx, rest = i / nx, bh = rest % nbh, li = rest / nbh;
+  const int pi = i % TP::kNParts, rest = i / TP::kNParts;
+  const int tx = rest % nx, rest2 = rest / nx, bh = rest2 % nbh, li = rest2 / nbh;
   if (li >= p.n_layers) return;
   const int b = bh / p.d.H, h = bh % p.d.H;
+  const int kv = TP::part(pi);
   const TileSpan sp = TP::span(p, tx);
   if (sp.n <= 0) return;
-  stage_rows<TP::kParts>(p, li, b, h, sp, rows);
+  stage_rows(p, li, b, h, kv, sp, rows);
   cp_async_commit();
   // the head's region map, once for the CTA while its copies are in flight
   // (64-bit arithmetic that would otherwise run in every thread)
   if (threadIdx.x == 0) s_hd = head_geom(p.d, layer_geom(p.d, p.lt.mask[li]), h);
   cp_async_wait<0>();
-  __syncthreads();
-  TP::process(p, li, b, sp, rows, s_hd);
+  __syncwarp();
+  TP::process(p, li, b, kv, sp, rows, s_hd);
 }
 
 // ---------------------------------------------------------------------------
@@ -1004,8 +1023,8 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 // Launch of the quantizer kernel over every tile of the launch's layers.
 template <class TP>
 cudaError_t launch_tiles(const QuantizeParams& p, int tiles_x, cudaStream_t s) {
-  const long long total = (long long)tiles_x * p.d.B * p.d.H * p.n_layers;
-  quantize_tiles_kernel<TP><<<(unsigned)total, TP::kBlock, 0, s>>>(p);
+  const long long total = (long long)tiles_x * TP::kNParts * p.d.B * p.d.H * p.n_layers;
+  quantize_tiles_kernel<TP><<<(unsigned)total, 32, 0, s>>>(p);
   return cudaGetLastError();
 }
 
