@@ -354,6 +354,45 @@ def test_minmax_quantize_exact_ties(bits, meta_bits):
     check_arena_layer(runner, 0, kb, vb, o)
 
 
+@pytest.mark.parametrize("base,bits,lo,hi", [(M, 2, -1.0, 1.375), (M, 2, -1.0, 5.25), (M, 3, -0.3125, 2.75),
+                                             (M, 3, -1.0, 1.375), (M, 4, 0.5, 7.5), (M, 4, 1.375, 9.5),
+                                             (K, 2, -2.5, 0.8125), (K, 2, -2.5, 12.0), (K, 3, -1.0, 1.375),
+                                             (K, 4, -0.3125, 7.5), (A, 4, -1.0, 1.375), (A, 2, -1.0, 5.25)],
+                         ids=["minmax2", "minmax2n", "minmax3", "minmax3n", "minmax4", "minmax4n", "kivi2",
+                              "kivi2n", "kivi3n", "kivi4n", "akvq4", "akvq2n"])
+def test_quantize_near_ties(base, bits, lo, hi):
+    """Every group (per-token rows, 32-channel value groups, 32-token key
+    groups) holds the same minimum lo and maximum hi, and the other entries
+    are the BF16 roundings of lo + (g + 1/2) * scale, scale = (hi - lo) /
+    levels not a power of two: a few per cent of the elements land within
+    2^-13 of a half-integer quotient, some of them exactly on it, which the
+    kernel decides without a division and the oracle by the IEEE quotient.
+    Arena bits must equal the oracle's."""
+    w = wl.custom("near%d" % bits, 1, 2, 8, 4, 7, 160, 9, base, bits, 0, decode_steps=1, seed=4,
+                  protected=[(0, 1)], residual=32)
+    runner = CacheRunner(w)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    gen = torch.Generator().manual_seed(23 + bits)
+    L = (1 << bits) - 1
+    scale = np.float32((np.float32(hi) - np.float32(lo)) / np.float32(L))
+    g = torch.randint(0, L, (2, B, H, T, 128), generator=gen).double()
+    x = float(lo) + (g + 0.5) * float(scale)
+    x[..., 0::32] = lo   # every 32-channel group and every token row: lo and hi
+    x[..., 1::32] = hi
+    off = (torch.arange(T) - w.img_start) % 32  # every 32-token key group of the image
+    x[:, :, :, off == 0, :] = lo
+    x[:, :, :, off == 1, :] = hi
+    xb = x.float().to(torch.bfloat16)
+    assert float(xb.float().min()) == lo and float(xb.float().max()) == hi
+    k = xb[0].contiguous().cuda()
+    v = xb[1].contiguous().cuda()
+    hg.hg_quantize_kv(runner.cache, 0, [k], [v])
+    torch.cuda.synchronize()
+    kb, vb = bits16(k), bits16(v)
+    o = oracle_layer(runner, 0, kb, vb)
+    check_arena_layer(runner, 0, kb, vb, o)
+
+
 @pytest.mark.parametrize("base,bits", [(M, 2), (M, 4), (K, 2), (A, 4)],
                          ids=["minmax2", "minmax4", "kivi2", "akvq4"])
 def test_meta16_extreme_ranges(base, bits):
