@@ -397,49 +397,70 @@ __device__ __forceinline__ void quantize_row_kivi_v(const char* row_s, uint32_t*
 }
 
 // ---------------------------------------------------------------------------
-// AKVQ-style keys (Sec. 4), one thread per vector: the BF16 row is widened
-// into 64 packed fp32 pairs (channels 2m, 2m + 1), rotated by the normalised
-// Hadamard-128 in registers -- stage h = 1 inside each pair, stages h = 2..64
-// on whole pairs (both halves of a pair meet the same partner offset), the
-// 1/sqrt(128) factor once at the end, the same butterflies in the same order
-// as the warp-wide transform -- and quantized per token like the min-max
-// rows above, with the same exact code rule.
+// AKVQ-style keys (Sec. 4): the BF16 row is widened into 64 packed fp32 pairs
+// (channels 2m, 2m + 1), rotated by the normalised Hadamard-128 in registers
+// -- stage h = 1 inside each pair, stages h = 2..64 on whole pairs (both
+// halves of a pair meet the same partner offset), the 1/sqrt(128) factor once
+// at the end, the same butterflies in the same order as the warp-wide
+// transform -- and quantized per token like the min-max rows above, with the
+// same exact code rule.  SPLIT = 2 spreads a row over the lanes hh = 0, 1 of
+// a lane pair (pmask): lane hh holds pairs 32 hh .. 32 hh + 31 (channels
+// 64 hh ..), runs stages 2..32 alone, meets its partner for stage 64 and for
+// the row's min / max by shuffles, and codes chunks 8 hh .. 8 hh + 7 into its
+// own words of the packed row (lane 0 stores the metadata).  Half the pairs
+// per thread: twice the rows resident.
 // ---------------------------------------------------------------------------
 __device__ __forceinline__ float pair_lo(uint64_t x) { return __uint_as_float((uint32_t)x); }
 __device__ __forceinline__ float pair_hi(uint64_t x) { return __uint_as_float((uint32_t)(x >> 32)); }
 
-template <int BITS, bool M16>
-__device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
-  const uint32_t* r32 = reinterpret_cast<const uint32_t*>(row_s);
-  uint64_t xp[64];
+__device__ __forceinline__ uint64_t shfl_xor_pair(unsigned mask, uint64_t x, int m) {
+  const uint32_t lo = __shfl_xor_sync(mask, (uint32_t)x, m), hi = __shfl_xor_sync(mask, (uint32_t)(x >> 32), m);
+  return ((uint64_t)hi << 32) | lo;
+}
+
+template <int BITS, bool M16, int SPLIT>
+__device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, unsigned pmask, uint32_t* codes,
+                                                     char* meta, size_t mi) {
+  constexpr int NP = 64 / SPLIT;  // pairs per thread
+  constexpr int NK = 16 / SPLIT;  // chunks per thread
+  const uint32_t* r32 = reinterpret_cast<const uint32_t*>(row_s) + NP * hh;
+  const int k0 = NK * hh;
+  uint64_t xp[NP];
 #pragma unroll
-  for (int m = 0; m < 64; ++m) {
+  for (int m = 0; m < NP; ++m) {
     const uint32_t w = r32[m];
     const float a = __uint_as_float(w << 16), b = __uint_as_float(w & 0xffff0000u);
     xp[m] = f32x2(__float_as_uint(__fadd_rn(a, b)), __float_as_uint(__fsub_rn(a, b)));  // stage h = 1
   }
 #pragma unroll
-  for (int hp = 1; hp < 64; hp <<= 1) {  // stage h = 2 hp
+  for (int hp = 1; hp < NP; hp <<= 1) {  // stage h = 2 hp
 #pragma unroll
-    for (int m = 0; m < 64; ++m) {
+    for (int m = 0; m < NP; ++m) {
       if (m & hp) continue;
       const uint64_t a = xp[m], b = xp[m + hp];
       xp[m] = f32x2_add(a, b);
       xp[m + hp] = f32x2_sub(a, b);
     }
   }
+  if (SPLIT == 2) {  // stage h = 64: pair m of lane 0 with pair m of lane 1
+#pragma unroll
+    for (int m = 0; m < NP; ++m) {
+      const uint64_t o = shfl_xor_pair(pmask, xp[m], 1);
+      xp[m] = hh ? f32x2_sub(o, xp[m]) : f32x2_add(xp[m], o);
+    }
+  }
   {
     const uint32_t cb = __float_as_uint(hadamard_c());
     const uint64_t c2 = f32x2(cb, cb);
 #pragma unroll
-    for (int m = 0; m < 64; ++m) xp[m] = f32x2_mul(xp[m], c2);
+    for (int m = 0; m < NP; ++m) xp[m] = f32x2_mul(xp[m], c2);
   }
   // min / max of the rotated vector (exact; signed zeros folded to +0)
   float mn = fminf(pair_lo(xp[0]), pair_hi(xp[0])), mx = fmaxf(pair_lo(xp[0]), pair_hi(xp[0]));
   {
     float mn1 = fminf(pair_lo(xp[1]), pair_hi(xp[1])), mx1 = fmaxf(pair_lo(xp[1]), pair_hi(xp[1]));
 #pragma unroll
-    for (int m = 2; m < 64; m += 2) {
+    for (int m = 2; m < NP; m += 2) {
       mn = fminf(mn, fminf(pair_lo(xp[m]), pair_hi(xp[m])));
       mx = fmaxf(mx, fmaxf(pair_lo(xp[m]), pair_hi(xp[m])));
       mn1 = fminf(mn1, fminf(pair_lo(xp[m + 1]), pair_hi(xp[m + 1])));
@@ -447,6 +468,10 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
     }
     mn = fminf(mn, mn1);
     mx = fmaxf(mx, mx1);
+  }
+  if (SPLIT == 2) {
+    mn = fminf(mn, __shfl_xor_sync(pmask, mn, 1));
+    mx = fmaxf(mx, __shfl_xor_sync(pmask, mx, 1));
   }
   mn = __fadd_rn(mn, 0.0f);
   mx = __fadd_rn(mx, 0.0f);
@@ -457,18 +482,18 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
     scale = half_sat(scale);
     mn = half_sat(mn);
   }
-  store_meta(meta, mi, scale, mn, M16);
-  constexpr int W = 4 * BITS;
+  if (hh == 0) store_meta(meta, mi, scale, mn, M16);
+  uint32_t prev = 0u, plane = 0u;
   if (scale == 0.0f) {
+    const uint32_t z8[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
 #pragma unroll
-    for (int i = 0; i < W; ++i) codes[i] = 0u;
+    for (int k = 0; k < NK; ++k) emit_chunk<BITS>(k0 + k, z8, codes, prev, plane);
     return;
   }
-  uint32_t prev = 0u, plane = 0u;
   if (M16) {  // as the min-max rows: the quotient clamped, then the same near-tie rule
     const float r = __frcp_rn(scale);
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < NK; ++k) {
       uint32_t c8[8];
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
@@ -479,7 +504,7 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
         const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
         c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
       }
-      emit_chunk<BITS>(k, c8, codes, prev, plane);
+      emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
     }
     return;
   }
@@ -490,35 +515,40 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, uint32_t
     const uint32_t cbits = __float_as_uint(192.50006103515625f);  // 192.5 + 4 * 2^-16
     const uint64_t c2 = f32x2(cbits, cbits);
 #pragma unroll
-    for (int k = 0; k < 16; ++k) {
+    for (int k = 0; k < NK; ++k) {
       const uint64_t x2[4] = {xp[4 * k], xp[4 * k + 1], xp[4 * k + 2], xp[4 * k + 3]};
       uint32_t a[8];
       if (chunk_T(x2, mn2, r2, c2, a)) {
-        emit_from_T<BITS>(k, a, codes, prev, plane);
+        emit_from_T<BITS>(k0 + k, a, codes, prev, plane);
       } else {
         uint32_t c8[8];
         chunk_near_tie<BITS>(a, [&](int i) { return (i & 1) ? pair_hi(x2[i >> 1]) : pair_lo(x2[i >> 1]); }, mn,
                              scale, c8);
-        emit_chunk<BITS>(k, c8, codes, prev, plane);
+        emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
       }
     }
     return;
   }
 #pragma unroll
-  for (int k = 0; k < 16; ++k) {  // tiny scale: the exact rule throughout
+  for (int k = 0; k < NK; ++k) {  // tiny scale: the exact rule throughout
     uint32_t c8[8];
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
       const uint64_t x2 = xp[4 * k + (i >> 1)];
       c8[i] = exact_code(__fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn), scale, levels);
     }
-    emit_chunk<BITS>(k, c8, codes, prev, plane);
+    emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
   }
 }
 
-__device__ __forceinline__ void copy_row(char* dst, const char* row_s) {
+// A BF16 row copied as it is (SPLIT = 2: lane hh of a pair copies its half).
+template <int SPLIT = 1>
+__device__ __forceinline__ void copy_row(char* dst, const char* row_s, int hh = 0) {
 #pragma unroll
-  for (int k = 0; k < 16; ++k) reinterpret_cast<uint4*>(dst)[k] = reinterpret_cast<const uint4*>(row_s)[k];
+  for (int k = 0; k < 16 / SPLIT; ++k) {
+    const int c = (16 / SPLIT) * hh + k;
+    reinterpret_cast<uint4*>(dst)[c] = reinterpret_cast<const uint4*>(row_s)[c];
+  }
 }
 
 // Staged rows of one warp tile: row r < n holds token t0 + r, 272-byte pitch.
@@ -562,11 +592,12 @@ struct TokenTiles {
     sp.n = min(kQTok, p.d.T - sp.t0);
     return sp;
   }
-  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int kv, const TileSpan& sp,
-                                                 const StagedRows& rows, const HeadGeom& hd) {
+  // Row r of the tile; SPLIT = 2: lane hh of the row's lane pair (pmask).
+  template <int SPLIT>
+  static __device__ __forceinline__ void row(const QuantizeParams& p, int li, int b, int kv, const TileSpan& sp,
+                                             const StagedRows& rows, const HeadGeom& hd, int r, int hh,
+                                             unsigned pmask) {
     const Dims& d = p.d;
-    const int r = threadIdx.x;
-    if (r >= sp.n) return;
     char* Lb = p.arena + p.lt.base[li];
     const int t = sp.t0 + r;
     const bool coded = t >= d.s && t < d.s + d.nq;
@@ -588,21 +619,36 @@ struct TokenTiles {
     if (kv == 0) {
       if (coded && hd.cls == kQuantized && !sal) {
         uint32_t* crow = reinterpret_cast<uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W;
-        if (BASE == kAkvq) quantize_row_rotated<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
-        else quantize_row_token<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
+        if (BASE == kAkvq)
+          quantize_row_rotated<BITS, M16, SPLIT>(row_s, hh, pmask, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
+        else if constexpr (SPLIT == 1)
+          quantize_row_token<BITS, M16>(row_s, crow, Lb + hd.kqm + b * hd.kqm_bs, ci);
         return;
       }
       char* dst = (coded && hd.cls == kKeysOnly && !sal) ? Lb + hd.kimg + b * hd.kimg_bs + (size_t)ci * 256
                                                          : Lb + hd.kb + b * hd.kb_bs + (size_t)pos * 256;
-      copy_row(dst, row_s);
-    } else {
+      copy_row<SPLIT>(dst, row_s, hh);
+    } else if constexpr (SPLIT == 1) {
       if (coded && hd.cls != kProtected && !sal) {
         quantize_row_token<BITS, M16>(row_s, reinterpret_cast<uint32_t*>(Lb + hd.vq + b * hd.vq_bs) + (size_t)ci * W,
                                       Lb + hd.vqm + b * hd.vqm_bs, ci);
         return;
       }
-      copy_row(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256, row_s);
+      copy_row<1>(Lb + hd.vb + b * hd.kb_bs + (size_t)pos * 256, row_s, 0);
     }
+  }
+  static __device__ __forceinline__ void process(const QuantizeParams& p, int li, int b, int kv, const TileSpan& sp,
+                                                 const StagedRows& rows, const HeadGeom& hd) {
+    if (BASE == kAkvq && PARTS == 1) {
+      // rotated key rows: two lanes per row, rows lane / 2 and 16 + lane / 2
+      // (both lanes of a pair take the same path, so the pair's shuffles meet)
+      const int hh = threadIdx.x & 1;
+      const unsigned pmask = 3u << (threadIdx.x & 30);
+#pragma unroll 1
+      for (int r = threadIdx.x >> 1; r < sp.n; r += 16) row<2>(p, li, b, kv, sp, rows, hd, r, hh, pmask);
+      return;
+    }
+    if ((int)threadIdx.x < sp.n) row<1>(p, li, b, kv, sp, rows, hd, threadIdx.x, 0, 0u);
   }
 };
 
