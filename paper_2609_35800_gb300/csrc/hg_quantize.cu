@@ -900,6 +900,64 @@ __device__ __forceinline__ uint32_t kivi_code(const uint32_t* row, int bits, int
   return (__ldg(row + e / per) >> (bits * (e % per))) & ((1u << bits) - 1u);
 }
 
+// Codes of token e of eight consecutive KIVI-style key rows (channels
+// 8j..8j+7: BITS words each, contiguous): at 2 and 3 bits the 16 or 24 words
+// arrive as 16-byte loads and each channel's word is selected in registers;
+// at 4 bits the one word a channel needs is loaded alone.
+template <int BITS>
+__device__ __forceinline__ void kivi_codes8(const uint32_t* rows, int e, uint32_t (&code)[8]) {
+  if (BITS == 4) {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) code[i] = kivi_code(rows + i * BITS, BITS, e);
+    return;
+  }
+  uint32_t w[8 * BITS];
+#pragma unroll
+  for (int v = 0; v < 2 * BITS; ++v) {
+    const uint4 x = ldg16(rows + 4 * v);
+    w[4 * v] = x.x;
+    w[4 * v + 1] = x.y;
+    w[4 * v + 2] = x.z;
+    w[4 * v + 3] = x.w;
+  }
+  const bool hi = e >= 16;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const uint32_t lo = ((hi ? w[i * BITS + 1] : w[i * BITS]) >> (2 * (e & 15))) & 3u;
+    if (BITS == 3) {
+      const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
+      code[i] = lo | (((w[i * BITS + 2] >> pp) & 1u) << 2);
+    } else {
+      code[i] = lo;
+    }
+  }
+}
+
+// Metadata pairs of eight consecutive KIVI-style key rows from index i0 (a
+// multiple of 8, so 64 or 32 contiguous bytes on a 16-byte boundary).
+template <bool M16>
+__device__ __forceinline__ void kivi_meta8(const char* base, size_t i0, float2 (&m)[8]) {
+  if (M16) {
+    const uint4* p = reinterpret_cast<const uint4*>(base + i0 * 4);
+#pragma unroll
+    for (int v = 0; v < 2; ++v) {
+      const uint4 x = __ldg(p + v);
+      m[4 * v] = half2_bits_to_float2(x.x);
+      m[4 * v + 1] = half2_bits_to_float2(x.y);
+      m[4 * v + 2] = half2_bits_to_float2(x.z);
+      m[4 * v + 3] = half2_bits_to_float2(x.w);
+    }
+  } else {
+    const float4* p = reinterpret_cast<const float4*>(base + i0 * 8);
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const float4 x = __ldg(p + v);
+      m[2 * v] = make_float2(x.x, x.y);
+      m[2 * v + 1] = make_float2(x.z, x.w);
+    }
+  }
+}
+
 // Normalised Hadamard-128 of a vector spread over a half-warp, lane j holding
 // channels 8j..8j+7: stages h = 1, 2, 4 in the lane, h = 8..64 with lane
 // j ^ (h / 8); butterflies (a, b) -> (a + b, a - b), one multiply at the end.
@@ -991,12 +1049,8 @@ __global__ void __launch_bounds__(kDqThreads, 6) dequantize_kernel(const __grid_
             const int grp = ti / kKiviGroup, e = ti % kKiviGroup;
             const uint32_t* codes = reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) +
                                     ((size_t)grp * kD + 8 * j) * BITS;
-            const char* meta = Lb + hd.kqm + b * hd.kqm_bs;
-#pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              code[i] = kivi_code(codes + i * BITS, BITS, e);
-              m[i] = load_meta(meta, (size_t)grp * kD + 8 * j + i, M16);
-            }
+            kivi_codes8<BITS>(codes, e, code);
+            kivi_meta8<M16>(Lb + hd.kqm + b * hd.kqm_bs, (size_t)grp * kD + 8 * j, m);
           } else {
             row_codes8(reinterpret_cast<const uint32_t*>(Lb + hd.kq + b * hd.kq_bs) + (size_t)ci * W, BITS, j,
                        code);
