@@ -492,9 +492,9 @@ def run_gpu(args):
     sigma = 0.0
     quant_b, dec_b, app_b = geometry_bytes(runner)
     step_bytes = quant_b + sum(dec_b) + S * app_b
-    # quantize: per 64 layers one launch (two for the AKVQ-style base: keys, values),
-    # preceded by the salient-token selection when on
-    q_launches = (L + 63) // 64 * ((2 if w.base == wl.BASE_AKVQ else 1)
+    # quantize: per 64 layers one launch (two for the AKVQ- and KIVI-style bases:
+    # keys, values), preceded by the salient-token selection when on
+    q_launches = (L + 63) // 64 * ((2 if w.base in (wl.BASE_AKVQ, wl.BASE_KIVI) else 1)
                                    + (1 if (w.salient_permille > 0 and w.image > 0) else 0))
     launches_per_step = q_launches + S * ((L + 63) // 64)
 

@@ -663,14 +663,14 @@ struct TokenTiles {
 // the BF16 residual window and a trailing partial group, protected heads,
 // keys of keys-only heads) is copied.
 // ---------------------------------------------------------------------------
-template <int BITS, bool M16>
+template <int BITS, bool M16, int PARTS>
 struct KiviTiles {
-  static constexpr int kNParts = 2;
+  static constexpr int kNParts = PARTS == 3 ? 2 : 1;
   // tile x: [origin - 32 + 32 x, + 32) clipped to [0, T), origin = s mod 32
   static __device__ __forceinline__ int count(const QuantizeParams& p) {
     return (p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
   }
-  static __device__ __forceinline__ int part(int i) { return i; }
+  static __device__ __forceinline__ int part(int i) { return PARTS == 3 ? i : (PARTS == 1 ? 0 : 1); }
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
     sp.tlo = p.tile_origin - kKiviGroup + kQTok * tx;
@@ -906,29 +906,29 @@ __device__ __forceinline__ uint32_t kivi_code(const uint32_t* row, int bits, int
 // at 4 bits the one word a channel needs is loaded alone.
 template <int BITS>
 __device__ __forceinline__ void kivi_codes8(const uint32_t* rows, int e, uint32_t (&code)[8]) {
-  if (BITS == 4) {
+  if constexpr (BITS == 4) {
 #pragma unroll
     for (int i = 0; i < 8; ++i) code[i] = kivi_code(rows + i * BITS, BITS, e);
-    return;
-  }
-  uint32_t w[8 * BITS];
+  } else {
+    uint32_t w[8 * BITS];
 #pragma unroll
-  for (int v = 0; v < 2 * BITS; ++v) {
-    const uint4 x = ldg16(rows + 4 * v);
-    w[4 * v] = x.x;
-    w[4 * v + 1] = x.y;
-    w[4 * v + 2] = x.z;
-    w[4 * v + 3] = x.w;
-  }
-  const bool hi = e >= 16;
+    for (int v = 0; v < 2 * BITS; ++v) {
+      const uint4 x = ldg16(rows + 4 * v);
+      w[4 * v] = x.x;
+      w[4 * v + 1] = x.y;
+      w[4 * v + 2] = x.z;
+      w[4 * v + 3] = x.w;
+    }
+    const bool hi = e >= 16;
 #pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const uint32_t lo = ((hi ? w[i * BITS + 1] : w[i * BITS]) >> (2 * (e & 15))) & 3u;
-    if (BITS == 3) {
-      const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
-      code[i] = lo | (((w[i * BITS + 2] >> pp) & 1u) << 2);
-    } else {
-      code[i] = lo;
+    for (int i = 0; i < 8; ++i) {
+      const uint32_t lo = ((hi ? w[i * BITS + 1] : w[i * BITS]) >> (2 * (e & 15))) & 3u;
+      if (BITS == 3) {
+        const int pp = (e & 7) | (((e >> 4) & 1) << 3) | (((e >> 3) & 1) << 4);
+        code[i] = lo | (((w[i * BITS + 2] >> pp) & 1u) << 2);
+      } else {
+        code[i] = lo;
+      }
     }
   }
 }
@@ -1133,7 +1133,11 @@ cudaError_t launch_quantize_bits(const QuantizeParams& p, cudaStream_t s) {
   const Dims& d = p.d;
   if (d.base == kKivi) {
     const int tx = (d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
-    return launch_tiles<KiviTiles<BITS, M16>>(p, tx, s);
+    // keys and values in launches of their own: each kernel holds one of the
+    // two code paths, so the warps of an SM share less instruction cache
+    const cudaError_t e = launch_tiles<KiviTiles<BITS, M16, 1>>(p, tx, s);
+    if (e != cudaSuccess) return e;
+    return launch_tiles<KiviTiles<BITS, M16, 2>>(p, tx, s);
   }
   const int tx = (d.T + kQTok - 1) / kQTok;
   if (d.base == kAkvq) {
