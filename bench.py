@@ -350,8 +350,9 @@ def oracle_sample(w, n_layers, n_steps, parts=None):
 
 
 def cpu_baseline_fields(w, n_layers, n_steps, parts):
-    """The oracle's quantize GB/s and decode tokens/s from one timed sample
-    (decode tokens/s scaled to all layers when the sample holds fewer)."""
+    """The oracle's quantize GB/s and decode tokens/s from timed samples
+    holding n_steps decode steps in all (decode tokens/s scaled to all layers
+    when the sample holds fewer)."""
     dec_tok = w.batch * n_steps / parts["dec_s"] * (n_layers / w.layers) if parts["dec_s"] > 0 else None
     return {"quantize_GBps": round(parts["quant_bytes"] / parts["quant_s"] / 1e9, 4),
             "decode_GBps": round(parts["dec_bytes"] / parts["dec_s"] / 1e9, 4),
@@ -380,11 +381,30 @@ def _decode_bytes_layer(w, mask_row, nq, appended, ns=0):
 
 
 def cpu_sample_plan(w):
-    """Bounded sample sizes: about 10-30 s of oracle work."""
+    """One sample of the oracle: the whole workload step (every layer's
+    quantization, then every decode step) on the small caches; the first layer
+    and two decode steps on the large ones."""
     per_layer_tokens = w.batch * w.kv_heads * w.seq_len
     if per_layer_tokens <= 10000:
-        return min(w.layers, 28), min(w.decode_steps, 8)
+        return w.layers, w.decode_steps
     return 1, 2
+
+
+def timed_oracle_samples(w, n_layers, n_steps, min_seconds=10.0, max_reps=50):
+    """Repeat the oracle sample until at least min_seconds of timed oracle
+    calls have accumulated (a bounded CPU baseline).  Returns (bytes, seconds,
+    threads, repetitions, parts) summed over the repetitions."""
+    tot_b, tot_s, reps, threads = 0, 0.0, 0, 1
+    parts = {"quant_bytes": 0, "quant_s": 0.0, "dec_bytes": 0, "dec_s": 0.0}
+    while reps < max_reps and (reps == 0 or tot_s < min_seconds):
+        one = {}
+        nb, secs, threads = oracle_sample(w, n_layers, n_steps, one)
+        tot_b += nb
+        tot_s += secs
+        reps += 1
+        for k in parts:
+            parts[k] += one[k]
+    return tot_b, tot_s, threads, reps, parts
 
 
 def _workload(args):
@@ -612,13 +632,13 @@ def run_gpu(args):
         line["e2e"] = e2e
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         n_layers, n_steps = cpu_sample_plan(w)
-        parts = {}
-        nb, secs, threads = oracle_sample(w, n_layers, n_steps, parts)
+        nb, secs, threads, reps, parts = timed_oracle_samples(w, n_layers, n_steps)
         line["cpu_baseline"] = dict({
             "value": round(nb / secs / 1e9, 4), "unit": "GB/s", "cores": threads, "kind": "oracle",
-            "sample": "%s: oracle quantize of %d layer(s) then %d decode step(s) of fp64 attention "
-                      "over them; timed oracle calls only" % (w.name, n_layers, n_steps)},
-            **cpu_baseline_fields(w, n_layers, n_steps, parts))
+            "sample": "%s: %d repetition(s) of oracle quantize of %d layer(s) then %d decode step(s) of "
+                      "fp64 attention over them, %.1f s of timed oracle calls" % (w.name, reps, n_layers,
+                                                                                   n_steps, secs)},
+            **cpu_baseline_fields(w, n_layers, n_steps * reps, parts))
     if rank == 0:
         print(json.dumps(line))
     if dist is not None:
