@@ -291,8 +291,9 @@ constexpr int kChunksPerUnit = BITS == 4 ? 1 : (BITS == 2 ? 2 : 4);
 // min / max over bf16x2 pairs (exact), signed zeros folded to +0,
 // scale = fl((max - min) / levels), metadata stored at index mi (binary16
 // pair with M16: codes against the rounded pair), codes 0 when scale == 0,
-// each chunk's codes emitted into the packed row.  The chunk loop stays rolled
-// (by two) so that the code is small and stays in the instruction cache.
+// each chunk's codes emitted into the packed row.  The chunk loop is unrolled
+// by four only (a KIVI-style value group whole; eight measured slower on the
+// per-token rows), so that the code stays small in the instruction cache.
 // A chunk with an element near a tie (fast rule) is emitted with its fast
 // codes and flagged; after the loop each thread codes the store units of its
 // flagged chunks again, the flagged elements by the exact rule, and stores
@@ -336,7 +337,7 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
   const uint32_t cbits = __float_as_uint(192.50006103515625f);  // C = 192.5 + 4 * 2^-16
   const uint64_t c2 = f32x2(cbits, cbits);
   uint32_t ties = 0u;  // bit k - k0: chunk k has an element near a tie
-#pragma unroll 2
+#pragma unroll 4
   for (int k = k0; k < k0 + nk; ++k) {
     const uint4 v = r4[k];
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
