@@ -1014,14 +1014,13 @@ __global__ void __launch_bounds__(kDqThreads, 6) dequantize_kernel(const __grid_
 
 #pragma unroll 1
   for (int x = blockIdx.x * span; x < x1; ++x) {
-    // unit u: K (u < 16 * kDqTile) or V, token (u >> 4) % kDqTile of the
-    // tile; unrolled so that the loads of a thread's four units are in flight
-    // together
+    // a thread's two tokens (rows 16 apart), each with its K and V unit: the
+    // token's coded slot and BF16 position found once for both
+    int tk[2], ck[2], pk[2];
+    bool codedk[2], salk[2];
 #pragma unroll
-    for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
-      const bool is_k = u < kDqTile * 16;
-      const int t = x * kDqTile + ((u >> 4) & (kDqTile - 1));
-      if (t >= Tt) continue;  // uniform over the half-warp
+    for (int r = 0; r < 2; ++r) {
+      const int t = x * kDqTile + ((threadIdx.x >> 4) + 16 * r);
       const bool coded = (t >= qs) && (t < qe);
       const int ti = t - qs;
       int ci = ti, spos = 0;  // coded slot; BF16 position of a salient token (Sec. 4)
@@ -1036,7 +1035,23 @@ __global__ void __launch_bounds__(kDqThreads, 6) dequantize_kernel(const __grid_
         ci = ti - rank;
         spos = qs + rank;
       }
-      const int pos = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
+      tk[r] = t;
+      ck[r] = ci;
+      codedk[r] = coded;
+      salk[r] = sal;
+      pk[r] = (t >= d.T) ? hd.bf16_prefill + (t - d.T) : (sal ? spos : bf16_pos(d, hd.cls, t));
+    }
+    // unit u: K (u < 16 * kDqTile) or V, token (u >> 4) % kDqTile of the
+    // tile; unrolled so that the loads of a thread's four units are in flight
+    // together
+#pragma unroll
+    for (int u = threadIdx.x; u < 2 * kDqTile * 16; u += kDqThreads) {
+      const bool is_k = u < kDqTile * 16;
+      const int r = ((u - threadIdx.x) / kDqThreads) & 1;  // the thread's token of this unit
+      const int t = tk[r];
+      if (t >= Tt) continue;  // uniform over the half-warp
+      const bool coded = codedk[r], sal = salk[r];
+      const int ti = t - qs, ci = ck[r], pos = pk[r];
       const size_t o = (out_row0 + t) * kD + 8 * j;
       void* dst = is_k ? p.k_out : p.v_out;
       float x8[8];
