@@ -171,19 +171,30 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
   float mn[2] = {__fadd_rn(__low2float(mn2), 0.0f), __fadd_rn(__high2float(mn2), 0.0f)};
   const float mx[2] = {__fadd_rn(__low2float(mx2), 0.0f), __fadd_rn(__high2float(mx2), 0.0f)};
   float sc[2];
+  bool fast = true;  // both channels: the fast rule applies (see quantize_row_group)
 #pragma unroll
   for (int j = 0; j < 2; ++j) {
     sc[j] = __fdiv_rn(__fsub_rn(mx[j], mn[j]), levels);
+    const float mn_x = mn[j];
     if (M16) {
       sc[j] = half_sat(sc[j]);
       mn[j] = half_sat(mn[j]);
+      if (sc[j] > 0.0f) {
+        const float rj = __frcp_rn(sc[j]);
+        const float qlo = __fmul_rn(__fsub_rn(mn_x, mn[j]), rj), qhi = __fmul_rn(__fsub_rn(mx[j], mn[j]), rj);
+        fast = fast && qlo > -0.25f && qhi < levels + 0.25f;
+      } else {
+        fast = false;
+      }
+    } else {
+      fast = fast && sc[j] >= 2.3509887e-38f;
     }
     store_meta(meta, mi + j, sc[j], mn[j], M16);
   }
   uint32_t wd0[BITS], wd1[BITS];  // the two channels' packed words, filled code by code
 #pragma unroll
   for (int i = 0; i < BITS; ++i) wd0[i] = wd1[i] = 0u;
-  if (!M16 && sc[0] >= 2.3509887e-38f && sc[1] >= 2.3509887e-38f) {
+  if (fast) {
     const float r0 = __frcp_rn(sc[0]), r1 = __frcp_rn(sc[1]);
     const uint64_t mn2p = f32x2(__float_as_uint(mn[0]), __float_as_uint(mn[1]));
     const uint64_t r2 = f32x2(__float_as_uint(r0), __float_as_uint(r1));
@@ -325,13 +336,23 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
   mx = __fadd_rn(mx, 0.0f);
   const float levels = (float)((1u << BITS) - 1u);
   float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  const float mn_x = mn;  // the group's own minimum
   if (M16) {  // binary16 metadata: codes against the stored pair
     scale = half_sat(scale);
     mn = half_sat(mn);
   }
   store_meta(meta, mi, scale, mn, M16);
-  const bool fast = !M16 && scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
+  bool fast = !M16 && scale >= 2.3509887e-38f;  // 2^-125: 1 / scale is finite
   const float r = (M16 || fast) ? __frcp_rn(scale) : 1.0f;
+  if (M16 && scale > 0.0f) {
+    // With the rounded pair the quotients fl(fl(x - min16) r) of the group run
+    // monotonically from the group minimum's to the maximum's.  When both lie
+    // well inside (-1/2, levels + 1/2), every code is in [0, levels] without a
+    // clamp, and the fast rule of the fp32 pairs (exact against the IEEE
+    // quotient, with the same near-tie window) applies to the stored pair.
+    const float qlo = __fmul_rn(__fsub_rn(mn_x, mn), r), qhi = __fmul_rn(__fsub_rn(mx, mn), r);
+    fast = qlo > -0.25f && qhi < levels + 0.25f;
+  }
   const uint64_t mnp = f32x2(__float_as_uint(mn), __float_as_uint(mn));
   const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
   const uint32_t cbits = __float_as_uint(192.50006103515625f);  // C = 192.5 + 4 * 2^-16
@@ -479,6 +500,7 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
   constexpr uint32_t L = (1u << BITS) - 1u;
   const float levels = (float)L;
   float scale = __fdiv_rn(__fsub_rn(mx, mn), levels);
+  const float mn_x = mn;
   if (M16) {
     scale = half_sat(scale);
     mn = half_sat(mn);
@@ -491,7 +513,13 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
     for (int k = 0; k < NK; ++k) emit_chunk<BITS>(k0 + k, z8, codes, prev, plane);
     return;
   }
-  if (M16) {  // as the min-max rows: the quotient clamped, then the same near-tie rule
+  bool fast = scale >= 2.3509887e-38f;  // the fast rule of the min-max rows (chunk_T)
+  if (M16) {  // with the stored pair: when every quotient is well inside the levels (quantize_row_group)
+    const float r = __frcp_rn(scale);
+    const float qlo = __fmul_rn(__fsub_rn(mn_x, mn), r), qhi = __fmul_rn(__fsub_rn(mx, mn), r);
+    fast = qlo > -0.25f && qhi < levels + 0.25f;
+  }
+  if (M16 && !fast) {  // as the min-max rows: the quotient clamped, then the same near-tie rule
     const float r = __frcp_rn(scale);
 #pragma unroll
     for (int k = 0; k < NK; ++k) {
@@ -509,7 +537,7 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
     }
     return;
   }
-  if (scale >= 2.3509887e-38f) {  // the fast rule of the min-max rows (chunk_T)
+  if (fast) {  // the fast rule of the min-max rows (chunk_T)
     const float r = __frcp_rn(scale);
     const uint64_t mn2 = f32x2(__float_as_uint(mn), __float_as_uint(mn));
     const uint64_t r2 = f32x2(__float_as_uint(r), __float_as_uint(r));
