@@ -360,16 +360,18 @@ def test_minmax_quantize_exact_ties(bits, meta_bits):
                                              (K, 4, -0.3125, 7.5), (A, 4, -1.0, 1.375), (A, 2, -1.0, 5.25)],
                          ids=["minmax2", "minmax2n", "minmax3", "minmax3n", "minmax4", "minmax4n", "kivi2",
                               "kivi2n", "kivi3n", "kivi4n", "akvq4", "akvq2n"])
-def test_quantize_near_ties(base, bits, lo, hi):
+@pytest.mark.parametrize("meta_bits", [64, 32])
+def test_quantize_near_ties(base, bits, lo, hi, meta_bits):
     """Every group (per-token rows, 32-channel value groups, 32-token key
     groups) holds the same minimum lo and maximum hi, and the other entries
     are the BF16 roundings of lo + (g + 1/2) * scale, scale = (hi - lo) /
     levels not a power of two: a few per cent of the elements land within
     2^-13 of a half-integer quotient, some of them exactly on it, which the
     kernel decides without a division and the oracle by the IEEE quotient.
+    With binary16 metadata the codes are taken against the rounded pair.
     Arena bits must equal the oracle's."""
     w = wl.custom("near%d" % bits, 1, 2, 8, 4, 7, 160, 9, base, bits, 0, decode_steps=1, seed=4,
-                  protected=[(0, 1)], residual=32)
+                  protected=[(0, 1)], residual=32, meta_bits=meta_bits)
     runner = CacheRunner(w)
     B, H, T = w.batch, w.kv_heads, w.seq_len
     gen = torch.Generator().manual_seed(23 + bits)
