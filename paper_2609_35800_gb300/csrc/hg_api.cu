@@ -69,9 +69,6 @@ hg_status validate(const hg_shape* sh, const hg_quant_config* c, const uint8_t* 
   const int64_t tok = (int64_t)sh->seq_len + sh->max_new_tokens;
   if (tok > (1 << 28)) return HG_ERR_UNSUPPORTED;
   if ((int64_t)sh->batch * sh->num_kv_heads > 65535) return HG_ERR_UNSUPPORTED;  // grid.y
-  // the quantizer's one-dimensional grid: 64-token tiles x rows x heads x 64 layers
-  if ((((int64_t)sh->seq_len + 32 + 63) / 64) * sh->batch * sh->num_kv_heads * kMaxLayersPerLaunch > INT32_MAX)
-    return HG_ERR_UNSUPPORTED;
 
   d->B = sh->batch;
   d->L = sh->num_layers;

@@ -595,10 +595,12 @@ __device__ __forceinline__ void stage_rows(const QuantizeParams& p, int li, int 
                                            StagedRows& rows) {
   const Dims& d = p.d;
   const size_t row0 = ((size_t)b * d.H + h) * (size_t)d.T + sp.t0;
-  const char* src = reinterpret_cast<const char*>((kv ? p.v[li] : p.k[li]) + row0 * kD);
-  for (int c = threadIdx.x; c < sp.n * 16; c += 32) {
-    const int r = c >> 4, col = c & 15;
-    cp_async16(smem_u32(&rows[r][col * 16]), src + (size_t)r * 256 + col * 16, 16);
+  const int col = threadIdx.x & 15;  // lane l: chunk l % 16 of rows l / 16, l / 16 + 2, ...
+  const char* src = reinterpret_cast<const char*>((kv ? p.v[li] : p.k[li]) + row0 * kD) + col * 16;
+#pragma unroll
+  for (int i = 0; i < kQTok / 2; ++i) {
+    const int r = (threadIdx.x >> 4) + 2 * i;
+    if (r < sp.n) cp_async16(smem_u32(&rows[r][col * 16]), src + (size_t)r * 256, 16);
   }
 }
 
@@ -749,8 +751,8 @@ struct KiviTiles {
   }
 };
 
-// The quantizer kernel: one CTA of one warp per (tile, part), numbered
-// (part, tile, batch row x KV head, layer) with the part fastest.  A warp
+// The quantizer kernel: one CTA of one warp per (tile, part); grid x = tile
+// x part (part fastest), y = batch row x KV head, z = layer.  A warp
 // stages its 32 rows, waits for its own copies and codes them; no CTA-wide
 // barrier, so the warps of an SM (23 resident) run out of step and one
 // warp's loads overlap another's coding.
@@ -758,12 +760,8 @@ template <class TP>
 __global__ void __launch_bounds__(32) quantize_tiles_kernel(const __grid_constant__ QuantizeParams p) {
   __shared__ __align__(16) StagedRows rows;
   __shared__ HeadGeom s_hd;
-  const int nx = TP::count(p), nbh = p.d.B * p.d.H;
-  const int i = blockIdx.x;
-  const int pi = i % TP::kNParts, rest = i / TP::kNParts;
-  const int tx = rest % nx, rest2 = rest / nx, bh = rest2 % nbh, li = rest2 / nbh;
-  if (li >= p.n_layers) return;
-  const int b = bh / p.d.H, h = bh % p.d.H;
+  const int pi = blockIdx.x % TP::kNParts, tx = blockIdx.x / TP::kNParts;
+  const int li = blockIdx.z, b = blockIdx.y / p.d.H, h = blockIdx.y % p.d.H;
   const int kv = TP::part(pi);
   const TileSpan sp = TP::span(p, tx);
   if (sp.n <= 0) return;
@@ -1167,8 +1165,8 @@ __global__ void __launch_bounds__(64) append_kernel(const __grid_constant__ Appe
 // Launch of the quantizer kernel over every tile of the launch's layers.
 template <class TP>
 cudaError_t launch_tiles(const QuantizeParams& p, int tiles_x, cudaStream_t s) {
-  const long long total = (long long)tiles_x * TP::kNParts * p.d.B * p.d.H * p.n_layers;
-  quantize_tiles_kernel<TP><<<(unsigned)total, 32, 0, s>>>(p);
+  const dim3 grid((unsigned)(tiles_x * TP::kNParts), (unsigned)(p.d.B * p.d.H), (unsigned)p.n_layers);
+  quantize_tiles_kernel<TP><<<grid, 32, 0, s>>>(p);
   return cudaGetLastError();
 }
 

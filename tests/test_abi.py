@@ -78,7 +78,6 @@ def _status(f, *a):
     (dict(img_len=-1), {}, 1),
     (dict(seq_len=1 << 28, img_start=0), {}, 3),          # token index range
     (dict(batch=20000), {}, 3),                            # batch x KV heads > grid.y
-    (dict(batch=4096, seq_len=1 << 20, img_start=0, img_len=0), {}, 3),  # quantizer tiles > 2^31
     ({}, dict(base=1, kivi_group_channels=16), 3),
     (dict(seq_len=60100, img_start=50, img_len=60000), dict(base=2, salient_permille=20), 3),
 ])
