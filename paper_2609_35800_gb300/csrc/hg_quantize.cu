@@ -801,16 +801,29 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
   __shared__ int red_i[kSalThreads / 32];
 
   const uint16_t* K = p.k[li] + (((size_t)b * d.H + h) * d.T + d.s) * kD;
-  for (int i = warp; i < nq; i += kSalThreads / 32) {
-    float x[4];
-    bf16x4_to_f32(ldg8(K + (size_t)i * kD + lane * 4), x);
-    float a = __fmul_rn(x[0], x[0]);
-    a = __fadd_rn(a, __fmul_rn(x[1], x[1]));
-    a = __fadd_rn(a, __fmul_rn(x[2], x[2]));
-    a = __fadd_rn(a, __fmul_rn(x[3], x[3]));
+  // four rows per warp in flight: their loads first, then each row's sum in
+  // the same order as one row at a time
+  constexpr int kRows = 4, kWarps = kSalThreads / 32;
+  for (int i0 = warp; i0 < nq; i0 += kRows * kWarps) {
+    uint2 w[kRows];
 #pragma unroll
-    for (int m = 16; m >= 1; m >>= 1) a = __fadd_rn(a, __shfl_xor_sync(kFull, a, m));
-    if (lane == 0) score[i] = a;
+    for (int u = 0; u < kRows; ++u) {
+      const int i = i0 + u * kWarps;
+      w[u] = (i < nq) ? ldg8(K + (size_t)i * kD + lane * 4) : make_uint2(0u, 0u);
+    }
+#pragma unroll
+    for (int u = 0; u < kRows; ++u) {
+      const int i = i0 + u * kWarps;
+      float x[4];
+      bf16x4_to_f32(w[u], x);
+      float a = __fmul_rn(x[0], x[0]);
+      a = __fadd_rn(a, __fmul_rn(x[1], x[1]));
+      a = __fadd_rn(a, __fmul_rn(x[2], x[2]));
+      a = __fadd_rn(a, __fmul_rn(x[3], x[3]));
+#pragma unroll
+      for (int m = 16; m >= 1; m >>= 1) a = __fadd_rn(a, __shfl_xor_sync(kFull, a, m));
+      if (lane == 0 && i < nq) score[i] = a;
+    }
   }
   for (int w = tid; w < nblk; w += kSalThreads) bits[w] = 0u;
   __syncthreads();
