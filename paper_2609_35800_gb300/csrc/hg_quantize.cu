@@ -797,8 +797,6 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
   extern __shared__ __align__(16) float sal_smem[];
   float* score = sal_smem;                                     // [nq]
   uint32_t* bits = reinterpret_cast<uint32_t*>(sal_smem + nq);  // [nblk]
-  __shared__ float red_v[kSalThreads / 32];
-  __shared__ int red_i[kSalThreads / 32];
 
   const uint16_t* K = p.k[li] + (((size_t)b * d.H + h) * d.T + d.s) * kD;
   // four rows per warp in flight: their loads first, then each row's sum in
@@ -825,48 +823,97 @@ __global__ void __launch_bounds__(kSalThreads) salient_kernel(const __grid_const
       if (lane == 0 && i < nq) score[i] = a;
     }
   }
-  for (int w = tid; w < nblk; w += kSalThreads) bits[w] = 0u;
   __syncthreads();
 
+  // The ns largest scores, ties to the lower index -- the set that ns rounds
+  // of arg-max (taken tokens dropping out) would pick -- by a radix select on
+  // the scores' bit patterns (non-negative floats order as their bits): four
+  // 8-bit digits from the top, each pass a histogram of the candidates that
+  // match the digits chosen so far and the digit where the count of larger
+  // keys reaches ns.  Then every key above the final threshold T is taken,
+  // and of the keys equal to T the first `need` by index.
+  static_assert(kSalThreads == 256, "one histogram bin per thread");
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t s_prefix, s_need, s_eq;
+  uint32_t prefix = 0u, pmask = 0u, need = (uint32_t)d.ns;
 #pragma unroll 1
-  for (int r = 0; r < d.ns; ++r) {
-    // a thread scans increasing indices, so a strict > keeps the lower index
-    float bv = -INFINITY;
-    int bi = INT_MAX;
-    for (int i = tid; i < nq; i += kSalThreads) {
-      const float v = score[i];
-      if (v > bv) {
-        bv = v;
-        bi = i;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    hist[tid] = 0u;  // kSalThreads == 256 bins
+    __syncthreads();
+    for (int i0 = warp * 32; i0 < nq; i0 += kSalThreads) {  // warp-uniform: lane i0 + lane
+      const int i = i0 + lane;
+      const uint32_t key = i < nq ? __float_as_uint(score[i]) : 0u;
+      const bool cand = i < nq && (key & pmask) == prefix;
+      const uint32_t dg = (key >> shift) & 255u;
+      // one atomic per distinct digit of the warp's candidates
+      const uint32_t act = __ballot_sync(kFull, cand);
+      if (cand) {
+        const uint32_t same = __match_any_sync(act, dg);
+        if ((__ffs(same) - 1) == lane) atomicAdd(&hist[dg], (uint32_t)__popc(same));
       }
     }
+    __syncthreads();
+    if (warp == 0) {
+      // lane l holds bins 255 - 8l .. 248 - 8l (largest digits first)
+      uint32_t c[8], tot = 0u;
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float ov = __shfl_xor_sync(kFull, bv, o);
-      const int oi = __shfl_xor_sync(kFull, bi, o);
-      if (ov > bv || (ov == bv && oi < bi)) {
-        bv = ov;
-        bi = oi;
+      for (int j = 0; j < 8; ++j) {
+        c[j] = hist[255 - 8 * lane - j];
+        tot += c[j];
       }
-    }
-    if (lane == 0) {
-      red_v[warp] = bv;
-      red_i[warp] = bi;
-    }
-    __syncthreads();
-    if (tid == 0) {
-      for (int w = 1; w < kSalThreads / 32; ++w)
-        if (red_v[w] > bv || (red_v[w] == bv && red_i[w] < bi)) {
-          bv = red_v[w];
-          bi = red_i[w];
+      uint32_t incl = tot;  // keys in this lane's bins and all larger digits
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t v = __shfl_up_sync(kFull, incl, o);
+        if (lane >= o) incl += v;
+      }
+      const uint32_t excl = incl - tot;
+      if (excl < need && need <= incl) {  // exactly one lane
+        uint32_t above = excl;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (above + c[j] >= need) {
+            const uint32_t dg = 255u - 8u * lane - j;
+            s_prefix = prefix | (dg << shift);
+            s_need = need - above;
+            s_eq = c[j];
+            break;
+          }
+          above += c[j];
         }
-      if (bi < nq) {  // taken tokens drop out of later rounds
-        score[bi] = -INFINITY;
-        bits[bi >> 5] |= 1u << (bi & 31);
       }
     }
     __syncthreads();
+    prefix = s_prefix;
+    need = s_need;
+    pmask |= 255u << shift;
   }
+  // T = prefix: `need` of the s_eq keys equal to T are taken, by index
+  const uint32_t T = prefix;
+  if (s_eq == need) {
+    for (int w = warp; w < nblk; w += kSalThreads / 32) {
+      const int i = w * 32 + lane;
+      const bool take = i < nq && __float_as_uint(score[i]) >= T;
+      const uint32_t word = __ballot_sync(kFull, take);
+      if (lane == 0) bits[w] = word;
+    }
+  } else if (warp == 0) {
+    uint32_t left = need;  // equal keys still to take, in index order
+    for (int w = 0; w < nblk; ++w) {
+      const int i = w * 32 + lane;
+      const uint32_t key = i < nq ? __float_as_uint(score[i]) : 0u;
+      const bool eq = i < nq && key == T;
+      const uint32_t eqm = __ballot_sync(kFull, eq);
+      const uint32_t before = __popc(eqm & ((1u << lane) - 1u));
+      const bool take = i < nq && (key > T || (eq && before < left));
+      const uint32_t word = __ballot_sync(kFull, take);
+      const uint32_t ne = __popc(eqm);
+      left = left > ne ? left - ne : 0u;
+      if (lane == 0) bits[w] = word;
+    }
+  }
+  __syncthreads();
 
   char* dst = p.arena + p.lt.base[li] + hd.sal + b * hd.sal_bs;
   uint32_t* out_bits = reinterpret_cast<uint32_t*>(dst);
