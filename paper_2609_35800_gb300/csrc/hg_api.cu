@@ -7,6 +7,7 @@
 #include <cuda_runtime.h>
 
 #include <algorithm>
+#include <atomic>
 #include <climits>
 #include <cmath>
 #include <cstdint>
@@ -138,15 +139,16 @@ bool range_ok(const hg_cache* c, int32_t begin, int32_t count) {
 // multiples of 64 tokens and depend only on the layer range and the device,
 // so the workspace bound holds for every appended count.
 int sm_count() {
-  static int cached[64] = {};
+  // per device, filled on first use; concurrent first calls store the same value
+  static std::atomic<int> cached[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 152;
-  if (cached[dev] == 0) {
-    int n = 0;
+  int n = cached[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
     if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 152;
-    cached[dev] = n;
+    cached[dev].store(n, std::memory_order_relaxed);
   }
-  return cached[dev];
+  return n;
 }
 
 int round_up_to(int x, int g) { return ((x + g - 1) / g) * g; }

@@ -1,12 +1,13 @@
 // Quantize-pack, dequantize and append kernels of the HeadGuard KV cache.
 //
 // Quantize (Sec. 3 "Applying protection" over the Sec. 1 / Sec. 4 bases).
-// Every base stages a 64-token tile of one (layer, batch row, KV head) in
-// shared memory with coalesced asynchronous copies and then works one thread
-// per vector: per-token min-max rows (Sec. 1), AKVQ-style rows (Sec. 4: keys
-// rotated by the Hadamard-128 in registers first), KIVI-style value rows
-// (four 32-channel groups) and KIVI-style key groups (one thread per channel
-// over 32 consecutive image tokens).  The head's class and the image span are
+// A CTA is one warp: it stages the K rows or the V rows of a 32-token tile of
+// one (layer, batch row, KV head) in shared memory with coalesced asynchronous
+// copies and then works one lane per vector: per-token min-max rows (Sec. 1),
+// AKVQ-style rows (Sec. 4: keys rotated by the Hadamard-128 in registers
+// first, a row over a lane pair), KIVI-style value rows (four 32-channel
+// groups) and KIVI-style key groups (one lane per channel pair over the 32
+// image tokens of the tile).  The head's class and the image span are
 // resolved once per CTA, so protected heads and text tokens take a uniform
 // BF16 copy path.  Codes, scales and zeros follow the group quantizer exactly
 // (round half to even of the IEEE quotient, no contraction).
@@ -34,11 +35,11 @@ __device__ __forceinline__ void bf16x4_to_f32(uint2 w, float (&x)[4]) {
 // ---------------------------------------------------------------------------
 // Per-token min-max base: one thread per (token, K or V) vector.
 //
-// A CTA takes 64 tokens of one (layer, row, KV head): the K and V rows are
-// staged in shared memory with coalesced loads (272-byte row pitch, so that
-// a thread's 16-byte reads of its own row are conflict free), then thread i
-// owns K row i, thread 64 + i V row i.  A coded vector is quantized by its
-// thread alone -- min / max over bf16x2 pairs (exact), then per element
+// A CTA takes the K rows or the V rows of 32 tokens of one (layer, row, KV
+// head), staged in shared memory with coalesced loads (272-byte row pitch, so
+// that a lane's 16-byte reads of its own row are conflict free); lane i owns
+// row i.  A coded vector is quantized by its lane alone -- min / max over
+// bf16x2 pairs (exact), then per element
 //   T = RN(d * r + 192), d = fl(x - min), r = RN(1 / scale):
 // T lies in [128, 256), so its low 16 mantissa bits hold d * r to 2^-16 and
 // bits 16.. hold floor(d * r + 0.5) once 0x8000 is added.  Within 2^-16 of
