@@ -9,6 +9,7 @@ import numpy as np
 import pytest
 import torch
 
+import oracle
 import paper_2609_35800_gb300 as hg
 from paper_2609_35800_gb300 import workloads as wl
 from paper_2609_35800_gb300.runner import CacheRunner
@@ -238,6 +239,36 @@ def test_salient_ties_and_meta16():
     hg.hg_quantize_kv(runner.cache, 0, [k], [v])
     torch.cuda.synchronize()
     kb, vb = bits16(k), bits16(v)
+    o = oracle_layer(runner, 0, kb, vb)
+    check_arena_layer(runner, 0, kb, vb, o)
+
+
+@pytest.mark.parametrize("mode", ["all_equal", "one_salient", "overflow"])
+def test_salient_select_extremes(mode):
+    """The selection's edge cases against the oracle: every image key the same
+    (all scores tie: the first ns tokens by index), a single salient token per
+    head, and keys whose squared norm overflows to +inf (they rank above every
+    finite score, ties among them to the lower index)."""
+    permille = 1 if mode == "one_salient" else 20
+    w = wl.custom("sal_x_" + mode, 1, 2, 8, 4, 7, 160, 9, A, 4, 0, decode_steps=1, seed=5,
+                  protected=[(0, 2)], salient_permille=permille)
+    runner = CacheRunner(w)
+    B, H, T = w.batch, w.kv_heads, w.seq_len
+    gen = torch.Generator().manual_seed(31)
+    k = torch.randn((B, H, T, 128), generator=gen)
+    v = torch.randn((B, H, T, 128), generator=gen)
+    s0 = w.img_start
+    if mode == "all_equal":
+        k[:, :, s0:s0 + w.image] = k[:, :, s0:s0 + 1]
+    elif mode == "overflow":
+        ns = oracle.salient_count(w.image, permille)
+        rows = torch.tensor([3, 17, 17 + 64, 150])[:ns - 1]  # fewer than ns, so all are taken
+        k[:, :, s0 + rows, 5] = 1e20  # squared in binary32: +inf
+    kb16 = k.to(torch.bfloat16).contiguous().cuda()
+    vb16 = v.to(torch.bfloat16).contiguous().cuda()
+    hg.hg_quantize_kv(runner.cache, 0, [kb16], [vb16])
+    torch.cuda.synchronize()
+    kb, vb = bits16(kb16), bits16(vb16)
     o = oracle_layer(runner, 0, kb, vb)
     check_arena_layer(runner, 0, kb, vb, o)
 
