@@ -293,11 +293,29 @@ __device__ __forceinline__ void chunk_near_tie(const uint32_t (&a)[8], X x, floa
     c8[i] = (a[i] & 0xfff8u) ? ((a[i] >> 16) & L) : exact_code(__fsub_rn(x(i), mn), scale, (float)L);
 }
 
-// Chunks per store unit of the packed row: the chunks whose codes share the
-// words that a chunk's codes go into (4 bits: one word per chunk; 2 bits: two
-// chunks per word; 3 bits: four chunks per plane word).
+// Chunk k's codes written over its bits of a packed row that this thread has
+// already stored: word k (4 bits), or half k % 2 of word k / 2 (2 and 3 bits)
+// and, at 3 bits, byte ((k >> 1) & 1) | ((k & 1) << 1) of plane word 8 + k / 4
+// (the layout of store_chunk).  The other chunks' bits are read back.
 template <int BITS>
-constexpr int kChunksPerUnit = BITS == 4 ? 1 : (BITS == 2 ? 2 : 4);
+__device__ __forceinline__ void patch_chunk(int k, const uint32_t (&c)[8], uint32_t* codes) {
+  uint32_t lo = 0u, hb = 0u;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    lo |= (BITS == 4) ? (c[i] << (4 * i)) : ((c[i] & 3u) << (2 * i));
+    if (BITS == 3) hb |= ((c[i] >> 2) & 1u) << i;
+  }
+  if (BITS == 4) {
+    codes[k] = lo;
+    return;
+  }
+  const int sh = 16 * (k & 1);
+  codes[k >> 1] = (codes[k >> 1] & ~(0xffffu << sh)) | (lo << sh);
+  if (BITS == 3) {
+    const int pb = 8 * (((k >> 1) & 1) | ((k & 1) << 1));
+    codes[8 + (k >> 2)] = (codes[8 + (k >> 2)] & ~(0xffu << pb)) | (hb << pb);
+  }
+}
 
 // One group of a BF16 row: chunks [k0, k0 + nk) (8 channels each) with their
 // min / max over bf16x2 pairs (exact), signed zeros folded to +0,
@@ -307,11 +325,12 @@ constexpr int kChunksPerUnit = BITS == 4 ? 1 : (BITS == 2 ? 2 : 4);
 // by four only (a KIVI-style value group whole; eight measured slower on the
 // per-token rows), so that the code stays small in the instruction cache.
 // A chunk with an element near a tie (fast rule) is emitted with its fast
-// codes and flagged; after the loop each thread codes the store units of its
-// flagged chunks again, the flagged elements by the exact rule, and stores
-// them over the first ones.  The threads of a warp do this side by side, so a
-// warp pays for the largest number of flagged units of one thread instead of
-// running every thread's near ties one after another inside the loop.
+// codes and flagged; after the loop each thread codes its flagged chunks again,
+// the flagged elements by the exact rule, and writes each chunk's bits over
+// the stored ones (patch_chunk).  The threads of a warp do this side by side,
+// so a warp pays for the largest number of flagged chunks of one thread
+// instead of running every thread's near ties one after another inside the
+// loop.
 template <int BITS, bool M16>
 __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int nk, uint32_t* codes, char* meta,
                                                    size_t mi, uint32_t& prev, uint32_t& plane) {
@@ -380,24 +399,19 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
     }
     emit_chunk<BITS>(k, c8, codes, prev, plane);
   }
-  constexpr int U = kChunksPerUnit<BITS>;
   while (ties) {
-    const int u0 = k0 + (((__ffs(ties) - 1) / U) * U);  // first chunk of the unit
-    ties &= ~(((1u << U) - 1u) << (u0 - k0));
-    uint32_t up = 0u, upl = 0u;
-#pragma unroll 1
-    for (int k = u0; k < u0 + U; ++k) {
-      const uint4 v = r4[k];
-      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-      uint64_t x2[4];
+    const int k = k0 + (__ffs(ties) - 1);
+    ties &= ties - 1;
+    const uint4 v = r4[k];
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    uint64_t x2[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);
-      uint32_t a[8], c8[8];
-      chunk_T(x2, mnp, r2, c2, a);
-      chunk_near_tie<BITS>(a, [&](int i) { return __uint_as_float((i & 1) ? (w[i >> 1] & 0xffff0000u) : (w[i >> 1] << 16)); },
-                           mn, scale, c8);
-      emit_chunk<BITS>(k, c8, codes, up, upl);
-    }
+    for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);
+    uint32_t a[8], c8[8];
+    chunk_T(x2, mnp, r2, c2, a);
+    chunk_near_tie<BITS>(a, [&](int i) { return __uint_as_float((i & 1) ? (w[i >> 1] & 0xffff0000u) : (w[i >> 1] << 16)); },
+                         mn, scale, c8);
+    patch_chunk<BITS>(k, c8, codes);
   }
 }
 
