@@ -59,48 +59,26 @@ __device__ __noinline__ uint32_t exact_code(float d, float scale, float levels) 
   return (uint32_t)fminf(fmaxf(rintf(__fdiv_rn(d, scale)), 0.0f), levels);
 }
 
-// Eight codes of channels 8k..8k+7 into the packed row: 4 bits -> word k;
-// 2 bits -> half of word k/2; 3 bits -> the same 2-bit half plus one byte of
-// plane word 8 + k/4 (byte ((k >> 1) & 1) | ((k & 1) << 1): channel index bits
-// 3 and 4 exchanged), each word stored once complete.  `lo` holds the chunk's
-// 32 (4-bit) or 16 (2- and 3-bit) code bits, `hb` the 8 bit-2 bits (3-bit).
+// The packed bits of one 8-channel chunk: `lo` its 32 (4-bit) or 16 (2- and
+// 3-bit) low code bits in channel order, `hb` its 8 bit-2 bits (3-bit).
 template <int BITS>
-__device__ __forceinline__ void store_chunk(int k, uint32_t lo, uint32_t hb, uint32_t* codes, uint32_t& prev,
-                                            uint32_t& plane) {
-  if (BITS == 4) {
-    codes[k] = lo;
-    return;
-  }
-  if (k & 1) codes[k >> 1] = prev | (lo << 16);
-  else prev = lo;
-  if (BITS == 3) {
-    plane |= hb << (8 * (((k >> 1) & 1) | ((k & 1) << 1)));
-    if ((k & 3) == 3) {
-      codes[8 + (k >> 2)] = plane;
-      plane = 0u;
-    }
-  }
-}
-
-template <int BITS>
-__device__ __forceinline__ void emit_chunk(int k, const uint32_t (&c)[8], uint32_t* codes, uint32_t& prev,
-                                           uint32_t& plane) {
-  uint32_t lo = 0u, hb = 0u;
+__device__ __forceinline__ void chunk_bits(const uint32_t (&c)[8], uint32_t& lo, uint32_t& hb) {
+  lo = 0u;
+  hb = 0u;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     lo |= (BITS == 4) ? (c[i] << (4 * i)) : ((c[i] & 3u) << (2 * i));
     if (BITS == 3) hb |= ((c[i] >> 2) & 1u) << i;
   }
-  store_chunk<BITS>(k, lo, hb, codes, prev, plane);
 }
 
 // The same from the eight T' words of the fast rule (code in bits 16..): each
 // code is shifted straight into its packed position (one shift and one
 // and-or per element instead of extracting it first).
 template <int BITS>
-__device__ __forceinline__ void emit_from_T(int k, const uint32_t (&a)[8], uint32_t* codes, uint32_t& prev,
-                                            uint32_t& plane) {
-  uint32_t lo = 0u, hb = 0u;
+__device__ __forceinline__ void chunk_bits_T(const uint32_t (&a)[8], uint32_t& lo, uint32_t& hb) {
+  lo = 0u;
+  hb = 0u;
 #pragma unroll
   for (int i = 0; i < 8; ++i) {
     if (BITS == 4) {
@@ -111,7 +89,23 @@ __device__ __forceinline__ void emit_from_T(int k, const uint32_t (&a)[8], uint3
       if (BITS == 3) hb |= (a[i] >> (18 - i)) & (1u << i);
     }
   }
-  store_chunk<BITS>(k, lo, hb, codes, prev, plane);
+}
+
+// Chunks kg..kg+3 (kg a multiple of 4) into the packed row, one vector store
+// per word run: 4 bits -> words kg..kg+3 (16 bytes); 2 and 3 bits -> words
+// kg/2, kg/2 + 1 (8 bytes, chunk k in half k % 2 of word k / 2); 3 bits also
+// plane word 8 + kg/4, chunk k's bit-2 byte at ((k >> 1) & 1) | ((k & 1) << 1)
+// (channel index bits 3 and 4 exchanged).  A packed row is 16 x bits bytes on
+// a 16-byte boundary.
+template <int BITS>
+__device__ __forceinline__ void store_group(int kg, const uint32_t (&lo)[4], const uint32_t (&hb)[4],
+                                            uint32_t* codes) {
+  if (BITS == 4) {
+    *reinterpret_cast<uint4*>(codes + kg) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+    return;
+  }
+  *reinterpret_cast<uint2*>(codes + (kg >> 1)) = make_uint2(lo[0] | (lo[1] << 16), lo[2] | (lo[3] << 16));
+  if (BITS == 3) codes[8 + (kg >> 2)] = hb[0] | (hb[2] << 8) | (hb[1] << 16) | (hb[3] << 24);
 }
 
 // T' = RN(fl(x - min) r + C) for the four channel pairs of a chunk (the fast
@@ -225,10 +219,21 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
       }
     }
   }
-#pragma unroll
-  for (int i = 0; i < BITS; ++i) {
-    dst0[i] = wd0[i];
-    dst1[i] = wd1[i];
+  // both channels' rows are contiguous (dst1 = dst0 + BITS) and start on a
+  // 16-byte (2, 4 bits) or 8-byte (3 bits) boundary: vector stores
+  if (BITS == 3) {
+    uint2* d2 = reinterpret_cast<uint2*>(dst0);
+    d2[0] = make_uint2(wd0[0], wd0[1]);
+    d2[1] = make_uint2(wd0[2 % BITS], wd1[0]);
+    d2[2] = make_uint2(wd1[1], wd1[2 % BITS]);
+  } else {
+    uint4* d4 = reinterpret_cast<uint4*>(dst0);
+    if (BITS == 2) {
+      d4[0] = make_uint4(wd0[0], wd0[1 % BITS], wd1[0], wd1[1 % BITS]);
+    } else {
+      d4[0] = make_uint4(wd0[0], wd0[1 % BITS], wd0[2 % BITS], wd0[3 % BITS]);
+      d4[1] = make_uint4(wd1[0], wd1[1 % BITS], wd1[2 % BITS], wd1[3 % BITS]);
+    }
   }
 }
 
@@ -254,7 +259,7 @@ __device__ __forceinline__ void quantize_key_pair(const char* col, uint32_t* dst
 //     reference division, 1 for the tie-break), so every element within two
 //     units of the half-integer boundary -- T' low bits in [2, 6] -- is among
 //     those with low bits in [0, 7], which take the exact rule (chunk_T,
-//     emit_from_T; a chunk with such an element goes through chunk_near_tie).
+//     chunk_bits_T; a chunk with such an element goes through chunk_near_tie).
 //   otherwise (tiny scale): the exact rule for every element.
 template <int BITS, bool M16>
 __device__ __forceinline__ void chunk_codes(const uint32_t (&w)[4], float mn, float scale, float r,
@@ -296,7 +301,7 @@ __device__ __forceinline__ void chunk_near_tie(const uint32_t (&a)[8], X x, floa
 // Chunk k's codes written over its bits of a packed row that this thread has
 // already stored: word k (4 bits), or half k % 2 of word k / 2 (2 and 3 bits)
 // and, at 3 bits, byte ((k >> 1) & 1) | ((k & 1) << 1) of plane word 8 + k / 4
-// (the layout of store_chunk).  The other chunks' bits are read back.
+// (the layout of store_group).  The other chunks' bits are read back.
 template <int BITS>
 __device__ __forceinline__ void patch_chunk(int k, const uint32_t (&c)[8], uint32_t* codes) {
   uint32_t lo = 0u, hb = 0u;
@@ -333,7 +338,7 @@ __device__ __forceinline__ void patch_chunk(int k, const uint32_t (&c)[8], uint3
 // loop.
 template <int BITS, bool M16>
 __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int nk, uint32_t* codes, char* meta,
-                                                   size_t mi, uint32_t& prev, uint32_t& plane) {
+                                                   size_t mi) {
   __nv_bfloat162 mn2, mx2;
   {
     const uint4 v = r4[k0];
@@ -378,26 +383,33 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
   const uint32_t cbits = __float_as_uint(192.50006103515625f);  // C = 192.5 + 4 * 2^-16
   const uint64_t c2 = f32x2(cbits, cbits);
   uint32_t ties = 0u;  // bit k - k0: chunk k has an element near a tie
-#pragma unroll 4
-  for (int k = k0; k < k0 + nk; ++k) {
-    const uint4 v = r4[k];
-    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-    uint32_t c8[8];
-    if (fast) {
-      uint64_t x2[4];
+#pragma unroll 1
+  for (int kg = k0; kg < k0 + nk; kg += 4) {
+    uint32_t lo[4], hb[4];
 #pragma unroll
-      for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1
-      uint32_t a[8];
-      if (!chunk_T(x2, mnp, r2, c2, a)) ties |= 1u << (k - k0);  // about one chunk in 100
-      emit_from_T<BITS>(k, a, codes, prev, plane);
-      continue;
-    } else if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
+    for (int kk = 0; kk < 4; ++kk) {
+      const int k = kg + kk;
+      const uint4 v = r4[k];
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+      if (fast) {
+        uint64_t x2[4];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) c8[i] = 0u;
-    } else {
-      chunk_codes<BITS, M16>(w, mn, scale, r, c8);
+        for (int i = 0; i < 4; ++i) x2[i] = f32x2(w[i] << 16, w[i] & 0xffff0000u);  // channels 2i, 2i + 1
+        uint32_t a[8];
+        if (!chunk_T(x2, mnp, r2, c2, a)) ties |= 1u << (k - k0);  // about one chunk in 100
+        chunk_bits_T<BITS>(a, lo[kk], hb[kk]);
+      } else {
+        uint32_t c8[8];
+        if (scale == 0.0f) {  // constant group (or a step below binary16 range): every code 0
+#pragma unroll
+          for (int i = 0; i < 8; ++i) c8[i] = 0u;
+        } else {
+          chunk_codes<BITS, M16>(w, mn, scale, r, c8);
+        }
+        chunk_bits<BITS>(c8, lo[kk], hb[kk]);
+      }
     }
-    emit_chunk<BITS>(k, c8, codes, prev, plane);
+    store_group<BITS>(kg, lo, hb, codes);
   }
   while (ties) {
     const int k = k0 + (__ffs(ties) - 1);
@@ -418,19 +430,16 @@ __device__ __forceinline__ void quantize_row_group(const uint4* r4, int k0, int 
 // Per-token min-max over the whole 128-channel row (Sec. 1), one group.
 template <int BITS, bool M16>
 __device__ __forceinline__ void quantize_row_token(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
-  uint32_t prev = 0u, plane = 0u;
-  quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 0, 16, codes, meta, mi, prev, plane);
+  quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 0, 16, codes, meta, mi);
 }
 
 // KIVI-style values (Sec. 4): four groups of 32 channels per token
 // (metadata mi .. mi + 3); the packing is the per-token one (channel order).
 template <int BITS, bool M16>
 __device__ __forceinline__ void quantize_row_kivi_v(const char* row_s, uint32_t* codes, char* meta, size_t mi) {
-  uint32_t prev = 0u, plane = 0u;
 #pragma unroll 1
   for (int j = 0; j < 4; ++j)
-    quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 4 * j, 4, codes, meta, mi + j, prev,
-                                  plane);
+    quantize_row_group<BITS, M16>(reinterpret_cast<const uint4*>(row_s), 4 * j, 4, codes, meta, mi + j);
 }
 
 // ---------------------------------------------------------------------------
@@ -521,11 +530,19 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
     mn = half_sat(mn);
   }
   if (hh == 0) store_meta(meta, mi, scale, mn, M16);
-  uint32_t prev = 0u, plane = 0u;
-  if (scale == 0.0f) {
-    const uint32_t z8[8] = {0u, 0u, 0u, 0u, 0u, 0u, 0u, 0u};
+  uint32_t lo[NK], hb[NK];  // this thread's chunks k0..k0+NK-1, stored four at a time at the end
+  auto store_all = [&]() {
 #pragma unroll
-    for (int k = 0; k < NK; ++k) emit_chunk<BITS>(k0 + k, z8, codes, prev, plane);
+    for (int g = 0; g < NK / 4; ++g) {
+      const uint32_t l4[4] = {lo[4 * g], lo[4 * g + 1], lo[4 * g + 2], lo[4 * g + 3]};
+      const uint32_t h4[4] = {hb[4 * g], hb[4 * g + 1], hb[4 * g + 2], hb[4 * g + 3]};
+      store_group<BITS>(k0 + 4 * g, l4, h4, codes);
+    }
+  };
+  if (scale == 0.0f) {
+#pragma unroll
+    for (int k = 0; k < NK; ++k) lo[k] = hb[k] = 0u;
+    store_all();
     return;
   }
   bool fast = scale >= 2.3509887e-38f;  // the fast rule of the min-max rows (chunk_T)
@@ -548,8 +565,9 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
         const int cu = min(max((int)(a >> 16) - 0x4340, 0), (int)L);
         c8[i] = ((a & 0xffffu) < 3u) ? exact_code(d, scale, levels) : (uint32_t)cu;
       }
-      emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
+      chunk_bits<BITS>(c8, lo[k], hb[k]);
     }
+    store_all();
     return;
   }
   if (fast) {  // the fast rule of the min-max rows (chunk_T)
@@ -563,14 +581,15 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
       const uint64_t x2[4] = {xp[4 * k], xp[4 * k + 1], xp[4 * k + 2], xp[4 * k + 3]};
       uint32_t a[8];
       if (chunk_T(x2, mn2, r2, c2, a)) {
-        emit_from_T<BITS>(k0 + k, a, codes, prev, plane);
+        chunk_bits_T<BITS>(a, lo[k], hb[k]);
       } else {
         uint32_t c8[8];
         chunk_near_tie<BITS>(a, [&](int i) { return (i & 1) ? pair_hi(x2[i >> 1]) : pair_lo(x2[i >> 1]); }, mn,
                              scale, c8);
-        emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
+        chunk_bits<BITS>(c8, lo[k], hb[k]);
       }
     }
+    store_all();
     return;
   }
 #pragma unroll
@@ -581,8 +600,9 @@ __device__ __forceinline__ void quantize_row_rotated(const char* row_s, int hh, 
       const uint64_t x2 = xp[4 * k + (i >> 1)];
       c8[i] = exact_code(__fsub_rn((i & 1) ? pair_hi(x2) : pair_lo(x2), mn), scale, levels);
     }
-    emit_chunk<BITS>(k0 + k, c8, codes, prev, plane);
+    chunk_bits<BITS>(c8, lo[k], hb[k]);
   }
+  store_all();
 }
 
 // A BF16 row copied as it is (SPLIT = 2: lane hh of a pair copies its half).
