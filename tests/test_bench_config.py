@@ -85,6 +85,34 @@ def test_cpu_baseline_fields_split_quantize_and_decode():
     assert "extrapolated from 7 of 28" in g["decode_tokens_per_s_basis"]
 
 
+def test_cpu_sample_plan_and_timed_repetitions(monkeypatch):
+    """The CPU baseline samples the whole workload step on the small caches
+    and one layer with two decode steps on the large ones, and repeats the
+    sample until the timed oracle calls reach the floor (at least once, at most
+    max_reps times), summing bytes, seconds and the quantize / decode parts."""
+    import bench
+    from paper_2609_35800_gb300 import workloads as wl
+    assert bench.cpu_sample_plan(wl.WORKLOADS["qwen25vl7b"]) == (28, 32)
+    assert bench.cpu_sample_plan(wl.WORKLOADS["qwen25vl72b"]) == (1, 2)
+    calls = []
+
+    def fake(w, n_layers, n_steps, parts=None):
+        calls.append((n_layers, n_steps))
+        parts.update(quant_bytes=10, quant_s=0.5, dec_bytes=30, dec_s=1.5)
+        return 40, 2.0, 7
+
+    monkeypatch.setattr(bench, "oracle_sample", fake)
+    w = wl.WORKLOADS["qwen25vl7b"]
+    nb, secs, threads, reps, parts = bench.timed_oracle_samples(w, 28, 32, min_seconds=5.0)
+    assert (reps, nb, secs, threads) == (3, 120, 6.0, 7) and calls == [(28, 32)] * 3
+    assert parts == {"quant_bytes": 30, "quant_s": 1.5, "dec_bytes": 90, "dec_s": 4.5}
+    f = bench.cpu_baseline_fields(w, 28, 32 * reps, parts)
+    assert f["decode_tokens_per_s"] == 1 * 96 / 4.5  # batch 1, 3 x 32 steps in 4.5 s
+    calls.clear()
+    assert bench.timed_oracle_samples(w, 28, 32, min_seconds=0.0)[3] == 1   # at least once
+    assert bench.timed_oracle_samples(w, 28, 32, min_seconds=1e9, max_reps=4)[3] == 4
+
+
 def test_floors_on_stubbed_events(monkeypatch):
     """measure_floors times three things with the same L2 flush before each
     repetition and reports medians; driven here with stub events on CPU."""
