@@ -107,7 +107,7 @@ def test_cpu_sample_plan_and_timed_repetitions(monkeypatch):
     assert (reps, nb, secs, threads) == (3, 120, 6.0, 7) and calls == [(28, 32)] * 3
     assert parts == {"quant_bytes": 30, "quant_s": 1.5, "dec_bytes": 90, "dec_s": 4.5}
     f = bench.cpu_baseline_fields(w, 28, 32 * reps, parts)
-    assert f["decode_tokens_per_s"] == 1 * 96 / 4.5  # batch 1, 3 x 32 steps in 4.5 s
+    assert f["decode_tokens_per_s"] == round(1 * 96 / 4.5, 3)  # batch 1, 3 x 32 steps in 4.5 s
     calls.clear()
     assert bench.timed_oracle_samples(w, 28, 32, min_seconds=0.0)[3] == 1   # at least once
     assert bench.timed_oracle_samples(w, 28, 32, min_seconds=1e9, max_reps=4)[3] == 4
