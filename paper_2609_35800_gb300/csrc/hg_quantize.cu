@@ -687,7 +687,6 @@ __device__ __forceinline__ bool copy_tile_whole(const QuantizeParams& p, int li,
 template <int BITS, bool M16, int BASE, int PARTS>
 struct TokenTiles {
   static constexpr int kNParts = PARTS == 3 ? 2 : 1;
-  static __device__ __forceinline__ int count(const QuantizeParams& p) { return (p.d.T + kQTok - 1) / kQTok; }
   static __device__ __forceinline__ int part(int i) { return PARTS == 3 ? i : (PARTS == 1 ? 0 : 1); }
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
@@ -770,11 +769,8 @@ struct TokenTiles {
 template <int BITS, bool M16, int PARTS>
 struct KiviTiles {
   static constexpr int kNParts = PARTS == 3 ? 2 : 1;
-  // tile x: [origin - 32 + 32 x, + 32) clipped to [0, T), origin = s mod 32
-  static __device__ __forceinline__ int count(const QuantizeParams& p) {
-    return (p.d.T - p.tile_origin + kKiviGroup + kQTok - 1) / kQTok;
-  }
   static __device__ __forceinline__ int part(int i) { return PARTS == 3 ? i : (PARTS == 1 ? 0 : 1); }
+  // tile x: [origin - 32 + 32 x, + 32) clipped to [0, T), origin = s mod 32
   static __device__ __forceinline__ TileSpan span(const QuantizeParams& p, int tx) {
     TileSpan sp;
     sp.tlo = p.tile_origin - kKiviGroup + kQTok * tx;
