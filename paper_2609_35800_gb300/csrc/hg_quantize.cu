@@ -325,10 +325,11 @@ __device__ __forceinline__ void patch_chunk(int k, const uint32_t (&c)[8], uint3
 // One group of a BF16 row: chunks [k0, k0 + nk) (8 channels each) with their
 // min / max over bf16x2 pairs (exact), signed zeros folded to +0,
 // scale = fl((max - min) / levels), metadata stored at index mi (binary16
-// pair with M16: codes against the rounded pair), codes 0 when scale == 0,
-// each chunk's codes emitted into the packed row.  The chunk loop is unrolled
-// by four only (a KIVI-style value group whole; eight measured slower on the
-// per-token rows), so that the code stays small in the instruction cache.
+// pair with M16: codes against the rounded pair), codes 0 when scale == 0.
+// The chunks go in groups of four (a KIVI-style value group whole), each
+// group's packed words written by one vector store (store_group); the group
+// loop stays rolled so that the code stays small in the instruction cache
+// (eight chunks per step measured slower on the per-token rows).
 // A chunk with an element near a tie (fast rule) is emitted with its fast
 // codes and flagged; after the loop each thread codes its flagged chunks again,
 // the flagged elements by the exact rule, and writes each chunk's bits over
